@@ -1,0 +1,397 @@
+#!/usr/bin/env python
+"""Benchmark of the MISA-T batched routing decision on GB300.
+
+One step = one pass of the whole hot path over one batch: misat_route (block hash,
+longest-prefix probe, caps, scoring, admission rounds) + misat_commit (index insert,
+session update, eviction).  Workload: the throughput-stress configuration, 128
+instances x 262,144 KV blocks filled to 95% (33.5M resident block hashes), batches of
+65,536 mixed RLVR/RLHF/agentic requests (40/30/30), synthetic and seeded.
+
+Every timed step starts from the same router state (a device checkpoint restored
+before the step, outside the step's CUDA events), so the K steps do identical work.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl gb300|reference]
+
+Under torchrun (N > 1) every rank runs an independent replica (the path does not
+shard across GPUs in this build): weak scaling, value = all ranks' requests / max time.
+"""
+
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "routed requests/s (route+commit)"
+UNIT = "requests/s"
+CLOCK_QUERY = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+               "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+               "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+
+def kernels_per_step(rounds):
+    """Kernels one route+commit launches: route = prologue 2 + hash + caps + probe 2 + 5 per round +
+    finalize; commit = insert + sessions + eviction select + compaction."""
+    return 7 + 5 * rounds + 4
+
+
+def parse_args():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=30)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
+    ap.add_argument("--n", type=int, default=65536, help="requests per batch")
+    ap.add_argument("--fill", type=float, default=0.95, help="resident fraction of the KV block capacity")
+    ap.add_argument("--e2e-steps", type=int, default=5)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    return ap.parse_args()
+
+
+def peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        d = json.load(open(p))
+        return float(d["hbm_gbs"]), "measured"
+    return 6800.0, "fallback"
+
+
+def workload(args):
+    from paper_2608_11152_gb300 import workload as wl
+
+    return wl.config5(n=args.n, fill=args.fill)
+
+
+def workload_config(args, sc):
+    return {"workload": f"throughput stress: {sc.W} instances x {int(sc.cap_blocks[0])} blocks, "
+                        f"fill {int(round(args.fill * 100))}%, {args.n} requests/batch 40/30/30 RLVR/RLHF/agentic",
+            "instances": int(sc.W), "cap_blocks": int(sc.cap_blocks[0]), "fill": args.fill,
+            "batch_requests": int(args.n), "batch_tokens": int(sc.batch.n_tokens), "block_tokens": 16,
+            "rounds": int(sc.rounds), "mode": "MISA-T",
+            "l2": "inputs larger than L2 (tokens %.2f GB, tables %.2f GB) and a state restore of the "
+                  "tables between steps" % (sc.batch.n_tokens * 4 / 1e9, sc.W * 2 * int(sc.cap_blocks[0]) * 16 / 1e9)}
+
+
+class ClockSampler:
+    """nvidia-smi clocks and throttle reasons sampled every 100 ms while active."""
+
+    def __init__(self, index):
+        self.index = index
+        self.f = tempfile.NamedTemporaryFile("w+", suffix=".csv", delete=False)
+        self.p = None
+        self.t0 = self.t1 = None
+
+    def start(self):
+        try:
+            self.p = subprocess.Popen(["nvidia-smi", f"--id={self.index}", f"--query-gpu={CLOCK_QUERY}",
+                                       "--format=csv,noheader,nounits", "-lms", "100"], stdout=self.f,
+                                      stderr=subprocess.DEVNULL)
+        except Exception:
+            self.p = None
+
+    def stop(self):
+        if self.p is not None:
+            self.p.terminate()
+            try:
+                self.p.wait(timeout=5)
+            except Exception:
+                self.p.kill()
+        self.f.flush()
+
+    def summary(self):
+        rows = []
+        try:
+            for line in open(self.f.name):
+                parts = [x.strip() for x in line.split(",")]
+                if len(parts) >= 9 and parts[1].replace(".", "").isdigit():
+                    rows.append(parts)
+        except Exception:
+            pass
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no nvidia-smi samples"], "samples": 0}
+        sm = [float(r[1]) for r in rows]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in rows for i in range(4) if r[5 + i].lower().startswith("active")})
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(float(r[2]) for r in rows),
+                "reasons": reasons, "samples": len(rows), "power_w_max": max(float(r[3]) for r in rows)}
+
+
+def setup_router(sc, torch):
+    from paper_2608_11152_gb300 import misat
+
+    r = misat.Router(sc.cap_blocks, max_batch=sc.max_batch, max_tokens=sc.max_tokens,
+                     protected_frac_q16=sc.protected_frac_q16, rounds=sc.rounds, mode=sc.mode,
+                     hold_delay_q=sc.hold_delay_q, prior_kbar=sc.prior_kbar, prior_T_us=sc.prior_T_us)
+    r.set_mixture(sc.rho_ppm)
+    r.set_instance_state(sc.backlog_q, sc.tokcost_q, sc.contraction)
+    for f in sc.fillers:
+        r.load_entries(f.w, f.keys, f.metas)
+    for b, c in sc.warm:
+        r.route(r.device_batch(b))
+        r.commit()
+        r.complete(c.session, c.cls, c.total_blocks, c.residency_us, c.done)
+    r.sync()
+    return r
+
+
+def setup_oracle(sc):
+    import oracle
+
+    o = oracle.Oracle(sc.cap_blocks, protected_frac_q16=sc.protected_frac_q16, rounds=sc.rounds, mode=sc.mode,
+                      hold_delay_q=sc.hold_delay_q, prior_kbar=sc.prior_kbar, prior_T_us=sc.prior_T_us)
+    o.set_mixture(sc.rho_ppm)
+    o.set_instance_state(sc.backlog_q, sc.tokcost_q, sc.contraction)
+    for f in sc.fillers:
+        o.load_entries(f.w, f.keys, f.metas)
+    for b, c in sc.warm:
+        o.route(b.cls, b.session, b.tok_off, b.tokens)
+        o.commit()
+        o.complete(c.session, c.cls, c.total_blocks, c.residency_us, c.done)
+    return o
+
+
+def cpu_step(o, b):
+    t = time.perf_counter()
+    o.route(b.cls, b.session, b.tok_off, b.tokens)
+    o.commit()
+    return time.perf_counter() - t
+
+
+def algorithmic_bytes(sc, st):
+    """Algorithmic HBM bytes per launch of the hash and probe kernels (see the design notes)."""
+    b = sc.batch
+    L = np.diff(b.tok_off)
+    nb = L // 16
+    n_blocks = int(nb.sum())
+    # K1: every full block's 16 token ids are read once (64 B) and its key written once (8 B),
+    # plus two 8-byte offsets per request
+    hash_b = 72 * n_blocks + 16 * b.n
+    # K2 phase 1: one 32-byte key group per block-0 probe, the H row written (2 B per pair),
+    # block-0 key, block count and key base read per request
+    first_b = 32 * st.probes_first + 2 * b.n * sc.W + 20 * b.n
+    # K2 phase 2: one 32-byte key group per probe of the binary searches
+    search_b = 32 * (st.probes - st.probes_first)
+    return {"hash": hash_b, "probe_first": first_b, "probe_search": search_b, "n_blocks": n_blocks}
+
+
+def run_gb300(args):
+    import torch
+
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    import __graft_entry__
+
+    if rank == 0 or world == 1:
+        __graft_entry__.build()
+    if dist:
+        dist.barrier()
+    from paper_2608_11152_gb300 import misat
+
+    sc = workload(args)
+    r = setup_router(sc, torch)
+    ckpt = r.checkpoint_save()
+    db = r.device_batch(sc.batch)
+    out = r.alloc_decisions(sc.batch.n)
+    stream = r.stream
+    r.set_timing(True)
+
+    def step():
+        r.route(db, out)
+        r.commit()
+
+    for _ in range(args.warmup):
+        r.checkpoint_restore(ckpt)
+        step()
+        r.phase_times()
+    torch.cuda.synchronize()
+    K = args.steps
+    starts = [torch.cuda.Event(enable_timing=True) for _ in range(K)]
+    ends = [torch.cuda.Event(enable_timing=True) for _ in range(K)]
+    phase_tot = {p: 0.0 for p in misat.PHASES}
+    sampler = ClockSampler(local)
+    sampler.start()
+    time.sleep(0.3)
+    if dist:
+        dist.barrier()
+    torch.cuda.synchronize()
+    t_wall = time.perf_counter()
+    for k in range(K):
+        r.checkpoint_restore(ckpt)
+        torch.cuda.nvtx.range_push("misat_step")
+        starts[k].record(stream)
+        step()
+        ends[k].record(stream)
+        torch.cuda.nvtx.range_pop()
+        for p, v in r.phase_times().items():  # waits for the step (outside its events)
+            phase_tot[p] += v
+    torch.cuda.synchronize()
+    if dist:
+        dist.barrier()
+    wall = time.perf_counter() - t_wall
+    sampler.stop()
+    step_ms = [starts[k].elapsed_time(ends[k]) for k in range(K)]
+    total_ms = float(sum(step_ms))
+    st = r.stats()
+    r.sync()
+    if dist:
+        t = torch.tensor([total_ms], device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        total_ms = float(t.item())
+    n = sc.batch.n
+    value = world * n * K / (total_ms / 1e3)
+
+    # end to end through the public host API: H2D of the batch from pinned memory, route, commit,
+    # D2H of the decisions, every step
+    b = sc.batch
+    pin = {}
+    for name, arr in (("cls", b.cls), ("session", b.session.view(np.int64)), ("tok_off", b.tok_off),
+                      ("tokens", b.tokens)):
+        t = torch.from_numpy(arr).pin_memory()
+        pin[name] = t
+    from paper_2608_11152_gb300.workload import Batch
+
+    hb = Batch(cls=pin["cls"].numpy(), session=pin["session"].numpy().view(np.uint64), group=b.group,
+               tok_off=pin["tok_off"].numpy(), tokens=pin["tokens"].numpy())
+    hout = {k: torch.empty(n, dtype=d).pin_memory().numpy() for k, d in
+            (("inst", torch.int32), ("reason", torch.uint8), ("hit_blocks", torch.int32))}
+    r.checkpoint_restore(ckpt)
+    r.route_host(hb, hout)
+    r.commit()
+    torch.cuda.synchronize()
+    e2e_ms = 0.0
+    for k in range(args.e2e_steps):
+        r.checkpoint_restore(ckpt)
+        torch.cuda.synchronize()
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        r.route_host(hb, hout)
+        r.commit()
+        e1.record(stream)
+        e1.synchronize()
+        e2e_ms += e0.elapsed_time(e1)
+    if dist:
+        t = torch.tensor([e2e_ms], device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        e2e_ms = float(t.item())
+    e2e = world * n * args.e2e_steps / (e2e_ms / 1e3)
+    h2d = int(b.cls.nbytes + b.session.nbytes + b.tok_off.nbytes + b.tokens.nbytes)
+    d2h = int(n * (4 + 1 + 4))
+
+    # roofline: dominant kernel of the step, plus the hash and probe kernels
+    peak, peak_kind = peaks()
+    ab = algorithmic_bytes(sc, st)
+    phase_ms = {p: phase_tot[p] / K for p in phase_tot}
+    dom = max(phase_ms, key=lambda p: phase_ms[p])
+
+    def roof(kind):
+        ms = phase_ms[kind]
+        byts = ab.get(kind)
+        if byts is None or ms <= 0:
+            return None
+        ach = byts / (ms / 1e3) / 1e9
+        return {"bound": "hbm", "achieved": round(ach, 1), "peak": peak, "unit": "GB/s",
+                "frac": round(ach / peak, 4), "traffic": None, "bytes_per_launch": int(byts),
+                "ms_per_launch": round(ms, 4), "peak_kind": peak_kind}
+
+    kernels = {k: roof(k) for k in ("hash", "probe_first", "probe_search")}
+    dom_roof = roof(dom)
+    if dom_roof is None:
+        dom_roof = {"bound": "hbm", "achieved": None, "peak": peak, "unit": "GB/s", "frac": None, "traffic": None,
+                    "kernel": dom, "ms_per_launch": round(phase_ms[dom], 4),
+                    "note": "no algorithmic byte model for this phase yet"}
+    dom_roof["kernel"] = dom
+
+    clocks = sampler.summary()
+    line = {
+        "metric": METRIC, "value": round(value, 1), "unit": UNIT, "n_gpus": world, "steps": K,
+        "warmup": args.warmup, "ms_per_step": round(total_ms / K, 4), "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "u64", "data": "synthetic (seeded, shaped after the paper's workloads)",
+        "config": workload_config(args, sc),
+        "probes_per_s": round(world * st.probes * K / (total_ms / 1e3), 1),
+        "e2e": {"value": round(e2e, 1), "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
+        "gpu_launches": kernels_per_step(sc.rounds) * K,
+        "roofline": dom_roof,
+        "kernels": kernels,
+        "phase_ms": {p: round(v, 4) for p, v in phase_ms.items()},
+        "clocks": clocks,
+        "wall_s_timed_loop": round(wall, 3),
+        "stats": {"admitted": st.n_admitted, "held": st.n_held, "probes": st.probes, "bucket_reads": st.bucket_reads,
+                  "new_keys": st.new_keys, "evicted": st.evicted, "hit_tokens": st.hit_tokens,
+                  "query_tokens": st.query_tokens, "dtv_ppm": st.dtv_ppm},
+    }
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        o = setup_oracle(sc)
+        t = cpu_step(o, sc.batch)
+        line["cpu_baseline"] = {"value": round(n / t, 1), "unit": UNIT, "cores": 1, "kind": "oracle",
+                                "sample": f"one full {n}-request batch (route+commit) from the same warmed state, "
+                                          f"single-threaded C++ oracle, {t:.2f} s; host has {os.cpu_count()} cores"}
+    else:
+        line["cpu_baseline"] = None
+    ckpt.free()
+    r.close()
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if dist:
+        dist.destroy_process_group()
+
+
+def run_reference(args):
+    """The CPU oracle, as it stands, on this host's cores: same workload, metric and unit; every
+    step restarts from the same warmed state (a copy of the oracle state, untimed)."""
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    if rank != 0:
+        return
+    sc = workload(args)
+    base = setup_oracle(sc)
+    n = sc.batch.n
+    total = 0.0
+    for k in range(args.warmup + args.steps):
+        o = base.clone()
+        t = cpu_step(o, sc.batch)
+        o.close()
+        if k >= args.warmup:
+            total += t
+    value = n * args.steps / total
+    line = {
+        "impl": "reference", "metric": METRIC, "value": round(value, 1), "unit": UNIT, "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(1e3 * total / args.steps, 3),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "u64",
+        "data": "synthetic (seeded, shaped after the paper's workloads)", "config": workload_config(args, sc),
+        "cpu_baseline": {"value": round(value, 1), "unit": UNIT, "cores": 1, "kind": "oracle",
+                         "sample": f"each step one full {n}-request batch from the same warmed state "
+                                   f"(single-threaded C++ oracle; host has {os.cpu_count()} cores)"},
+        "e2e": {"value": round(value, 1), "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    args = parse_args()
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_gb300(args)
+
+
+if __name__ == "__main__":
+    main()

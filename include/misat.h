@@ -1,0 +1,276 @@
+/*
+ * misat.h -- C ABI of the GB300 (sm_103a) MISA-T batched routing decision.
+ *
+ * MISA-T ("Scheduling Mixed RL Rollouts Beyond Prefix Locality") is a routing-layer
+ * admission policy for mixed RLVR / RLHF / agentic rollout serving.  For each
+ * request r the router outputs pi(r) in W u {HOLD} (Sec. 3.1): it admits and
+ * places the request on an inference instance, or holds it for re-evaluation.
+ * This library computes that decision for a whole batch on one GPU:
+ *
+ *   1. chained 16-token block hashes of every prompt (Sec. 4.5),
+ *   2. the longest cached prefix H_rw of every request on every instance's
+ *      resident-block index, held as GPU open-addressing hash tables (Sec. 4.5),
+ *   3. caps K_w and K_wb (Sec. 4.1, Eqs. 9-13), eligibility (Eq. 6), prefill
+ *      cost (Eq. 1) and the hold-vs-cold rule (Eq. 7), argmin placement,
+ *   4. arrival-order admission under the global and class caps (Eq. 6, Sec. 4.2),
+ *      then a deterministic commit: index insert, session table update and
+ *      eviction down to each instance's KV block capacity.
+ *
+ * Conventions
+ *   - Return value: MISAT_OK (0) or a negative MISAT_ERR_* code.  Calls validate
+ *     their host-visible arguments before enqueueing anything; an invalid call
+ *     changes no state.
+ *   - Streams: every call is stream-ordered on the stream given to misat_create.
+ *     Calls marked [async] return after enqueueing; calls marked [sync] wait.
+ *   - Device errors (a malformed batch found on the device, a full table) are
+ *     sticky: they are recorded on the device and returned by the next
+ *     misat_sync, misat_stats or misat_dump_* call.  Kernels skip their work once
+ *     an error is recorded, and no device loop is unbounded.
+ *   - Ownership: the caller owns every buffer it passes (batch inputs, decision
+ *     outputs, host arrays); the library owns its tables, counters and scratch
+ *     and frees them in misat_destroy.  Device pointers are raw CUDA device
+ *     addresses on the context's device (e.g. torch tensor data_ptr()).
+ *   - Block size is 16 tokens.  Limits: W <= 1024 instances, capacity <= 2^26
+ *     blocks per instance, <= 2^20 requests per batch, prompts < 2^20 tokens,
+ *     < 2^28 commits per context.
+ */
+#ifndef MISAT_H
+#define MISAT_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* ---- return codes ---- */
+#define MISAT_OK 0
+#define MISAT_ERR_INVALID_ARG (-1)     /* argument outside its documented range */
+#define MISAT_ERR_OOM (-2)             /* device or pinned host allocation failed */
+#define MISAT_ERR_CUDA (-3)            /* a CUDA runtime call failed */
+#define MISAT_ERR_STATE (-4)           /* commit without a pending route */
+#define MISAT_ERR_TABLE_FULL (-5)      /* a bounded probe found no free slot */
+#define MISAT_ERR_BATCH_TOO_LARGE (-6) /* batch exceeds max_batch / max_tokens */
+
+/* ---- policy modes (Sec. 5.2 ablation variants) ---- */
+#define MISAT_MODE_MISA_T 0            /* block-time quota, Eqs. (11),(13) (default) */
+#define MISAT_MODE_MISA 1              /* spatial quota, Eqs. (9)-(10) */
+#define MISAT_MODE_SESSION_ADMISSION 2 /* global cap only (class-agnostic) */
+#define MISAT_MODE_PLACEMENT_ONLY 3    /* no admission control (cache-aware placement) */
+
+/* ---- decision reasons ---- */
+#define MISAT_ADMIT_CONT 1         /* session already protected on the instance (Eq. 6, case 1) */
+#define MISAT_ADMIT_NEW 2          /* new, released or rebound session admitted with headroom */
+#define MISAT_ADMIT_FOLLOW 3       /* later request of a session whose leader was admitted */
+#define MISAT_HOLD_GLOBAL_CAP 16   /* no global headroom on the chosen instance */
+#define MISAT_HOLD_CLASS_CAP 17    /* no class headroom on the chosen instance */
+#define MISAT_HOLD_NO_ELIGIBLE 18  /* no instance has headroom for this session */
+#define MISAT_HOLD_PREFER_CACHE 19 /* Eq. (7): waiting for the cached instance is cheaper */
+#define MISAT_HOLD_LEADER_HELD 20  /* later request of a session whose leader was held */
+
+typedef struct misat_ctx misat_ctx;
+
+/* Router configuration (misat_create).  All sizes in KV blocks of 16 tokens. */
+typedef struct misat_config {
+  int32_t n_instances;          /* W, 1..1024 */
+  const int64_t* cap_blocks;    /* host [W]: resident-block capacity Cap_w, 1..2^26 */
+  int32_t protected_frac_q16;   /* C_w = floor(Cap_w * q / 65536), 1..65536 (0.9 -> 58982) */
+  int32_t rounds;               /* selection rounds per batch, 1..64 (default 4) */
+  int32_t mode;                 /* MISAT_MODE_* */
+  int32_t max_batch;            /* largest n passed to misat_route, 1..2^20 */
+  int64_t max_tokens;           /* largest total prompt tokens of one batch, >= 16 */
+  int32_t max_sessions;         /* expected live sessions (table is sized 2x and grows) */
+  int32_t hist_window;          /* completed sessions kept per class, 1..4096 (256) */
+  int32_t min_obs;              /* observations before T_b leaves the prior, >= 1 (8) */
+  int64_t hold_delay_q;         /* Delta_r of Eq. (7), cost units, 0..2^61 */
+  int64_t prior_kbar_blocks[3]; /* conservative class footprint priors, 1..2^30 */
+  int64_t prior_T_us;           /* shared neutral residency prior (Sec. 4.3), 0..2^40 */
+  uint64_t hash_seed;           /* a_{-1} of the block-hash chain (0x9e3779b97f4a7c15) */
+  double table_load;            /* max load of an instance table before it grows, 0.25..0.9 (0.75) */
+} misat_config;
+
+/* One routing batch.  Device pointers, except n and n_tokens. */
+typedef struct misat_batch {
+  int32_t n;                /* requests, 0..max_batch */
+  int64_t n_tokens;         /* tok_off[n] */
+  const uint8_t* cls;       /* [n] workload class b_r: 0 RLVR, 1 RLHF, 2 agentic */
+  const uint64_t* session;  /* [n] session id s_r, nonzero; a session keeps one class */
+  const uint64_t* group;    /* [n] prompt group g_r, may be NULL (carried, not used) */
+  const int64_t* tok_off;   /* [n+1] CSR offsets into tokens, tok_off[0] = 0, non-decreasing,
+                               each prompt < 2^20 tokens */
+  const int32_t* tokens;    /* [n_tokens] token ids; 16-byte aligned and readable up to the
+                               next 16-byte boundary past n_tokens */
+  uint16_t* out_H;          /* optional [n*W] device output: H_rw in blocks, row-major */
+} misat_batch;
+
+/* Decisions of one batch.  Device pointers (misat_route) or host pointers
+ * (misat_route_host). */
+typedef struct misat_decisions {
+  int32_t* inst;        /* [n] instance, -1 = HOLD */
+  uint8_t* reason;      /* [n] MISAT_ADMIT_* / MISAT_HOLD_* */
+  int32_t* hit_blocks;  /* [n] H on the chosen instance; for HOLD the max over instances */
+} misat_decisions;
+
+/* Index entry (dump / load).  meta = seq<<36 | arrival<<16 | (65535 - depth):
+ * ascending (meta, key) is the eviction order (oldest commit first, deeper block
+ * first).  key >= 2. */
+typedef struct misat_entry {
+  uint64_t key;
+  uint64_t meta;
+} misat_entry;
+
+/* Statistics of the last route and commit (misat_stats). */
+typedef struct misat_batch_stats {
+  int64_t n_requests, n_admitted, n_held;
+  int64_t by_reason[8];          /* CONT NEW FOLLOW GLOBAL CLASS NO_ELIGIBLE PREFER_CACHE LEADER_HELD */
+  int64_t admitted_by_class[3];
+  int64_t held_by_class[3];
+  int64_t hit_tokens;            /* 16 * hit blocks over admitted requests */
+  int64_t query_tokens;          /* prompt tokens of admitted requests */
+  int64_t dtv_ppm;               /* D_TV(admitted class mix, rho) in ppm, -1 if none admitted */
+  int64_t probes;                /* key lookups executed by the probe kernels */
+  int64_t bucket_reads;          /* 32-byte key groups read by the probe kernels */
+  int64_t probes_first;          /* of which: block-0 probes (phase 1) */
+  int64_t bucket_reads_first;    /* of which: key groups read by phase 1 */
+  int64_t new_keys;              /* keys inserted by the last commit */
+  int64_t evicted;               /* keys evicted by the last commit */
+  int64_t seq;                   /* commits applied so far */
+} misat_batch_stats;
+
+/* Create a router on the current CUDA device.  cuda_stream: a cudaStream_t (NULL =
+ * legacy default stream).  [sync] Errors: INVALID_ARG, OOM, CUDA. */
+int misat_create(const misat_config* cfg, void* cuda_stream, misat_ctx** out);
+
+/* Free all device and host memory of ctx (waits for the stream). */
+int misat_destroy(misat_ctx* ctx);
+
+/* Trainer target mixture rho (Sec. 3.1), ppm per class, sum = 10^6.  Used only for
+ * D_TV (Sec. 3.3) and for splitting C_w when no class has demand.  [host] */
+int misat_set_mixture(misat_ctx* ctx, const uint32_t rho_ppm[3]);
+
+/* Per-instance runtime state from the serving layer, host arrays [W], each may be NULL
+ * to keep the previous values:
+ *   backlog_q       d_w of Eq. (1), fixed-point cost units, 0..2^61
+ *   tokcost_q       1/mu_w of Eq. (1), cost units per prompt token, 0..2^32
+ *   cap_contraction overload contraction of K_w (Sec. 4.1), >= 0
+ * [async] */
+int misat_set_instance_state(misat_ctx* ctx, const int64_t* backlog_q, const int64_t* tokcost_q,
+                             const int32_t* cap_contraction);
+
+/* Route one batch against the state at batch start (Sec. 3.1, Sec. 4).  Inputs and
+ * outputs are device pointers; outputs are written before the call's work ends on the
+ * stream.  A second route without a commit replaces the pending one.  [async]
+ * Errors: INVALID_ARG, BATCH_TOO_LARGE; malformed contents are reported by misat_sync. */
+int misat_route(misat_ctx* ctx, const misat_batch* batch, misat_decisions* out);
+
+/* misat_route with HOST batch arrays (pinned memory recommended) and host outputs:
+ * copies the batch to library staging buffers, routes, and copies the decisions
+ * back.  out_H must be NULL.  [sync] */
+int misat_route_host(misat_ctx* ctx, const misat_batch* host_batch, misat_decisions* host_out);
+
+/* Apply the pending route: insert every admitted request's blocks into its instance's
+ * index (tick = commit number and arrival index, depth = block index, max-merge), make
+ * newly admitted sessions protected on their instance (a rebound session leaves its old
+ * instance), then evict each instance down to Cap_w (Sec. 4.1, Sec. 4.5).  Waits for the
+ * route's small summary, then enqueues.  Errors: STATE (no pending route). */
+int misat_commit(misat_ctx* ctx);
+
+/* Completion events, host arrays [n] with distinct sessions:
+ *   done != 0: the session finished: (total_blocks, residency_us) join class cls's
+ *              bounded histories (Sec. 4.1, Sec. 4.3) and the session leaves the
+ *              protected set and is forgotten;
+ *   done == 0: protection is released but the session is remembered; its next
+ *              request is a continuation that must reacquire admission (Eq. 7).
+ * Unknown sessions only update the histories.  [async] */
+int misat_complete(misat_ctx* ctx, int32_t n, const uint64_t* session, const uint8_t* cls,
+                   const int32_t* total_blocks, const int64_t* residency_us, const uint8_t* done);
+
+/* Engine removal events (Sec. 4.5): remove the listed keys (host array) from instance
+ * w's index.  The removed set must be suffix-closed (no remaining block may lose its
+ * parent).  [sync] */
+int misat_evict(misat_ctx* ctx, int32_t w, const uint64_t* keys, int64_t n);
+
+/* Cache reset of instance w (e.g. after a weight sync): its index becomes empty. [async] */
+int misat_reset_instance(misat_ctx* ctx, int32_t w);
+
+/* Warm-up of prompt chains, host arrays: chain c (tokens tok_off[c]..tok_off[c+1]) is
+ * hashed and its first min(full blocks, max_blocks[c]) blocks are inserted on inst[c]
+ * with tick (seq[c] < 2^28, arr[c] < 2^20), then every instance is evicted to Cap.
+ * [sync] */
+int misat_load_chains(misat_ctx* ctx, int32_t n_chains, const int64_t* tok_off,
+                      const int32_t* tokens, const int32_t* inst, const uint64_t* seq,
+                      const uint32_t* arr, const int32_t* max_blocks);
+
+/* Load index entries (host array) into instance w with max-merge of meta, then evict w
+ * to Cap.  Loaded state must be prefix-closed.  [sync] */
+int misat_load_entries(misat_ctx* ctx, int32_t w, const misat_entry* entries, int64_t n);
+
+/* Number of resident blocks of instance w.  [sync] */
+int misat_index_size(misat_ctx* ctx, int32_t w, int64_t* out);
+
+/* Copy instance w's index to host_out sorted by key (cap entries available; *n_out =
+ * count).  [sync] */
+int misat_dump_index(misat_ctx* ctx, int32_t w, misat_entry* host_out, int64_t cap,
+                     int64_t* n_out);
+
+/* Block keys of the last routed batch, request order (host, cap entries). [sync] */
+int misat_dump_keys(misat_ctx* ctx, uint64_t* host_out, int64_t cap, int64_t* n_out);
+
+/* Caps of the last route (host arrays): K_w [W], K_wb [W*3], N_wb [W*3], kbar_w [W],
+ * kbar_b [3], T_b [3].  Any pointer may be NULL.  [sync] */
+int misat_dump_caps(misat_ctx* ctx, int64_t* K_w, int64_t* K_wb, int64_t* N_wb, int64_t* kbar_w,
+                    int64_t* kbar_b, int64_t* T_b);
+
+/* Protected session counts per (w, b), host [W*3].  [sync] */
+int misat_dump_counts(misat_ctx* ctx, int32_t* prot);
+
+/* Live sessions sorted by id (host arrays, cap entries): state 1 = protected,
+ * 2 = released; inst; class.  [sync] */
+int misat_dump_sessions(misat_ctx* ctx, uint64_t* ids, int32_t* state, int32_t* inst,
+                        int32_t* cls, int64_t cap, int64_t* n_out);
+
+/* Statistics of the last route / commit.  [sync] */
+int misat_stats(misat_ctx* ctx, misat_batch_stats* host_out);
+
+/* ---- checkpoint / resume (the paper has no counterpart: state snapshots of the router) ----
+ * A checkpoint is a device-resident copy of the whole router state: every instance index
+ * (with its table geometry), the session table, protected counts, per-instance inputs,
+ * class histories and the commit counter.  save [sync]; restore [async, stream-ordered]:
+ * the context returns to exactly the saved state (tables that grew since are shrunk back);
+ * a pending route is dropped.  free releases the copy. */
+typedef struct misat_checkpoint misat_checkpoint;
+int misat_checkpoint_save(misat_ctx* ctx, misat_checkpoint** out);
+int misat_checkpoint_restore(misat_ctx* ctx, const misat_checkpoint* ckpt);
+int misat_checkpoint_free(misat_checkpoint* ckpt);
+
+/* ---- per-phase device time (measurement; the paper has no counterpart) ----
+ * With timing enabled, CUDA events on the context's stream bracket each phase of
+ * misat_route and misat_commit.  misat_phase_times waits and writes the durations (ms)
+ * of the last route / commit, indexed by MISAT_PHASE_*. */
+#define MISAT_PHASE_PROLOGUE 0      /* validation, session snapshot, leaders */
+#define MISAT_PHASE_HASH 1          /* K1 chained block hash */
+#define MISAT_PHASE_CAPS 2          /* K3a caps */
+#define MISAT_PHASE_PROBE_FIRST 3   /* K2 block-0 probe of every (request, instance) pair */
+#define MISAT_PHASE_PROBE_SEARCH 4  /* K2 binary search of the hit pairs */
+#define MISAT_PHASE_ROUNDS 5        /* K3b score + K4a admission, all rounds */
+#define MISAT_PHASE_FINALIZE 6      /* holds, followers, outputs */
+#define MISAT_PHASE_INSERT 7        /* K4b index insert */
+#define MISAT_PHASE_SESSIONS 8      /* session table update */
+#define MISAT_PHASE_EVICT 9         /* K4c eviction select + compaction */
+#define MISAT_N_PHASES 10
+int misat_set_timing(misat_ctx* ctx, int enable);
+int misat_phase_times(misat_ctx* ctx, float* ms_out);
+
+/* Wait for the stream and return the sticky device error (0 if none), then clear it and
+ * drop any pending route.  A batch rejected on the device changes no persistent state;
+ * after TABLE_FULL during a commit the index of the affected instance may hold part of
+ * that commit's blocks.  [sync] */
+int misat_sync(misat_ctx* ctx);
+
+/* Static description of an error code. */
+const char* misat_strerror(int code);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* MISAT_H */

@@ -88,6 +88,7 @@ def _load():
         "oracle_dump_sessions": (C.c_int, [p, p, p, p, p, i64, p]),
         "oracle_seq": (u64, [p]),
         "oracle_check_invariants": (C.c_int, [p]),
+        "oracle_clone": (p, [p]),
     }
     for name, (res, args) in sig.items():
         f = getattr(lib, name)
@@ -257,6 +258,15 @@ class Oracle:
 
     def seq(self):
         return int(self._lib.oracle_seq(self._h))
+
+    def clone(self):
+        """Deep copy of this oracle state."""
+        o = object.__new__(Oracle)
+        o._lib = self._lib
+        o.W = self.W
+        o.n = self.n
+        o._h = self._lib.oracle_clone(self._h)
+        return o
 
     def check_invariants(self):
         return int(self._lib.oracle_check_invariants(self._h))

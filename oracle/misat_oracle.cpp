@@ -847,3 +847,8 @@ int oracle_check_invariants(void* h) {
 }
 
 }  // extern "C"
+
+extern "C" {
+// Deep copy of an oracle state (used to restart a timed step from the same state).
+void* oracle_clone(void* h) { return new Oracle(*(Oracle*)h); }
+}

@@ -1,0 +1,1200 @@
+// C ABI of the MISA-T routing library: context, orchestration of the kernels, class
+// histories (host), table growth and state dumps.  See include/misat.h.
+#include <algorithm>
+#include <cstring>
+#include <deque>
+#include <new>
+#include <unordered_set>
+#include <vector>
+
+#include "common.cuh"
+#include "kernels.h"
+
+using namespace misat;
+
+namespace {
+
+constexpr int kTileReq = 1024;
+constexpr int kMaxRounds = 64;
+
+// Small device block copied to the host in one transfer after each route / commit.
+// Layout (8-byte words): stats[32] | U[W] | size[W] | sess_used | err | cand[3] | work | n_hits
+struct MetaLayout {
+  size_t stats = 0, U = 0, size = 0, sess_used = 0, err = 0, cand = 0, work = 0, n_hits = 0, words = 0;
+  void init(int W) {
+    stats = 0;
+    U = 32;
+    size = U + W;
+    sess_used = size + W;
+    err = sess_used + 1;
+    cand = err + 1;
+    work = cand + 3;
+    n_hits = work + 1;
+    words = n_hits + 1;
+  }
+};
+
+inline int ceil_log2(uint64_t x) {
+  int l = 0;
+  while ((1ull << l) < x) ++l;
+  return l;
+}
+
+}  // namespace
+
+struct misat_ctx {
+  int device = 0, num_sms = 1;
+  cudaStream_t stream = nullptr;
+  // configuration
+  int32_t W = 0, pf_q16 = 0, rounds = 1, mode = 0, max_batch = 0, max_sessions = 0, hist_window = 256,
+          min_obs = 8;
+  int64_t max_tokens = 0, hold_delay_q = 0, prior_kbar[3] = {1, 1, 1}, prior_T = 0;
+  uint64_t seed = kGold;
+  double table_load = 0.75;
+  std::vector<int64_t> cap;
+  // host state
+  std::deque<int64_t> hist_blocks[3], hist_res[3];
+  uint32_t rho[3] = {333334, 333333, 333333};
+  uint64_t seq = 0;
+  bool routed = false;
+  int32_t last_n = 0;
+  int64_t last_ntok = 0;
+  int64_t kbar_b[3] = {0, 0, 0}, T_b[3] = {0, 0, 0};
+  // instance tables
+  std::vector<InstDesc> h_desc;
+  std::vector<uint32_t*> h_bitmap;
+  std::vector<uint4*> h_ca, h_cb;
+  InstDesc* d_desc = nullptr;
+  uint32_t** d_bitmap = nullptr;
+  uint4** d_ca = nullptr;
+  uint4** d_cb = nullptr;
+  // per-instance inputs and state
+  int64_t* d_backlog = nullptr;
+  int64_t* d_tokcost = nullptr;
+  int32_t* d_contraction = nullptr;
+  int32_t* d_prot = nullptr;
+  unsigned long long* d_theta = nullptr;
+  int32_t* d_active = nullptr;
+  int32_t* d_onew = nullptr;
+  InstArrays ia{};
+  // sessions
+  SessTable sess{};
+  // per-request scratch
+  ReqArrays rq{};
+  uint64_t* d_keys = nullptr;
+  int64_t keys_cap = 0;
+  uint16_t* d_H = nullptr;
+  int2* d_hits = nullptr;
+  int64_t hits_cap = 0;
+  unsigned long long* d_bm_key = nullptr;
+  int32_t* d_bm_val = nullptr;
+  int32_t* d_tile = nullptr;
+  // one small block of counters, mirrored to pinned host memory
+  MetaLayout ml;
+  unsigned long long* d_meta = nullptr;
+  unsigned long long* h_meta = nullptr;
+  cudaEvent_t ev_meta = nullptr;
+  // staging of misat_route_host and of host-array calls
+  int32_t* d_stage_tok = nullptr;
+  int64_t* d_stage_off = nullptr;
+  uint8_t* d_stage_cls = nullptr;
+  uint64_t* d_stage_ses = nullptr;
+  int32_t* d_out_inst = nullptr;
+  uint8_t* d_out_reason = nullptr;
+  int32_t* d_out_hit = nullptr;
+  std::vector<void*> owned;  // fixed allocations freed in destroy
+  // phase timing: events 0..7 bracket the route phases, 8..11 the commit phases
+  bool timing = false;
+  cudaEvent_t ev[12] = {};
+
+  void mark(int i) {
+    if (timing) cudaEventRecord(ev[i], stream);
+  }
+
+  long long* size_ptr() { return reinterpret_cast<long long*>(d_meta + ml.size); }
+  long long* U_ptr() { return reinterpret_cast<long long*>(d_meta + ml.U); }
+  int32_t* err_ptr() { return reinterpret_cast<int32_t*>(d_meta + ml.err); }
+  long long* cand_ptr() { return reinterpret_cast<long long*>(d_meta + ml.cand); }
+  unsigned* work_ptr() { return reinterpret_cast<unsigned*>(d_meta + ml.work); }
+  unsigned* nhits_ptr() { return reinterpret_cast<unsigned*>(d_meta + ml.n_hits); }
+  unsigned long long* stats_ptr() { return d_meta + ml.stats; }
+  long long h_size(int w) const { return reinterpret_cast<const long long*>(h_meta + ml.size)[w]; }
+  long long h_U(int w) const { return reinterpret_cast<const long long*>(h_meta + ml.U)[w]; }
+  int32_t h_err() const { return *reinterpret_cast<const int32_t*>(h_meta + ml.err); }
+};
+
+namespace {
+
+#define CK(x)                                    \
+  do {                                           \
+    if ((x) != cudaSuccess) return MISAT_ERR_CUDA; \
+  } while (0)
+
+int dalloc(misat_ctx* c, void** p, size_t bytes) {
+  *p = nullptr;
+  if (bytes == 0) bytes = 16;
+  if (cudaMalloc(p, bytes) != cudaSuccess) {
+    cudaGetLastError();
+    return MISAT_ERR_OOM;
+  }
+  if (cudaMemset(*p, 0, bytes) != cudaSuccess) return MISAT_ERR_CUDA;
+  c->owned.push_back(*p);
+  return MISAT_OK;
+}
+
+template <typename T>
+int dalloc_n(misat_ctx* c, T** p, size_t n) {
+  return dalloc(c, reinterpret_cast<void**>(p), n * sizeof(T));
+}
+
+// Allocate instance w's table (zeroed), bitmap and candidate lists for 2^lg buckets.
+int alloc_instance(misat_ctx* c, int w, uint32_t lg, InstDesc* out, uint32_t** bm, uint4** ca, uint4** cb) {
+  const size_t nb = (size_t)1 << lg;
+  void *t = nullptr, *b = nullptr, *x = nullptr, *y = nullptr;
+  if (cudaMalloc(&t, nb * sizeof(Bucket)) != cudaSuccess || cudaMalloc(&b, (nb / 32 + 1) * 4) != cudaSuccess ||
+      cudaMalloc(&x, nb * 4 * sizeof(uint4)) != cudaSuccess || cudaMalloc(&y, nb * 4 * sizeof(uint4)) != cudaSuccess) {
+    cudaGetLastError();
+    cudaFree(t);
+    cudaFree(b);
+    cudaFree(x);
+    cudaFree(y);
+    return MISAT_ERR_OOM;
+  }
+  CK(cudaMemsetAsync(t, 0, nb * sizeof(Bucket), c->stream));
+  CK(cudaMemsetAsync(b, 0, (nb / 32 + 1) * 4, c->stream));
+  out->tab = (Bucket*)t;
+  out->log2nb = lg;
+  out->pad = 0;
+  out->cap = c->cap[w];
+  *bm = (uint32_t*)b;
+  *ca = (uint4*)x;
+  *cb = (uint4*)y;
+  return MISAT_OK;
+}
+
+int push_desc(misat_ctx* c, int w) {
+  CK(cudaMemcpyAsync(c->d_desc + w, &c->h_desc[w], sizeof(InstDesc), cudaMemcpyHostToDevice, c->stream));
+  CK(cudaMemcpyAsync(c->d_bitmap + w, &c->h_bitmap[w], sizeof(uint32_t*), cudaMemcpyHostToDevice, c->stream));
+  CK(cudaMemcpyAsync(c->d_ca + w, &c->h_ca[w], sizeof(uint4*), cudaMemcpyHostToDevice, c->stream));
+  CK(cudaMemcpyAsync(c->d_cb + w, &c->h_cb[w], sizeof(uint4*), cudaMemcpyHostToDevice, c->stream));
+  return MISAT_OK;
+}
+
+uint32_t buckets_log2_for(int64_t entries, double load) {
+  // smallest power-of-two bucket count whose slots hold `entries` at `load`
+  const double slots = (double)entries / load;
+  uint32_t lg = 1;
+  while ((double)((uint64_t)4 << lg) < slots) ++lg;
+  return lg;
+}
+
+// Grow instance w so that `need` entries fit at half load; entries are re-inserted.
+int grow_instance(misat_ctx* c, int w, int64_t need) {
+  const uint32_t lg = std::max(buckets_log2_for(need, 0.5), c->h_desc[w].log2nb + 1);
+  InstDesc nd;
+  uint32_t* bm;
+  uint4 *ca, *cb;
+  int rc = alloc_instance(c, w, lg, &nd, &bm, &ca, &cb);
+  if (rc) return rc;
+  RehashArgs ra{c->h_desc[w], nd, c->err_ptr()};
+  launch_rehash(ra, c->stream);
+  CK(cudaGetLastError());
+  CK(cudaStreamSynchronize(c->stream));
+  cudaFree(c->h_desc[w].tab);
+  cudaFree(c->h_bitmap[w]);
+  cudaFree(c->h_ca[w]);
+  cudaFree(c->h_cb[w]);
+  c->h_desc[w] = nd;
+  c->h_bitmap[w] = bm;
+  c->h_ca[w] = ca;
+  c->h_cb[w] = cb;
+  return push_desc(c, w);
+}
+
+// Make room for `add[w]` more entries on every instance (current sizes must be on the host).
+int ensure_capacity(misat_ctx* c, const std::vector<int64_t>& sizes, const std::vector<int64_t>& add) {
+  for (int w = 0; w < c->W; ++w) {
+    const int64_t need = sizes[w] + add[w];
+    const double slots = (double)((uint64_t)4 << c->h_desc[w].log2nb);
+    if ((double)need > c->table_load * slots) {
+      int rc = grow_instance(c, w, need);
+      if (rc) return rc;
+    }
+  }
+  return MISAT_OK;
+}
+
+// Read the counters block (sync).
+int read_meta(misat_ctx* c) {
+  CK(cudaMemcpyAsync(c->h_meta, c->d_meta, c->ml.words * 8, cudaMemcpyDeviceToHost, c->stream));
+  CK(cudaStreamSynchronize(c->stream));
+  return MISAT_OK;
+}
+
+int enqueue_meta(misat_ctx* c) {
+  CK(cudaMemcpyAsync(c->h_meta, c->d_meta, c->ml.words * 8, cudaMemcpyDeviceToHost, c->stream));
+  CK(cudaEventRecord(c->ev_meta, c->stream));
+  return MISAT_OK;
+}
+
+// Session table rebuild when claimed slots (live + finished) pass 70% of it.
+int maybe_rebuild_sessions(misat_ctx* c, int64_t incoming) {
+  const uint64_t used = c->h_meta[c->ml.sess_used];
+  const uint64_t capn = 1ull << c->sess.log2n;
+  if ((double)(used + incoming) <= 0.7 * (double)capn) return MISAT_OK;
+  // count live sessions on the host from a copy (rare path)
+  std::vector<SessSlot> hs(capn);
+  CK(cudaMemcpyAsync(hs.data(), c->sess.slots, capn * sizeof(SessSlot), cudaMemcpyDeviceToHost, c->stream));
+  CK(cudaStreamSynchronize(c->stream));
+  uint64_t live = 0;
+  for (auto& s : hs)
+    if (s.key && (sess_state(s.val) == kSessProtected || sess_state(s.val) == kSessReleased)) ++live;
+  const uint64_t want = std::max<uint64_t>(2 * (uint64_t)c->max_sessions, 2 * (live + (uint64_t)incoming));
+  const uint32_t lg = (uint32_t)std::max(4, ceil_log2(want));
+  SessSlot* ns = nullptr;
+  if (cudaMalloc(&ns, ((size_t)1 << lg) * sizeof(SessSlot)) != cudaSuccess) {
+    cudaGetLastError();
+    return MISAT_ERR_OOM;
+  }
+  CK(cudaMemsetAsync(ns, 0, ((size_t)1 << lg) * sizeof(SessSlot), c->stream));
+  CK(cudaMemsetAsync(c->d_meta + c->ml.sess_used, 0, 8, c->stream));
+  SessTable to{ns, lg, c->d_meta + c->ml.sess_used};
+  SessRehashArgs a{c->sess, to, c->err_ptr()};
+  launch_sess_rehash(a, c->stream);
+  CK(cudaGetLastError());
+  CK(cudaStreamSynchronize(c->stream));
+  cudaFree(c->sess.slots);
+  c->sess = to;
+  return read_meta(c);
+}
+
+void estimate_classes(misat_ctx* c) {
+  for (int b = 0; b < 3; ++b) {
+    const auto& h = c->hist_blocks[b];
+    if (h.empty()) {
+      c->kbar_b[b] = c->prior_kbar[b];
+    } else {
+      std::vector<int64_t> v(h.begin(), h.end());
+      std::sort(v.begin(), v.end());
+      const int64_t m = (int64_t)v.size();
+      const int64_t rank = (9 * m + 9) / 10;  // nearest-rank 90th percentile
+      c->kbar_b[b] = std::max(c->prior_kbar[b], v[rank - 1]);
+    }
+    const auto& t = c->hist_res[b];
+    if ((int64_t)t.size() < c->min_obs) {
+      c->T_b[b] = c->prior_T;
+    } else {
+      int64_t s = 0;
+      for (int64_t x : t) s += x;
+      c->T_b[b] = s / (int64_t)t.size();
+    }
+  }
+}
+
+int evict_all(misat_ctx* c, unsigned long long* evicted_counter) {
+  EvictArgs ev{};
+  ev.desc = c->d_desc;
+  ev.W = c->W;
+  ev.only_w = nullptr;
+  ev.size = c->size_ptr();
+  ev.cur_seq = c->seq + 1;
+  ev.bitmaps = c->d_bitmap;
+  ev.cand_a = c->d_ca;
+  ev.cand_b = c->d_cb;
+  ev.theta = c->d_theta;
+  ev.active = c->d_active;
+  ev.evicted = evicted_counter;
+  ev.err = c->err_ptr();
+  uint32_t maxlg = 1;
+  for (auto& d : c->h_desc) maxlg = std::max(maxlg, d.log2nb);
+  // compaction threads per instance: about 64 buckets each, at most 32 CTAs of 256
+  int chunks = (int)std::min<uint64_t>(32, std::max<uint64_t>(1, ((uint64_t)1 << maxlg) / (64 * 256)));
+  launch_evict(ev, chunks, c->stream);
+  CK(cudaGetLastError());
+  return MISAT_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+const char* misat_strerror(int code) {
+  switch (code) {
+    case MISAT_OK: return "ok";
+    case MISAT_ERR_INVALID_ARG: return "invalid argument";
+    case MISAT_ERR_OOM: return "out of memory";
+    case MISAT_ERR_CUDA: return "CUDA runtime error";
+    case MISAT_ERR_STATE: return "no pending route to commit";
+    case MISAT_ERR_TABLE_FULL: return "table full";
+    case MISAT_ERR_BATCH_TOO_LARGE: return "batch exceeds max_batch or max_tokens";
+    default: return "unknown error";
+  }
+}
+
+int misat_destroy(misat_ctx* c) {
+  if (!c) return MISAT_ERR_INVALID_ARG;
+  cudaStreamSynchronize(c->stream);
+  for (size_t w = 0; w < c->h_desc.size(); ++w) {
+    cudaFree(c->h_desc[w].tab);
+    cudaFree(c->h_bitmap[w]);
+    cudaFree(c->h_ca[w]);
+    cudaFree(c->h_cb[w]);
+  }
+  cudaFree(c->sess.slots);
+  for (void* p : c->owned) cudaFree(p);
+  if (c->h_meta) cudaFreeHost(c->h_meta);
+  if (c->ev_meta) cudaEventDestroy(c->ev_meta);
+  for (auto& e : c->ev)
+    if (e) cudaEventDestroy(e);
+  delete c;
+  return MISAT_OK;
+}
+
+int misat_create(const misat_config* cfg, void* cuda_stream, misat_ctx** out) {
+  if (!cfg || !out || !cfg->cap_blocks) return MISAT_ERR_INVALID_ARG;
+  *out = nullptr;
+  const int W = cfg->n_instances;
+  if (W < 1 || W > kMaxW) return MISAT_ERR_INVALID_ARG;
+  for (int w = 0; w < W; ++w)
+    if (cfg->cap_blocks[w] < 1 || cfg->cap_blocks[w] > ((int64_t)1 << 26)) return MISAT_ERR_INVALID_ARG;
+  if (cfg->protected_frac_q16 < 1 || cfg->protected_frac_q16 > 65536) return MISAT_ERR_INVALID_ARG;
+  if (cfg->rounds < 1 || cfg->rounds > kMaxRounds) return MISAT_ERR_INVALID_ARG;
+  if (cfg->mode < 0 || cfg->mode > 3) return MISAT_ERR_INVALID_ARG;
+  if (cfg->max_batch < 1 || cfg->max_batch > (1 << 20)) return MISAT_ERR_INVALID_ARG;
+  if (cfg->max_tokens < 16 || cfg->max_tokens > ((int64_t)1 << 36)) return MISAT_ERR_INVALID_ARG;
+  if (cfg->max_sessions < 1 || cfg->max_sessions > (1 << 28)) return MISAT_ERR_INVALID_ARG;
+  if (cfg->hist_window < 1 || cfg->hist_window > 4096 || cfg->min_obs < 1) return MISAT_ERR_INVALID_ARG;
+  if (cfg->hold_delay_q < 0 || cfg->hold_delay_q > kBacklogMax) return MISAT_ERR_INVALID_ARG;
+  for (int b = 0; b < 3; ++b)
+    if (cfg->prior_kbar_blocks[b] < 1 || cfg->prior_kbar_blocks[b] > ((int64_t)1 << 30)) return MISAT_ERR_INVALID_ARG;
+  if (cfg->prior_T_us < 0 || cfg->prior_T_us > ((int64_t)1 << 40)) return MISAT_ERR_INVALID_ARG;
+  if (!(cfg->table_load >= 0.25 && cfg->table_load <= 0.9)) return MISAT_ERR_INVALID_ARG;
+
+  misat_ctx* c = new (std::nothrow) misat_ctx();
+  if (!c) return MISAT_ERR_OOM;
+  int rc = MISAT_OK;
+  auto fail = [&](int code) {
+    misat_destroy(c);
+    return code;
+  };
+  if (cudaGetDevice(&c->device) != cudaSuccess) return fail(MISAT_ERR_CUDA);
+  if (cudaDeviceGetAttribute(&c->num_sms, cudaDevAttrMultiProcessorCount, c->device) != cudaSuccess)
+    return fail(MISAT_ERR_CUDA);
+  c->stream = (cudaStream_t)cuda_stream;
+  c->W = W;
+  c->cap.assign(cfg->cap_blocks, cfg->cap_blocks + W);
+  c->pf_q16 = cfg->protected_frac_q16;
+  c->rounds = cfg->rounds;
+  c->mode = cfg->mode;
+  c->max_batch = cfg->max_batch;
+  c->max_tokens = cfg->max_tokens;
+  c->max_sessions = cfg->max_sessions;
+  c->hist_window = cfg->hist_window;
+  c->min_obs = cfg->min_obs;
+  c->hold_delay_q = cfg->hold_delay_q;
+  for (int b = 0; b < 3; ++b) c->prior_kbar[b] = cfg->prior_kbar_blocks[b];
+  c->prior_T = cfg->prior_T_us;
+  c->seed = cfg->hash_seed;
+  c->table_load = cfg->table_load;
+  c->ml.init(W);
+  if (cudaEventCreateWithFlags(&c->ev_meta, cudaEventDisableTiming) != cudaSuccess) return fail(MISAT_ERR_CUDA);
+  if (cudaMallocHost(&c->h_meta, c->ml.words * 8) != cudaSuccess) return fail(MISAT_ERR_OOM);
+  std::memset(c->h_meta, 0, c->ml.words * 8);
+
+  const size_t NB = (size_t)c->max_batch, Ws = (size_t)W;
+  c->keys_cap = c->max_tokens / 16 + 1;
+  c->hits_cap = (int64_t)std::min<size_t>(NB * Ws, (size_t)1 << 27);
+  const int bm_log2 = std::max(1, ceil_log2(2 * NB));
+  const size_t n_tiles = (NB + kTileReq - 1) / kTileReq;
+  if ((rc = dalloc_n(c, &c->d_meta, c->ml.words)) || (rc = dalloc_n(c, &c->d_keys, (size_t)c->keys_cap)) ||
+      (rc = dalloc_n(c, &c->d_H, NB * Ws)) || (rc = dalloc_n(c, &c->d_hits, (size_t)c->hits_cap)) ||
+      (rc = dalloc_n(c, &c->d_bm_key, (size_t)1 << bm_log2)) ||
+      (rc = dalloc_n(c, &c->d_bm_val, (size_t)1 << bm_log2)) || (rc = dalloc_n(c, &c->d_tile, n_tiles * 3 * Ws)) ||
+      (rc = dalloc_n(c, &c->rq.nb, NB)) || (rc = dalloc_n(c, &c->rq.kbase, NB)) || (rc = dalloc_n(c, &c->rq.L, NB)) ||
+      (rc = dalloc_n(c, &c->rq.cls, NB)) || (rc = dalloc_n(c, &c->rq.session, NB)) ||
+      (rc = dalloc_n(c, &c->rq.sst, NB)) || (rc = dalloc_n(c, &c->rq.sinst, NB)) ||
+      (rc = dalloc_n(c, &c->rq.leader, NB)) || (rc = dalloc_n(c, &c->rq.status, NB)) ||
+      (rc = dalloc_n(c, &c->rq.choice, NB)) || (rc = dalloc_n(c, &c->rq.last_reason, NB)) ||
+      (rc = dalloc_n(c, &c->rq.inst, NB)) || (rc = dalloc_n(c, &c->rq.reason, NB)) ||
+      (rc = dalloc_n(c, &c->ia.K_w, Ws)) || (rc = dalloc_n(c, &c->ia.K_wb, 3 * Ws)) ||
+      (rc = dalloc_n(c, &c->ia.N_wb, 3 * Ws)) || (rc = dalloc_n(c, &c->ia.kbar_w, Ws)) ||
+      (rc = dalloc_n(c, &c->ia.tot, Ws)) || (rc = dalloc_n(c, &c->ia.gh, Ws)) || (rc = dalloc_n(c, &c->ia.ch, 3 * Ws)) ||
+      (rc = dalloc_n(c, &c->ia.delta, 3 * Ws)) || (rc = dalloc_n(c, &c->ia.backlog_k, Ws)) ||
+      (rc = dalloc_n(c, &c->ia.prefill, Ws)) || (rc = dalloc_n(c, &c->d_backlog, Ws)) ||
+      (rc = dalloc_n(c, &c->d_tokcost, Ws)) || (rc = dalloc_n(c, &c->d_contraction, Ws)) ||
+      (rc = dalloc_n(c, &c->d_prot, 3 * Ws)) || (rc = dalloc_n(c, &c->d_theta, 2 * Ws)) ||
+      (rc = dalloc_n(c, &c->d_active, Ws)) || (rc = dalloc_n(c, &c->d_onew, 1)) ||
+      (rc = dalloc_n(c, &c->d_desc, Ws)) || (rc = dalloc_n(c, &c->d_bitmap, Ws)) || (rc = dalloc_n(c, &c->d_ca, Ws)) ||
+      (rc = dalloc_n(c, &c->d_cb, Ws)) || (rc = dalloc_n(c, &c->d_stage_tok, (size_t)c->max_tokens + 8)) ||
+      (rc = dalloc_n(c, &c->d_stage_off, NB + 1)) || (rc = dalloc_n(c, &c->d_stage_cls, NB)) ||
+      (rc = dalloc_n(c, &c->d_stage_ses, NB)) || (rc = dalloc_n(c, &c->d_out_inst, NB)) ||
+      (rc = dalloc_n(c, &c->d_out_reason, NB)) || (rc = dalloc_n(c, &c->d_out_hit, NB)))
+    return fail(rc);
+  c->ia.U = c->U_ptr();
+  // instance tables: at most half full after eviction
+  c->h_desc.resize(W);
+  c->h_bitmap.assign(W, nullptr);
+  c->h_ca.assign(W, nullptr);
+  c->h_cb.assign(W, nullptr);
+  for (int w = 0; w < W; ++w) {
+    if ((rc = alloc_instance(c, w, buckets_log2_for(c->cap[w], 0.5), &c->h_desc[w], &c->h_bitmap[w], &c->h_ca[w],
+                             &c->h_cb[w])))
+      return fail(rc);
+    if ((rc = push_desc(c, w))) return fail(rc);
+  }
+  // session table
+  {
+    const uint32_t lg = (uint32_t)std::max(4, ceil_log2(2ull * (uint64_t)c->max_sessions));
+    if (cudaMalloc(&c->sess.slots, ((size_t)1 << lg) * sizeof(SessSlot)) != cudaSuccess) {
+      cudaGetLastError();
+      return fail(MISAT_ERR_OOM);
+    }
+    if (cudaMemsetAsync(c->sess.slots, 0, ((size_t)1 << lg) * sizeof(SessSlot), c->stream) != cudaSuccess)
+      return fail(MISAT_ERR_CUDA);
+    c->sess.log2n = lg;
+    c->sess.used = c->d_meta + c->ml.sess_used;
+  }
+  if (cudaStreamSynchronize(c->stream) != cudaSuccess) return fail(MISAT_ERR_CUDA);
+  *out = c;
+  return MISAT_OK;
+}
+
+int misat_set_mixture(misat_ctx* c, const uint32_t rho_ppm[3]) {
+  if (!c || !rho_ppm) return MISAT_ERR_INVALID_ARG;
+  if ((uint64_t)rho_ppm[0] + rho_ppm[1] + rho_ppm[2] != 1000000) return MISAT_ERR_INVALID_ARG;
+  for (int b = 0; b < 3; ++b) c->rho[b] = rho_ppm[b];
+  return MISAT_OK;
+}
+
+int misat_set_instance_state(misat_ctx* c, const int64_t* backlog_q, const int64_t* tokcost_q,
+                             const int32_t* cap_contraction) {
+  if (!c) return MISAT_ERR_INVALID_ARG;
+  for (int w = 0; w < c->W; ++w) {
+    if (backlog_q && (backlog_q[w] < 0 || backlog_q[w] > kBacklogMax)) return MISAT_ERR_INVALID_ARG;
+    if (tokcost_q && (tokcost_q[w] < 0 || tokcost_q[w] > ((int64_t)1 << 32))) return MISAT_ERR_INVALID_ARG;
+    if (cap_contraction && cap_contraction[w] < 0) return MISAT_ERR_INVALID_ARG;
+  }
+  if (backlog_q) CK(cudaMemcpyAsync(c->d_backlog, backlog_q, c->W * 8, cudaMemcpyHostToDevice, c->stream));
+  if (tokcost_q) CK(cudaMemcpyAsync(c->d_tokcost, tokcost_q, c->W * 8, cudaMemcpyHostToDevice, c->stream));
+  if (cap_contraction)
+    CK(cudaMemcpyAsync(c->d_contraction, cap_contraction, c->W * 4, cudaMemcpyHostToDevice, c->stream));
+  return MISAT_OK;
+}
+
+int misat_route(misat_ctx* c, const misat_batch* b, misat_decisions* out) {
+  if (!c || !b || !out) return MISAT_ERR_INVALID_ARG;
+  const int32_t n = b->n;
+  if (n < 0 || b->n_tokens < 0) return MISAT_ERR_INVALID_ARG;
+  if (n > c->max_batch || b->n_tokens > c->max_tokens) return MISAT_ERR_BATCH_TOO_LARGE;
+  if (n > 0 && (!b->cls || !b->session || !b->tok_off || !out->inst || !out->reason || !out->hit_blocks))
+    return MISAT_ERR_INVALID_ARG;
+  if (b->n_tokens > 0 && (!b->tokens || ((uintptr_t)b->tokens & 15) != 0)) return MISAT_ERR_INVALID_ARG;
+  cudaStream_t st = c->stream;
+  c->routed = false;
+  estimate_classes(c);
+  // reset the per-batch counters: stats, U, cand, work, n_hits (size and sess_used persist)
+  CK(cudaMemsetAsync(c->d_meta + c->ml.stats, 0, 32 * 8, st));
+  CK(cudaMemsetAsync(c->d_meta + c->ml.U, 0, c->W * 8, st));
+  CK(cudaMemsetAsync(c->d_meta + c->ml.cand, 0, 5 * 8, st));
+  c->last_n = n;
+  c->last_ntok = b->n_tokens;
+  CapsArgs ca{};
+  ca.W = c->W;
+  ca.desc = c->d_desc;
+  ca.prot = c->d_prot;
+  ca.cand = c->cand_ptr();
+  for (int i = 0; i < 3; ++i) {
+    ca.kbar_b[i] = c->kbar_b[i];
+    ca.T_b[i] = c->T_b[i];
+    ca.rho[i] = c->rho[i];
+  }
+  ca.pf_q16 = c->pf_q16;
+  ca.mode = c->mode;
+  ca.contraction = c->d_contraction;
+  ca.backlog = c->d_backlog;
+  ca.ia = c->ia;
+  ca.err = c->err_ptr();
+  if (n == 0) {
+    // the caps of an empty batch are still defined (no candidate sessions)
+    launch_caps(ca, st);
+    CK(cudaGetLastError());
+    CK(enqueue_meta(c));
+    c->routed = true;
+    return MISAT_OK;
+  }
+  const int bm_log2 = std::max(1, ceil_log2(2 * (uint64_t)n));
+  CK(cudaMemsetAsync(c->d_bm_key, 0, ((size_t)1 << bm_log2) * 8, st));
+  CK(cudaMemsetAsync(c->d_bm_val, 0x7f, ((size_t)1 << bm_log2) * 4, st));
+
+  c->mark(0);
+  PrologueArgs pa{};
+  pa.n = n;
+  pa.n_tokens = b->n_tokens;
+  pa.cls = b->cls;
+  pa.session = b->session;
+  pa.tok_off = b->tok_off;
+  pa.rq = c->rq;
+  pa.st = c->sess;
+  pa.bm_key = c->d_bm_key;
+  pa.bm_val = c->d_bm_val;
+  pa.bm_log2 = (uint32_t)bm_log2;
+  pa.cand = c->cand_ptr();
+  pa.err = c->err_ptr();
+  launch_prologue(pa, st);
+  c->mark(1);
+
+  HashArgs ha{};
+  ha.tok_off = b->tok_off;
+  ha.tokens = b->tokens;
+  ha.n_tokens = b->n_tokens;
+  ha.n = n;
+  ha.seed = c->seed;
+  ha.keys = c->d_keys;
+  ha.keys_cap = c->keys_cap;
+  ha.work = c->work_ptr();
+  ha.err = c->err_ptr();
+  launch_block_hash(ha, c->num_sms, st);
+  c->mark(2);
+  launch_caps(ca, st);
+  c->mark(3);
+
+  ProbeArgs pr{};
+  pr.desc = c->d_desc;
+  pr.W = c->W;
+  pr.n = n;
+  pr.nb = c->rq.nb;
+  pr.kbase = c->rq.kbase;
+  pr.keys = c->d_keys;
+  pr.H = c->d_H;
+  pr.hits = c->d_hits;
+  pr.n_hits = c->nhits_ptr();
+  pr.hits_cap = c->hits_cap;
+  pr.stats = c->stats_ptr() + 16;
+  pr.stats_search = c->stats_ptr() + 22;
+  pr.err = c->err_ptr();
+  launch_probe_first(pr, c->num_sms, st);
+  c->mark(4);
+  launch_probe_search(pr, c->num_sms, st);
+  c->mark(5);
+  if (b->out_H)
+    CK(cudaMemcpyAsync(b->out_H, c->d_H, (size_t)n * c->W * sizeof(uint16_t), cudaMemcpyDeviceToDevice, st));
+
+  RoundArgs ra{};
+  ra.n = n;
+  ra.W = c->W;
+  ra.rq = c->rq;
+  ra.ia = c->ia;
+  ra.H = c->d_H;
+  ra.tokcost = c->d_tokcost;
+  ra.hold_delay_q = c->hold_delay_q;
+  ra.tile_counts = c->d_tile;
+  ra.n_tiles = (n + kTileReq - 1) / kTileReq;
+  ra.err = c->err_ptr();
+  for (int k = 0; k < c->rounds; ++k) launch_round(ra, c->num_sms, st);
+  c->mark(6);
+
+  FinalizeArgs fa{};
+  fa.n = n;
+  fa.W = c->W;
+  fa.rq = c->rq;
+  fa.H = c->d_H;
+  fa.out_inst = out->inst;
+  fa.out_reason = out->reason;
+  fa.out_hit = out->hit_blocks;
+  fa.U = c->U_ptr();
+  fa.stats = c->stats_ptr();
+  fa.err = c->err_ptr();
+  launch_finalize(fa, st);
+  c->mark(7);
+  CK(cudaGetLastError());
+  CK(enqueue_meta(c));
+  c->routed = true;
+  return MISAT_OK;
+}
+
+int misat_route_host(misat_ctx* c, const misat_batch* hb, misat_decisions* ho) {
+  if (!c || !hb || !ho || hb->out_H) return MISAT_ERR_INVALID_ARG;
+  const int32_t n = hb->n;
+  if (n < 0 || hb->n_tokens < 0) return MISAT_ERR_INVALID_ARG;
+  if (n > c->max_batch || hb->n_tokens > c->max_tokens) return MISAT_ERR_BATCH_TOO_LARGE;
+  if (n > 0 && (!hb->cls || !hb->session || !hb->tok_off || !ho->inst || !ho->reason || !ho->hit_blocks))
+    return MISAT_ERR_INVALID_ARG;
+  if (hb->n_tokens > 0 && !hb->tokens) return MISAT_ERR_INVALID_ARG;
+  cudaStream_t st = c->stream;
+  if (n > 0) {
+    CK(cudaMemcpyAsync(c->d_stage_off, hb->tok_off, (size_t)(n + 1) * 8, cudaMemcpyHostToDevice, st));
+    CK(cudaMemcpyAsync(c->d_stage_cls, hb->cls, (size_t)n, cudaMemcpyHostToDevice, st));
+    CK(cudaMemcpyAsync(c->d_stage_ses, hb->session, (size_t)n * 8, cudaMemcpyHostToDevice, st));
+    if (hb->n_tokens > 0)
+      CK(cudaMemcpyAsync(c->d_stage_tok, hb->tokens, (size_t)hb->n_tokens * 4, cudaMemcpyHostToDevice, st));
+  }
+  misat_batch db = *hb;
+  db.cls = c->d_stage_cls;
+  db.session = c->d_stage_ses;
+  db.tok_off = c->d_stage_off;
+  db.tokens = c->d_stage_tok;
+  db.group = nullptr;
+  db.out_H = nullptr;
+  misat_decisions dd{c->d_out_inst, c->d_out_reason, c->d_out_hit};
+  int rc = misat_route(c, &db, &dd);
+  if (rc) return rc;
+  if (n > 0) {
+    CK(cudaMemcpyAsync(ho->inst, c->d_out_inst, (size_t)n * 4, cudaMemcpyDeviceToHost, st));
+    CK(cudaMemcpyAsync(ho->reason, c->d_out_reason, (size_t)n, cudaMemcpyDeviceToHost, st));
+    CK(cudaMemcpyAsync(ho->hit_blocks, c->d_out_hit, (size_t)n * 4, cudaMemcpyDeviceToHost, st));
+  }
+  CK(cudaStreamSynchronize(st));
+  return MISAT_OK;
+}
+
+int misat_commit(misat_ctx* c) {
+  if (!c) return MISAT_ERR_INVALID_ARG;
+  if (!c->routed) return MISAT_ERR_STATE;
+  cudaStream_t st = c->stream;
+  CK(cudaEventSynchronize(c->ev_meta));
+  if (c->h_err()) return c->h_err();
+  c->routed = false;
+  const int n = c->last_n;
+  if (n > 0) {
+    std::vector<int64_t> sizes(c->W), add(c->W);
+    for (int w = 0; w < c->W; ++w) {
+      sizes[w] = c->h_size(w);
+      add[w] = c->h_U(w);
+    }
+    int rc = ensure_capacity(c, sizes, add);
+    if (rc) return rc;
+    rc = maybe_rebuild_sessions(c, n);
+    if (rc) return rc;
+  }
+  CK(cudaMemsetAsync(c->stats_ptr() + 18, 0, 2 * 8, st));
+  c->mark(8);
+  if (n > 0) {
+    InsertArgs ia{};
+    ia.desc = c->d_desc;
+    ia.n = n;
+    ia.n_slots = c->last_ntok / 16;
+    ia.nb = c->rq.nb;
+    ia.kbase = c->rq.kbase;
+    ia.inst = c->rq.inst;
+    ia.keys = c->d_keys;
+    ia.seq = c->seq + 1;
+    ia.size = c->size_ptr();
+    ia.new_keys = c->stats_ptr() + 18;
+    ia.err = c->err_ptr();
+    launch_insert(ia, c->num_sms, st);
+    c->mark(9);
+    SessUpdateArgs sa{n, c->rq, c->sess, c->d_prot, c->err_ptr()};
+    launch_session_update(sa, st);
+    c->mark(10);
+    int rc = evict_all(c, c->stats_ptr() + 19);
+    if (rc) return rc;
+  } else {
+    c->mark(9);
+    c->mark(10);
+  }
+  c->mark(11);
+  CK(cudaGetLastError());
+  CK(enqueue_meta(c));
+  c->seq += 1;
+  return MISAT_OK;
+}
+
+int misat_complete(misat_ctx* c, int32_t n, const uint64_t* session, const uint8_t* cls, const int32_t* total_blocks,
+                   const int64_t* residency_us, const uint8_t* done) {
+  if (!c || n < 0) return MISAT_ERR_INVALID_ARG;
+  if (n == 0) return MISAT_OK;
+  if (!session || !cls || !total_blocks || !residency_us || !done) return MISAT_ERR_INVALID_ARG;
+  std::unordered_set<uint64_t> seen;
+  seen.reserve((size_t)n * 2);
+  for (int i = 0; i < n; ++i) {
+    if (cls[i] > 2 || total_blocks[i] < 0 || residency_us[i] < 0 || session[i] == 0) return MISAT_ERR_INVALID_ARG;
+    if (!seen.insert(session[i]).second) return MISAT_ERR_INVALID_ARG;
+  }
+  for (int i = 0; i < n; ++i) {
+    if (!done[i]) continue;
+    const int b = cls[i];
+    c->hist_blocks[b].push_back(total_blocks[i]);
+    c->hist_res[b].push_back(residency_us[i]);
+    while ((int32_t)c->hist_blocks[b].size() > c->hist_window) c->hist_blocks[b].pop_front();
+    while ((int32_t)c->hist_res[b].size() > c->hist_window) c->hist_res[b].pop_front();
+  }
+  // device part: sessions and done flags through the route staging buffers (in chunks)
+  cudaStream_t st = c->stream;
+  for (int off = 0; off < n; off += c->max_batch) {
+    const int m = std::min(c->max_batch, n - off);
+    CK(cudaMemcpyAsync(c->d_stage_ses, session + off, (size_t)m * 8, cudaMemcpyHostToDevice, st));
+    CK(cudaMemcpyAsync(c->d_stage_cls, done + off, (size_t)m, cudaMemcpyHostToDevice, st));
+    CompleteArgs a{m, c->d_stage_ses, c->d_stage_cls, c->sess, c->d_prot};
+    launch_complete(a, st);
+    CK(cudaGetLastError());
+    CK(cudaStreamSynchronize(st));  // staging is reused
+  }
+  return MISAT_OK;
+}
+
+int misat_reset_instance(misat_ctx* c, int32_t w) {
+  if (!c || w < 0 || w >= c->W) return MISAT_ERR_INVALID_ARG;
+  CK(cudaMemsetAsync(c->h_desc[w].tab, 0, ((size_t)1 << c->h_desc[w].log2nb) * sizeof(Bucket), c->stream));
+  CK(cudaMemsetAsync(c->size_ptr() + w, 0, 8, c->stream));
+  return MISAT_OK;
+}
+
+int misat_evict(misat_ctx* c, int32_t w, const uint64_t* keys, int64_t n) {
+  if (!c || w < 0 || w >= c->W || n < 0 || (n > 0 && !keys)) return MISAT_ERR_INVALID_ARG;
+  cudaStream_t st = c->stream;
+  uint64_t* dk = nullptr;
+  if (n > 0) {
+    if (cudaMalloc(&dk, (size_t)n * 8) != cudaSuccess) {
+      cudaGetLastError();
+      return MISAT_ERR_OOM;
+    }
+    CK(cudaMemcpyAsync(dk, keys, (size_t)n * 8, cudaMemcpyHostToDevice, st));
+  }
+  CK(cudaMemcpyAsync(c->d_onew, &w, 4, cudaMemcpyHostToDevice, st));
+  MarkArgs ma{c->h_desc[w], n, dk, c->size_ptr() + w, c->h_bitmap[w], c->d_active + w};
+  EvictArgs ev{};
+  ev.desc = c->d_desc;
+  ev.W = c->W;
+  ev.only_w = c->d_onew;
+  ev.size = c->size_ptr();
+  ev.cur_seq = c->seq + 1;
+  ev.bitmaps = c->d_bitmap;
+  ev.cand_a = c->d_ca;
+  ev.cand_b = c->d_cb;
+  ev.theta = c->d_theta;
+  ev.active = c->d_active;
+  ev.evicted = c->stats_ptr() + 20;
+  ev.err = c->err_ptr();
+  launch_mark_evict(ma, w, ev, st);
+  CK(cudaGetLastError());
+  CK(cudaStreamSynchronize(st));
+  cudaFree(dk);
+  return MISAT_OK;
+}
+
+static int load_common_evict(misat_ctx* c) {
+  int rc = evict_all(c, c->stats_ptr() + 20);
+  if (rc) return rc;
+  CK(cudaStreamSynchronize(c->stream));
+  return read_meta(c);
+}
+
+int misat_load_entries(misat_ctx* c, int32_t w, const misat_entry* entries, int64_t n) {
+  if (!c || w < 0 || w >= c->W || n < 0 || (n > 0 && !entries)) return MISAT_ERR_INVALID_ARG;
+  for (int64_t i = 0; i < n; ++i)
+    if (entries[i].key < 2 || (entries[i].meta & 0xffff) == 0 || (entries[i].meta >> 36) >= (1ull << 28))
+      return MISAT_ERR_INVALID_ARG;
+  int rc = read_meta(c);
+  if (rc) return rc;
+  if (c->h_err()) return c->h_err();
+  std::vector<int64_t> sizes(c->W), add(c->W, 0);
+  for (int x = 0; x < c->W; ++x) sizes[x] = c->h_size(x);
+  add[w] = n;
+  if ((rc = ensure_capacity(c, sizes, add))) return rc;
+  misat_entry* de = nullptr;
+  if (n > 0) {
+    if (cudaMalloc(&de, (size_t)n * sizeof(misat_entry)) != cudaSuccess) {
+      cudaGetLastError();
+      return MISAT_ERR_OOM;
+    }
+    CK(cudaMemcpyAsync(de, entries, (size_t)n * sizeof(misat_entry), cudaMemcpyHostToDevice, c->stream));
+    EntryInsertArgs a{c->h_desc[w], n, de, c->size_ptr() + w, c->err_ptr()};
+    launch_insert_entries(a, c->stream);
+    CK(cudaGetLastError());
+  }
+  rc = load_common_evict(c);
+  cudaFree(de);
+  if (rc) return rc;
+  return c->h_err();
+}
+
+int misat_load_chains(misat_ctx* c, int32_t n_chains, const int64_t* tok_off, const int32_t* tokens,
+                      const int32_t* inst, const uint64_t* seq, const uint32_t* arr, const int32_t* max_blocks) {
+  if (!c || n_chains < 0) return MISAT_ERR_INVALID_ARG;
+  if (n_chains == 0) return MISAT_OK;
+  if (!tok_off || !inst || !seq || !arr || !max_blocks) return MISAT_ERR_INVALID_ARG;
+  if (n_chains > c->max_batch) return MISAT_ERR_BATCH_TOO_LARGE;
+  if (tok_off[0] != 0) return MISAT_ERR_INVALID_ARG;
+  const int64_t ntok = tok_off[n_chains];
+  if (ntok > c->max_tokens) return MISAT_ERR_BATCH_TOO_LARGE;
+  if (ntok > 0 && !tokens) return MISAT_ERR_INVALID_ARG;
+  std::vector<int64_t> add(c->W, 0);
+  for (int i = 0; i < n_chains; ++i) {
+    const int64_t L = tok_off[i + 1] - tok_off[i];
+    if (L < 0 || L >= (1 << 20) || inst[i] < 0 || inst[i] >= c->W || seq[i] >= (1ull << 28) ||
+        arr[i] >= (1u << 20) || max_blocks[i] < 0)
+      return MISAT_ERR_INVALID_ARG;
+    add[inst[i]] += std::min<int64_t>(L / 16, max_blocks[i]);
+  }
+  if (c->routed) return MISAT_ERR_STATE;  // the staging and key buffers hold a pending route
+  int rc = read_meta(c);
+  if (rc) return rc;
+  if (c->h_err()) return c->h_err();
+  std::vector<int64_t> sizes(c->W);
+  for (int x = 0; x < c->W; ++x) sizes[x] = c->h_size(x);
+  if ((rc = ensure_capacity(c, sizes, add))) return rc;
+  cudaStream_t st = c->stream;
+  // stage: offsets, tokens, per-chain inst / tick / limit (reuse request scratch arrays)
+  CK(cudaMemcpyAsync(c->d_stage_off, tok_off, (size_t)(n_chains + 1) * 8, cudaMemcpyHostToDevice, st));
+  if (ntok > 0) CK(cudaMemcpyAsync(c->d_stage_tok, tokens, (size_t)ntok * 4, cudaMemcpyHostToDevice, st));
+  std::vector<int32_t> nbv(n_chains);
+  std::vector<int64_t> kbv(n_chains);
+  for (int i = 0; i < n_chains; ++i) {
+    nbv[i] = (int32_t)((tok_off[i + 1] - tok_off[i]) >> 4);
+    kbv[i] = tok_off[i] >> 4;
+  }
+  CK(cudaMemcpyAsync(c->rq.nb, nbv.data(), (size_t)n_chains * 4, cudaMemcpyHostToDevice, st));
+  CK(cudaMemcpyAsync(c->rq.kbase, kbv.data(), (size_t)n_chains * 8, cudaMemcpyHostToDevice, st));
+  CK(cudaMemcpyAsync(c->rq.inst, inst, (size_t)n_chains * 4, cudaMemcpyHostToDevice, st));
+  CK(cudaMemcpyAsync(c->rq.session, seq, (size_t)n_chains * 8, cudaMemcpyHostToDevice, st));
+  CK(cudaMemcpyAsync(c->rq.choice, max_blocks, (size_t)n_chains * 4, cudaMemcpyHostToDevice, st));
+  CK(cudaMemcpyAsync(c->d_out_hit, arr, (size_t)n_chains * 4, cudaMemcpyHostToDevice, st));
+  CK(cudaMemsetAsync(c->work_ptr(), 0, 4, st));
+  HashArgs ha{};
+  ha.tok_off = c->d_stage_off;
+  ha.tokens = c->d_stage_tok;
+  ha.n_tokens = ntok;
+  ha.n = n_chains;
+  ha.seed = c->seed;
+  ha.keys = c->d_keys;
+  ha.keys_cap = c->keys_cap;
+  ha.work = c->work_ptr();
+  ha.err = c->err_ptr();
+  launch_block_hash(ha, c->num_sms, st);
+  InsertArgs ia{};
+  ia.desc = c->d_desc;
+  ia.n = n_chains;
+  ia.n_slots = ntok / 16;
+  ia.nb = c->rq.nb;
+  ia.kbase = c->rq.kbase;
+  ia.inst = c->rq.inst;
+  ia.keys = c->d_keys;
+  ia.meta_seq = c->rq.session;
+  ia.meta_arr = reinterpret_cast<const uint32_t*>(c->d_out_hit);
+  ia.max_blocks = c->rq.choice;
+  ia.size = c->size_ptr();
+  ia.new_keys = c->stats_ptr() + 21;
+  ia.err = c->err_ptr();
+  launch_insert(ia, c->num_sms, st);
+  CK(cudaGetLastError());
+  rc = load_common_evict(c);
+  if (rc) return rc;
+  return c->h_err();
+}
+
+int misat_index_size(misat_ctx* c, int32_t w, int64_t* out) {
+  if (!c || !out || w < 0 || w >= c->W) return MISAT_ERR_INVALID_ARG;
+  int rc = read_meta(c);
+  if (rc) return rc;
+  *out = c->h_size(w);
+  return c->h_err();
+}
+
+int misat_dump_index(misat_ctx* c, int32_t w, misat_entry* host_out, int64_t cap, int64_t* n_out) {
+  if (!c || !n_out || w < 0 || w >= c->W || cap < 0 || (cap > 0 && !host_out)) return MISAT_ERR_INVALID_ARG;
+  const size_t nb = (size_t)1 << c->h_desc[w].log2nb;
+  std::vector<Bucket> hb(nb);
+  CK(cudaMemcpyAsync(hb.data(), c->h_desc[w].tab, nb * sizeof(Bucket), cudaMemcpyDeviceToHost, c->stream));
+  int rc = read_meta(c);
+  if (rc) return rc;
+  std::vector<misat_entry> v;
+  for (auto& B : hb)
+    for (int s = 0; s < 4; ++s)
+      if (B.key[s] != kEmpty) v.push_back(misat_entry{B.key[s], B.meta[s]});
+  std::sort(v.begin(), v.end(), [](const misat_entry& a, const misat_entry& b) { return a.key < b.key; });
+  *n_out = (int64_t)v.size();
+  if ((int64_t)v.size() > cap) return MISAT_ERR_INVALID_ARG;
+  std::copy(v.begin(), v.end(), host_out);
+  return c->h_err();
+}
+
+int misat_dump_keys(misat_ctx* c, uint64_t* host_out, int64_t cap, int64_t* n_out) {
+  if (!c || !n_out || cap < 0 || (cap > 0 && !host_out)) return MISAT_ERR_INVALID_ARG;
+  const int n = c->last_n;
+  std::vector<int32_t> nb(n);
+  std::vector<int64_t> kb(n);
+  const int64_t slots = c->last_ntok / 16;
+  std::vector<uint64_t> keys(slots);
+  if (n > 0) {
+    CK(cudaMemcpyAsync(nb.data(), c->rq.nb, (size_t)n * 4, cudaMemcpyDeviceToHost, c->stream));
+    CK(cudaMemcpyAsync(kb.data(), c->rq.kbase, (size_t)n * 8, cudaMemcpyDeviceToHost, c->stream));
+  }
+  if (slots > 0) CK(cudaMemcpyAsync(keys.data(), c->d_keys, (size_t)slots * 8, cudaMemcpyDeviceToHost, c->stream));
+  int rc = read_meta(c);
+  if (rc) return rc;
+  int64_t k = 0;
+  for (int r = 0; r < n; ++r)
+    for (int j = 0; j < nb[r]; ++j) {
+      if (k >= cap) return MISAT_ERR_INVALID_ARG;
+      host_out[k++] = keys[kb[r] + j];
+    }
+  *n_out = k;
+  return c->h_err();
+}
+
+int misat_dump_caps(misat_ctx* c, int64_t* K_w, int64_t* K_wb, int64_t* N_wb, int64_t* kbar_w, int64_t* kbar_b,
+                    int64_t* T_b) {
+  if (!c) return MISAT_ERR_INVALID_ARG;
+  cudaStream_t st = c->stream;
+  if (K_w) CK(cudaMemcpyAsync(K_w, c->ia.K_w, c->W * 8, cudaMemcpyDeviceToHost, st));
+  if (K_wb) CK(cudaMemcpyAsync(K_wb, c->ia.K_wb, c->W * 24, cudaMemcpyDeviceToHost, st));
+  if (N_wb) CK(cudaMemcpyAsync(N_wb, c->ia.N_wb, c->W * 24, cudaMemcpyDeviceToHost, st));
+  if (kbar_w) CK(cudaMemcpyAsync(kbar_w, c->ia.kbar_w, c->W * 8, cudaMemcpyDeviceToHost, st));
+  CK(cudaStreamSynchronize(st));
+  for (int b = 0; b < 3; ++b) {
+    if (kbar_b) kbar_b[b] = c->kbar_b[b];
+    if (T_b) T_b[b] = c->T_b[b];
+  }
+  return MISAT_OK;
+}
+
+int misat_dump_counts(misat_ctx* c, int32_t* prot) {
+  if (!c || !prot) return MISAT_ERR_INVALID_ARG;
+  CK(cudaMemcpyAsync(prot, c->d_prot, c->W * 12, cudaMemcpyDeviceToHost, c->stream));
+  CK(cudaStreamSynchronize(c->stream));
+  return MISAT_OK;
+}
+
+int misat_dump_sessions(misat_ctx* c, uint64_t* ids, int32_t* state, int32_t* inst, int32_t* cls, int64_t cap,
+                        int64_t* n_out) {
+  if (!c || !n_out || cap < 0) return MISAT_ERR_INVALID_ARG;
+  const size_t N = (size_t)1 << c->sess.log2n;
+  std::vector<SessSlot> hs(N);
+  CK(cudaMemcpyAsync(hs.data(), c->sess.slots, N * sizeof(SessSlot), cudaMemcpyDeviceToHost, c->stream));
+  CK(cudaStreamSynchronize(c->stream));
+  std::vector<SessSlot> v;
+  for (auto& s : hs)
+    if (s.key && (sess_state(s.val) == kSessProtected || sess_state(s.val) == kSessReleased)) v.push_back(s);
+  std::sort(v.begin(), v.end(), [](const SessSlot& a, const SessSlot& b) { return a.key < b.key; });
+  *n_out = (int64_t)v.size();
+  if ((int64_t)v.size() > cap) return MISAT_ERR_INVALID_ARG;
+  for (size_t i = 0; i < v.size(); ++i) {
+    if (ids) ids[i] = v[i].key;
+    if (state) state[i] = (int32_t)sess_state(v[i].val);
+    if (inst) inst[i] = (int32_t)sess_inst(v[i].val);
+    if (cls) cls[i] = (int32_t)sess_cls(v[i].val);
+  }
+  return MISAT_OK;
+}
+
+int misat_stats(misat_ctx* c, misat_batch_stats* o) {
+  if (!c || !o) return MISAT_ERR_INVALID_ARG;
+  int rc = read_meta(c);
+  if (rc) return rc;
+  const unsigned long long* s = c->h_meta + c->ml.stats;
+  std::memset(o, 0, sizeof(*o));
+  o->n_requests = c->last_n;
+  for (int i = 0; i < 8; ++i) o->by_reason[i] = (int64_t)s[i];
+  for (int b = 0; b < 3; ++b) {
+    o->admitted_by_class[b] = (int64_t)s[8 + b];
+    o->held_by_class[b] = (int64_t)s[11 + b];
+    o->n_admitted += (int64_t)s[8 + b];
+    o->n_held += (int64_t)s[11 + b];
+  }
+  o->hit_tokens = (int64_t)s[14];
+  o->query_tokens = (int64_t)s[15];
+  o->probes = (int64_t)(s[16] + s[22]);
+  o->bucket_reads = (int64_t)(s[17] + s[23]);
+  o->probes_first = (int64_t)s[16];
+  o->bucket_reads_first = (int64_t)s[17];
+  o->new_keys = (int64_t)s[18];
+  o->evicted = (int64_t)s[19];
+  o->seq = (int64_t)c->seq;
+  // D_TV (Sec. 3.3) of the admitted class mix against rho, in ppm
+  const int64_t A = o->n_admitted;
+  if (A > 0) {
+    __int128 acc = 0;
+    for (int b = 0; b < 3; ++b) {
+      const __int128 d = (__int128)1000000 * o->admitted_by_class[b] - (__int128)c->rho[b] * A;
+      acc += d < 0 ? -d : d;
+    }
+    o->dtv_ppm = (int64_t)(acc / (2 * (__int128)A));
+  } else {
+    o->dtv_ppm = -1;
+  }
+  return c->h_err();
+}
+
+int misat_set_timing(misat_ctx* c, int enable) {
+  if (!c) return MISAT_ERR_INVALID_ARG;
+  if (enable && !c->ev[0])
+    for (auto& e : c->ev) CK(cudaEventCreate(&e));
+  c->timing = enable != 0;
+  return MISAT_OK;
+}
+
+int misat_phase_times(misat_ctx* c, float* ms) {
+  if (!c || !ms) return MISAT_ERR_INVALID_ARG;
+  if (!c->timing) return MISAT_ERR_STATE;
+  CK(cudaStreamSynchronize(c->stream));
+  // route phases: consecutive events 0..7; commit phases: 8..11
+  const int from[MISAT_N_PHASES] = {0, 1, 2, 3, 4, 5, 6, 8, 9, 10};
+  for (int i = 0; i < MISAT_N_PHASES; ++i) {
+    float t = 0.f;
+    if (cudaEventElapsedTime(&t, c->ev[from[i]], c->ev[from[i] + 1]) != cudaSuccess) {
+      cudaGetLastError();
+      t = 0.f;  // phase not recorded (e.g. empty batch)
+    }
+    ms[i] = t;
+  }
+  return MISAT_OK;
+}
+
+}  // extern "C"
+
+// ---- checkpoint / resume ----
+struct misat_checkpoint {
+  int W = 0;
+  std::vector<InstDesc> desc;  // saved tables (device copies) with their geometry
+  std::vector<int64_t> size;
+  SessSlot* sess = nullptr;
+  uint32_t sess_log2 = 0;
+  uint64_t sess_used = 0;
+  int32_t* prot = nullptr;
+  int64_t* backlog = nullptr;
+  int64_t* tokcost = nullptr;
+  int32_t* contraction = nullptr;
+  std::deque<int64_t> hist_blocks[3], hist_res[3];
+  uint32_t rho[3] = {0, 0, 0};
+  uint64_t seq = 0;
+};
+
+extern "C" {
+
+int misat_checkpoint_free(misat_checkpoint* k) {
+  if (!k) return MISAT_ERR_INVALID_ARG;
+  for (auto& d : k->desc) cudaFree(d.tab);
+  cudaFree(k->sess);
+  cudaFree(k->prot);
+  cudaFree(k->backlog);
+  cudaFree(k->tokcost);
+  cudaFree(k->contraction);
+  delete k;
+  return MISAT_OK;
+}
+
+int misat_checkpoint_save(misat_ctx* c, misat_checkpoint** out) {
+  if (!c || !out) return MISAT_ERR_INVALID_ARG;
+  *out = nullptr;
+  int rc = read_meta(c);
+  if (rc) return rc;
+  if (c->h_err()) return c->h_err();
+  misat_checkpoint* k = new (std::nothrow) misat_checkpoint();
+  if (!k) return MISAT_ERR_OOM;
+  cudaStream_t st = c->stream;
+  k->W = c->W;
+  k->desc = c->h_desc;
+  for (auto& d : k->desc) d.tab = nullptr;
+  bool oom = false;
+  for (int w = 0; w < c->W && !oom; ++w) {
+    const size_t bytes = ((size_t)1 << c->h_desc[w].log2nb) * sizeof(Bucket);
+    if (cudaMalloc(&k->desc[w].tab, bytes) != cudaSuccess) {
+      oom = true;
+      break;
+    }
+    if (cudaMemcpyAsync(k->desc[w].tab, c->h_desc[w].tab, bytes, cudaMemcpyDeviceToDevice, st) != cudaSuccess)
+      oom = true;
+  }
+  const size_t sbytes = ((size_t)1 << c->sess.log2n) * sizeof(SessSlot);
+  if (!oom && (cudaMalloc(&k->sess, sbytes) != cudaSuccess || cudaMalloc(&k->prot, c->W * 12) != cudaSuccess ||
+               cudaMalloc(&k->backlog, c->W * 8) != cudaSuccess || cudaMalloc(&k->tokcost, c->W * 8) != cudaSuccess ||
+               cudaMalloc(&k->contraction, c->W * 4) != cudaSuccess))
+    oom = true;
+  if (oom) {
+    cudaGetLastError();
+    misat_checkpoint_free(k);
+    return MISAT_ERR_OOM;
+  }
+  CK(cudaMemcpyAsync(k->sess, c->sess.slots, sbytes, cudaMemcpyDeviceToDevice, st));
+  CK(cudaMemcpyAsync(k->prot, c->d_prot, c->W * 12, cudaMemcpyDeviceToDevice, st));
+  CK(cudaMemcpyAsync(k->backlog, c->d_backlog, c->W * 8, cudaMemcpyDeviceToDevice, st));
+  CK(cudaMemcpyAsync(k->tokcost, c->d_tokcost, c->W * 8, cudaMemcpyDeviceToDevice, st));
+  CK(cudaMemcpyAsync(k->contraction, c->d_contraction, c->W * 4, cudaMemcpyDeviceToDevice, st));
+  CK(cudaStreamSynchronize(st));
+  k->sess_log2 = c->sess.log2n;
+  k->sess_used = c->h_meta[c->ml.sess_used];
+  k->size.resize(c->W);
+  for (int w = 0; w < c->W; ++w) k->size[w] = c->h_size(w);
+  for (int b = 0; b < 3; ++b) {
+    k->hist_blocks[b] = c->hist_blocks[b];
+    k->hist_res[b] = c->hist_res[b];
+    k->rho[b] = c->rho[b];
+  }
+  k->seq = c->seq;
+  *out = k;
+  return MISAT_OK;
+}
+
+int misat_checkpoint_restore(misat_ctx* c, const misat_checkpoint* k) {
+  if (!c || !k || k->W != c->W) return MISAT_ERR_INVALID_ARG;
+  cudaStream_t st = c->stream;
+  // the counters block is mirrored in pinned host memory: let pending copies land first
+  CK(cudaStreamSynchronize(st));
+  for (int w = 0; w < c->W; ++w) {
+    if (c->h_desc[w].log2nb != k->desc[w].log2nb) {
+      // the table grew after the save: return to the saved geometry
+      CK(cudaStreamSynchronize(st));
+      InstDesc nd;
+      uint32_t* bm;
+      uint4 *ca, *cb;
+      int rc = alloc_instance(c, w, k->desc[w].log2nb, &nd, &bm, &ca, &cb);
+      if (rc) return rc;
+      cudaFree(c->h_desc[w].tab);
+      cudaFree(c->h_bitmap[w]);
+      cudaFree(c->h_ca[w]);
+      cudaFree(c->h_cb[w]);
+      c->h_desc[w] = nd;
+      c->h_bitmap[w] = bm;
+      c->h_ca[w] = ca;
+      c->h_cb[w] = cb;
+      if ((rc = push_desc(c, w))) return rc;
+    }
+    CK(cudaMemcpyAsync(c->h_desc[w].tab, k->desc[w].tab, ((size_t)1 << k->desc[w].log2nb) * sizeof(Bucket),
+                       cudaMemcpyDeviceToDevice, st));
+  }
+  if (c->sess.log2n != k->sess_log2) {
+    CK(cudaStreamSynchronize(st));
+    SessSlot* ns = nullptr;
+    if (cudaMalloc(&ns, ((size_t)1 << k->sess_log2) * sizeof(SessSlot)) != cudaSuccess) {
+      cudaGetLastError();
+      return MISAT_ERR_OOM;
+    }
+    cudaFree(c->sess.slots);
+    c->sess.slots = ns;
+    c->sess.log2n = k->sess_log2;
+  }
+  CK(cudaMemcpyAsync(c->sess.slots, k->sess, ((size_t)1 << k->sess_log2) * sizeof(SessSlot),
+                     cudaMemcpyDeviceToDevice, st));
+  CK(cudaMemcpyAsync(c->d_prot, k->prot, c->W * 12, cudaMemcpyDeviceToDevice, st));
+  CK(cudaMemcpyAsync(c->d_backlog, k->backlog, c->W * 8, cudaMemcpyDeviceToDevice, st));
+  CK(cudaMemcpyAsync(c->d_tokcost, k->tokcost, c->W * 8, cudaMemcpyDeviceToDevice, st));
+  CK(cudaMemcpyAsync(c->d_contraction, k->contraction, c->W * 4, cudaMemcpyDeviceToDevice, st));
+  // sizes and the session-slot counter live in the counters block
+  for (int w = 0; w < c->W; ++w) reinterpret_cast<long long*>(c->h_meta + c->ml.size)[w] = k->size[w];
+  c->h_meta[c->ml.sess_used] = k->sess_used;
+  CK(cudaMemcpyAsync(c->d_meta + c->ml.size, c->h_meta + c->ml.size, (c->W + 1) * 8, cudaMemcpyHostToDevice, st));
+  for (int b = 0; b < 3; ++b) {
+    c->hist_blocks[b] = k->hist_blocks[b];
+    c->hist_res[b] = k->hist_res[b];
+    c->rho[b] = k->rho[b];
+  }
+  c->seq = k->seq;
+  c->routed = false;
+  return MISAT_OK;
+}
+
+int misat_sync(misat_ctx* c) {
+  if (!c) return MISAT_ERR_INVALID_ARG;
+  int rc = read_meta(c);
+  if (rc) return rc;
+  const int32_t e = c->h_err();
+  if (e) {
+    // reported once: clear the device error word so that the context can be reused
+    CK(cudaMemsetAsync(c->err_ptr(), 0, 4, c->stream));
+    CK(cudaStreamSynchronize(c->stream));
+    c->routed = false;
+  }
+  return e;
+}
+
+}  // extern "C"

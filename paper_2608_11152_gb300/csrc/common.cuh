@@ -1,0 +1,152 @@
+// Shared device-side definitions of the MISA-T routing library (sm_103a).
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "../../include/misat.h"
+
+namespace misat {
+
+constexpr int kBlockTokens = 16;
+constexpr uint64_t kGold = 0x9e3779b97f4a7c15ull;  // SplitMix64 increment, chain multiplier
+constexpr uint64_t kEmpty = 0;                     // empty slot key (block keys are >= 2)
+constexpr int kSlots = 4;                          // keys per bucket: one 32-byte sector
+constexpr int64_t kCapInf = 2147483647;            // "no cap"
+constexpr int64_t kBacklogMax = (int64_t)1 << 61;  // saturation of the in-batch backlog
+constexpr int kMaxW = 1024;
+
+// Session states in the device session table.
+constexpr uint32_t kSessProtected = 1;  // in O_w u P_w of `inst`
+constexpr uint32_t kSessReleased = 2;   // admitted before, protected nowhere
+constexpr uint32_t kSessDead = 3;       // finished; slot reusable
+
+// Request status during the selection rounds.
+constexpr uint8_t kStUnresolved = 0;
+constexpr uint8_t kStResolved = 1;
+constexpr uint8_t kStFollower = 2;
+
+// One bucket of an instance's resident-block table: four keys in one 32-byte
+// sector (what a probe reads) followed by their four metas (what a commit
+// updates), 64 bytes aligned.  meta = seq<<36 | arrival<<16 | (65535 - depth);
+// an empty slot has key 0 and meta 0.
+struct alignas(64) Bucket {
+  unsigned long long key[kSlots];
+  unsigned long long meta[kSlots];
+};
+static_assert(sizeof(Bucket) == 64, "bucket must be 64 bytes");
+
+// Per-instance table descriptor (device copy kept in sync by the host).
+struct InstDesc {
+  Bucket* tab;
+  uint32_t log2nb;  // number of buckets = 2^log2nb, log2nb >= 1
+  uint32_t pad;
+  int64_t cap;      // Cap_w
+};
+
+// Session table slot: key = session id (0 = never used), val = state<<40 | cls<<32 | inst.
+struct alignas(16) SessSlot {
+  unsigned long long key;
+  unsigned long long val;
+};
+
+__host__ __device__ __forceinline__ uint64_t sess_val(uint32_t state, uint32_t cls, uint32_t inst) {
+  return ((uint64_t)state << 40) | ((uint64_t)cls << 32) | (uint64_t)inst;
+}
+__host__ __device__ __forceinline__ uint32_t sess_state(uint64_t v) { return (uint32_t)(v >> 40); }
+__host__ __device__ __forceinline__ uint32_t sess_cls(uint64_t v) { return (uint32_t)(v >> 32) & 0xff; }
+__host__ __device__ __forceinline__ uint32_t sess_inst(uint64_t v) { return (uint32_t)v; }
+
+__host__ __device__ __forceinline__ uint64_t pack_meta(uint64_t seq, uint64_t arrival, uint64_t depth) {
+  return (seq << 36) | (arrival << 16) | (65535ull - depth);
+}
+
+// SplitMix64 finaliser (Steele, Lea & Flood 2014).
+__device__ __forceinline__ uint64_t mix64(uint64_t z) {
+  z = (z ^ (z >> 30)) * 0xbf58476d1ce4e5b9ull;
+  z = (z ^ (z >> 27)) * 0x94d049bb133111ebull;
+  return z ^ (z >> 31);
+}
+
+// Home bucket of a key: its top log2nb bits (keys are uniformly mixed).
+__device__ __forceinline__ uint32_t home_bucket(uint64_t key, uint32_t log2nb) {
+  return (uint32_t)(key >> (64 - log2nb));
+}
+
+// Home slot of a session id in the session table.
+__device__ __forceinline__ uint32_t sess_home(uint64_t s, uint32_t log2n) {
+  return (uint32_t)(mix64(s) >> (64 - log2n));
+}
+
+// Block-uniform early exit once a device error is recorded (safe before __syncthreads).
+__device__ __forceinline__ bool block_error(const int32_t* err) {
+  __shared__ int32_t s_err;
+  if (threadIdx.x == 0) s_err = *(volatile const int32_t*)err;
+  __syncthreads();
+  return s_err != 0;
+}
+
+// Signed 64-bit atomic add (two's complement through the unsigned overload).
+__device__ __forceinline__ void atomic_add_i64(long long* p, long long v) {
+  atomicAdd(reinterpret_cast<unsigned long long*>(p), (unsigned long long)v);
+}
+
+// Record the first device error (sticky).
+__device__ __forceinline__ void set_error(int32_t* err, int32_t code) { atomicCAS(err, 0, code); }
+
+__device__ __forceinline__ uint32_t lanemask_lt() {
+  uint32_t m;
+  asm("mov.u32 %0, %%lanemask_lt;" : "=r"(m));
+  return m;
+}
+
+// Streaming 16-byte read-only load (read once: no L1 allocation, 256-byte L2 prefetch).
+__device__ __forceinline__ int4 ld_stream_v4(const int4* p) {
+  int4 v;
+  asm volatile("ld.global.nc.L1::no_allocate.L2::256B.v4.s32 {%0,%1,%2,%3}, [%4];"
+               : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+               : "l"(p));
+  return v;
+}
+
+// Read the four keys of a bucket (one 32-byte sector) through the read-only path.
+__device__ __forceinline__ void ld_bucket_keys(const Bucket* b, unsigned long long k[4]) {
+  const ulonglong2* p = reinterpret_cast<const ulonglong2*>(b->key);
+  ulonglong2 a = __ldg(p);
+  ulonglong2 c = __ldg(p + 1);
+  k[0] = a.x;
+  k[1] = a.y;
+  k[2] = c.x;
+  k[3] = c.y;
+}
+
+// Coherent (L2) read of the four keys, for kernels that modify tables concurrently.
+__device__ __forceinline__ void ld_bucket_keys_cg(const Bucket* b, unsigned long long k[4]) {
+  const ulonglong2* p = reinterpret_cast<const ulonglong2*>(b->key);
+  ulonglong2 a = __ldcg(p);
+  ulonglong2 c = __ldcg(p + 1);
+  k[0] = a.x;
+  k[1] = a.y;
+  k[2] = c.x;
+  k[3] = c.y;
+}
+
+// Look a key up in one instance table (no concurrent writers).  Returns 1 if
+// resident.  Adds the number of buckets read to *reads.  Bounded by the table size.
+__device__ __forceinline__ int table_contains(const InstDesc& d, uint64_t key, uint32_t* reads) {
+  const uint32_t mask = (1u << d.log2nb) - 1;
+  uint32_t b = home_bucket(key, d.log2nb);
+  for (uint32_t it = 0; it <= mask; ++it) {
+    unsigned long long k[4];
+    ld_bucket_keys(d.tab + b, k);
+    *reads += 1;
+    bool hit = (k[0] == key) | (k[1] == key) | (k[2] == key) | (k[3] == key);
+    if (hit) return 1;
+    bool open = (k[0] == kEmpty) | (k[1] == kEmpty) | (k[2] == kEmpty) | (k[3] == kEmpty);
+    if (open) return 0;
+    b = (b + 1) & mask;
+  }
+  return 0;
+}
+
+}  // namespace misat

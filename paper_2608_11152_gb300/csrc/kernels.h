@@ -1,0 +1,230 @@
+// Kernel argument blocks and host-side launchers of the MISA-T routing library.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "common.cuh"
+
+namespace misat {
+
+// ---- K1 ----
+struct HashArgs {
+  const int64_t* tok_off;
+  const int32_t* tokens;
+  int64_t n_tokens;
+  int32_t n;
+  uint64_t seed;
+  uint64_t* keys;       // key of (r, j) at floor(tok_off[r]/16) + j
+  int64_t keys_cap;
+  unsigned* work;       // zeroed before the launch
+  const int32_t* err;
+};
+void launch_block_hash(const HashArgs& a, int num_sms, cudaStream_t st);
+
+// ---- per-request derived data shared by the route and commit kernels ----
+struct ReqArrays {
+  int32_t* nb;          // full blocks
+  int64_t* kbase;       // first key index
+  int32_t* L;           // prompt tokens
+  uint8_t* cls;         // copy of the batch classes
+  uint64_t* session;    // copy of the batch sessions
+  uint8_t* sst;         // session state at batch start (0 absent, 1 protected, 2 released)
+  int32_t* sinst;       // protected / last instance
+  int32_t* leader;      // first request of the session in the batch
+  uint8_t* status;      // kStUnresolved / kStResolved / kStFollower
+  int32_t* choice;      // this round's choice of an unresolved leader needing headroom
+  uint8_t* last_reason; // hold reason if it stays unresolved
+  int32_t* inst;        // decision (internal copy)
+  uint8_t* reason;      // reason (internal copy)
+};
+
+// ---- per-instance round state ----
+struct InstArrays {
+  int64_t* K_w;         // [W]
+  int64_t* K_wb;        // [W*3]
+  int64_t* N_wb;        // [W*3]
+  int64_t* kbar_w;      // [W]
+  int32_t* tot;         // [W] protected sessions at batch start
+  int32_t* gh;          // [W] global headroom at the start of the round
+  int32_t* ch;          // [W*3] class headroom at the start of the round
+  int32_t* delta;       // [W*3] admissions of the current round
+  int64_t* backlog_k;   // [W] in-batch backlog
+  unsigned long long* prefill;  // [W] admitted prefill tokens of the current round
+  long long* U;         // [W] upper bound of new keys of the pending commit
+};
+
+// ---- K2 ----
+struct ProbeArgs {
+  const InstDesc* desc;
+  int32_t W;
+  int32_t n;
+  const int32_t* nb;
+  const int64_t* kbase;
+  const uint64_t* keys;
+  uint16_t* H;                 // [n*W]
+  int2* hits;                  // (r, w) pairs with block 0 resident and nb >= 2
+  unsigned* n_hits;
+  int64_t hits_cap;
+  unsigned long long* stats;         // phase 1: [0] probes, [1] bucket reads
+  unsigned long long* stats_search;  // phase 2: [0] probes, [1] bucket reads
+  int32_t* err;
+};
+void launch_probe_first(const ProbeArgs& a, int num_sms, cudaStream_t st);
+void launch_probe_search(const ProbeArgs& a, int num_sms, cudaStream_t st);
+
+// ---- route ----
+struct SessTable {
+  SessSlot* slots;
+  uint32_t log2n;
+  unsigned long long* used;    // slots ever claimed
+};
+
+struct PrologueArgs {
+  int32_t n;
+  int64_t n_tokens;
+  const uint8_t* cls;
+  const uint64_t* session;
+  const int64_t* tok_off;
+  ReqArrays rq;
+  SessTable st;
+  unsigned long long* bm_key;  // batch-local session map
+  int32_t* bm_val;
+  uint32_t bm_log2;
+  long long* cand;             // [3]
+  int32_t* err;
+};
+void launch_prologue(const PrologueArgs& a, cudaStream_t st);
+
+struct CapsArgs {
+  int32_t W;
+  const InstDesc* desc;
+  const int32_t* prot;         // [W*3]
+  const long long* cand;       // [3]
+  int64_t kbar_b[3];
+  int64_t T_b[3];
+  uint32_t rho[3];
+  int32_t pf_q16;
+  int32_t mode;
+  const int32_t* contraction;  // [W]
+  const int64_t* backlog;      // [W]
+  InstArrays ia;
+  const int32_t* err;
+};
+void launch_caps(const CapsArgs& a, cudaStream_t st);
+
+struct RoundArgs {
+  int32_t n;
+  int32_t W;
+  ReqArrays rq;
+  InstArrays ia;
+  const uint16_t* H;
+  const int64_t* tokcost;      // [W]
+  int64_t hold_delay_q;
+  int32_t* tile_counts;        // [n_tiles * 3W]
+  int32_t n_tiles;
+  const int32_t* err;
+};
+void launch_round(const RoundArgs& a, int num_sms, cudaStream_t st);
+
+struct FinalizeArgs {
+  int32_t n;
+  int32_t W;
+  ReqArrays rq;
+  const uint16_t* H;
+  int32_t* out_inst;
+  uint8_t* out_reason;
+  int32_t* out_hit;
+  long long* U;
+  unsigned long long* stats;   // route stats block (see api)
+  const int32_t* err;
+};
+void launch_finalize(const FinalizeArgs& a, cudaStream_t st);
+
+// ---- commit ----
+struct InsertArgs {
+  const InstDesc* desc;
+  int32_t n;
+  int64_t n_slots;             // key slots to scan: floor(n_tokens / 16)
+  const int32_t* nb;
+  const int64_t* kbase;
+  const int32_t* inst;         // instance per request (-1: skip)
+  const uint64_t* keys;
+  const uint64_t* meta_seq;    // per request tick source: NULL -> (seq, r)
+  const uint32_t* meta_arr;    // per request arrival when meta_seq != NULL
+  const int32_t* max_blocks;   // per request insert limit (NULL: all)
+  uint64_t seq;
+  long long* size;             // [W] live entries
+  unsigned long long* new_keys;
+  int32_t* err;
+};
+void launch_insert(const InsertArgs& a, int num_sms, cudaStream_t st);
+
+struct EntryInsertArgs {
+  InstDesc desc;
+  int64_t n;
+  const misat_entry* entries;
+  long long* size;             // &size[w]
+  int32_t* err;
+};
+void launch_insert_entries(const EntryInsertArgs& a, cudaStream_t st);
+
+struct SessUpdateArgs {
+  int32_t n;
+  ReqArrays rq;
+  SessTable st;
+  int32_t* prot;               // [W*3]
+  int32_t* err;
+};
+void launch_session_update(const SessUpdateArgs& a, cudaStream_t st);
+
+struct CompleteArgs {
+  int32_t n;
+  const uint64_t* session;
+  const uint8_t* done;
+  SessTable st;
+  int32_t* prot;
+};
+void launch_complete(const CompleteArgs& a, cudaStream_t st);
+
+struct EvictArgs {
+  const InstDesc* desc;
+  int32_t W;
+  const int32_t* only_w;       // if not NULL: evict only instance *only_w
+  long long* size;             // [W]
+  uint64_t cur_seq;
+  uint32_t* const* bitmaps;    // [W] per instance fullness bitmap (NB/32 words)
+  uint4* const* cand_a;        // [W] candidate lists (meta, key) as uint4
+  uint4* const* cand_b;
+  unsigned long long* theta;   // [W*2] (meta, key)
+  int32_t* active;             // [W] 1: delete entries <= theta
+  unsigned long long* evicted;
+  int32_t* err;
+};
+void launch_evict(const EvictArgs& a, int chunks_per_inst, cudaStream_t st);
+
+struct MarkArgs {
+  InstDesc desc;
+  int64_t n;
+  const uint64_t* keys;
+  long long* size;             // &size[w]
+  uint32_t* bitmap;
+  int32_t* active;             // &active[w], set to 0
+};
+void launch_mark_evict(const MarkArgs& a, int32_t w, const EvictArgs& ev, cudaStream_t st);
+
+struct RehashArgs {
+  InstDesc from;
+  InstDesc to;
+  int32_t* err;
+};
+void launch_rehash(const RehashArgs& a, cudaStream_t st);
+
+struct SessRehashArgs {
+  SessTable from;
+  SessTable to;
+  int32_t* err;
+};
+void launch_sess_rehash(const SessRehashArgs& a, cudaStream_t st);
+
+}  // namespace misat

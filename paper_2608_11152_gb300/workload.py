@@ -136,15 +136,26 @@ class Scenario:
 
 
 class _AgentSession:
-    __slots__ = ("sid", "prompt", "turn", "max_turns", "decode_sum", "last_decode")
+    """Session history kept in one growing buffer; each turn's prompt is a prefix view."""
+    __slots__ = ("sid", "buf", "plen", "turn", "max_turns", "decode_sum", "last_decode")
 
-    def __init__(self, sid, prompt, max_turns):
+    def __init__(self, sid, first, max_turns, capacity):
         self.sid = sid
-        self.prompt = prompt
+        self.buf = np.empty(max(capacity, len(first)), dtype=np.int32)
+        self.buf[: len(first)] = first
+        self.plen = len(first)
         self.turn = 0
         self.max_turns = max_turns
         self.decode_sum = 0
         self.last_decode = 0
+
+    @property
+    def prompt(self):
+        return self.buf[: self.plen]
+
+    def append(self, toks):
+        self.buf[self.plen: self.plen + len(toks)] = toks
+        self.plen += len(toks)
 
 
 class MixedStream:
@@ -172,7 +183,7 @@ class MixedStream:
         s = self.spec
         L0 = int(self.rng.integers(s.agent_initial[0], s.agent_initial[1] + 1))
         mt = int(self.rng.integers(s.agent_max_turns[0], s.agent_max_turns[1] + 1))
-        return _AgentSession(self._sid(), self._tokens(L0), mt)
+        return _AgentSession(self._sid(), self._tokens(L0), mt, s.agent_hist_cap + s.agent_append[1])
 
     def next_batch(self, n: int) -> tuple[Batch, Completion]:
         s = self.spec
@@ -215,8 +226,7 @@ class MixedStream:
                 k = base + (1 if i < extra else 0)
                 for t in range(k):
                     if a.turn > 0:
-                        app = self._tokens(rng.integers(s.agent_append[0], s.agent_append[1] + 1))
-                        a.prompt = np.concatenate([a.prompt, app])
+                        a.append(self._tokens(rng.integers(s.agent_append[0], s.agent_append[1] + 1)))
                     a.turn += 1
                     dec = self._lognormal(s.agent_decode_median, 1.45, s.agent_decode_cap)
                     a.decode_sum += dec
@@ -305,9 +315,14 @@ def _stream_scenario(name, seed, W, cap, n, n_warm, spec: MixSpec, fill=0.0):
     if fill > 0:
         nf = int(fill * cap)
         for w in range(W):
-            keys = np.unique(rng.integers(2, np.iinfo(np.int64).max, size=nf + 64, dtype=np.int64)
-                             .astype(np.uint64))[:nf]
-            rng.shuffle(keys)
+            keys = rng.integers(2, np.iinfo(np.int64).max, size=nf + 64, dtype=np.int64).astype(np.uint64)
+            srt = np.sort(keys)
+            dup = np.zeros(len(keys), bool)
+            dup[1:] = srt[1:] == srt[:-1]
+            if dup.any():  # keep distinct keys only (2^-63 collisions: practically never)
+                keys = np.array(sorted(set(keys.tolist())), dtype=np.uint64)
+                rng.shuffle(keys)
+            keys = keys[:nf]
             arr = rng.integers(0, 1 << 20, size=len(keys), dtype=np.int64)
             sc.fillers.append(Filler(w=w, keys=keys, metas=entry_meta(0, arr, 0)))
     stream = MixedStream(spec, seed, sid_base=(seed % 4096) << 40)

@@ -1,0 +1,297 @@
+"""CUDA path (through the C ABI) vs the CPU oracle, element by element (bit-exact:
+every output of this path is integer or index work).
+
+Covers keys, the H matrix, caps, decisions, reasons, hit blocks, statistics, protected
+counts, the session table and the full sorted index of every instance after every
+commit; on random small scenarios (all modes, caps and eviction binding often), the five
+workload configurations and the edge cases of the API."""
+
+import numpy as np
+import pytest
+
+torch = pytest.importorskip("torch")
+if not torch.cuda.is_available():  # pragma: no cover
+    pytestmark = pytest.mark.skip(reason="needs a CUDA GPU")
+else:
+    pytestmark = pytest.mark.gpu
+
+import oracle  # noqa: E402
+from paper_2608_11152_gb300 import workload as wl  # noqa: E402
+from tests.gpu_helpers import assert_equal, compare_state, make_router, route_both, run_parity  # noqa: E402
+from tests.helpers import make_oracle  # noqa: E402
+
+pytestmark = [pytest.mark.gpu]
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    import __graft_entry__
+
+    __graft_entry__.build()
+    from paper_2608_11152_gb300 import misat  # noqa: F401
+
+
+def _mk(cls, sessions, lens, seed=0, offset_tokens=None):
+    rng = np.random.default_rng(seed)
+    off = np.zeros(len(cls) + 1, np.int64)
+    np.cumsum(lens, out=off[1:])
+    toks = offset_tokens if offset_tokens is not None else rng.integers(0, wl.VOCAB, size=int(off[-1]), dtype=np.int32)
+    return wl.Batch(cls=np.array(cls, np.uint8), session=np.array(sessions, np.uint64),
+                    group=np.zeros(len(cls), np.uint64), tok_off=off, tokens=np.ascontiguousarray(toks, np.int32))
+
+
+# ------------------------------------------------------------------ random small scenarios
+
+@pytest.mark.parametrize("seed", list(range(40)))
+def test_parity_random_small(seed):
+    rng = np.random.default_rng(seed)
+    sc = wl.small_random(5000 + seed, W=int(rng.integers(1, 9)), cap=int(rng.integers(8, 160)),
+                         n=int(rng.integers(1, 80)), rounds=int(rng.integers(1, 6)), mode=seed % 4,
+                         n_warm=int(rng.integers(0, 6)))
+    r, o = run_parity(sc)
+    r.close()
+
+
+@pytest.mark.parametrize("seed", list(range(10)))
+def test_parity_with_releases_and_rebounds(seed):
+    """Completions with done=0 release sessions (Eq. 7 continuations); backlogs change
+    between batches so continuations rebind; caps are contracted on some instances."""
+    sc = wl.small_random(7000 + seed, W=4, cap=96, n=48, rounds=3, mode=0, n_warm=6)
+    r, o = make_router(sc), make_oracle(sc)
+    rng = np.random.default_rng(seed)
+    steps = list(sc.warm) + [(sc.batch, None)]
+    for i, (b, comp) in enumerate(steps):
+        bk = rng.integers(0, 3_000_000, size=sc.W)
+        cont = rng.integers(0, 3, size=sc.W).astype(np.int32)
+        for x in (r, o):
+            x.set_instance_state(bk, None, cont)
+        route_both(r, o, b, sc.W)
+        r.commit()
+        o.commit()
+        compare_state(r, o, sc.W)
+        if comp is not None:
+            for x in (r, o):
+                x.complete(comp.session, comp.cls, comp.total_blocks, comp.residency_us, comp.done)
+        ids, st, ins, cl = o.sessions()
+        pick = ids[rng.random(len(ids)) < 0.35]
+        if len(pick):
+            z8, z32, z64 = np.zeros(len(pick), np.uint8), np.zeros(len(pick), np.int32), np.zeros(len(pick), np.int64)
+            for x in (r, o):
+                x.complete(pick, z8, z32, z64, z8)
+        compare_state(r, o, sc.W, index=False)
+    r.close()
+
+
+# ------------------------------------------------------------------ workload configurations
+
+@pytest.mark.parametrize("cfg", [1, 2, 3])
+def test_parity_config(cfg):
+    sc = wl.CONFIGS[cfg]()
+    r, o = run_parity(sc, index_every_step=cfg == 1)
+    r.close()
+
+
+def test_parity_config4_agentic_long_sessions():
+    sc = wl.config4()
+    r, o = run_parity(sc, index_every_step=False)
+    r.close()
+
+
+def test_parity_config5_reduced():
+    sc = wl.config5(n=4096, fill=0.5)
+    r, o = run_parity(sc, index_every_step=False)
+    r.close()
+
+
+def test_parity_config5_full_size():
+    """The benchmark workload itself: 128 x 262,144 blocks at 95% fill, 65,536 requests,
+    in the launch configuration the benchmark times."""
+    sc = wl.config5(n=65536, fill=0.95)
+    r, o = run_parity(sc, index_every_step=False, check_keys=True)
+    r.close()
+
+
+# ------------------------------------------------------------------ edge cases
+
+def test_empty_batch_and_commit_state():
+    from paper_2608_11152_gb300 import misat
+
+    sc = wl.small_random(11, n_warm=1)
+    r, o = make_router(sc), make_oracle(sc)
+    with pytest.raises(misat.MisatError) as e:
+        r.commit()
+    assert e.value.code == misat.ERR_STATE
+    empty = _mk([], [], [])
+    route_both(r, o, empty, sc.W)
+    r.commit()
+    o.commit()
+    assert r.stats().seq == o.seq() == 1
+    b, c = sc.warm[0]
+    route_both(r, o, b, sc.W)
+    r.commit()
+    o.commit()
+    compare_state(r, o, sc.W)
+    r.close()
+
+
+def test_short_prompts_alignments_and_partial_blocks():
+    """Prompts of 0..40 tokens (no full block, exactly one, a trailing partial block) at every
+    16-byte misalignment of their first token."""
+    lens = [0, 1, 3, 15, 16, 17, 31, 32, 33, 40, 5, 16, 47, 48, 2, 64]
+    n = len(lens)
+    sc = wl.small_random(12, W=3, cap=64, n=4, n_warm=0)
+    r, o = make_router(sc, max_batch=64, max_tokens=4096), make_oracle(sc)
+    rng = np.random.default_rng(3)
+    shared = rng.integers(0, wl.VOCAB, size=64, dtype=np.int32)
+    toks = np.concatenate([shared[:L] for L in lens])
+    b = _mk([i % 3 for i in range(n)], list(range(1, n + 1)), lens, offset_tokens=toks)
+    for _ in range(3):
+        route_both(r, o, b, sc.W)
+        r.commit()
+        o.commit()
+        compare_state(r, o, sc.W)
+    r.close()
+
+
+def test_longest_prompt_65535_blocks():
+    sc = wl.small_random(13, W=2, cap=70000, n=2, n_warm=0)
+    L = (1 << 20) - 1
+    r, o = make_router(sc, max_batch=4, max_tokens=2 * L), make_oracle(sc)
+    rng = np.random.default_rng(4)
+    t = rng.integers(0, wl.VOCAB, size=L, dtype=np.int32)
+    b = _mk([2, 2], [7, 8], [L, L], offset_tokens=np.concatenate([t, t]))
+    route_both(r, o, b, sc.W)
+    r.commit()
+    o.commit()
+    compare_state(r, o, sc.W)
+    # the same prompt again: fully cached on its instance (H = 65535)
+    b2 = _mk([2], [7], [L], offset_tokens=t)
+    out = route_both(r, o, b2, sc.W)
+    assert int(out["hit_blocks"][0]) == 65535
+    r.close()
+
+
+def test_many_instances_w1024():
+    sc = wl.small_random(14, W=1024, cap=32, n=300, rounds=3, n_warm=2)
+    r, o = run_parity(sc)
+    r.close()
+
+
+def test_one_instance():
+    sc = wl.small_random(15, W=1, cap=256, n=60, rounds=2, n_warm=3)
+    r, o = run_parity(sc)
+    r.close()
+
+
+def test_table_growth_and_session_rebuild():
+    """Tiny tables and a tiny session table: growth and rebuild paths run and stay exact."""
+    sc = wl.small_random(16, W=3, cap=8, n=70, rounds=4, mode=3, n_warm=5)
+    r, o = run_parity(sc, max_sessions=1, table_load=0.25)
+    r.close()
+
+
+def test_batch_too_large_and_invalid_device_input():
+    from paper_2608_11152_gb300 import misat
+
+    sc = wl.small_random(17, W=2, cap=64, n=8, n_warm=0)
+    r = make_router(sc, max_batch=8, max_tokens=2048)
+    big = _mk([0] * 9, list(range(1, 10)), [16] * 9)
+    with pytest.raises(misat.MisatError) as e:
+        r.route(r.device_batch(big))
+    assert e.value.code == misat.ERR_BATCH_TOO_LARGE
+    # a zero session id and a class id of 7 are found on the device: sticky error, no state change
+    bad = _mk([0, 7], [0, 5], [32, 32])
+    r.route(r.device_batch(bad))
+    with pytest.raises(misat.MisatError) as e:
+        r.sync()
+    assert e.value.code == misat.ERR_INVALID_ARG
+    # non-monotone offsets
+    bad2 = _mk([0, 1], [4, 5], [32, 32])
+    bad2.tok_off[1] = 40
+    bad2.tok_off[2] = 32
+    r.route(r.device_batch(bad2))
+    with pytest.raises(misat.MisatError):
+        r.sync()
+    # the context is usable again and still matches the oracle
+    o = make_oracle(sc)
+    good = _mk([0, 1, 2], [4, 5, 6], [48, 40, 33])
+    route_both(r, o, good, sc.W)
+    r.commit()
+    o.commit()
+    compare_state(r, o, sc.W)
+    r.close()
+
+
+def test_route_host_matches_device_route():
+    sc = wl.config1()
+    r1, r2, o = make_router(sc), make_router(sc), make_oracle(sc)
+    for b, comp in list(sc.warm) + [(sc.batch, None)]:
+        dev = route_both(r1, o, b, sc.W)
+        host = r2.route_host(b)
+        for k in ("inst", "reason", "hit_blocks"):
+            assert_equal(k, host[k][: b.n], dev[k][: b.n].cpu().numpy())
+        for x in (r1, r2, o):
+            x.commit()
+        if comp is not None:
+            for x in (r1, r2, o):
+                x.complete(comp.session, comp.cls, comp.total_blocks, comp.residency_us, comp.done)
+    for w in range(sc.W):
+        assert_equal("index", r1.dump_index(w)[1], r2.dump_index(w)[1])
+    r1.close()
+    r2.close()
+
+
+def test_external_evict_reset_and_load_chains():
+    sc = wl.small_random(18, W=3, cap=200, n=20, n_warm=2)
+    r, o = run_parity(sc)
+    # engine removal events: drop a suffix of one resident chain on every instance
+    for w in range(sc.W):
+        gk, gm = r.dump_index(w)
+        if len(gk) == 0:
+            continue
+        depth = 65535 - (gm & 0xFFFF).astype(np.int64)
+        drop = gk[depth >= max(1, int(depth.max()) - 1)]
+        r.evict(w, drop)
+        o.evict(w, drop)
+    compare_state(r, o, sc.W)
+    assert o.check_invariants() == 0
+    # cache reset of one instance (weight sync)
+    r.reset_instance(1)
+    o.reset_instance(1)
+    compare_state(r, o, sc.W)
+    # warm chains with explicit ticks and block limits
+    rng = np.random.default_rng(5)
+    lens = [100, 35, 300, 16, 0, 77]
+    off = np.zeros(len(lens) + 1, np.int64)
+    np.cumsum(lens, out=off[1:])
+    toks = rng.integers(0, wl.VOCAB, size=int(off[-1]), dtype=np.int32)
+    inst, seq, arr, mb = [0, 1, 2, 1, 0, 2], [1, 1, 2, 0, 1, 3], [5, 6, 7, 8, 9, 10], [3, 100, 12, 1, 4, 0]
+    r.load_chains(off, toks, inst, seq, arr, mb)
+    o.load_chains(off, toks, inst, seq, arr, mb)
+    compare_state(r, o, sc.W)
+    route_both(r, o, sc.batch, sc.W)
+    r.commit()
+    o.commit()
+    compare_state(r, o, sc.W)
+    r.close()
+
+
+def test_all_four_modes_on_config1():
+    for mode in range(4):
+        sc = wl.config1()
+        sc.mode = mode
+        r, o = run_parity(sc)
+        r.close()
+
+
+def test_rounds_sweep_on_config2_first_batch():
+    sc = wl.config2()
+    b = sc.warm[0][0]
+    for rounds in (1, 2, 8):
+        r = make_router(sc, rounds=rounds)
+        o = make_oracle(sc, rounds=rounds)
+        route_both(r, o, b, sc.W)
+        r.commit()
+        o.commit()
+        compare_state(r, o, sc.W)
+        r.close()
