@@ -33,6 +33,13 @@ ROOT = os.path.dirname(os.path.abspath(__file__))
 if ROOT not in sys.path:
     sys.path.insert(0, ROOT)
 
+T_START = time.perf_counter()
+
+
+def log(msg):
+    print(f"[bench {time.perf_counter() - T_START:8.1f}s] {msg}", file=sys.stderr, flush=True)
+
+
 METRIC = "routed requests/s (route+commit)"
 UNIT = "requests/s"
 CLOCK_QUERY = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
@@ -137,11 +144,13 @@ def setup_router(sc, torch):
     r.set_instance_state(sc.backlog_q, sc.tokcost_q, sc.contraction)
     for f in sc.fillers:
         r.load_entries(f.w, f.keys, f.metas)
+    log("gpu: filler entries loaded")
     for b, c in sc.warm:
         r.route(r.device_batch(b))
         r.commit()
         r.complete(c.session, c.cls, c.total_blocks, c.residency_us, c.done)
     r.sync()
+    log("gpu: warm-up batches routed and committed")
     return r
 
 
@@ -154,10 +163,12 @@ def setup_oracle(sc):
     o.set_instance_state(sc.backlog_q, sc.tokcost_q, sc.contraction)
     for f in sc.fillers:
         o.load_entries(f.w, f.keys, f.metas)
+    log("oracle: filler entries loaded")
     for b, c in sc.warm:
         o.route(b.cls, b.session, b.tok_off, b.tokens)
         o.commit()
         o.complete(c.session, c.cls, c.total_blocks, c.residency_us, c.done)
+    log("oracle: warm-up batches routed and committed")
     return o
 
 
@@ -206,21 +217,23 @@ def run_gb300(args):
     from paper_2608_11152_gb300 import misat
 
     sc = workload(args)
+    log(f"workload generated: {sc.name}, {sc.batch.n_tokens} tokens in the measured batch")
     r = setup_router(sc, torch)
     ckpt = r.checkpoint_save()
     db = r.device_batch(sc.batch)
     out = r.alloc_decisions(sc.batch.n)
     stream = r.stream
     r.set_timing(True)
+    log("checkpoint saved, batch resident")
 
     def step():
         r.route(db, out)
         r.commit()
 
-    for _ in range(args.warmup):
+    for i in range(args.warmup):
         r.checkpoint_restore(ckpt)
         step()
-        r.phase_times()
+        log(f"warm-up step {i}: " + ", ".join(f"{k} {v:.3f}" for k, v in r.phase_times().items()))
     torch.cuda.synchronize()
     K = args.steps
     starts = [torch.cuda.Event(enable_timing=True) for _ in range(K)]
@@ -249,6 +262,7 @@ def run_gb300(args):
     sampler.stop()
     step_ms = [starts[k].elapsed_time(ends[k]) for k in range(K)]
     total_ms = float(sum(step_ms))
+    log(f"timed steps done: {total_ms / K:.3f} ms/step (wall {wall:.2f} s for {K} steps incl. restores)")
     st = r.stats()
     r.sync()
     if dist:
@@ -292,7 +306,8 @@ def run_gb300(args):
         t = torch.tensor([e2e_ms], device="cuda")
         dist.all_reduce(t, op=dist.ReduceOp.MAX)
         e2e_ms = float(t.item())
-    e2e = world * n * args.e2e_steps / (e2e_ms / 1e3)
+    e2e = world * n * args.e2e_steps / max(e2e_ms / 1e3, 1e-9)
+    log(f"e2e done: {e2e_ms / max(1, args.e2e_steps):.3f} ms/step")
     h2d = int(b.cls.nbytes + b.session.nbytes + b.tok_off.nbytes + b.tokens.nbytes)
     d2h = int(n * (4 + 1 + 4))
 
@@ -341,6 +356,7 @@ def run_gb300(args):
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         o = setup_oracle(sc)
         t = cpu_step(o, sc.batch)
+        log(f"oracle step: {t:.2f} s")
         line["cpu_baseline"] = {"value": round(n / t, 1), "unit": UNIT, "cores": 1, "kind": "oracle",
                                 "sample": f"one full {n}-request batch (route+commit) from the same warmed state, "
                                           f"single-threaded C++ oracle, {t:.2f} s; host has {os.cpu_count()} cores"}

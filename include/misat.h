@@ -236,8 +236,9 @@ int misat_stats(misat_ctx* ctx, misat_batch_stats* host_out);
  * A checkpoint is a device-resident copy of the whole router state: every instance index
  * (with its table geometry), the session table, protected counts, per-instance inputs,
  * class histories and the commit counter.  save [sync]; restore [async, stream-ordered]:
- * the context returns to exactly the saved state (tables that grew since are shrunk back);
- * a pending route is dropped.  free releases the copy. */
+ * the context returns to exactly the saved state (a table that grew since keeps its
+ * larger size and receives the saved entries); a pending route is dropped.  free
+ * releases the copy. */
 typedef struct misat_checkpoint misat_checkpoint;
 int misat_checkpoint_save(misat_ctx* ctx, misat_checkpoint** out);
 int misat_checkpoint_restore(misat_ctx* ctx, const misat_checkpoint* ckpt);

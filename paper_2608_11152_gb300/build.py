@@ -73,6 +73,6 @@ def build(force: bool = False, verbose: bool = False, extra_flags=()) -> str:
 
 
 if __name__ == "__main__":
-    build(force="--force" in sys.argv, verbose=True,
+    build(force="--force" in sys.argv, verbose="--verbose" in sys.argv,
           extra_flags=["-Xptxas", "-v"] if "--ptxas" in sys.argv else [])
     print(LIB)

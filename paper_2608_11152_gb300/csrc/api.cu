@@ -1,6 +1,7 @@
 // C ABI of the MISA-T routing library: context, orchestration of the kernels, class
 // histories (host), table growth and state dumps.  See include/misat.h.
 #include <algorithm>
+#include <cstdlib>
 #include <cstring>
 #include <deque>
 #include <new>
@@ -572,6 +573,7 @@ int misat_route(misat_ctx* c, const misat_batch* b, misat_decisions* out) {
   pr.stats = c->stats_ptr() + 16;
   pr.stats_search = c->stats_ptr() + 22;
   pr.err = c->err_ptr();
+  pr.flat = getenv("MISAT_PROBE_FLAT") ? 1 : 0;
   launch_probe_first(pr, c->num_sms, st);
   c->mark(4);
   launch_probe_search(pr, c->num_sms, st);
@@ -1131,8 +1133,16 @@ int misat_checkpoint_restore(misat_ctx* c, const misat_checkpoint* k) {
   // the counters block is mirrored in pinned host memory: let pending copies land first
   CK(cudaStreamSynchronize(st));
   for (int w = 0; w < c->W; ++w) {
+    if (c->h_desc[w].log2nb > k->desc[w].log2nb) {
+      // the table grew after the save: keep the larger table and re-insert the saved
+      // entries into it (same entry set, so every later result is the same)
+      CK(cudaMemsetAsync(c->h_desc[w].tab, 0, ((size_t)1 << c->h_desc[w].log2nb) * sizeof(Bucket), st));
+      RehashArgs ra{k->desc[w], c->h_desc[w], c->err_ptr()};
+      launch_rehash(ra, st);
+      CK(cudaGetLastError());
+      continue;
+    }
     if (c->h_desc[w].log2nb != k->desc[w].log2nb) {
-      // the table grew after the save: return to the saved geometry
       CK(cudaStreamSynchronize(st));
       InstDesc nd;
       uint32_t* bm;

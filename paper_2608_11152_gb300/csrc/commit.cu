@@ -524,12 +524,13 @@ __global__ void __launch_bounds__(256) k_mark(MarkArgs a) {
       b = (b + 1) & mask;
     }
   }
-  if (threadIdx.x == 0 && blockIdx.x == 0) *a.active = 2;
   (void)cnt;
 }
 
 __global__ void __launch_bounds__(256) k_bitmap_keys(MarkArgs a) {
   const uint32_t NB = 1u << a.desc.log2nb;
+  // compaction of this instance deletes marked entries only
+  if (threadIdx.x == 0 && blockIdx.x == 0) *a.active = 2;
   for (uint32_t b0 = blockIdx.x * blockDim.x; b0 < NB; b0 += gridDim.x * blockDim.x) {
     const uint32_t b = b0 + threadIdx.x;
     bool full = false;

@@ -68,9 +68,10 @@ __device__ __forceinline__ uint64_t mix64(uint64_t z) {
   return z ^ (z >> 31);
 }
 
-// Home bucket of a key: its top log2nb bits (keys are uniformly mixed).
+// Home bucket of a key: top log2nb bits of key * G (multiplicative hashing), so that
+// loaded entries with skewed keys (e.g. 63-bit values) still spread over the table.
 __device__ __forceinline__ uint32_t home_bucket(uint64_t key, uint32_t log2nb) {
-  return (uint32_t)(key >> (64 - log2nb));
+  return (uint32_t)((key * kGold) >> (64 - log2nb));
 }
 
 // Home slot of a session id in the session table.

@@ -69,6 +69,7 @@ struct ProbeArgs {
   unsigned long long* stats;         // phase 1: [0] probes, [1] bucket reads
   unsigned long long* stats_search;  // phase 2: [0] probes, [1] bucket reads
   int32_t* err;
+  int32_t flat;                      // 1: thread-per-pair phase 1 (comparison layout)
 };
 void launch_probe_first(const ProbeArgs& a, int num_sms, cudaStream_t st);
 void launch_probe_search(const ProbeArgs& a, int num_sms, cudaStream_t st);

@@ -102,6 +102,82 @@ __global__ void __launch_bounds__(256) k2_probe_first(ProbeArgs a) {
   block_add_stats(a.stats, probes, reads);
 }
 
+// Phase 1, sub-warp layout: a group of S lanes (S = min(32, pow2 >= W)) owns one request;
+// its block-0 key is read once and broadcast, each lane probes instances w = lane, lane+S,
+// ... with up to kIlp independent sector loads in flight before any of them is consumed.
+template <int S>
+__global__ void __launch_bounds__(256) k2_probe_first_group(ProbeArgs a) {
+  constexpr int kIlp = 4;
+  __shared__ Bucket* s_tab[kMaxW];
+  __shared__ uint32_t s_lg[kMaxW];
+  if (block_error(a.err)) return;
+  for (int w = threadIdx.x; w < a.W; w += blockDim.x) {
+    s_tab[w] = a.desc[w].tab;
+    s_lg[w] = a.desc[w].log2nb;
+  }
+  __syncthreads();
+  const int lane = threadIdx.x & 31;
+  const int sub = lane & (S - 1);
+  const int gid = (blockIdx.x * blockDim.x + threadIdx.x) / S;  // group index
+  const int ngroups = (gridDim.x * blockDim.x) / S;
+  unsigned long long probes = 0, reads = 0;
+  // groups per warp iterate in lockstep so that the warp-wide ballots see every lane
+  const int warp_first_group = ((blockIdx.x * blockDim.x + (threadIdx.x & ~31)) / S);
+  for (int rb = warp_first_group; rb < a.n; rb += ngroups) {
+    const int r = rb + (gid - warp_first_group);
+    const bool live = r < a.n;
+    int32_t nb = 0;
+    uint64_t key = 0;
+    if (live) {
+      nb = a.nb[r];
+      if (nb > 0) key = a.keys[a.kbase[r]];
+    }
+    for (int w0 = 0; w0 < a.W; w0 += S * kIlp) {
+      int res[kIlp];
+      uint32_t rd[kIlp];
+#pragma unroll
+      for (int i = 0; i < kIlp; ++i) {
+        const int w = w0 + i * S + sub;
+        res[i] = 0;
+        rd[i] = 0;
+        if (live && nb > 0 && w < a.W) {
+          InstDesc d;
+          d.tab = s_tab[w];
+          d.log2nb = s_lg[w];
+          res[i] = table_contains(d, key, &rd[i]);
+        }
+      }
+#pragma unroll
+      for (int i = 0; i < kIlp; ++i) {
+        const int w = w0 + i * S + sub;
+        const bool valid = live && w < a.W;
+        if (valid) {
+          a.H[(int64_t)r * a.W + w] = (uint16_t)res[i];
+          if (nb > 0) {
+            probes += 1;
+            reads += rd[i];
+          }
+        }
+        const bool hl = valid && res[i] && nb > 1;
+        const unsigned m = __ballot_sync(0xffffffffu, hl);
+        if (m) {
+          unsigned pos = 0;
+          const int leader = __ffs(m) - 1;
+          if (lane == leader) pos = atomicAdd(a.n_hits, (unsigned)__popc(m));
+          pos = __shfl_sync(0xffffffffu, pos, leader) + __popc(m & lanemask_lt());
+          if (hl) {
+            if ((int64_t)pos < a.hits_cap)
+              a.hits[pos] = make_int2(r, w);
+            else
+              set_error(a.err, MISAT_ERR_TABLE_FULL);
+          }
+        }
+      }
+    }
+  }
+  block_add_stats(a.stats, probes, reads);
+}
+
 __global__ void __launch_bounds__(256) k2_probe_search(ProbeArgs a) {
   if (block_error(a.err)) return;
   const unsigned nh = *a.n_hits;
@@ -139,9 +215,25 @@ __global__ void __launch_bounds__(256) k2_probe_search(ProbeArgs a) {
 void launch_probe_first(const ProbeArgs& a, int num_sms, cudaStream_t st) {
   const int64_t total = (int64_t)a.n * a.W;
   if (total <= 0) return;
-  int64_t blocks = (total + 255) / 256;
-  int grid = (int)(blocks < (int64_t)num_sms * 8 ? blocks : (int64_t)num_sms * 8);
-  k2_probe_first<<<grid, 256, 0, st>>>(a);
+  if (a.flat) {
+    int64_t blocks = (total + 255) / 256;
+    int grid = (int)(blocks < (int64_t)num_sms * 8 ? blocks : (int64_t)num_sms * 8);
+    k2_probe_first<<<grid, 256, 0, st>>>(a);
+    return;
+  }
+  int S = 1;
+  while (S < a.W && S < 32) S <<= 1;
+  const int64_t threads = (int64_t)a.n * S;
+  int64_t blocks = (threads + 255) / 256;
+  const int grid = (int)(blocks < (int64_t)num_sms * 8 ? blocks : (int64_t)num_sms * 8);
+  switch (S) {
+    case 1: k2_probe_first_group<1><<<grid, 256, 0, st>>>(a); break;
+    case 2: k2_probe_first_group<2><<<grid, 256, 0, st>>>(a); break;
+    case 4: k2_probe_first_group<4><<<grid, 256, 0, st>>>(a); break;
+    case 8: k2_probe_first_group<8><<<grid, 256, 0, st>>>(a); break;
+    case 16: k2_probe_first_group<16><<<grid, 256, 0, st>>>(a); break;
+    default: k2_probe_first_group<32><<<grid, 256, 0, st>>>(a); break;
+  }
 }
 
 void launch_probe_search(const ProbeArgs& a, int num_sms, cudaStream_t st) {

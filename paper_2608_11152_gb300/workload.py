@@ -315,11 +315,12 @@ def _stream_scenario(name, seed, W, cap, n, n_warm, spec: MixSpec, fill=0.0):
     if fill > 0:
         nf = int(fill * cap)
         for w in range(W):
-            keys = rng.integers(2, np.iinfo(np.int64).max, size=nf + 64, dtype=np.int64).astype(np.uint64)
+            # full 64-bit keys (like block hashes), 0 and 1 excluded
+            keys = rng.integers(2, np.iinfo(np.uint64).max, size=nf + 64, dtype=np.uint64, endpoint=True)
             srt = np.sort(keys)
             dup = np.zeros(len(keys), bool)
             dup[1:] = srt[1:] == srt[:-1]
-            if dup.any():  # keep distinct keys only (2^-63 collisions: practically never)
+            if dup.any():  # keep distinct keys only (2^-64 collisions: practically never)
                 keys = np.array(sorted(set(keys.tolist())), dtype=np.uint64)
                 rng.shuffle(keys)
             keys = keys[:nf]

@@ -4,6 +4,9 @@ inputs, and every output is compared element by element."""
 
 from __future__ import annotations
 
+import os
+import time
+
 import numpy as np
 
 import oracle
@@ -77,6 +80,14 @@ def compare_state(r, o, W, index=True):
             assert_equal(f"index metas w={w}", gm, om)
 
 
+_T0 = time.perf_counter()
+
+
+def progress(msg):
+    if os.environ.get("MISAT_TEST_VERBOSE"):
+        print(f"[{time.perf_counter() - _T0:8.1f}s] {msg}", flush=True)
+
+
 def run_parity(sc, index_every_step=True, check_H=True, check_keys=True, final_index=True, **router_over):
     """Run a whole scenario through both implementations, comparing every step."""
     r = make_router(sc, **router_over)
@@ -84,14 +95,21 @@ def run_parity(sc, index_every_step=True, check_H=True, check_keys=True, final_i
     try:
         for f in sc.fillers:
             r.load_entries(f.w, f.keys, f.metas)
+        progress("gpu fillers loaded")
+        for f in sc.fillers:
             o.load_entries(f.w, f.keys, f.metas)
+        progress("oracle fillers loaded")
         steps = list(sc.warm) + [(sc.batch, None)]
         for i, (b, comp) in enumerate(steps):
             route_both(r, o, b, sc.W, check_H=check_H, check_keys=check_keys)
+            progress(f"batch {i} routed and compared")
             r.commit()
+            progress(f"batch {i} gpu commit")
             o.commit()
+            progress(f"batch {i} oracle commit")
             last = i == len(steps) - 1
             compare_state(r, o, sc.W, index=index_every_step or (final_index and last))
+            progress(f"batch {i} state compared")
             s = r.stats()
             os_ = o.stats()
             assert s.new_keys == os_[21], f"new keys {s.new_keys} vs {os_[21]}"

@@ -155,6 +155,7 @@ def test_short_prompts_alignments_and_partial_blocks():
 
 def test_longest_prompt_65535_blocks():
     sc = wl.small_random(13, W=2, cap=70000, n=2, n_warm=0)
+    sc.cap_blocks = np.array([70000, 70000], np.int64)
     L = (1 << 20) - 1
     r, o = make_router(sc, max_batch=4, max_tokens=2 * L), make_oracle(sc)
     rng = np.random.default_rng(4)
@@ -295,3 +296,33 @@ def test_rounds_sweep_on_config2_first_batch():
         o.commit()
         compare_state(r, o, sc.W)
         r.close()
+
+
+def test_checkpoint_restore_replays_identically():
+    """A restored checkpoint gives the same decisions and the same committed state again,
+    including after a commit that grew a table (the restore shrinks it back)."""
+    sc = wl.small_random(19, W=3, cap=16, n=60, rounds=3, mode=3, n_warm=2)
+    r, o = run_parity(sc, table_load=0.25)
+    ck = r.checkpoint_save()
+    o2 = o.clone()
+    outs = []
+    for _ in range(2):
+        r.checkpoint_restore(ck)
+        oc = o2.clone()
+        out = route_both(r, oc, sc.batch, sc.W)
+        outs.append({k: v[: sc.batch.n].cpu().numpy() for k, v in out.items()})
+        r.commit()
+        oc.commit()
+        compare_state(r, oc, sc.W)
+        oc.close()
+    for k in outs[0]:
+        assert_equal(k, outs[0][k], outs[1][k])
+    r.set_timing(True)
+    r.checkpoint_restore(ck)
+    r.route(r.device_batch(sc.batch))
+    r.commit()
+    ph = r.phase_times()
+    assert set(ph) >= {"hash", "probe_first", "evict"} and all(v >= 0 for v in ph.values())
+    ck.free()
+    o2.close()
+    r.close()
