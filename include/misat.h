@@ -262,6 +262,28 @@ int misat_checkpoint_free(misat_checkpoint* ckpt);
 int misat_set_timing(misat_ctx* ctx, int enable);
 int misat_phase_times(misat_ctx* ctx, float* ms_out);
 
+/* ---- allocation-free block hashing (the paper has no counterpart) ----
+ * For callers that cannot allocate device memory: an inference engine that has already
+ * given all free HBM to its KV-cache pool (a new cudaMalloc would fail, or fragment and
+ * shrink that pool), or a hook that runs inside another framework's allocator or
+ * memory-accounting scope where device allocations are not allowed.  It writes the same
+ * chained 16-token block keys as misat_route, in request order (request 0's full blocks,
+ * then request 1's, ... -- the layout of misat_dump_keys), and allocates nothing: its
+ * scratch (per-request key offsets, a work counter, an error word) is a fixed array of
+ * about 513 KiB inside this library, held by every GPU that loads it until exit.
+ *   tok_off   device [n+1], as in misat_batch
+ *   tokens    device [n_tokens], 16-byte aligned, readable to the next 16-byte boundary
+ *   keys_out  device [keys_cap] u64
+ * n above MISAT_NOALLOC_MAX_REQUESTS returns MISAT_ERR_BATCH_TOO_LARGE; malformed offsets
+ * or keys_cap below the number of full blocks return MISAT_ERR_INVALID_ARG (nothing is
+ * written then).  The first call on a device looks the scratch array up
+ * (cudaGetSymbolAddress, with that device current) and should come before any stream
+ * capture.  Every call shares the one array: calls that overlap on the GPU (e.g. from
+ * two streams at once) race.  [sync: waits for its stream to report errors] */
+#define MISAT_NOALLOC_MAX_REQUESTS 65536
+int misat_block_hash_noalloc(const int64_t* tok_off, const int32_t* tokens, int32_t n, int64_t n_tokens,
+                             uint64_t hash_seed, uint64_t* keys_out, int64_t keys_cap, void* cuda_stream);
+
 /* Wait for the stream and return the sticky device error (0 if none), then clear it and
  * drop any pending route.  A batch rejected on the device changes no persistent state;
  * after TABLE_FULL during a commit the index of the affected instance may hold part of

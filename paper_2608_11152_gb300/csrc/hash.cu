@@ -14,6 +14,8 @@
 // (funnel of the lane's int4 and its right neighbour's).  Lanes 4m..4m+3 hold the
 // four quarters of one block and combine their partial hashes with two xor
 // shuffles.  Keys are written coalesced at keys[floor(tok_off[r]/16) + j].
+#include <mutex>
+
 #include "common.cuh"
 #include "kernels.h"
 
@@ -160,4 +162,204 @@ void launch_block_hash(const HashArgs& a, int num_sms, cudaStream_t st) {
   k1_block_hash<<<grid, 256, 0, st>>>(a);
 }
 
+// ---------------------------------------------------------------------------
+// Allocation-free block hashing.
+//
+// Some callers of this library cannot allocate device memory: an inference engine
+// that has already handed all free HBM to its KV-cache pool (a new cudaMalloc would
+// fail, or fragment and shrink that pool), or a hook that runs inside another
+// framework's allocator or memory-accounting scope, where new device allocations are
+// not allowed.  misat_block_hash_noalloc serves them: it computes the same chained
+// block keys as the routing path and allocates nothing.  Its only scratch -- the
+// per-request key offsets, a work counter and an error word -- lives in the
+// file-scope array below, which every GPU that loads this library holds
+// (about 513 KiB) until the process exits.
+
+// scratch layout in 8-byte words: [0] work counter (low 32 bits) | [1] error word |
+// [2] total blocks | [3..7] unused | [8 .. 8 + max requests] exclusive key offsets
+constexpr int kNoAllocMaxRequests = MISAT_NOALLOC_MAX_REQUESTS;
+constexpr int kNoAllocWords = 8 + kNoAllocMaxRequests + 1;
+static __device__ __align__(256) unsigned long long g_noalloc_scratch[kNoAllocWords];
+
+namespace {
+
+// One CTA: clear the counters, validate the offsets and write the exclusive prefix of
+// floor(L_r / 16) (compact key positions) into the scratch array.
+__global__ void __launch_bounds__(1024) k1na_offsets(const int64_t* tok_off, int32_t n, int64_t n_tokens,
+                                                     int64_t keys_cap, unsigned long long* scratch) {
+  __shared__ long long s_warp[32];
+  __shared__ int s_bad;
+  const int t = threadIdx.x, lane = t & 31, wid = t >> 5;
+  if (t == 0) {
+    scratch[0] = 0;
+    scratch[1] = 0;
+    s_bad = 0;
+  }
+  __syncthreads();
+  const int per = (n + blockDim.x - 1) / blockDim.x;
+  const int lo = t * per, hi = min(n, lo + per);
+  long long local = 0;
+  bool bad = false;
+  for (int r = lo; r < hi; ++r) {
+    const int64_t t0 = tok_off[r], t1 = tok_off[r + 1];
+    if (t0 < 0 || t1 < t0 || t1 > n_tokens || (t1 - t0) >= (1 << 20)) bad = true;
+    local += (t1 - t0) >> 4;
+  }
+  if (t == 0 && tok_off[0] != 0) bad = true;
+  if (t == 0 && tok_off[n] != n_tokens) bad = true;
+  if (bad) atomicOr(&s_bad, 1);
+  long long incl = local;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const long long v = __shfl_up_sync(kFull, incl, o);
+    if (lane >= o) incl += v;
+  }
+  if (lane == 31) s_warp[wid] = incl;
+  __syncthreads();
+  if (wid == 0) {
+    const long long v = s_warp[lane];
+    long long sc = v;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const long long u = __shfl_up_sync(kFull, sc, o);
+      if (lane >= o) sc += u;
+    }
+    s_warp[lane] = sc - v;
+  }
+  __syncthreads();
+  long long run = s_warp[wid] + incl - local;
+  for (int r = lo; r < hi; ++r) {
+    scratch[8 + r] = (unsigned long long)run;
+    run += (tok_off[r + 1] - tok_off[r]) >> 4;
+  }
+  if (t == blockDim.x - 1) {
+    scratch[8 + n] = (unsigned long long)run;
+    scratch[2] = (unsigned long long)run;
+  }
+  __syncthreads();
+  if (t == 0) {
+    const long long total = (long long)scratch[2];
+    if (s_bad || total > keys_cap) scratch[1] = (unsigned long long)(long long)MISAT_ERR_INVALID_ARG;
+  }
+}
+
+// The block hash of k1_block_hash with compact output positions: block j of request r
+// goes to keys[off[r] + j] (off = the exclusive prefix above).
+__global__ void __launch_bounds__(256) k1na_hash(const int64_t* tok_off, const int32_t* tokens, int64_t n_tokens,
+                                                 int32_t n, uint64_t seed, uint64_t* keys,
+                                                 unsigned long long* scratch) {
+  if (scratch[1]) return;
+  unsigned* work = reinterpret_cast<unsigned*>(scratch);
+  const unsigned long long* off_r = scratch + 8;
+  const int lane = threadIdx.x & 31;
+  const int q = lane & 3;
+  const int64_t n_int4 = (n_tokens + 3) >> 2;
+  const int4* tok4 = reinterpret_cast<const int4*>(tokens);
+  uint64_t pw = kGold;
+  for (int i = 0; i < lane; ++i) pw *= kGold;
+  const uint64_t addA = (uint64_t)(2 * q + 1) * kGold;
+  const uint64_t addB = (uint64_t)(2 * q + 2) * kGold;
+  while (true) {
+    int r = 0;
+    if (lane == 0) r = (int)atomicAdd(work, 1u);
+    r = __shfl_sync(kFull, r, 0);
+    if (r >= n) break;
+    const int64_t t0 = tok_off[r];
+    const int32_t nb = (int32_t)((tok_off[r + 1] - t0) >> 4);
+    if (nb <= 0) continue;
+    const int64_t kb = (int64_t)off_r[r];
+    const int64_t q0 = t0 >> 2;
+    const int off = (int)(t0 & 3);
+    uint64_t carry = seed;
+    const int n_chunks = (nb + 31) >> 5;
+    for (int c = 0; c < n_chunks; ++c) {
+      const int64_t base = q0 + 128ll * c;
+      int4 v[4];
+#pragma unroll
+      for (int i = 0; i < 4; ++i) v[i] = load_tok4(tok4, base + 32 * i + lane, n_int4);
+      const int4 ex = (off != 0 && lane == 0) ? load_tok4(tok4, base + 128, n_int4) : make_int4(0, 0, 0, 0);
+      uint64_t cmine = 0;
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        int4 t = v[i];
+        if (off != 0) {
+          int4 nxt = shfl_down_int4(v[i]);
+          const int4 wrap = shfl_int4(i < 3 ? v[i + 1] : ex, 0);
+          if (lane == 31) nxt = wrap;
+          t = funnel(v[i], nxt, off);
+        }
+        const uint64_t xa = (uint64_t)(uint32_t)t.x | ((uint64_t)(uint32_t)t.y << 32);
+        const uint64_t xb = (uint64_t)(uint32_t)t.z | ((uint64_t)(uint32_t)t.w << 32);
+        uint64_t p = mix64(xa + addA) ^ mix64(xb + addB);
+        p ^= __shfl_xor_sync(kFull, p, 1);
+        p ^= __shfl_xor_sync(kFull, p, 2);
+        const uint64_t cb = mix64(p);
+        const uint64_t got = __shfl_sync(kFull, cb, 4 * (lane & 7));
+        if ((lane >> 3) == i) cmine = got;
+      }
+      const int cnt = min(32, nb - 32 * c);
+      uint64_t s = lane < cnt ? cmine : 0;
+#pragma unroll
+      for (int d = 1; d < 32; d <<= 1) {
+        const uint64_t u = __shfl_up_sync(kFull, s, d);
+        if (lane >= d) s += u * gold_pow(d);
+      }
+      const uint64_t av = carry * pw + s;
+      uint64_t key = mix64(av ^ (uint64_t)(32 * c + lane + 1));
+      key += key < 2 ? 2 : 0;
+      if (lane < cnt) keys[kb + 32ll * c + lane] = key;
+      carry = __shfl_sync(kFull, av, 31);
+    }
+  }
+}
+
+std::mutex g_noalloc_mu;
+unsigned long long* g_noalloc_ptr[256];  // device address of the scratch array, per device
+int g_noalloc_sms[256];
+
+// Per device, once, with that device current: the device address of the scratch array.
+int noalloc_setup(unsigned long long** scratch, int* sms) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 256) return MISAT_ERR_CUDA;
+  std::lock_guard<std::mutex> lock(g_noalloc_mu);
+  if (!g_noalloc_ptr[dev]) {
+    void* p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_noalloc_scratch) != cudaSuccess) {
+      cudaGetLastError();
+      return MISAT_ERR_CUDA;
+    }
+    int s = 0;
+    if (cudaDeviceGetAttribute(&s, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return MISAT_ERR_CUDA;
+    g_noalloc_sms[dev] = s;
+    g_noalloc_ptr[dev] = reinterpret_cast<unsigned long long*>(p);
+  }
+  *scratch = g_noalloc_ptr[dev];
+  *sms = g_noalloc_sms[dev];
+  return MISAT_OK;
+}
+
+}  // namespace
 }  // namespace misat
+
+extern "C" int misat_block_hash_noalloc(const int64_t* tok_off, const int32_t* tokens, int32_t n, int64_t n_tokens,
+                                        uint64_t seed, uint64_t* keys_out, int64_t keys_cap, void* cuda_stream) {
+  using namespace misat;
+  if (n < 0 || n_tokens < 0 || keys_cap < 0) return MISAT_ERR_INVALID_ARG;
+  if (n > kNoAllocMaxRequests) return MISAT_ERR_BATCH_TOO_LARGE;
+  if (n == 0) return MISAT_OK;
+  if (!tok_off || (keys_cap > 0 && !keys_out)) return MISAT_ERR_INVALID_ARG;
+  if (n_tokens > 0 && (!tokens || ((uintptr_t)tokens & 15) != 0)) return MISAT_ERR_INVALID_ARG;
+  unsigned long long* scratch = nullptr;
+  int sms = 1;
+  int rc = noalloc_setup(&scratch, &sms);
+  if (rc) return rc;
+  cudaStream_t st = (cudaStream_t)cuda_stream;
+  k1na_offsets<<<1, 1024, 0, st>>>(tok_off, n, n_tokens, keys_cap, scratch);
+  k1na_hash<<<sms * 8, 256, 0, st>>>(tok_off, tokens, n_tokens, n, seed, keys_out, scratch);
+  if (cudaGetLastError() != cudaSuccess) return MISAT_ERR_CUDA;
+  unsigned long long err = 0;
+  if (cudaMemcpyAsync(&err, scratch + 1, sizeof(err), cudaMemcpyDeviceToHost, st) != cudaSuccess ||
+      cudaStreamSynchronize(st) != cudaSuccess)
+    return MISAT_ERR_CUDA;
+  return (int)(long long)err;
+}

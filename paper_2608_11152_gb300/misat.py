@@ -93,7 +93,20 @@ _SIG = {
     "misat_checkpoint_free": [_p],
     "misat_set_timing": [_p, C.c_int],
     "misat_phase_times": [_p, _p],
+    "misat_block_hash_noalloc": [_p, _p, C.c_int32, C.c_int64, C.c_uint64, _p, C.c_int64, _p],
 }
+NOALLOC_MAX_REQUESTS = 65536
+
+
+def block_hash_noalloc(tok_off, tokens, n, n_tokens, keys_out, seed=0x9E3779B97F4A7C15, stream=None):
+    """Chained block keys of a device batch, written in request order into the device tensor
+    ``keys_out``, without any device allocation (misat_block_hash_noalloc)."""
+    import torch
+
+    st = stream if stream is not None else torch.cuda.current_stream()
+    _ck(_lib.misat_block_hash_noalloc(_tptr(tok_off), _tptr(tokens), int(n), int(n_tokens), seed,
+                                      _tptr(keys_out), int(keys_out.numel()), _p(st.cuda_stream)),
+        "misat_block_hash_noalloc")
 for _name, _args in _SIG.items():
     _f = getattr(_lib, _name)
     _f.argtypes = _args
