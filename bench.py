@@ -63,6 +63,7 @@ def parse_args():
     ap.add_argument("--fill", type=float, default=0.95, help="resident fraction of the KV block capacity")
     ap.add_argument("--e2e-steps", type=int, default=5)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--instances", type=int, default=128, help="fewer only for small profiling captures")
     return ap.parse_args()
 
 
@@ -77,7 +78,7 @@ def peaks():
 def workload(args):
     from paper_2608_11152_gb300 import workload as wl
 
-    return wl.config5(n=args.n, fill=args.fill)
+    return wl.config5(n=args.n, fill=args.fill, instances=args.instances)
 
 
 def workload_config(args, sc):

@@ -15,7 +15,7 @@ using namespace misat;
 
 namespace {
 
-constexpr int kTileReq = 1024;
+constexpr int kTileReq = kAdmitTile;
 constexpr int kMaxRounds = 64;
 
 // Small device block copied to the host in one transfer after each route / commit.
@@ -41,6 +41,28 @@ inline int ceil_log2(uint64_t x) {
   return l;
 }
 
+// Eviction work buffers of one instance table (sized with the table).
+struct InstBufs {
+  uint32_t* bitmap = nullptr;  // fullness, 1 bit per bucket
+  uint32_t* dmask = nullptr;   // deleted slots, 4 bits per bucket
+  uint4* ca = nullptr;         // collected candidates (meta, key)
+  uint4* cb = nullptr;         // narrowing work lists
+  uint4* cc = nullptr;
+  uint32_t* slots = nullptr;   // slot of each collected candidate
+  uint32_t* dslots = nullptr;  // slots certainly evicted
+};
+
+void free_bufs(InstBufs& b) {
+  cudaFree(b.bitmap);
+  cudaFree(b.dmask);
+  cudaFree(b.ca);
+  cudaFree(b.cb);
+  cudaFree(b.cc);
+  cudaFree(b.slots);
+  cudaFree(b.dslots);
+  b = InstBufs{};
+}
+
 }  // namespace
 
 struct misat_ctx {
@@ -63,12 +85,18 @@ struct misat_ctx {
   int64_t kbar_b[3] = {0, 0, 0}, T_b[3] = {0, 0, 0};
   // instance tables
   std::vector<InstDesc> h_desc;
-  std::vector<uint32_t*> h_bitmap;
-  std::vector<uint4*> h_ca, h_cb;
+  std::vector<InstBufs> h_bufs;
   InstDesc* d_desc = nullptr;
   uint32_t** d_bitmap = nullptr;
+  uint32_t** d_dmask = nullptr;
   uint4** d_ca = nullptr;
   uint4** d_cb = nullptr;
+  uint4** d_cc = nullptr;
+  uint32_t** d_slots = nullptr;
+  uint32_t** d_dslots = nullptr;
+  unsigned* d_ncand = nullptr;
+  unsigned* d_nd = nullptr;
+  unsigned long long* d_thr = nullptr;  // [2W] bracket lo | hi
   // per-instance inputs and state
   int64_t* d_backlog = nullptr;
   int64_t* d_tokcost = nullptr;
@@ -83,6 +111,7 @@ struct misat_ctx {
   // per-request scratch
   ReqArrays rq{};
   uint64_t* d_keys = nullptr;
+  int32_t* d_owner = nullptr;
   int64_t keys_cap = 0;
   uint16_t* d_H = nullptr;
   int2* d_hits = nullptr;
@@ -148,37 +177,57 @@ int dalloc_n(misat_ctx* c, T** p, size_t n) {
   return dalloc(c, reinterpret_cast<void**>(p), n * sizeof(T));
 }
 
-// Allocate instance w's table (zeroed), bitmap and candidate lists for 2^lg buckets.
-int alloc_instance(misat_ctx* c, int w, uint32_t lg, InstDesc* out, uint32_t** bm, uint4** ca, uint4** cb) {
+// Allocate instance w's table (zeroed) and its eviction buffers for 2^lg buckets.
+int alloc_instance(misat_ctx* c, int w, uint32_t lg, InstDesc* out, InstBufs* bufs) {
   const size_t nb = (size_t)1 << lg;
-  void *t = nullptr, *b = nullptr, *x = nullptr, *y = nullptr;
-  if (cudaMalloc(&t, nb * sizeof(Bucket)) != cudaSuccess || cudaMalloc(&b, (nb / 32 + 1) * 4) != cudaSuccess ||
-      cudaMalloc(&x, nb * 4 * sizeof(uint4)) != cudaSuccess || cudaMalloc(&y, nb * 4 * sizeof(uint4)) != cudaSuccess) {
+  void* t = nullptr;
+  InstBufs b;
+  if (cudaMalloc(&t, nb * sizeof(Bucket)) != cudaSuccess ||
+      cudaMalloc((void**)&b.bitmap, (nb / 32 + 1) * 4) != cudaSuccess ||
+      cudaMalloc((void**)&b.dmask, (nb / 8 + 1) * 4) != cudaSuccess ||
+      cudaMalloc((void**)&b.ca, nb * 4 * sizeof(uint4)) != cudaSuccess ||
+      cudaMalloc((void**)&b.cb, nb * 4 * sizeof(uint4)) != cudaSuccess ||
+      cudaMalloc((void**)&b.cc, nb * 4 * sizeof(uint4)) != cudaSuccess ||
+      cudaMalloc((void**)&b.slots, nb * 4 * sizeof(uint32_t)) != cudaSuccess ||
+      cudaMalloc((void**)&b.dslots, nb * 4 * sizeof(uint32_t)) != cudaSuccess) {
     cudaGetLastError();
     cudaFree(t);
-    cudaFree(b);
-    cudaFree(x);
-    cudaFree(y);
+    free_bufs(b);
     return MISAT_ERR_OOM;
   }
   CK(cudaMemsetAsync(t, 0, nb * sizeof(Bucket), c->stream));
-  CK(cudaMemsetAsync(b, 0, (nb / 32 + 1) * 4, c->stream));
+  CK(cudaMemsetAsync(b.bitmap, 0, (nb / 32 + 1) * 4, c->stream));
+  CK(cudaMemsetAsync(b.dmask, 0, (nb / 8 + 1) * 4, c->stream));
   out->tab = (Bucket*)t;
   out->log2nb = lg;
   out->pad = 0;
   out->cap = c->cap[w];
-  *bm = (uint32_t*)b;
-  *ca = (uint4*)x;
-  *cb = (uint4*)y;
+  *bufs = b;
   return MISAT_OK;
 }
 
 int push_desc(misat_ctx* c, int w) {
-  CK(cudaMemcpyAsync(c->d_desc + w, &c->h_desc[w], sizeof(InstDesc), cudaMemcpyHostToDevice, c->stream));
-  CK(cudaMemcpyAsync(c->d_bitmap + w, &c->h_bitmap[w], sizeof(uint32_t*), cudaMemcpyHostToDevice, c->stream));
-  CK(cudaMemcpyAsync(c->d_ca + w, &c->h_ca[w], sizeof(uint4*), cudaMemcpyHostToDevice, c->stream));
-  CK(cudaMemcpyAsync(c->d_cb + w, &c->h_cb[w], sizeof(uint4*), cudaMemcpyHostToDevice, c->stream));
+  cudaStream_t st = c->stream;
+  const InstBufs& b = c->h_bufs[w];
+  CK(cudaMemcpyAsync(c->d_desc + w, &c->h_desc[w], sizeof(InstDesc), cudaMemcpyHostToDevice, st));
+  CK(cudaMemcpyAsync(c->d_bitmap + w, &b.bitmap, sizeof(void*), cudaMemcpyHostToDevice, st));
+  CK(cudaMemcpyAsync(c->d_dmask + w, &b.dmask, sizeof(void*), cudaMemcpyHostToDevice, st));
+  CK(cudaMemcpyAsync(c->d_ca + w, &b.ca, sizeof(void*), cudaMemcpyHostToDevice, st));
+  CK(cudaMemcpyAsync(c->d_cb + w, &b.cb, sizeof(void*), cudaMemcpyHostToDevice, st));
+  CK(cudaMemcpyAsync(c->d_cc + w, &b.cc, sizeof(void*), cudaMemcpyHostToDevice, st));
+  CK(cudaMemcpyAsync(c->d_slots + w, &b.slots, sizeof(void*), cudaMemcpyHostToDevice, st));
+  CK(cudaMemcpyAsync(c->d_dslots + w, &b.dslots, sizeof(void*), cudaMemcpyHostToDevice, st));
   return MISAT_OK;
+}
+
+// Replace instance w's table and buffers (the old ones are freed after the stream drains).
+int swap_instance(misat_ctx* c, int w, const InstDesc& nd, const InstBufs& nb) {
+  CK(cudaStreamSynchronize(c->stream));
+  cudaFree(c->h_desc[w].tab);
+  free_bufs(c->h_bufs[w]);
+  c->h_desc[w] = nd;
+  c->h_bufs[w] = nb;
+  return push_desc(c, w);
 }
 
 uint32_t buckets_log2_for(int64_t entries, double load) {
@@ -193,23 +242,13 @@ uint32_t buckets_log2_for(int64_t entries, double load) {
 int grow_instance(misat_ctx* c, int w, int64_t need) {
   const uint32_t lg = std::max(buckets_log2_for(need, 0.5), c->h_desc[w].log2nb + 1);
   InstDesc nd;
-  uint32_t* bm;
-  uint4 *ca, *cb;
-  int rc = alloc_instance(c, w, lg, &nd, &bm, &ca, &cb);
+  InstBufs nb;
+  int rc = alloc_instance(c, w, lg, &nd, &nb);
   if (rc) return rc;
   RehashArgs ra{c->h_desc[w], nd, c->err_ptr()};
   launch_rehash(ra, c->stream);
   CK(cudaGetLastError());
-  CK(cudaStreamSynchronize(c->stream));
-  cudaFree(c->h_desc[w].tab);
-  cudaFree(c->h_bitmap[w]);
-  cudaFree(c->h_ca[w]);
-  cudaFree(c->h_cb[w]);
-  c->h_desc[w] = nd;
-  c->h_bitmap[w] = bm;
-  c->h_ca[w] = ca;
-  c->h_cb[w] = cb;
-  return push_desc(c, w);
+  return swap_instance(c, w, nd, nb);
 }
 
 // Make room for `add[w]` more entries on every instance (current sizes must be on the host).
@@ -292,24 +331,36 @@ void estimate_classes(misat_ctx* c) {
   }
 }
 
-int evict_all(misat_ctx* c, unsigned long long* evicted_counter) {
+EvictArgs evict_args(misat_ctx* c, unsigned long long* evicted_counter) {
   EvictArgs ev{};
   ev.desc = c->d_desc;
   ev.W = c->W;
   ev.only_w = nullptr;
   ev.size = c->size_ptr();
-  ev.cur_seq = c->seq + 1;
   ev.bitmaps = c->d_bitmap;
   ev.cand_a = c->d_ca;
   ev.cand_b = c->d_cb;
+  ev.cand_c = c->d_cc;
+  ev.slots = c->d_slots;
+  ev.dslots = c->d_dslots;
+  ev.dmask = c->d_dmask;
+  ev.n_cand = c->d_ncand;
+  ev.n_d = c->d_nd;
+  ev.thr_lo = c->d_thr;
+  ev.thr_hi = c->d_thr + c->W;
   ev.theta = c->d_theta;
   ev.active = c->d_active;
   ev.evicted = evicted_counter;
   ev.err = c->err_ptr();
+  return ev;
+}
+
+int evict_all(misat_ctx* c, unsigned long long* evicted_counter) {
+  const EvictArgs ev = evict_args(c, evicted_counter);
+  // streaming CTAs per instance: about 16 buckets per thread, at most 64 CTAs of 256
   uint32_t maxlg = 1;
   for (auto& d : c->h_desc) maxlg = std::max(maxlg, d.log2nb);
-  // compaction threads per instance: about 64 buckets each, at most 32 CTAs of 256
-  int chunks = (int)std::min<uint64_t>(32, std::max<uint64_t>(1, ((uint64_t)1 << maxlg) / (64 * 256)));
+  const int chunks = (int)std::min<uint64_t>(64, std::max<uint64_t>(1, ((uint64_t)1 << maxlg) / (16 * 256)));
   launch_evict(ev, chunks, c->stream);
   CK(cudaGetLastError());
   return MISAT_OK;
@@ -337,9 +388,7 @@ int misat_destroy(misat_ctx* c) {
   cudaStreamSynchronize(c->stream);
   for (size_t w = 0; w < c->h_desc.size(); ++w) {
     cudaFree(c->h_desc[w].tab);
-    cudaFree(c->h_bitmap[w]);
-    cudaFree(c->h_ca[w]);
-    cudaFree(c->h_cb[w]);
+    if (w < c->h_bufs.size()) free_bufs(c->h_bufs[w]);
   }
   cudaFree(c->sess.slots);
   for (void* p : c->owned) cudaFree(p);
@@ -408,6 +457,7 @@ int misat_create(const misat_config* cfg, void* cuda_stream, misat_ctx** out) {
   const int bm_log2 = std::max(1, ceil_log2(2 * NB));
   const size_t n_tiles = (NB + kTileReq - 1) / kTileReq;
   if ((rc = dalloc_n(c, &c->d_meta, c->ml.words)) || (rc = dalloc_n(c, &c->d_keys, (size_t)c->keys_cap)) ||
+      (rc = dalloc_n(c, &c->d_owner, (size_t)c->keys_cap)) ||
       (rc = dalloc_n(c, &c->d_H, NB * Ws)) || (rc = dalloc_n(c, &c->d_hits, (size_t)c->hits_cap)) ||
       (rc = dalloc_n(c, &c->d_bm_key, (size_t)1 << bm_log2)) ||
       (rc = dalloc_n(c, &c->d_bm_val, (size_t)1 << bm_log2)) || (rc = dalloc_n(c, &c->d_tile, n_tiles * 3 * Ws)) ||
@@ -426,7 +476,11 @@ int misat_create(const misat_config* cfg, void* cuda_stream, misat_ctx** out) {
       (rc = dalloc_n(c, &c->d_prot, 3 * Ws)) || (rc = dalloc_n(c, &c->d_theta, 2 * Ws)) ||
       (rc = dalloc_n(c, &c->d_active, Ws)) || (rc = dalloc_n(c, &c->d_onew, 1)) ||
       (rc = dalloc_n(c, &c->d_desc, Ws)) || (rc = dalloc_n(c, &c->d_bitmap, Ws)) || (rc = dalloc_n(c, &c->d_ca, Ws)) ||
-      (rc = dalloc_n(c, &c->d_cb, Ws)) || (rc = dalloc_n(c, &c->d_stage_tok, (size_t)c->max_tokens + 8)) ||
+      (rc = dalloc_n(c, &c->d_cb, Ws)) || (rc = dalloc_n(c, &c->d_cc, Ws)) || (rc = dalloc_n(c, &c->d_slots, Ws)) ||
+      (rc = dalloc_n(c, &c->d_dmask, Ws)) || (rc = dalloc_n(c, &c->d_ncand, Ws)) ||
+      (rc = dalloc_n(c, &c->d_dslots, Ws)) || (rc = dalloc_n(c, &c->d_nd, Ws)) ||
+      (rc = dalloc_n(c, &c->d_thr, 2 * Ws)) ||
+      (rc = dalloc_n(c, &c->d_stage_tok, (size_t)c->max_tokens + 8)) ||
       (rc = dalloc_n(c, &c->d_stage_off, NB + 1)) || (rc = dalloc_n(c, &c->d_stage_cls, NB)) ||
       (rc = dalloc_n(c, &c->d_stage_ses, NB)) || (rc = dalloc_n(c, &c->d_out_inst, NB)) ||
       (rc = dalloc_n(c, &c->d_out_reason, NB)) || (rc = dalloc_n(c, &c->d_out_hit, NB)))
@@ -434,12 +488,9 @@ int misat_create(const misat_config* cfg, void* cuda_stream, misat_ctx** out) {
   c->ia.U = c->U_ptr();
   // instance tables: at most half full after eviction
   c->h_desc.resize(W);
-  c->h_bitmap.assign(W, nullptr);
-  c->h_ca.assign(W, nullptr);
-  c->h_cb.assign(W, nullptr);
+  c->h_bufs.resize(W);
   for (int w = 0; w < W; ++w) {
-    if ((rc = alloc_instance(c, w, buckets_log2_for(c->cap[w], 0.5), &c->h_desc[w], &c->h_bitmap[w], &c->h_ca[w],
-                             &c->h_cb[w])))
+    if ((rc = alloc_instance(c, w, buckets_log2_for(c->cap[w], 0.5), &c->h_desc[w], &c->h_bufs[w])))
       return fail(rc);
     if ((rc = push_desc(c, w))) return fail(rc);
   }
@@ -552,6 +603,7 @@ int misat_route(misat_ctx* c, const misat_batch* b, misat_decisions* out) {
   ha.seed = c->seed;
   ha.keys = c->d_keys;
   ha.keys_cap = c->keys_cap;
+  ha.owner = c->d_owner;
   ha.work = c->work_ptr();
   ha.err = c->err_ptr();
   launch_block_hash(ha, c->num_sms, st);
@@ -679,6 +731,7 @@ int misat_commit(misat_ctx* c) {
     ia.kbase = c->rq.kbase;
     ia.inst = c->rq.inst;
     ia.keys = c->d_keys;
+    ia.owner = c->d_owner;
     ia.seq = c->seq + 1;
     ia.size = c->size_ptr();
     ia.new_keys = c->stats_ptr() + 18;
@@ -753,20 +806,9 @@ int misat_evict(misat_ctx* c, int32_t w, const uint64_t* keys, int64_t n) {
     CK(cudaMemcpyAsync(dk, keys, (size_t)n * 8, cudaMemcpyHostToDevice, st));
   }
   CK(cudaMemcpyAsync(c->d_onew, &w, 4, cudaMemcpyHostToDevice, st));
-  MarkArgs ma{c->h_desc[w], n, dk, c->size_ptr() + w, c->h_bitmap[w], c->d_active + w};
-  EvictArgs ev{};
-  ev.desc = c->d_desc;
-  ev.W = c->W;
+  MarkArgs ma{c->h_desc[w], n, dk, c->size_ptr() + w, c->h_bufs[w].bitmap, c->d_active + w};
+  EvictArgs ev = evict_args(c, c->stats_ptr() + 20);
   ev.only_w = c->d_onew;
-  ev.size = c->size_ptr();
-  ev.cur_seq = c->seq + 1;
-  ev.bitmaps = c->d_bitmap;
-  ev.cand_a = c->d_ca;
-  ev.cand_b = c->d_cb;
-  ev.theta = c->d_theta;
-  ev.active = c->d_active;
-  ev.evicted = c->stats_ptr() + 20;
-  ev.err = c->err_ptr();
   launch_mark_evict(ma, w, ev, st);
   CK(cudaGetLastError());
   CK(cudaStreamSynchronize(st));
@@ -860,6 +902,7 @@ int misat_load_chains(misat_ctx* c, int32_t n_chains, const int64_t* tok_off, co
   ha.seed = c->seed;
   ha.keys = c->d_keys;
   ha.keys_cap = c->keys_cap;
+  ha.owner = c->d_owner;
   ha.work = c->work_ptr();
   ha.err = c->err_ptr();
   launch_block_hash(ha, c->num_sms, st);
@@ -871,6 +914,7 @@ int misat_load_chains(misat_ctx* c, int32_t n_chains, const int64_t* tok_off, co
   ia.kbase = c->rq.kbase;
   ia.inst = c->rq.inst;
   ia.keys = c->d_keys;
+  ia.owner = c->d_owner;
   ia.meta_seq = c->rq.session;
   ia.meta_arr = reinterpret_cast<const uint32_t*>(c->d_out_hit);
   ia.max_blocks = c->rq.choice;
@@ -1143,21 +1187,11 @@ int misat_checkpoint_restore(misat_ctx* c, const misat_checkpoint* k) {
       continue;
     }
     if (c->h_desc[w].log2nb != k->desc[w].log2nb) {
-      CK(cudaStreamSynchronize(st));
       InstDesc nd;
-      uint32_t* bm;
-      uint4 *ca, *cb;
-      int rc = alloc_instance(c, w, k->desc[w].log2nb, &nd, &bm, &ca, &cb);
+      InstBufs nb;
+      int rc = alloc_instance(c, w, k->desc[w].log2nb, &nd, &nb);
       if (rc) return rc;
-      cudaFree(c->h_desc[w].tab);
-      cudaFree(c->h_bitmap[w]);
-      cudaFree(c->h_ca[w]);
-      cudaFree(c->h_cb[w]);
-      c->h_desc[w] = nd;
-      c->h_bitmap[w] = bm;
-      c->h_ca[w] = ca;
-      c->h_cb[w] = cb;
-      if ((rc = push_desc(c, w))) return rc;
+      if ((rc = swap_instance(c, w, nd, nb))) return rc;
     }
     CK(cudaMemcpyAsync(c->h_desc[w].tab, k->desc[w].tab, ((size_t)1 << k->desc[w].log2nb) * sizeof(Bucket),
                        cudaMemcpyDeviceToDevice, st));

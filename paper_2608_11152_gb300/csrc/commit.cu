@@ -56,32 +56,11 @@ __device__ int table_insert(const InstDesc& d, uint64_t key, uint64_t meta) {
   return -1;
 }
 
-// Owner request of key slot q (keys of request r live at kbase[r] .. kbase[r]+nb[r]-1,
-// kbase non-decreasing): the last r with kbase[r] <= q, or -1 if q is a gap.
-__device__ __forceinline__ int owner_of(int64_t q, const int64_t* kbase, const int32_t* nb, int n) {
-  int lo = 0, hi = n - 1, r = -1;
-  while (lo <= hi) {
-    const int mid = (lo + hi) >> 1;
-    if (kbase[mid] <= q) {
-      r = mid;
-      lo = mid + 1;
-    } else {
-      hi = mid - 1;
-    }
-  }
-  // several requests can share kbase when earlier ones have no full block; the owner is
-  // the last of them, which is the one found.
-  if (r < 0 || q >= kbase[r] + nb[r]) return -1;
-  return r;
-}
-
-__device__ __forceinline__ bool le128(uint64_t ma, uint64_t ka, uint64_t mb, uint64_t kb) {
-  return ma < mb || (ma == mb && ka <= kb);
-}
 }  // namespace
 
 // ---------------------------------------------------------------------------
-// Insert: one thread per key slot of the batch; owner request found by binary search.
+// Insert: one thread per key slot of the batch; the owning request comes from the owner
+// map the hash kernel wrote next to the keys.
 __global__ void __launch_bounds__(256) k4_insert(InsertArgs a) {
   if (block_error(a.err)) return;
   const int lane = threadIdx.x & 31;
@@ -92,7 +71,7 @@ __global__ void __launch_bounds__(256) k4_insert(InsertArgs a) {
     const int64_t q = base + lane;
     int w = -1, isnew = 0;
     if (q < a.n_slots) {
-      const int r = owner_of(q, a.kbase, a.nb, a.n);
+      const int r = a.owner[q];
       if (r >= 0) {
         w = a.inst[r];
         const int64_t j = q - a.kbase[r];
@@ -118,7 +97,8 @@ __global__ void __launch_bounds__(256) k4_insert(InsertArgs a) {
       nnew += c;
     }
   }
-  if (nnew) atomicAdd(a.new_keys, nnew);
+  const long long tot = block_sum((long long)nnew);
+  if (threadIdx.x == 0 && tot) atomicAdd(a.new_keys, (unsigned long long)tot);
 }
 
 void launch_insert(const InsertArgs& a, int num_sms, cudaStream_t st) {
@@ -139,7 +119,8 @@ __global__ void __launch_bounds__(256) k4_insert_entries(EntryInsertArgs a) {
     else
       nnew += res;
   }
-  if (nnew) atomic_add_i64(a.size, nnew);
+  const long long tot = block_sum(nnew);
+  if (threadIdx.x == 0 && tot) atomic_add_i64(a.size, tot);
 }
 
 void launch_insert_entries(const EntryInsertArgs& a, cudaStream_t st) {
@@ -220,287 +201,6 @@ void launch_complete(const CompleteArgs& a, cudaStream_t st) {
   k_complete<<<(a.n + 255) / 256, 256, 0, st>>>(a);
 }
 
-// ---------------------------------------------------------------------------
-// Eviction select: one CTA per instance with E = size - Cap > 0 finds theta, the E-th
-// smallest (meta, key) (ascending = oldest commit first, deeper block first, key last).
-// Pass A: histogram of the commit age of every entry (12-bit digit) and the fullness
-// bitmap of the buckets.  Pass B: entries of the threshold age bin become candidates
-// (copied with their values).  Then radix passes over the candidates, each on the 12
-// bits below the highest bit in which candidates still differ, until one is left.
-constexpr int kSelThreads = 1024;
-constexpr int kBins = 4096;
-
-__device__ __forceinline__ uint32_t age_digit(uint64_t meta, uint64_t cur_seq) {
-  const uint64_t seq = meta >> 36;
-  const uint64_t age = cur_seq > seq ? cur_seq - seq : 0;
-  return (uint32_t)(kBins - 1 - (age < (uint64_t)(kBins - 1) ? age : (uint64_t)(kBins - 1)));
-}
-
-// Block-wide: find bin t with cum(<t) < E <= cum(<=t); returns t, writes cum(<t).
-__device__ int find_threshold_bin(uint32_t* hist, long long E, long long* below, long long* s_tmp) {
-  // each thread owns 4 consecutive bins
-  const int t = threadIdx.x;
-  long long local = (long long)hist[4 * t] + hist[4 * t + 1] + hist[4 * t + 2] + hist[4 * t + 3];
-  // block exclusive scan of `local` (1024 threads) via warp scans
-  const int lane = t & 31, wid = t >> 5;
-  long long incl = local;
-#pragma unroll
-  for (int o = 1; o < 32; o <<= 1) {
-    const long long v = __shfl_up_sync(kFull, incl, o);
-    if (lane >= o) incl += v;
-  }
-  if (lane == 31) s_tmp[wid] = incl;
-  __syncthreads();
-  if (wid == 0) {
-    long long v = s_tmp[lane];
-    long long sc = v;
-#pragma unroll
-    for (int o = 1; o < 32; o <<= 1) {
-      const long long u = __shfl_up_sync(kFull, sc, o);
-      if (lane >= o) sc += u;
-    }
-    s_tmp[lane] = sc - v;  // exclusive warp offsets
-  }
-  __syncthreads();
-  const long long excl = s_tmp[wid] + incl - local;
-  __shared__ int s_bin;
-  __shared__ long long s_below;
-  if (t == 0) s_bin = -1;
-  __syncthreads();
-  long long c = excl;
-  for (int i = 0; i < 4; ++i) {
-    const long long h = hist[4 * t + i];
-    if (c < E && E <= c + h) {
-      s_bin = 4 * t + i;
-      s_below = c;
-    }
-    c += h;
-  }
-  __syncthreads();
-  *below = s_below;
-  const int bin = s_bin;
-  __syncthreads();
-  return bin;
-}
-
-__device__ __forceinline__ uint32_t digit128(uint64_t hi, uint64_t lo, int shift) {
-  // 12 bits of the 128-bit value (hi:lo) starting at bit `shift`
-  if (shift >= 64) return (uint32_t)(hi >> (shift - 64)) & (kBins - 1);
-  uint64_t v = lo >> shift;
-  if (shift > 0 && shift + 12 > 64) v |= hi << (64 - shift);
-  return (uint32_t)v & (kBins - 1);
-}
-
-__global__ void __launch_bounds__(kSelThreads) k4_evict_select(EvictArgs a) {
-  __shared__ uint32_t hist[kBins];
-  __shared__ long long s_tmp[32];
-  __shared__ unsigned s_cnt;
-  __shared__ unsigned long long s_or_hi, s_or_lo, s_v0_hi, s_v0_lo;
-  const int w = a.only_w ? *a.only_w : blockIdx.x;
-  if (block_error(a.err)) return;
-  const long long E = a.size[w] - a.desc[w].cap;
-  if (threadIdx.x == 0) a.active[w] = E > 0 ? 1 : 0;
-  if (E <= 0) return;
-  const InstDesc d = a.desc[w];
-  const uint32_t NB = 1u << d.log2nb;
-  uint32_t* bitmap = a.bitmaps[w];
-  for (int i = threadIdx.x; i < kBins; i += blockDim.x) hist[i] = 0;
-  __syncthreads();
-  // pass A: age histogram + fullness bitmap
-  for (uint32_t b0 = 0; b0 < NB; b0 += blockDim.x) {
-    const uint32_t b = b0 + threadIdx.x;
-    bool full = false;
-    if (b < NB) {
-      const ulonglong2* mp = reinterpret_cast<const ulonglong2*>(d.tab[b].meta);
-      const ulonglong2 m01 = __ldcg(mp), m23 = __ldcg(mp + 1);
-      const unsigned long long m[4] = {m01.x, m01.y, m23.x, m23.y};
-      full = true;
-#pragma unroll
-      for (int s = 0; s < 4; ++s) {
-        if (m[s]) atomicAdd(&hist[age_digit(m[s], a.cur_seq)], 1u);
-        else full = false;
-      }
-    }
-    const unsigned bits = __ballot_sync(kFull, full);
-    if ((threadIdx.x & 31) == 0 && b < NB) bitmap[b >> 5] = bits;
-  }
-  __syncthreads();
-  long long below;
-  int t1 = find_threshold_bin(hist, E, &below, s_tmp);
-  long long Erem = E - below;
-  // pass B: candidates of the threshold bin
-  if (threadIdx.x == 0) s_cnt = 0;
-  __syncthreads();
-  uint4* cur = a.cand_a[w];
-  uint4* nxt = a.cand_b[w];
-  for (uint32_t b = threadIdx.x; b < NB; b += blockDim.x) {
-    const Bucket* B = d.tab + b;
-#pragma unroll
-    for (int s = 0; s < 4; ++s) {
-      const unsigned long long m = __ldcg(&B->meta[s]);
-      if (m && age_digit(m, a.cur_seq) == (uint32_t)t1) {
-        const unsigned long long k = __ldcg(&B->key[s]);
-        const unsigned pos = atomicAdd(&s_cnt, 1u);
-        cur[pos] = make_uint4((uint32_t)m, (uint32_t)(m >> 32), (uint32_t)k, (uint32_t)(k >> 32));
-      }
-    }
-  }
-  __syncthreads();
-  unsigned cnt = s_cnt;
-  // radix narrowing over the candidates
-  for (int iter = 0; iter < 16 && cnt > 1; ++iter) {
-    if (threadIdx.x == 0) {
-      const uint4 v0 = cur[0];
-      s_v0_hi = ((unsigned long long)v0.y << 32) | v0.x;
-      s_v0_lo = ((unsigned long long)v0.w << 32) | v0.z;
-      s_or_hi = 0;
-      s_or_lo = 0;
-    }
-    for (int i = threadIdx.x; i < kBins; i += blockDim.x) hist[i] = 0;
-    __syncthreads();
-    unsigned long long oh = 0, ol = 0;
-    for (unsigned i = threadIdx.x; i < cnt; i += blockDim.x) {
-      const uint4 v = cur[i];
-      oh |= (((unsigned long long)v.y << 32) | v.x) ^ s_v0_hi;
-      ol |= (((unsigned long long)v.w << 32) | v.z) ^ s_v0_lo;
-    }
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
-      oh |= __shfl_xor_sync(kFull, oh, o);
-      ol |= __shfl_xor_sync(kFull, ol, o);
-    }
-    if ((threadIdx.x & 31) == 0) {
-      if (oh) atomicOr(&s_or_hi, oh);
-      if (ol) atomicOr(&s_or_lo, ol);
-    }
-    __syncthreads();
-    const unsigned long long dh = s_or_hi, dl = s_or_lo;
-    if (dh == 0 && dl == 0) break;  // all equal (cannot happen for distinct keys)
-    const int top = dh ? 64 + 63 - __clzll((long long)dh) : 63 - __clzll((long long)dl);
-    const int shift = top >= 11 ? top - 11 : 0;
-    for (unsigned i = threadIdx.x; i < cnt; i += blockDim.x) {
-      const uint4 v = cur[i];
-      atomicAdd(&hist[digit128(((unsigned long long)v.y << 32) | v.x, ((unsigned long long)v.w << 32) | v.z, shift)], 1u);
-    }
-    __syncthreads();
-    long long bl;
-    const int t = find_threshold_bin(hist, Erem, &bl, s_tmp);
-    Erem -= bl;
-    if (threadIdx.x == 0) s_cnt = 0;
-    __syncthreads();
-    for (unsigned i = threadIdx.x; i < cnt; i += blockDim.x) {
-      const uint4 v = cur[i];
-      if (digit128(((unsigned long long)v.y << 32) | v.x, ((unsigned long long)v.w << 32) | v.z, shift) == (uint32_t)t) {
-        const unsigned pos = atomicAdd(&s_cnt, 1u);
-        nxt[pos] = v;
-      }
-    }
-    __syncthreads();
-    cnt = s_cnt;
-    uint4* tmp = cur;
-    cur = nxt;
-    nxt = tmp;
-    __syncthreads();
-  }
-  if (threadIdx.x == 0) {
-    if (cnt < 1) set_error(a.err, MISAT_ERR_TABLE_FULL);
-    // the E-th smallest: with cnt == 1 the only candidate; if all remaining candidates
-    // are equal (impossible for distinct keys) theta is their common value
-    const uint4 v = cur[0];
-    a.theta[2 * w] = ((unsigned long long)v.y << 32) | v.x;
-    a.theta[2 * w + 1] = ((unsigned long long)v.w << 32) | v.z;
-  }
-}
-
-// Compaction of one instance table: delete entries with meta == 0 (marked) or
-// (meta, key) <= theta, then restore the probing invariant inside each run of full
-// buckets.  A run starts after a bucket that was not full before the pass and ends at
-// the next such bucket; runs are disjoint, so each is owned by one thread.
-__global__ void __launch_bounds__(256) k4_evict_compact(EvictArgs a) {
-  const int w = a.only_w ? *a.only_w : blockIdx.y;
-  if (block_error(a.err)) return;
-  // active: 0 nothing to do (bitmap not built), 1 theta eviction, 2 marked entries only
-  const int act = a.active[w];
-  if (act == 0) return;
-  const InstDesc d = a.desc[w];
-  const uint32_t NB = 1u << d.log2nb;
-  const uint32_t mask = NB - 1;
-  const uint32_t* bitmap = a.bitmaps[w];
-  const unsigned long long tm = a.theta[2 * w], tk = a.theta[2 * w + 1];
-  const uint32_t nthreads = gridDim.x * blockDim.x;
-  const uint32_t tid = blockIdx.x * blockDim.x + threadIdx.x;
-  const uint32_t per = (NB + nthreads - 1) / nthreads;
-  const uint32_t lo = tid * per;
-  const uint32_t hi = lo + per < NB ? lo + per : NB;
-  long long deleted = 0;
-  auto is_full = [&](uint32_t b) { return (bitmap[b >> 5] >> (b & 31)) & 1u; };
-  for (uint32_t x0 = lo; x0 < hi; ++x0) {
-    if (is_full((x0 - 1) & mask)) continue;  // not a run start
-    // run [x0, e]: e = first bucket at or after x0 that was not full
-    uint32_t e = x0, len = 0;
-    while (is_full(e) && len < NB) {
-      e = (e + 1) & mask;
-      ++len;
-    }
-    // delete
-    for (uint32_t i = 0; i <= len; ++i) {
-      Bucket* B = d.tab + ((x0 + i) & mask);
-#pragma unroll
-      for (int s = 0; s < 4; ++s) {
-        const unsigned long long k = B->key[s];
-        if (k == kEmpty) continue;
-        const unsigned long long m = B->meta[s];
-        if (m == 0 || (act == 1 && le128(m, k, tm, tk))) {
-          B->key[s] = kEmpty;
-          B->meta[s] = 0;
-          ++deleted;
-        }
-      }
-    }
-    if (len == 0) continue;
-    // backward shift: fill free slots of bucket x from the first later entry of the run
-    // whose home lies in [x0, x]
-    for (uint32_t i = 0; i < len; ++i) {
-      Bucket* X = d.tab + ((x0 + i) & mask);
-      for (int s = 0; s < 4; ++s) {
-        if (X->key[s] != kEmpty) continue;
-        bool moved = false;
-        for (uint32_t j = i + 1; j <= len && !moved; ++j) {
-          Bucket* Y = d.tab + ((x0 + j) & mask);
-          for (int t = 0; t < 4; ++t) {
-            const unsigned long long k = Y->key[t];
-            if (k == kEmpty) continue;
-            const uint32_t rel = (home_bucket(k, d.log2nb) - x0) & mask;
-            if (rel <= i) {
-              X->key[s] = k;
-              X->meta[s] = Y->meta[t];
-              Y->key[t] = kEmpty;
-              Y->meta[t] = 0;
-              moved = true;
-              break;
-            }
-          }
-        }
-        if (!moved) break;  // no later entry can move into x
-      }
-    }
-  }
-  if (deleted) {
-    atomic_add_i64(&a.size[w], -deleted);
-    atomicAdd(a.evicted, (unsigned long long)deleted);
-  }
-}
-
-void launch_evict(const EvictArgs& a, int chunks_per_inst, cudaStream_t st) {
-  if (a.only_w) {
-    k4_evict_select<<<1, kSelThreads, 0, st>>>(a);
-    k4_evict_compact<<<dim3(chunks_per_inst, 1), 256, 0, st>>>(a);
-  } else {
-    k4_evict_select<<<a.W, kSelThreads, 0, st>>>(a);
-    k4_evict_compact<<<dim3(chunks_per_inst, a.W), 256, 0, st>>>(a);
-  }
-}
-
 // External removal (Sec. 4.5 engine events): mark listed keys (meta = 0), rebuild the
 // fullness bitmap from the keys, then compact with theta inactive.
 __global__ void __launch_bounds__(256) k_mark(MarkArgs a) {
@@ -551,7 +251,7 @@ void launch_mark_evict(const MarkArgs& a, int32_t w, const EvictArgs& ev, cudaSt
   }
   const uint32_t NB = 1u << a.desc.log2nb;
   k_bitmap_keys<<<(NB + 255) / 256 < 4096 ? (NB + 255) / 256 : 4096, 256, 0, st>>>(a);
-  k4_evict_compact<<<dim3(8, 1), 256, 0, st>>>(ev);
+  launch_compact_marked(ev, st);
 }
 
 // Growth: re-insert every entry of `from` into the empty, larger table `to`.

@@ -92,6 +92,22 @@ __device__ __forceinline__ void atomic_add_i64(long long* p, long long v) {
   atomicAdd(reinterpret_cast<unsigned long long*>(p), (unsigned long long)v);
 }
 
+// Sum of v over the block (every thread must call it); the total is valid in thread 0.
+// Used so that per-kernel counters cost one global atomic per CTA, not per thread.
+__device__ __forceinline__ long long block_sum(long long v) {
+  __shared__ long long s_part[32];
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+  __syncthreads();  // s_part may still be read by a previous call
+  if (lane == 0) s_part[wid] = v;
+  __syncthreads();
+  long long t = 0;
+  if (threadIdx.x == 0)
+    for (int i = 0; i < (int)((blockDim.x + 31) >> 5); ++i) t += s_part[i];
+  return t;
+}
+
 // Record the first device error (sticky).
 __device__ __forceinline__ void set_error(int32_t* err, int32_t code) { atomicCAS(err, 0, code); }
 

@@ -1,0 +1,549 @@
+// Eviction down to capacity (K4c): after a commit's inserts, each instance whose index
+// holds E = size - Cap_w > 0 entries too many loses its E smallest (meta, key): the
+// least recently committed blocks, deepest first among equal ticks (Sec. 4.5 reading:
+// LRU; the commit-tick order keeps every index prefix-closed).
+//
+// Admissions concentrate on few instances (every cold request of a round prefers the
+// same cheapest instance), so E ranges from 0 to a large part of an instance; the work
+// is spread over many CTAs per instance and the one serial step is kept small:
+//   k4_evict_estimate  (1 CTA / instance)  sorted sample of up to 4096 metas -> a meta
+//                      bracket [lo, hi] that contains the E-th smallest w.h.p.
+//   k4_evict_collect   (many CTAs / instance, streaming)  fullness bitmap; entries with
+//                      meta < lo are certainly evicted (slot list D), entries with
+//                      lo <= meta <= hi go to a short list U with their values and slots
+//   k4_evict_select    (1 CTA / instance)  theta = the (E - |D|)-th smallest of U by
+//                      radix narrowing; if the bracket missed, the CTA re-collects the
+//                      whole instance and selects exactly anyway
+//   k4_evict_delete    deletes D and the entries of U at or below theta
+//   k4_evict_shift     refills the holes of every run of full buckets that lost an entry
+//                      with backward shifts (no tombstones), one thread per run
+#include "common.cuh"
+#include "kernels.h"
+
+namespace misat {
+
+namespace {
+constexpr unsigned kFull = 0xffffffffu;
+constexpr int kSelThreads = 1024;
+constexpr int kBins = 4096;
+constexpr int kSamples = 4096;  // 4 slots of up to 1024 sampled buckets
+
+__device__ __forceinline__ bool le128(uint64_t ma, uint64_t ka, uint64_t mb, uint64_t kb) {
+  return ma < mb || (ma == mb && ka <= kb);
+}
+
+__device__ __forceinline__ uint64_t v_hi(const uint4& v) { return ((unsigned long long)v.y << 32) | v.x; }
+__device__ __forceinline__ uint64_t v_lo(const uint4& v) { return ((unsigned long long)v.w << 32) | v.z; }
+
+// Block-wide (1024 threads, 4096 bins): bin t with cum(<t) < E <= cum(<=t); cum(<t) in *below.
+__device__ int find_threshold_bin(uint32_t* hist, long long E, long long* below, long long* s_tmp) {
+  const int t = threadIdx.x;
+  long long local = (long long)hist[4 * t] + hist[4 * t + 1] + hist[4 * t + 2] + hist[4 * t + 3];
+  const int lane = t & 31, wid = t >> 5;
+  long long incl = local;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const long long v = __shfl_up_sync(kFull, incl, o);
+    if (lane >= o) incl += v;
+  }
+  if (lane == 31) s_tmp[wid] = incl;
+  __syncthreads();
+  if (wid == 0) {
+    long long v = s_tmp[lane];
+    long long sc = v;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const long long u = __shfl_up_sync(kFull, sc, o);
+      if (lane >= o) sc += u;
+    }
+    s_tmp[lane] = sc - v;
+  }
+  __syncthreads();
+  const long long excl = s_tmp[wid] + incl - local;
+  __shared__ int s_bin;
+  __shared__ long long s_below;
+  if (t == 0) s_bin = -1;
+  __syncthreads();
+  long long c = excl;
+  for (int i = 0; i < 4; ++i) {
+    const long long h = hist[4 * t + i];
+    if (c < E && E <= c + h) {
+      s_bin = 4 * t + i;
+      s_below = c;
+    }
+    c += h;
+  }
+  __syncthreads();
+  *below = s_below;
+  const int bin = s_bin;
+  __syncthreads();
+  return bin;
+}
+
+// 12 bits of the 128-bit value (hi:lo) starting at bit `shift`.
+__device__ __forceinline__ uint32_t digit128(uint64_t hi, uint64_t lo, int shift) {
+  if (shift >= 64) return (uint32_t)(hi >> (shift - 64)) & (kBins - 1);
+  uint64_t v = lo >> shift;
+  if (shift > 0 && shift + 12 > 64) v |= hi << (64 - shift);
+  return (uint32_t)v & (kBins - 1);
+}
+
+__device__ __forceinline__ bool bit_of(const uint32_t* bm, uint32_t b) { return (bm[b >> 5] >> (b & 31)) & 1u; }
+// deleted-slot mask of bucket b (4 bits per bucket, 8 buckets per word)
+__device__ __forceinline__ uint32_t dmask_of(const uint32_t* dm, uint32_t b) { return (dm[b >> 3] >> ((b & 7) * 4)) & 0xFu; }
+}  // namespace
+
+
+__global__ void __launch_bounds__(kSelThreads) k4_evict_estimate(EvictArgs a) {
+  __shared__ unsigned long long s_buf[kSamples];
+  __shared__ unsigned s_m;
+  const int w = a.only_w ? *a.only_w : blockIdx.x;
+  if (block_error(a.err)) return;
+  const long long size = a.size[w];
+  const long long E = size - a.desc[w].cap;
+  const int tid = threadIdx.x;
+  if (tid == 0) {
+    a.active[w] = E > 0 ? 1 : 0;
+    a.n_d[w] = 0;
+    a.n_cand[w] = 0;
+  }
+  if (E <= 0) return;
+  const InstDesc d = a.desc[w];
+  const uint32_t NB = 1u << d.log2nb;
+  if (tid == 0) s_m = 0;
+  __syncthreads();
+  {
+    const uint32_t nsb = NB < 1024u ? NB : 1024u;
+    unsigned occ = 0;
+    for (int s = 0; s < 4; ++s) s_buf[4 * tid + s] = ~0ull;
+    if ((uint32_t)tid < nsb) {
+      const uint32_t b = (uint32_t)(((uint64_t)tid * NB) / nsb);
+      const ulonglong2* mp = reinterpret_cast<const ulonglong2*>(d.tab[b].meta);
+      const ulonglong2 m01 = __ldcg(mp), m23 = __ldcg(mp + 1);
+      const unsigned long long m[4] = {m01.x, m01.y, m23.x, m23.y};
+      for (int s = 0; s < 4; ++s)
+        if (m[s]) {
+          s_buf[4 * tid + s] = m[s];
+          ++occ;
+        }
+    }
+    if (occ) atomicAdd(&s_m, occ);
+  }
+  __syncthreads();
+  for (int k = 2; k <= kSamples; k <<= 1) {
+    for (int j = k >> 1; j > 0; j >>= 1) {
+      for (int i = tid; i < kSamples; i += kSelThreads) {
+        const int ixj = i ^ j;
+        if (ixj > i) {
+          const unsigned long long x = s_buf[i], y = s_buf[ixj];
+          if ((x > y) == ((i & k) == 0)) {
+            s_buf[i] = y;
+            s_buf[ixj] = x;
+          }
+        }
+      }
+      __syncthreads();
+    }
+  }
+  if (tid == 0) {
+    // the E-th smallest sits near sample index p = E m / size; bracket it by ~3 standard
+    // deviations of the sample count plus a constant on both sides
+    const unsigned m = s_m;
+    unsigned long long lo = 0, hi = ~0ull;
+    if (m > 0 && size > 0) {
+      const double p = (double)E * (double)m / (double)size;
+      const double margin = 3.0 * sqrt(p + 1.0) + 16.0;
+      const double il = p - margin, ih = p + margin;
+      if (il >= 0.0) lo = s_buf[(int)il];
+      if (ih < (double)m) hi = s_buf[(int)ih];
+    }
+    a.thr_lo[w] = lo;
+    a.thr_hi[w] = hi;
+  }
+}
+
+// Streaming pass over the instance's metas (grid.x CTAs per instance).
+__global__ void __launch_bounds__(256) k4_evict_collect(EvictArgs a) {
+  const int w = a.only_w ? *a.only_w : blockIdx.y;
+  if (block_error(a.err)) return;
+  if (a.active[w] != 1) return;
+  const InstDesc d = a.desc[w];
+  const uint32_t NB = 1u << d.log2nb;
+  const unsigned long long lo = a.thr_lo[w], hi = a.thr_hi[w];
+  uint32_t* bitmap = a.bitmaps[w];
+  uint32_t* dmask = a.dmask[w];
+  uint32_t* dsl = a.dslots[w];
+  uint4* u = a.cand_a[w];
+  uint32_t* usl = a.slots[w];
+  const int lane = threadIdx.x & 31;
+  const uint32_t stride = gridDim.x * blockDim.x;
+  for (uint32_t b0 = blockIdx.x * blockDim.x; b0 < NB; b0 += stride) {
+    const uint32_t b = b0 + threadIdx.x;
+    unsigned long long m[4] = {0, 0, 0, 0};
+    bool full = false;
+    if (b < NB) {
+      const ulonglong2* mp = reinterpret_cast<const ulonglong2*>(d.tab[b].meta);
+      const ulonglong2 m01 = __ldcg(mp), m23 = __ldcg(mp + 1);
+      m[0] = m01.x;
+      m[1] = m01.y;
+      m[2] = m23.x;
+      m[3] = m23.y;
+      full = m[0] && m[1] && m[2] && m[3];
+    }
+    int nd = 0, nu = 0;
+#pragma unroll
+    for (int s = 0; s < 4; ++s) {
+      if (!m[s]) continue;
+      if (m[s] < lo) ++nd;
+      else if (m[s] <= hi) ++nu;
+    }
+    // warp-aggregated reservations in both lists
+    int id = nd, iu = nu;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int vd = __shfl_up_sync(kFull, id, o), vu = __shfl_up_sync(kFull, iu, o);
+      if (lane >= o) {
+        id += vd;
+        iu += vu;
+      }
+    }
+    const int td = __shfl_sync(kFull, id, 31), tu = __shfl_sync(kFull, iu, 31);
+    unsigned bd = 0, bu = 0;
+    if (lane == 31) {
+      if (td) bd = atomicAdd(&a.n_d[w], (unsigned)td);
+      if (tu) bu = atomicAdd(&a.n_cand[w], (unsigned)tu);
+    }
+    bd = __shfl_sync(kFull, bd, 31) + (unsigned)(id - nd);
+    bu = __shfl_sync(kFull, bu, 31) + (unsigned)(iu - nu);
+#pragma unroll
+    for (int s = 0; s < 4; ++s) {
+      if (!m[s]) continue;
+      if (m[s] < lo) {
+        dsl[bd++] = b * 4 + s;
+      } else if (m[s] <= hi) {
+        const unsigned long long key = __ldcg(&d.tab[b].key[s]);
+        u[bu] = make_uint4((uint32_t)m[s], (uint32_t)(m[s] >> 32), (uint32_t)key, (uint32_t)(key >> 32));
+        usl[bu] = b * 4 + s;
+        ++bu;
+      }
+    }
+    const unsigned bits = __ballot_sync(kFull, full);
+    if (lane == 0 && b < NB) bitmap[b >> 5] = bits;
+    if ((lane & 7) == 0 && b < NB) dmask[b >> 3] = 0;
+  }
+}
+
+__global__ void __launch_bounds__(kSelThreads) k4_evict_select(EvictArgs a) {
+  __shared__ uint32_t hist[kBins];
+  __shared__ long long s_tmp[32];
+  __shared__ unsigned s_cnt;
+  __shared__ unsigned long long s_or_hi, s_or_lo, s_v0_hi, s_v0_lo;
+  const int w = a.only_w ? *a.only_w : blockIdx.x;
+  if (block_error(a.err)) return;
+  if (a.active[w] != 1) return;
+  const long long E = a.size[w] - a.desc[w].cap;
+  const int tid = threadIdx.x;
+  const InstDesc d = a.desc[w];
+  const uint32_t NB = 1u << d.log2nb;
+  uint4* c0 = a.cand_a[w];
+  unsigned cnt = a.n_cand[w];
+  const unsigned nd = a.n_d[w];
+  long long Erem = E - (long long)nd;
+  if (Erem <= 0 || Erem > (long long)cnt) {
+    // the bracket missed the E-th smallest: collect every entry of the instance here
+    if (tid == 0) s_cnt = 0;
+    __syncthreads();
+    uint32_t* usl = a.slots[w];
+    for (uint32_t b = tid; b < NB; b += kSelThreads) {
+      for (int s = 0; s < 4; ++s) {
+        const unsigned long long m = __ldcg(&d.tab[b].meta[s]);
+        if (!m) continue;
+        const unsigned long long key = __ldcg(&d.tab[b].key[s]);
+        const unsigned pos = atomicAdd(&s_cnt, 1u);
+        c0[pos] = make_uint4((uint32_t)m, (uint32_t)(m >> 32), (uint32_t)key, (uint32_t)(key >> 32));
+        usl[pos] = b * 4 + s;
+      }
+    }
+    __syncthreads();
+    cnt = s_cnt;
+    Erem = E;
+    if (tid == 0) {
+      a.n_cand[w] = cnt;
+      a.n_d[w] = 0;
+    }
+  }
+  // radix narrowing over the candidates: each pass takes the 12 bits below the highest
+  // bit in which the remaining candidates differ and keeps the bin holding the target
+  uint4* cur = c0;
+  uint4* nxt = a.cand_b[w];
+  uint4* spare = a.cand_c[w];
+  for (int iter = 0; iter < 16 && cnt > 1; ++iter) {
+    if (tid == 0) {
+      s_v0_hi = v_hi(cur[0]);
+      s_v0_lo = v_lo(cur[0]);
+      s_or_hi = 0;
+      s_or_lo = 0;
+    }
+    for (int i = tid; i < kBins; i += kSelThreads) hist[i] = 0;
+    __syncthreads();
+    unsigned long long oh = 0, ol = 0;
+    for (unsigned i = tid; i < cnt; i += kSelThreads) {
+      const uint4 v = cur[i];
+      oh |= v_hi(v) ^ s_v0_hi;
+      ol |= v_lo(v) ^ s_v0_lo;
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      oh |= __shfl_xor_sync(kFull, oh, o);
+      ol |= __shfl_xor_sync(kFull, ol, o);
+    }
+    if ((tid & 31) == 0) {
+      if (oh) atomicOr(&s_or_hi, oh);
+      if (ol) atomicOr(&s_or_lo, ol);
+    }
+    __syncthreads();
+    const unsigned long long dh = s_or_hi, dl = s_or_lo;
+    if (dh == 0 && dl == 0) break;  // all equal (cannot happen for distinct keys)
+    const int top = dh ? 64 + 63 - __clzll((long long)dh) : 63 - __clzll((long long)dl);
+    const int shift = top >= 11 ? top - 11 : 0;
+    for (unsigned i = tid; i < cnt; i += kSelThreads) {
+      const uint4 v = cur[i];
+      atomicAdd(&hist[digit128(v_hi(v), v_lo(v), shift)], 1u);
+    }
+    __syncthreads();
+    long long bl;
+    const int t = find_threshold_bin(hist, Erem, &bl, s_tmp);
+    Erem -= bl;
+    if (tid == 0) s_cnt = 0;
+    __syncthreads();
+    for (unsigned i = tid; i < cnt; i += kSelThreads) {
+      const uint4 v = cur[i];
+      if (digit128(v_hi(v), v_lo(v), shift) == (uint32_t)t) nxt[atomicAdd(&s_cnt, 1u)] = v;
+    }
+    __syncthreads();
+    cnt = s_cnt;
+    uint4* done = cur;  // the collected list (with its slots) is kept for the delete pass
+    cur = nxt;
+    nxt = (done == c0) ? spare : done;
+    __syncthreads();
+  }
+  if (tid == 0) {
+    if (cnt < 1) set_error(a.err, MISAT_ERR_TABLE_FULL);
+    const uint4 v = cur[0];
+    a.theta[2 * w] = v_hi(v);
+    a.theta[2 * w + 1] = v_lo(v);
+  }
+}
+
+namespace {
+__device__ __forceinline__ void delete_slot(Bucket* tab, uint32_t* dmask, uint32_t sl) {
+  const uint32_t b = sl >> 2, s = sl & 3;
+  tab[b].key[s] = kEmpty;
+  tab[b].meta[s] = 0;
+  atomicOr(&dmask[b >> 3], 1u << ((b & 7) * 4 + s));
+}
+}  // namespace
+
+// Delete D and the candidates at or below theta; record them in the deleted-slot masks.
+__global__ void __launch_bounds__(256) k4_evict_delete(EvictArgs a) {
+  const int w = a.only_w ? *a.only_w : blockIdx.y;
+  if (block_error(a.err)) return;
+  if (a.active[w] != 1) return;
+  const unsigned nd = a.n_d[w], n = a.n_cand[w];
+  const uint32_t* dsl = a.dslots[w];
+  const uint4* c0 = a.cand_a[w];
+  const uint32_t* slots = a.slots[w];
+  uint32_t* dmask = a.dmask[w];
+  Bucket* tab = a.desc[w].tab;
+  const unsigned long long tm = a.theta[2 * w], tk = a.theta[2 * w + 1];
+  long long deleted = 0;
+  const unsigned stride = gridDim.x * blockDim.x;
+  for (unsigned i = blockIdx.x * blockDim.x + threadIdx.x; i < nd + n; i += stride) {
+    if (i < nd) {
+      delete_slot(tab, dmask, dsl[i]);
+      ++deleted;
+    } else {
+      const uint4 v = c0[i - nd];
+      if (!le128(v_hi(v), v_lo(v), tm, tk)) continue;
+      delete_slot(tab, dmask, slots[i - nd]);
+      ++deleted;
+    }
+  }
+  const long long tot = block_sum(deleted);
+  if (threadIdx.x == 0 && tot) {
+    atomic_add_i64(&a.size[w], -tot);
+    atomicAdd(a.evicted, (unsigned long long)tot);
+  }
+}
+
+// Refill the holes of every run of full buckets that lost an entry.  The thread of the
+// run's first deleted slot (lowest bucket, then lowest slot) owns the run.
+__global__ void __launch_bounds__(256) k4_evict_shift(EvictArgs a) {
+  const int w = a.only_w ? *a.only_w : blockIdx.y;
+  if (block_error(a.err)) return;
+  if (a.active[w] != 1) return;
+  const unsigned nd = a.n_d[w], n = a.n_cand[w];
+  const uint32_t* dsl = a.dslots[w];
+  const uint4* c0 = a.cand_a[w];
+  const uint32_t* slots = a.slots[w];
+  const uint32_t* full = a.bitmaps[w];
+  const uint32_t* dmask = a.dmask[w];
+  const InstDesc d = a.desc[w];
+  const uint32_t NB = 1u << d.log2nb, mask = NB - 1;
+  const unsigned long long tm = a.theta[2 * w], tk = a.theta[2 * w + 1];
+  const unsigned stride = gridDim.x * blockDim.x;
+  for (unsigned i = blockIdx.x * blockDim.x + threadIdx.x; i < nd + n; i += stride) {
+    uint32_t sl;
+    if (i < nd) {
+      sl = dsl[i];
+    } else {
+      const uint4 v = c0[i - nd];
+      if (!le128(v_hi(v), v_lo(v), tm, tk)) continue;
+      sl = slots[i - nd];
+    }
+    const uint32_t x = sl >> 2, sx = sl & 3;
+    // a hole in the last (not full) bucket of a run needs no refill
+    if (!bit_of(full, x)) continue;
+    // my deletion must be the lowest deleted slot of bucket x (the masks are not modified
+    // by this kernel, unlike the buckets)
+    if ((uint32_t)(__ffs(dmask_of(dmask, x)) - 1) != sx) continue;
+    // run start: walk back over full buckets; no earlier bucket of the run may hold a deletion
+    uint32_t s0 = x, len = 0;
+    bool lead = true;
+    while (bit_of(full, (s0 - 1) & mask) && len < NB) {
+      s0 = (s0 - 1) & mask;
+      ++len;
+      if (dmask_of(dmask, s0)) {
+        lead = false;
+        break;
+      }
+    }
+    if (!lead) continue;
+    // run end: the first bucket after x that was not full
+    uint32_t e = x, rl = 0;
+    while (bit_of(full, e) && rl < NB) {
+      e = (e + 1) & mask;
+      ++rl;
+    }
+    const uint32_t runlen = ((e - s0) & mask);  // buckets s0 .. e-1 are full, e ends the run
+    for (uint32_t ii = 0; ii < runlen; ++ii) {
+      Bucket* X = d.tab + ((s0 + ii) & mask);
+      for (int s = 0; s < 4; ++s) {
+        if (X->key[s] != kEmpty) continue;
+        bool moved = false;
+        for (uint32_t j = ii + 1; j <= runlen && !moved; ++j) {
+          Bucket* Y = d.tab + ((s0 + j) & mask);
+          for (int t = 0; t < 4; ++t) {
+            const unsigned long long k = Y->key[t];
+            if (k == kEmpty) continue;
+            const uint32_t rel = (home_bucket(k, d.log2nb) - s0) & mask;
+            if (rel <= ii) {
+              X->key[s] = k;
+              X->meta[s] = Y->meta[t];
+              Y->key[t] = kEmpty;
+              Y->meta[t] = 0;
+              moved = true;
+              break;
+            }
+          }
+        }
+        if (!moved) break;  // no later entry of the run can move into this bucket
+      }
+    }
+  }
+}
+
+void launch_evict(const EvictArgs& a, int chunks_per_inst, cudaStream_t st) {
+  const int W = a.only_w ? 1 : a.W;
+  k4_evict_estimate<<<W, kSelThreads, 0, st>>>(a);
+  k4_evict_collect<<<dim3(chunks_per_inst, W), 256, 0, st>>>(a);
+  k4_evict_select<<<W, kSelThreads, 0, st>>>(a);
+  k4_evict_delete<<<dim3(chunks_per_inst, W), 256, 0, st>>>(a);
+  k4_evict_shift<<<dim3(chunks_per_inst, W), 256, 0, st>>>(a);
+}
+
+// Compaction of one instance table: delete entries with meta == 0 (marked) or
+// (meta, key) <= theta, then restore the probing invariant inside each run of full
+// buckets.  A run starts after a bucket that was not full before the pass and ends at
+// the next such bucket; runs are disjoint, so each is owned by one thread.
+__global__ void __launch_bounds__(256) k4_evict_compact(EvictArgs a) {
+  const int w = a.only_w ? *a.only_w : blockIdx.y;
+  if (block_error(a.err)) return;
+  // active: 0 nothing to do (bitmap not built), 1 theta eviction, 2 marked entries only
+  const int act = a.active[w];
+  if (act == 0) return;
+  const InstDesc d = a.desc[w];
+  const uint32_t NB = 1u << d.log2nb;
+  const uint32_t mask = NB - 1;
+  const uint32_t* bitmap = a.bitmaps[w];
+  const unsigned long long tm = a.theta[2 * w], tk = a.theta[2 * w + 1];
+  const uint32_t nthreads = gridDim.x * blockDim.x;
+  const uint32_t tid = blockIdx.x * blockDim.x + threadIdx.x;
+  const uint32_t per = (NB + nthreads - 1) / nthreads;
+  const uint32_t lo = tid * per;
+  const uint32_t hi = lo + per < NB ? lo + per : NB;
+  long long deleted = 0;
+  auto is_full = [&](uint32_t b) { return (bitmap[b >> 5] >> (b & 31)) & 1u; };
+  for (uint32_t x0 = lo; x0 < hi; ++x0) {
+    if (is_full((x0 - 1) & mask)) continue;  // not a run start
+    // run [x0, e]: e = first bucket at or after x0 that was not full
+    uint32_t e = x0, len = 0;
+    while (is_full(e) && len < NB) {
+      e = (e + 1) & mask;
+      ++len;
+    }
+    // delete
+    for (uint32_t i = 0; i <= len; ++i) {
+      Bucket* B = d.tab + ((x0 + i) & mask);
+#pragma unroll
+      for (int s = 0; s < 4; ++s) {
+        const unsigned long long k = B->key[s];
+        if (k == kEmpty) continue;
+        const unsigned long long m = B->meta[s];
+        if (m == 0 || (act == 1 && le128(m, k, tm, tk))) {
+          B->key[s] = kEmpty;
+          B->meta[s] = 0;
+          ++deleted;
+        }
+      }
+    }
+    if (len == 0) continue;
+    // backward shift: fill free slots of bucket x from the first later entry of the run
+    // whose home lies in [x0, x]
+    for (uint32_t i = 0; i < len; ++i) {
+      Bucket* X = d.tab + ((x0 + i) & mask);
+      for (int s = 0; s < 4; ++s) {
+        if (X->key[s] != kEmpty) continue;
+        bool moved = false;
+        for (uint32_t j = i + 1; j <= len && !moved; ++j) {
+          Bucket* Y = d.tab + ((x0 + j) & mask);
+          for (int t = 0; t < 4; ++t) {
+            const unsigned long long k = Y->key[t];
+            if (k == kEmpty) continue;
+            const uint32_t rel = (home_bucket(k, d.log2nb) - x0) & mask;
+            if (rel <= i) {
+              X->key[s] = k;
+              X->meta[s] = Y->meta[t];
+              Y->key[t] = kEmpty;
+              Y->meta[t] = 0;
+              moved = true;
+              break;
+            }
+          }
+        }
+        if (!moved) break;  // no later entry can move into x
+      }
+    }
+  }
+  const long long tot = block_sum(deleted);
+  if (threadIdx.x == 0 && tot) {
+    atomic_add_i64(&a.size[w], -tot);
+    atomicAdd(a.evicted, (unsigned long long)tot);
+  }
+}
+
+void launch_compact_marked(const EvictArgs& a, cudaStream_t st) {
+  k4_evict_compact<<<dim3(8, 1), 256, 0, st>>>(a);
+}
+
+}  // namespace misat

@@ -89,8 +89,11 @@ __global__ void __launch_bounds__(256) k1_block_hash(HashArgs a) {
     const int64_t t0 = a.tok_off[r];
     const int64_t t1 = a.tok_off[r + 1];
     const int32_t nb = (int32_t)((t1 - t0) >> 4);
-    if (nb <= 0) continue;
     const int64_t kb = t0 >> 4;
+    // key slots kb .. kb+nb-1 belong to r; at most one slot before the next request's
+    // first slot floor(t1/16) belongs to nobody (the owner map marks it -1)
+    if (lane == 0 && a.owner && kb + nb < (t1 >> 4) && kb + nb < a.keys_cap) a.owner[kb + nb] = -1;
+    if (nb <= 0) continue;
     const int64_t q0 = t0 >> 2;
     const int off = (int)(t0 & 3);
     uint64_t carry = a.seed;
@@ -110,7 +113,9 @@ __global__ void __launch_bounds__(256) k1_block_hash(HashArgs a) {
       for (int i = 0; i < 4; ++i) vn[i] = more ? load_tok4(tok4, nbase + 32 * i + lane, n_int4) : make_int4(0, 0, 0, 0);
       if (more && off != 0 && lane == 0) exn = load_tok4(tok4, nbase + 128, n_int4);
 
-      uint64_t cmine = 0;
+      // pre-mix XOR of block 8i + lane/4 after sub-iteration i (same in its 4 lanes); lane
+      // 4m + i' keeps the one of sub-iteration i' = lane % 4, i.e. block 8(lane%4) + lane/4
+      uint64_t pkeep = 0;
 #pragma unroll
       for (int i = 0; i < 4; ++i) {
         int4 t = v[i];
@@ -126,10 +131,11 @@ __global__ void __launch_bounds__(256) k1_block_hash(HashArgs a) {
         uint64_t p = mix64(xa + addA) ^ mix64(xb + addB);
         p ^= __shfl_xor_sync(kFull, p, 1);
         p ^= __shfl_xor_sync(kFull, p, 2);
-        const uint64_t cb = mix64(p);
-        const uint64_t got = __shfl_sync(kFull, cb, 4 * (lane & 7));
-        if ((lane >> 3) == i) cmine = got;
+        if (q == i) pkeep = p;
       }
+      // one finishing mix per lane, then block j moves to lane j (it sits on lane 4(j%8) + j/8)
+      const uint64_t cown = mix64(pkeep);
+      const uint64_t cmine = __shfl_sync(kFull, cown, 4 * (lane & 7) + (lane >> 3));
       const int cnt = min(32, nb - 32 * c);
       uint64_t s = lane < cnt ? cmine : 0;
       {
@@ -148,7 +154,10 @@ __global__ void __launch_bounds__(256) k1_block_hash(HashArgs a) {
       uint64_t key = mix64(av ^ (uint64_t)(32 * c + lane + 1));
       key += key < 2 ? 2 : 0;
       const int64_t dst = kb + 32ll * c + lane;
-      if (lane < cnt && dst < a.keys_cap) a.keys[dst] = key;
+      if (lane < cnt && dst < a.keys_cap) {
+        a.keys[dst] = key;
+        if (a.owner) a.owner[dst] = r;
+      }
       carry = __shfl_sync(kFull, av, 31);
 #pragma unroll
       for (int i = 0; i < 4; ++i) v[i] = vn[i];

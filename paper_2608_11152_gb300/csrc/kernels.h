@@ -16,6 +16,7 @@ struct HashArgs {
   int32_t n;
   uint64_t seed;
   uint64_t* keys;       // key of (r, j) at floor(tok_off[r]/16) + j
+  int32_t* owner;       // request owning each key slot, -1 for a slot of no request (may be NULL)
   int64_t keys_cap;
   unsigned* work;       // zeroed before the launch
   const int32_t* err;
@@ -114,6 +115,8 @@ struct CapsArgs {
 };
 void launch_caps(const CapsArgs& a, cudaStream_t st);
 
+constexpr int kAdmitTile = 128;  // requests per admission tile
+
 struct RoundArgs {
   int32_t n;
   int32_t W;
@@ -147,6 +150,7 @@ struct InsertArgs {
   const InstDesc* desc;
   int32_t n;
   int64_t n_slots;             // key slots to scan: floor(n_tokens / 16)
+  const int32_t* owner;        // request of each key slot (-1: none), written by the hash kernel
   const int32_t* nb;
   const int64_t* kbase;
   const int32_t* inst;         // instance per request (-1: skip)
@@ -193,16 +197,24 @@ struct EvictArgs {
   int32_t W;
   const int32_t* only_w;       // if not NULL: evict only instance *only_w
   long long* size;             // [W]
-  uint64_t cur_seq;
   uint32_t* const* bitmaps;    // [W] per instance fullness bitmap (NB/32 words)
-  uint4* const* cand_a;        // [W] candidate lists (meta, key) as uint4
-  uint4* const* cand_b;
+  uint4* const* cand_a;        // [W] candidate lists (meta, key) as uint4: the collected list
+  uint4* const* cand_b;        //     and two work lists of the radix narrowing
+  uint4* const* cand_c;
+  uint32_t* const* slots;      // [W] slot (bucket*4+s) of each entry of cand_a
+  uint32_t* const* dslots;     // [W] slots certainly evicted (meta below the bracket)
+  uint32_t* const* dmask;      // [W] deleted-slot mask, 4 bits per bucket (NB/8 words)
+  unsigned* n_cand;            // [W] entries in cand_a
+  unsigned* n_d;               // [W] entries in dslots
+  unsigned long long* thr_lo;  // [W] meta bracket of the E-th smallest
+  unsigned long long* thr_hi;  // [W]
   unsigned long long* theta;   // [W*2] (meta, key)
-  int32_t* active;             // [W] 1: delete entries <= theta
+  int32_t* active;             // [W] 1: delete entries <= theta, 2: marked entries only
   unsigned long long* evicted;
   int32_t* err;
 };
 void launch_evict(const EvictArgs& a, int chunks_per_inst, cudaStream_t st);
+void launch_compact_marked(const EvictArgs& a, cudaStream_t st);
 
 struct MarkArgs {
   InstDesc desc;

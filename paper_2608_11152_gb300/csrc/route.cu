@@ -7,7 +7,7 @@ namespace misat {
 
 namespace {
 constexpr unsigned kFull = 0xffffffffu;
-constexpr int kTile = 1024;  // requests per admission tile
+constexpr int kTile = kAdmitTile;  // requests per admission tile
 }  // namespace
 
 // ---------------------------------------------------------------------------
@@ -299,18 +299,40 @@ __global__ void __launch_bounds__(256) k4_tile_count(RoundArgs a) {
   for (int k = threadIdx.x; k < nb; k += blockDim.x) out[k] = s_cnt[k];
 }
 
-__global__ void __launch_bounds__(256) k4_tile_scan(RoundArgs a) {
+// Exclusive scan of the tile counts over the tiles, per (instance, class) column: a CTA of
+// 32 warps owns 32 columns (lanes); warp k sums a stripe of tiles, the stripe sums are
+// scanned across warps, then each warp rewrites its stripe with running prefixes.
+__global__ void __launch_bounds__(1024) k4_tile_scan(RoundArgs a) {
+  __shared__ int32_t s_sum[32][33];
   if (block_error(a.err)) return;
   const int nb = 3 * a.W;
-  const int k = blockIdx.x * blockDim.x + threadIdx.x;
-  if (k >= nb) return;
-  int32_t acc = 0;
-  for (int t = 0; t < a.n_tiles; ++t) {
-    int32_t* p = a.tile_counts + (int64_t)t * nb + k;
-    const int32_t v = *p;
-    *p = acc;
-    acc += v;
+  const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+  const int col = blockIdx.x * 32 + lane;
+  const int T = a.n_tiles;
+  const int per = (T + 31) / 32;
+  const int t0 = wid * per, t1 = min(T, t0 + per);
+  int32_t sum = 0;
+  if (col < nb)
+    for (int t = t0; t < t1; ++t) sum += a.tile_counts[(int64_t)t * nb + col];
+  s_sum[wid][lane] = sum;
+  __syncthreads();
+  if (wid == 0) {
+    int32_t acc = 0;
+    for (int k = 0; k < 32; ++k) {
+      const int32_t v = s_sum[k][lane];
+      s_sum[k][lane] = acc;
+      acc += v;
+    }
   }
+  __syncthreads();
+  int32_t acc = s_sum[wid][lane];
+  if (col < nb)
+    for (int t = t0; t < t1; ++t) {
+      int32_t* p = a.tile_counts + (int64_t)t * nb + col;
+      const int32_t v = *p;
+      *p = acc;
+      acc += v;
+    }
 }
 
 __global__ void __launch_bounds__(32) k4_admit(RoundArgs a) {
@@ -388,8 +410,8 @@ void launch_round(const RoundArgs& a, int num_sms, cudaStream_t st) {
   if (score_grid < 1) score_grid = 1;
   k3_score<<<score_grid, 256, score_smem, st>>>(a);
   const size_t cnt_smem = (size_t)a.W * 3 * sizeof(int32_t);
-  k4_tile_count<<<a.n_tiles, 256, cnt_smem, st>>>(a);
-  k4_tile_scan<<<(3 * a.W + 255) / 256, 256, 0, st>>>(a);
+  k4_tile_count<<<a.n_tiles, 128, cnt_smem, st>>>(a);
+  k4_tile_scan<<<(3 * a.W + 31) / 32, 1024, 0, st>>>(a);
   k4_admit<<<a.n_tiles, 32, cnt_smem, st>>>(a);
   k4_round_end<<<1, 1024, 0, st>>>(a);
 }

@@ -445,10 +445,11 @@ def _concat_batches(batches, rng):
                  tokens=np.ascontiguousarray(np.concatenate([prompts[i] for i in order]), dtype=np.int32))
 
 
-def config5(n=65536, fill=0.95, seed=20260005, n_warm=1) -> Scenario:
-    """Throughput stress: 128 x 262,144 blocks filled to `fill`, batches of n requests 40/30/30."""
+def config5(n=65536, fill=0.95, seed=20260005, n_warm=1, instances=128, cap=262144) -> Scenario:
+    """Throughput stress: 128 x 262,144 blocks filled to `fill`, batches of n requests 40/30/30
+    (fewer instances only for small profiling captures)."""
     spec = MixSpec(rho_ppm=(400000, 300000, 300000), agent_sessions=max(1, round(0.3 * n / 4.8)), **MIX2)
-    return _stream_scenario(f"cfg5_stress_128x262144_n{n}_fill{int(fill * 100)}", seed, 128, 262144, n,
+    return _stream_scenario(f"cfg5_stress_{instances}x{cap}_n{n}_fill{int(fill * 100)}", seed, instances, cap, n,
                             n_warm, spec, fill=fill)
 
 
