@@ -357,10 +357,10 @@ EvictArgs evict_args(misat_ctx* c, unsigned long long* evicted_counter) {
 
 int evict_all(misat_ctx* c, unsigned long long* evicted_counter) {
   const EvictArgs ev = evict_args(c, evicted_counter);
-  // streaming CTAs per instance: about 16 buckets per thread, at most 64 CTAs of 256
+  // streaming CTAs per instance: about 4 buckets per thread, at most 256 CTAs of 256
   uint32_t maxlg = 1;
   for (auto& d : c->h_desc) maxlg = std::max(maxlg, d.log2nb);
-  const int chunks = (int)std::min<uint64_t>(64, std::max<uint64_t>(1, ((uint64_t)1 << maxlg) / (16 * 256)));
+  const int chunks = (int)std::min<uint64_t>(256, std::max<uint64_t>(1, ((uint64_t)1 << maxlg) / (4 * 256)));
   launch_evict(ev, chunks, c->stream);
   CK(cudaGetLastError());
   return MISAT_OK;
@@ -467,6 +467,7 @@ int misat_create(const misat_config* cfg, void* cuda_stream, misat_ctx** out) {
       (rc = dalloc_n(c, &c->rq.leader, NB)) || (rc = dalloc_n(c, &c->rq.status, NB)) ||
       (rc = dalloc_n(c, &c->rq.choice, NB)) || (rc = dalloc_n(c, &c->rq.last_reason, NB)) ||
       (rc = dalloc_n(c, &c->rq.inst, NB)) || (rc = dalloc_n(c, &c->rq.reason, NB)) ||
+      (rc = dalloc_n(c, &c->rq.hmax, NB)) ||
       (rc = dalloc_n(c, &c->ia.K_w, Ws)) || (rc = dalloc_n(c, &c->ia.K_wb, 3 * Ws)) ||
       (rc = dalloc_n(c, &c->ia.N_wb, 3 * Ws)) || (rc = dalloc_n(c, &c->ia.kbar_w, Ws)) ||
       (rc = dalloc_n(c, &c->ia.tot, Ws)) || (rc = dalloc_n(c, &c->ia.gh, Ws)) || (rc = dalloc_n(c, &c->ia.ch, 3 * Ws)) ||
@@ -725,6 +726,7 @@ int misat_commit(misat_ctx* c) {
   if (n > 0) {
     InsertArgs ia{};
     ia.desc = c->d_desc;
+    ia.n_inst = c->W;
     ia.n = n;
     ia.n_slots = c->last_ntok / 16;
     ia.nb = c->rq.nb;
@@ -908,6 +910,7 @@ int misat_load_chains(misat_ctx* c, int32_t n_chains, const int64_t* tok_off, co
   launch_block_hash(ha, c->num_sms, st);
   InsertArgs ia{};
   ia.desc = c->d_desc;
+  ia.n_inst = c->W;
   ia.n = n_chains;
   ia.n_slots = ntok / 16;
   ia.nb = c->rq.nb;

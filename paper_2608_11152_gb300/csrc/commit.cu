@@ -62,48 +62,66 @@ __device__ int table_insert(const InstDesc& d, uint64_t key, uint64_t meta) {
 // Insert: one thread per key slot of the batch; the owning request comes from the owner
 // map the hash kernel wrote next to the keys.
 __global__ void __launch_bounds__(256) k4_insert(InsertArgs a) {
+  __shared__ unsigned s_new[kMaxW];  // new keys per instance, flushed once per CTA
   if (block_error(a.err)) return;
+  for (int i = threadIdx.x; i < a.n_inst; i += blockDim.x) s_new[i] = 0;
+  __syncthreads();
+  constexpr int kPer = 4;  // independent key slots per thread per iteration
   const int lane = threadIdx.x & 31;
   unsigned long long nnew = 0;
-  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
-  const int64_t start = (int64_t)blockIdx.x * blockDim.x + (threadIdx.x & ~31);
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x * kPer;
+  // a warp covers 32*kPer consecutive slots per iteration; lane handles base + lane + 32 k
+  const int64_t start = ((int64_t)blockIdx.x * blockDim.x + (threadIdx.x & ~31)) * kPer;
   for (int64_t base = start; base < a.n_slots; base += stride) {
-    const int64_t q = base + lane;
-    int w = -1, isnew = 0;
-    if (q < a.n_slots) {
-      const int r = a.owner[q];
-      if (r >= 0) {
-        w = a.inst[r];
-        const int64_t j = q - a.kbase[r];
-        if (w >= 0 && a.max_blocks && j >= a.max_blocks[r]) w = -1;
-        if (w >= 0) {
-          const uint64_t meta = a.meta_seq ? pack_meta(a.meta_seq[r], a.meta_arr[r], (uint64_t)j)
-                                           : pack_meta(a.seq, (uint64_t)r, (uint64_t)j);
-          const int res = table_insert(a.desc[w], a.keys[q], meta);
-          if (res < 0) {
-            set_error(a.err, MISAT_ERR_TABLE_FULL);
-          } else {
-            isnew = res;
-          }
-        }
+    int r[kPer], w[kPer];
+#pragma unroll
+    for (int k = 0; k < kPer; ++k) {
+      const int64_t q = base + lane + 32 * k;
+      r[k] = q < a.n_slots ? a.owner[q] : -1;
+    }
+#pragma unroll
+    for (int k = 0; k < kPer; ++k) {
+      w[k] = -1;
+      if (r[k] >= 0) {
+        w[k] = a.inst[r[k]];
+        const int64_t j = base + lane + 32 * k - a.kbase[r[k]];
+        if (w[k] >= 0 && a.max_blocks && j >= a.max_blocks[r[k]]) w[k] = -1;
       }
     }
-    // per-instance size increments, aggregated over the warp's lanes with the same instance
-    const unsigned peers = __match_any_sync(kFull, isnew ? w : -1 - lane);
-    const unsigned newmask = __ballot_sync(kFull, isnew);
-    if (isnew && lane == __ffs(peers) - 1) {
-      const int c = __popc(peers & newmask);
-      atomic_add_i64(&a.size[w], (long long)c);
-      nnew += c;
+#pragma unroll
+    for (int k = 0; k < kPer; ++k) {
+      const int64_t q = base + lane + 32 * k;
+      int isnew = 0;
+      if (w[k] >= 0) {
+        const int64_t j = q - a.kbase[r[k]];
+        const uint64_t meta = a.meta_seq ? pack_meta(a.meta_seq[r[k]], a.meta_arr[r[k]], (uint64_t)j)
+                                         : pack_meta(a.seq, (uint64_t)r[k], (uint64_t)j);
+        const int res = table_insert(a.desc[w[k]], a.keys[q], meta);
+        if (res < 0)
+          set_error(a.err, MISAT_ERR_TABLE_FULL);
+        else
+          isnew = res;
+      }
+      // per-instance size increments, aggregated over the warp's lanes with the same instance
+      const unsigned peers = __match_any_sync(kFull, isnew ? w[k] : -1 - lane);
+      const unsigned newmask = __ballot_sync(kFull, isnew);
+      if (isnew && lane == __ffs(peers) - 1) {
+        const int c = __popc(peers & newmask);
+        atomicAdd(&s_new[w[k]], (unsigned)c);
+        nnew += c;
+      }
     }
   }
   const long long tot = block_sum((long long)nnew);
   if (threadIdx.x == 0 && tot) atomicAdd(a.new_keys, (unsigned long long)tot);
+  __syncthreads();
+  for (int i = threadIdx.x; i < a.n_inst; i += blockDim.x)
+    if (s_new[i]) atomic_add_i64(&a.size[i], (long long)s_new[i]);
 }
 
 void launch_insert(const InsertArgs& a, int num_sms, cudaStream_t st) {
   if (a.n_slots <= 0 || a.n <= 0) return;
-  int64_t blocks = (a.n_slots + 255) / 256;
+  int64_t blocks = (a.n_slots + 1023) / 1024;
   int grid = (int)(blocks < (int64_t)num_sms * 8 ? blocks : (int64_t)num_sms * 8);
   k4_insert<<<grid, 256, 0, st>>>(a);
 }

@@ -95,7 +95,11 @@ __device__ __forceinline__ uint32_t dmask_of(const uint32_t* dm, uint32_t b) { r
 
 
 __global__ void __launch_bounds__(kSelThreads) k4_evict_estimate(EvictArgs a) {
-  __shared__ unsigned long long s_buf[kSamples];
+  constexpr int kEst = 2048;  // 4 slots of up to 512 evenly spaced buckets
+  __shared__ unsigned long long s_smp[kEst];
+  __shared__ uint32_t hist[kBins];
+  __shared__ long long s_tmp[32];
+  __shared__ unsigned long long s_min, s_max;
   __shared__ unsigned s_m;
   const int w = a.only_w ? *a.only_w : blockIdx.x;
   if (block_error(a.err)) return;
@@ -110,53 +114,78 @@ __global__ void __launch_bounds__(kSelThreads) k4_evict_estimate(EvictArgs a) {
   if (E <= 0) return;
   const InstDesc d = a.desc[w];
   const uint32_t NB = 1u << d.log2nb;
-  if (tid == 0) s_m = 0;
+  if (tid == 0) {
+    s_m = 0;
+    s_min = ~0ull;
+    s_max = 0;
+  }
+  for (int i = tid; i < kBins; i += kSelThreads) hist[i] = 0;
   __syncthreads();
+  // samples: the metas of up to 512 evenly spaced buckets
+  unsigned long long mn = ~0ull, mx = 0;
   {
-    const uint32_t nsb = NB < 1024u ? NB : 1024u;
+    const uint32_t nsb = NB < 512u ? NB : 512u;
     unsigned occ = 0;
-    for (int s = 0; s < 4; ++s) s_buf[4 * tid + s] = ~0ull;
     if ((uint32_t)tid < nsb) {
       const uint32_t b = (uint32_t)(((uint64_t)tid * NB) / nsb);
       const ulonglong2* mp = reinterpret_cast<const ulonglong2*>(d.tab[b].meta);
       const ulonglong2 m01 = __ldcg(mp), m23 = __ldcg(mp + 1);
       const unsigned long long m[4] = {m01.x, m01.y, m23.x, m23.y};
-      for (int s = 0; s < 4; ++s)
+      for (int s = 0; s < 4; ++s) {
+        s_smp[4 * tid + s] = m[s];
         if (m[s]) {
-          s_buf[4 * tid + s] = m[s];
           ++occ;
-        }
-    }
-    if (occ) atomicAdd(&s_m, occ);
-  }
-  __syncthreads();
-  for (int k = 2; k <= kSamples; k <<= 1) {
-    for (int j = k >> 1; j > 0; j >>= 1) {
-      for (int i = tid; i < kSamples; i += kSelThreads) {
-        const int ixj = i ^ j;
-        if (ixj > i) {
-          const unsigned long long x = s_buf[i], y = s_buf[ixj];
-          if ((x > y) == ((i & k) == 0)) {
-            s_buf[i] = y;
-            s_buf[ixj] = x;
-          }
+          mn = m[s] < mn ? m[s] : mn;
+          mx = m[s] > mx ? m[s] : mx;
         }
       }
-      __syncthreads();
+    } else if (tid < kEst / 4) {
+      for (int s = 0; s < 4; ++s) s_smp[4 * tid + s] = 0;
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      const unsigned long long a1 = __shfl_xor_sync(kFull, mn, o), a2 = __shfl_xor_sync(kFull, mx, o);
+      mn = a1 < mn ? a1 : mn;
+      mx = a2 > mx ? a2 : mx;
+      occ += __shfl_xor_sync(kFull, occ, o);
+    }
+    if ((tid & 31) == 0 && occ) {
+      atomicAdd(&s_m, occ);
+      atomicMin(&s_min, mn);
+      atomicMax(&s_max, mx);
     }
   }
-  if (tid == 0) {
-    // the E-th smallest sits near sample index p = E m / size; bracket it by ~3 standard
-    // deviations of the sample count plus a constant on both sides
-    const unsigned m = s_m;
-    unsigned long long lo = 0, hi = ~0ull;
-    if (m > 0 && size > 0) {
-      const double p = (double)E * (double)m / (double)size;
-      const double margin = 3.0 * sqrt(p + 1.0) + 16.0;
-      const double il = p - margin, ih = p + margin;
-      if (il >= 0.0) lo = s_buf[(int)il];
-      if (ih < (double)m) hi = s_buf[(int)ih];
+  __syncthreads();
+  const unsigned m = s_m;
+  unsigned long long lo = 0, hi = ~0ull;
+  if (m > 0 && size > 0) {
+    // histogram of the samples over [min, max], 4096 equal bins
+    const unsigned long long smin = s_min;
+    const unsigned __int128 range = (unsigned __int128)(s_max - s_min) + 1;
+    auto bin_of = [&](unsigned long long x) {
+      return (uint32_t)((((unsigned __int128)(x - smin)) << 12) / range);
+    };
+    for (int i = tid; i < kEst; i += kSelThreads) {
+      const unsigned long long x = s_smp[i];
+      if (x) atomicAdd(&hist[bin_of(x)], 1u);
     }
+    __syncthreads();
+    // the E-th smallest sits near sample rank p = E m / size; bracket it by ~3 standard
+    // deviations of the sample count plus a constant on both sides
+    const double p = (double)E * (double)m / (double)size;
+    const double margin = 3.0 * sqrt(p + 1.0) + 16.0;
+    const long long rl = (long long)(p - margin), rh = (long long)(p + margin) + 1;
+    long long below;
+    const int bl = rl >= 1 ? find_threshold_bin(hist, rl, &below, s_tmp) : -1;
+    const int bh = rh <= (long long)m ? find_threshold_bin(hist, rh, &below, s_tmp) : -1;
+    // bin edges: every sample of bin b lies in [edge(b), edge(b + 1) - 1]
+    auto edge = [&](int b) {
+      return smin + (unsigned long long)((range * (unsigned)b + 4095) >> 12);
+    };
+    if (bl >= 0) lo = edge(bl);
+    if (bh >= 0) hi = edge(bh + 1) - 1;
+  }
+  if (tid == 0) {
     a.thr_lo[w] = lo;
     a.thr_hi[w] = hi;
   }
@@ -164,6 +193,7 @@ __global__ void __launch_bounds__(kSelThreads) k4_evict_estimate(EvictArgs a) {
 
 // Streaming pass over the instance's metas (grid.x CTAs per instance).
 __global__ void __launch_bounds__(256) k4_evict_collect(EvictArgs a) {
+  __shared__ unsigned s_wd[8], s_wu[8], s_bd, s_bu;
   const int w = a.only_w ? *a.only_w : blockIdx.y;
   if (block_error(a.err)) return;
   if (a.active[w] != 1) return;
@@ -197,7 +227,7 @@ __global__ void __launch_bounds__(256) k4_evict_collect(EvictArgs a) {
       if (m[s] < lo) ++nd;
       else if (m[s] <= hi) ++nu;
     }
-    // warp-aggregated reservations in both lists
+    // CTA-wide reservation in both lists: warp scans, then one atomic pair per CTA
     int id = nd, iu = nu;
 #pragma unroll
     for (int o = 1; o < 32; o <<= 1) {
@@ -207,14 +237,28 @@ __global__ void __launch_bounds__(256) k4_evict_collect(EvictArgs a) {
         iu += vu;
       }
     }
-    const int td = __shfl_sync(kFull, id, 31), tu = __shfl_sync(kFull, iu, 31);
-    unsigned bd = 0, bu = 0;
+    const int wid = threadIdx.x >> 5;
     if (lane == 31) {
-      if (td) bd = atomicAdd(&a.n_d[w], (unsigned)td);
-      if (tu) bu = atomicAdd(&a.n_cand[w], (unsigned)tu);
+      s_wd[wid] = id;
+      s_wu[wid] = iu;
     }
-    bd = __shfl_sync(kFull, bd, 31) + (unsigned)(id - nd);
-    bu = __shfl_sync(kFull, bu, 31) + (unsigned)(iu - nu);
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      unsigned td = 0, tu = 0;
+      for (int k = 0; k < (int)(blockDim.x >> 5); ++k) {
+        const unsigned xd = s_wd[k], xu = s_wu[k];
+        s_wd[k] = td;
+        s_wu[k] = tu;
+        td += xd;
+        tu += xu;
+      }
+      s_bd = td ? atomicAdd(&a.n_d[w], td) : 0;
+      s_bu = tu ? atomicAdd(&a.n_cand[w], tu) : 0;
+    }
+    __syncthreads();
+    unsigned bd = s_bd + s_wd[wid] + (unsigned)(id - nd);
+    unsigned bu = s_bu + s_wu[wid] + (unsigned)(iu - nu);
+    __syncthreads();  // the shared offsets are rewritten by the next iteration
 #pragma unroll
     for (int s = 0; s < 4; ++s) {
       if (!m[s]) continue;

@@ -38,6 +38,7 @@ struct ReqArrays {
   uint8_t* last_reason; // hold reason if it stays unresolved
   int32_t* inst;        // decision (internal copy)
   uint8_t* reason;      // reason (internal copy)
+  int32_t* hmax;        // max over instances of H_rw (set by the score kernel for leaders)
 };
 
 // ---- per-instance round state ----
@@ -159,6 +160,7 @@ struct InsertArgs {
   const uint32_t* meta_arr;    // per request arrival when meta_seq != NULL
   const int32_t* max_blocks;   // per request insert limit (NULL: all)
   uint64_t seq;
+  int32_t n_inst;              // W
   long long* size;             // [W] live entries
   unsigned long long* new_keys;
   int32_t* err;

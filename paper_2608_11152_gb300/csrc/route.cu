@@ -201,18 +201,40 @@ __global__ void __launch_bounds__(256) k3_score(RoundArgs a) {
   const int lane = threadIdx.x & 31;
   const int warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
   const int nwarps = (gridDim.x * blockDim.x) >> 5;
+  // the next request's fields and first H values are loaded while this one is reduced
+  constexpr int kPre = 4;  // H values per lane prefetched (instances lane + 32 i, i < kPre)
+  struct Next {
+    uint8_t st, b, sst;
+    int sinst;
+    int32_t L;
+    uint16_t h[kPre];
+  };
+  auto fetch = [&](int rr, Next& x) {
+    x.st = rr < a.n ? a.rq.status[rr] : kStResolved;
+    if (x.st != kStUnresolved) return;
+    x.b = a.rq.cls[rr];
+    x.sst = a.rq.sst[rr];
+    x.sinst = a.rq.sinst[rr];
+    x.L = a.rq.L[rr];
+    const uint16_t* Hr = a.H + (int64_t)rr * a.W;
+#pragma unroll
+    for (int i = 0; i < kPre; ++i) x.h[i] = (lane + 32 * i < a.W) ? Hr[lane + 32 * i] : 0;
+  };
+  Next nx;
+  fetch(warp, nx);
   for (int r = warp; r < a.n; r += nwarps) {
-    if (a.rq.status[r] != kStUnresolved) continue;
-    const int b = a.rq.cls[r];
-    const uint8_t sst = a.rq.sst[r];
-    const int pw = sst == kSessProtected ? a.rq.sinst[r] : -1;
-    const int64_t Lr = a.rq.L[r];
+    const Next cur = nx;
+    fetch(r + nwarps, nx);
+    if (cur.st != kStUnresolved) continue;
+    const int b = cur.b;
+    const uint8_t sst = cur.sst;
+    const int pw = sst == kSessProtected ? cur.sinst : -1;
+    const int64_t Lr = cur.L;
     const uint16_t* Hr = a.H + (int64_t)r * a.W;
     int64_t best_c = INT64_MAX;
     int best_w = INT32_MAX;
     int hmax = -1, whit = INT32_MAX;
-    for (int w = lane; w < a.W; w += 32) {
-      const int h = Hr[w];
+    auto visit = [&](int w, int h) {
       const bool elig = (w == pw) || (s_gh[w] > 0 && s_ch[w * 3 + b] > 0);
       if (elig) {
         const int64_t cost = s_bk[w] + (Lr - 16 * (int64_t)h) * s_tc[w];
@@ -225,7 +247,11 @@ __global__ void __launch_bounds__(256) k3_score(RoundArgs a) {
         hmax = h;
         whit = w;
       }
-    }
+    };
+#pragma unroll
+    for (int i = 0; i < kPre; ++i)
+      if (lane + 32 * i < a.W) visit(lane + 32 * i, cur.h[i]);
+    for (int w = lane + 32 * kPre; w < a.W; w += 32) visit(w, Hr[w]);
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) {
       const int64_t oc = __shfl_xor_sync(kFull, best_c, o);
@@ -242,6 +268,7 @@ __global__ void __launch_bounds__(256) k3_score(RoundArgs a) {
       }
     }
     if (lane == 0) {
+      a.rq.hmax[r] = hmax < 0 ? 0 : hmax;
       int choice = -1;
       uint8_t reason = 0;
       if (best_w == INT32_MAX) {
@@ -445,6 +472,8 @@ __global__ void __launch_bounds__(256) k4_finalize(FinalizeArgs a) {
     int hb = 0;
     if (w >= 0) {
       hb = Hr[w];
+    } else if (stv != kStFollower) {
+      hb = a.rq.hmax[r];  // every leader was scored at least once
     } else {
       for (int x = 0; x < a.W; ++x) hb = Hr[x] > hb ? Hr[x] : hb;
     }
