@@ -48,9 +48,11 @@ CLOCK_QUERY = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.ac
 
 
 def kernels_per_step(rounds):
-    """Kernels one route+commit launches: route = prologue 2 + hash + caps + probe 2 + 5 per round +
-    finalize; commit = insert + sessions + eviction select + compaction."""
-    return 7 + 5 * rounds + 4
+    """Kernels one route+commit launches.  Route: prologue, leaders, hash, caps, probe first,
+    probe search, 5 per selection round (score, tile count, tile scan, admit, round end),
+    finalize.  Commit: insert work list, insert, sessions, and the five eviction kernels
+    (estimate, collect, select, delete, shift)."""
+    return 7 + 5 * rounds + 8
 
 
 def parse_args():
@@ -64,6 +66,8 @@ def parse_args():
     ap.add_argument("--e2e-steps", type=int, default=5)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--instances", type=int, default=128, help="fewer only for small profiling captures")
+    ap.add_argument("--prefix-index", default="global", choices=["global", "per-instance"],
+                    help="block-0 probe through the global key->instance-mask index or per instance table")
     return ap.parse_args()
 
 
@@ -86,7 +90,7 @@ def workload_config(args, sc):
                         f"fill {int(round(args.fill * 100))}%, {args.n} requests/batch 40/30/30 RLVR/RLHF/agentic",
             "instances": int(sc.W), "cap_blocks": int(sc.cap_blocks[0]), "fill": args.fill,
             "batch_requests": int(args.n), "batch_tokens": int(sc.batch.n_tokens), "block_tokens": 16,
-            "rounds": int(sc.rounds), "mode": "MISA-T",
+            "rounds": int(sc.rounds), "mode": "MISA-T", "prefix_index": args.prefix_index,
             "l2": "inputs larger than L2 (tokens %.2f GB, tables %.2f GB) and a state restore of the "
                   "tables between steps" % (sc.batch.n_tokens * 4 / 1e9, sc.W * 2 * int(sc.cap_blocks[0]) * 16 / 1e9)}
 
@@ -135,12 +139,13 @@ class ClockSampler:
                 "reasons": reasons, "samples": len(rows), "power_w_max": max(float(r[3]) for r in rows)}
 
 
-def setup_router(sc, torch):
+def setup_router(sc, torch, prefix_index):
     from paper_2608_11152_gb300 import misat
 
     r = misat.Router(sc.cap_blocks, max_batch=sc.max_batch, max_tokens=sc.max_tokens,
                      protected_frac_q16=sc.protected_frac_q16, rounds=sc.rounds, mode=sc.mode,
-                     hold_delay_q=sc.hold_delay_q, prior_kbar=sc.prior_kbar, prior_T_us=sc.prior_T_us)
+                     hold_delay_q=sc.hold_delay_q, prior_kbar=sc.prior_kbar, prior_T_us=sc.prior_T_us,
+                     prefix_index=prefix_index)
     r.set_mixture(sc.rho_ppm)
     r.set_instance_state(sc.backlog_q, sc.tokcost_q, sc.contraction)
     for f in sc.fillers:
@@ -180,8 +185,9 @@ def cpu_step(o, b):
     return time.perf_counter() - t
 
 
-def algorithmic_bytes(sc, st):
-    """Algorithmic HBM bytes per launch of the hash and probe kernels (see the design notes)."""
+def algorithmic_bytes(sc, st, mask_words=None):
+    """Algorithmic HBM bytes per launch of the hash and probe kernels (see the design notes).
+    mask_words: words per key of the global prefix index, None for the per-instance probe."""
     b = sc.batch
     L = np.diff(b.tok_off)
     nb = L // 16
@@ -189,9 +195,14 @@ def algorithmic_bytes(sc, st):
     # K1: every full block's 16 token ids are read once (64 B) and its key written once (8 B),
     # plus two 8-byte offsets per request
     hash_b = 72 * n_blocks + 16 * b.n
-    # K2 phase 1: one 32-byte key group per block-0 probe, the H row written (2 B per pair),
-    # block-0 key, block count and key base read per request
-    first_b = 32 * st.probes_first + 2 * b.n * sc.W + 20 * b.n
+    if mask_words is None:
+        # K2 phase 1 per instance: one 32-byte key group per block-0 probe, the H row written
+        # (2 B per pair), block-0 key, block count and key base read per request
+        first_b = 32 * st.probes_first + 2 * b.n * sc.W + 20 * b.n
+    else:
+        # K2 phase 1 through the global index: one 32-byte key group per bucket read, the mask
+        # of each looked-up key, the H row, request fields (the hit list is not counted)
+        first_b = 32 * st.bucket_reads_first + 8 * mask_words * st.probes_first + 2 * b.n * sc.W + 20 * b.n
     # K2 phase 2: one 32-byte key group per probe of the binary searches
     search_b = 32 * (st.probes - st.probes_first)
     return {"hash": hash_b, "probe_first": first_b, "probe_search": search_b, "n_blocks": n_blocks}
@@ -219,7 +230,8 @@ def run_gb300(args):
 
     sc = workload(args)
     log(f"workload generated: {sc.name}, {sc.batch.n_tokens} tokens in the measured batch")
-    r = setup_router(sc, torch)
+    pidx = misat.PREFIX_GLOBAL if args.prefix_index == "global" else misat.PREFIX_PER_INSTANCE
+    r = setup_router(sc, torch, pidx)
     ckpt = r.checkpoint_save()
     db = r.device_batch(sc.batch)
     out = r.alloc_decisions(sc.batch.n)
@@ -314,7 +326,26 @@ def run_gb300(args):
 
     # roofline: dominant kernel of the step, plus the hash and probe kernels
     peak, peak_kind = peaks()
-    ab = algorithmic_bytes(sc, st)
+    gidx = None
+    if pidx == misat.PREFIX_GLOBAL:
+        # global prefix index: size, claimed slots and the cost of one rebuild from the
+        # instance tables, amortized over the steps a rebuild's headroom lasts at this
+        # workload's rate of new keys (rebuilds happen outside the steady-state step)
+        mw, slots, claimed = r.global_info()
+        live = sum(r.index_size(w) for w in range(sc.W))
+        torch.cuda.synchronize()
+        g0, g1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        g0.record(stream)
+        r.global_rebuild()
+        g1.record(stream)
+        g1.synchronize()
+        rb_ms = g0.elapsed_time(g1)
+        steps_between = max(1.0, (0.7 * slots - live) / max(1, st.new_keys))
+        gidx = {"mask_words": mw, "slots": slots, "claimed_after_step": claimed, "live_keys": live,
+                "rebuild_ms": round(rb_ms, 3), "steps_between_rebuilds": round(steps_between, 1),
+                "amortized_rebuild_ms_per_step": round(rb_ms / steps_between, 4)}
+        log(f"global index: {gidx}")
+    ab = algorithmic_bytes(sc, st, mask_words=gidx["mask_words"] if gidx else None)
     phase_ms = {p: phase_tot[p] / K for p in phase_tot}
     dom = max(phase_ms, key=lambda p: phase_ms[p])
 
@@ -347,6 +378,8 @@ def run_gb300(args):
         "gpu_launches": kernels_per_step(sc.rounds) * K,
         "roofline": dom_roof,
         "kernels": kernels,
+        "prefix_index": args.prefix_index,
+        "global_index": gidx,
         "phase_ms": {p: round(v, 4) for p, v in phase_ms.items()},
         "clocks": clocks,
         "wall_s_timed_loop": round(wall, 3),

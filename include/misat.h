@@ -51,6 +51,11 @@ extern "C" {
 #define MISAT_ERR_STATE (-4)           /* commit without a pending route */
 #define MISAT_ERR_TABLE_FULL (-5)      /* a bounded probe found no free slot */
 #define MISAT_ERR_BATCH_TOO_LARGE (-6) /* batch exceeds max_batch / max_tokens */
+#define MISAT_ERR_INTERNAL (-7)        /* the global index no longer mirrors the instance tables */
+
+/* ---- prefix index used by the block-0 probe (misat_config.prefix_index) ---- */
+#define MISAT_PREFIX_GLOBAL 0       /* key -> instance bitmask, one lookup per request (default) */
+#define MISAT_PREFIX_PER_INSTANCE 1 /* one lookup per (request, instance) pair */
 
 /* ---- policy modes (Sec. 5.2 ablation variants) ---- */
 #define MISAT_MODE_MISA_T 0            /* block-time quota, Eqs. (11),(13) (default) */
@@ -87,6 +92,7 @@ typedef struct misat_config {
   int64_t prior_T_us;           /* shared neutral residency prior (Sec. 4.3), 0..2^40 */
   uint64_t hash_seed;           /* a_{-1} of the block-hash chain (0x9e3779b97f4a7c15) */
   double table_load;            /* max load of an instance table before it grows, 0.25..0.9 (0.75) */
+  int32_t prefix_index;         /* MISAT_PREFIX_* (0 = global) */
 } misat_config;
 
 /* One routing batch.  Device pointers, except n and n_tokens. */
@@ -231,6 +237,23 @@ int misat_dump_sessions(misat_ctx* ctx, uint64_t* ids, int32_t* state, int32_t* 
 
 /* Statistics of the last route / commit.  [sync] */
 int misat_stats(misat_ctx* ctx, misat_batch_stats* host_out);
+
+/* Global prefix index (Sec. 4.5: the router maps every prefix block hash to the set of
+ * instances that currently cache it).  With MISAT_PREFIX_GLOBAL the library keeps, next to
+ * the per-instance tables, one table key -> W-bit instance mask that mirrors them exactly;
+ * the block-0 probe of a request reads one mask instead of W tables.
+ *
+ * misat_global_info [sync]: mask words per entry (ceil(W/64)), slots of the index and
+ *   slots claimed (live keys plus keys whose mask became empty; the index is rebuilt from
+ *   the instance tables when claimed slots pass 70% of the slots).  Any output may be NULL.
+ * misat_global_dump [sync]: the keys with a non-empty mask (unordered) and their masks,
+ *   host arrays keys[cap] and masks[cap * mask_words]; *n_out = number of such keys (may
+ *   exceed cap: only cap are written).
+ * misat_global_rebuild [async]: rebuild the index from the instance tables now.
+ * All three return MISAT_ERR_STATE when the context uses MISAT_PREFIX_PER_INSTANCE. */
+int misat_global_info(misat_ctx* ctx, int32_t* mask_words, int64_t* slots, int64_t* claimed);
+int misat_global_dump(misat_ctx* ctx, uint64_t* keys, uint64_t* masks, int64_t cap, int64_t* n_out);
+int misat_global_rebuild(misat_ctx* ctx);
 
 /* ---- checkpoint / resume (the paper has no counterpart: state snapshots of the router) ----
  * A checkpoint is a device-resident copy of the whole router state: every instance index

@@ -21,7 +21,7 @@ constexpr int kMaxRounds = 64;
 // Small device block copied to the host in one transfer after each route / commit.
 // Layout (8-byte words): stats[32] | U[W] | size[W] | sess_used | err | cand[3] | work | n_hits
 struct MetaLayout {
-  size_t stats = 0, U = 0, size = 0, sess_used = 0, err = 0, cand = 0, work = 0, n_hits = 0, words = 0;
+  size_t stats = 0, U = 0, size = 0, sess_used = 0, err = 0, cand = 0, work = 0, n_hits = 0, g_used = 0, words = 0;
   void init(int W) {
     stats = 0;
     U = 32;
@@ -31,7 +31,8 @@ struct MetaLayout {
     cand = err + 1;
     work = cand + 3;
     n_hits = work + 1;
-    words = n_hits + 1;
+    g_used = n_hits + 1;
+    words = g_used + 1;
   }
 };
 
@@ -111,7 +112,12 @@ struct misat_ctx {
   // per-request scratch
   ReqArrays rq{};
   uint64_t* d_keys = nullptr;
-  int32_t* d_owner = nullptr;
+  // global prefix index (MISAT_PREFIX_GLOBAL); its arrays are reallocated by rebuilds
+  bool use_gix = false;
+  GIndex gix{};
+  int2* d_units = nullptr;      // insert work list
+  unsigned* d_units_n = nullptr;
+  int64_t units_cap = 0;
   int64_t keys_cap = 0;
   uint16_t* d_H = nullptr;
   int2* d_hits = nullptr;
@@ -264,6 +270,64 @@ int ensure_capacity(misat_ctx* c, const std::vector<int64_t>& sizes, const std::
   return MISAT_OK;
 }
 
+// ---- global prefix index ----
+constexpr double kGixLoad = 0.35;  // load after a rebuild
+constexpr double kGixMax = 0.7;    // claimed slots that trigger a rebuild
+
+size_t gix_slots(const misat_ctx* c) { return (size_t)4 << c->gix.log2nb; }
+
+// Replace the index arrays by zeroed ones of 2^lg buckets (waits for the stream).
+int gix_alloc(misat_ctx* c, uint32_t lg) {
+  const size_t slots = (size_t)4 << lg;
+  unsigned long long *k = nullptr, *m = nullptr;
+  if (cudaMalloc(&k, slots * 8) != cudaSuccess || cudaMalloc(&m, slots * c->gix.mw * 8) != cudaSuccess) {
+    cudaGetLastError();
+    cudaFree(k);
+    return MISAT_ERR_OOM;
+  }
+  CK(cudaStreamSynchronize(c->stream));
+  cudaFree(c->gix.keys);
+  cudaFree(c->gix.masks);
+  c->gix.keys = k;
+  c->gix.masks = m;
+  c->gix.log2nb = lg;
+  CK(cudaMemsetAsync(k, 0, slots * 8, c->stream));
+  CK(cudaMemsetAsync(m, 0, slots * c->gix.mw * 8, c->stream));
+  return MISAT_OK;
+}
+
+// Rebuild the index from the instance tables, growing it so that `live` keys fill at
+// most kGixLoad of it.
+int gix_rebuild(misat_ctx* c, int64_t live) {
+  const uint32_t lg = std::max(c->gix.log2nb, buckets_log2_for(std::max<int64_t>(live, 1024), kGixLoad));
+  if (lg != c->gix.log2nb) {
+    int rc = gix_alloc(c, lg);
+    if (rc) return rc;
+  } else {
+    CK(cudaMemsetAsync(c->gix.keys, 0, gix_slots(c) * 8, c->stream));
+    CK(cudaMemsetAsync(c->gix.masks, 0, gix_slots(c) * c->gix.mw * 8, c->stream));
+  }
+  CK(cudaMemsetAsync(c->d_meta + c->ml.g_used, 0, 8, c->stream));
+  c->h_meta[c->ml.g_used] = 0;
+  uint32_t maxlg = 1;
+  for (auto& d : c->h_desc) maxlg = std::max(maxlg, d.log2nb);
+  launch_gix_build(c->d_desc, c->W, maxlg, c->gix, c->err_ptr(), c->stream);
+  CK(cudaGetLastError());
+  return MISAT_OK;
+}
+
+// Before up to `add` keys enter the tables (claimed-slot count must be on the host).
+int gix_ensure(misat_ctx* c, const std::vector<int64_t>& sizes, int64_t add) {
+  if (!c->use_gix) return MISAT_OK;
+  const uint64_t used = c->h_meta[c->ml.g_used];
+  if ((double)(used + (uint64_t)add) <= kGixMax * (double)gix_slots(c)) return MISAT_OK;
+  int64_t live = add;
+  for (int64_t x : sizes) live += x;
+  return gix_rebuild(c, live);
+}
+
+GIndex gix_or_null(const misat_ctx* c) { return c->use_gix ? c->gix : GIndex{}; }
+
 // Read the counters block (sync).
 int read_meta(misat_ctx* c) {
   CK(cudaMemcpyAsync(c->h_meta, c->d_meta, c->ml.words * 8, cudaMemcpyDeviceToHost, c->stream));
@@ -352,6 +416,7 @@ EvictArgs evict_args(misat_ctx* c, unsigned long long* evicted_counter) {
   ev.active = c->d_active;
   ev.evicted = evicted_counter;
   ev.err = c->err_ptr();
+  ev.gix = gix_or_null(c);
   return ev;
 }
 
@@ -376,9 +441,10 @@ const char* misat_strerror(int code) {
     case MISAT_ERR_INVALID_ARG: return "invalid argument";
     case MISAT_ERR_OOM: return "out of memory";
     case MISAT_ERR_CUDA: return "CUDA runtime error";
-    case MISAT_ERR_STATE: return "no pending route to commit";
+    case MISAT_ERR_STATE: return "call not valid in this state";
     case MISAT_ERR_TABLE_FULL: return "table full";
     case MISAT_ERR_BATCH_TOO_LARGE: return "batch exceeds max_batch or max_tokens";
+    case MISAT_ERR_INTERNAL: return "global prefix index out of step with the instance tables";
     default: return "unknown error";
   }
 }
@@ -391,6 +457,8 @@ int misat_destroy(misat_ctx* c) {
     if (w < c->h_bufs.size()) free_bufs(c->h_bufs[w]);
   }
   cudaFree(c->sess.slots);
+  cudaFree(c->gix.keys);
+  cudaFree(c->gix.masks);
   for (void* p : c->owned) cudaFree(p);
   if (c->h_meta) cudaFreeHost(c->h_meta);
   if (c->ev_meta) cudaEventDestroy(c->ev_meta);
@@ -419,6 +487,8 @@ int misat_create(const misat_config* cfg, void* cuda_stream, misat_ctx** out) {
     if (cfg->prior_kbar_blocks[b] < 1 || cfg->prior_kbar_blocks[b] > ((int64_t)1 << 30)) return MISAT_ERR_INVALID_ARG;
   if (cfg->prior_T_us < 0 || cfg->prior_T_us > ((int64_t)1 << 40)) return MISAT_ERR_INVALID_ARG;
   if (!(cfg->table_load >= 0.25 && cfg->table_load <= 0.9)) return MISAT_ERR_INVALID_ARG;
+  if (cfg->prefix_index != MISAT_PREFIX_GLOBAL && cfg->prefix_index != MISAT_PREFIX_PER_INSTANCE)
+    return MISAT_ERR_INVALID_ARG;
 
   misat_ctx* c = new (std::nothrow) misat_ctx();
   if (!c) return MISAT_ERR_OOM;
@@ -453,11 +523,12 @@ int misat_create(const misat_config* cfg, void* cuda_stream, misat_ctx** out) {
 
   const size_t NB = (size_t)c->max_batch, Ws = (size_t)W;
   c->keys_cap = c->max_tokens / 16 + 1;
+  c->units_cap = (int64_t)NB + c->keys_cap / 128 + 1;  // one unit per 128 blocks of a request
   c->hits_cap = (int64_t)std::min<size_t>(NB * Ws, (size_t)1 << 27);
   const int bm_log2 = std::max(1, ceil_log2(2 * NB));
   const size_t n_tiles = (NB + kTileReq - 1) / kTileReq;
   if ((rc = dalloc_n(c, &c->d_meta, c->ml.words)) || (rc = dalloc_n(c, &c->d_keys, (size_t)c->keys_cap)) ||
-      (rc = dalloc_n(c, &c->d_owner, (size_t)c->keys_cap)) ||
+      (rc = dalloc_n(c, &c->d_units, (size_t)c->units_cap)) || (rc = dalloc_n(c, &c->d_units_n, 1)) ||
       (rc = dalloc_n(c, &c->d_H, NB * Ws)) || (rc = dalloc_n(c, &c->d_hits, (size_t)c->hits_cap)) ||
       (rc = dalloc_n(c, &c->d_bm_key, (size_t)1 << bm_log2)) ||
       (rc = dalloc_n(c, &c->d_bm_val, (size_t)1 << bm_log2)) || (rc = dalloc_n(c, &c->d_tile, n_tiles * 3 * Ws)) ||
@@ -506,6 +577,16 @@ int misat_create(const misat_config* cfg, void* cuda_stream, misat_ctx** out) {
       return fail(MISAT_ERR_CUDA);
     c->sess.log2n = lg;
     c->sess.used = c->d_meta + c->ml.sess_used;
+  }
+  // global prefix index, sized for full tables (up to 2^26 keys; rebuilds grow it)
+  if (cfg->prefix_index == MISAT_PREFIX_GLOBAL) {
+    c->use_gix = true;
+    c->gix.mw = (uint32_t)((W + 63) / 64);
+    c->gix.used = c->d_meta + c->ml.g_used;
+    int64_t total_cap = 0;
+    for (int w = 0; w < W; ++w) total_cap += c->cap[w];
+    total_cap = std::min<int64_t>(total_cap, (int64_t)1 << 26);
+    if ((rc = gix_alloc(c, buckets_log2_for(std::max<int64_t>(total_cap, 1024), kGixLoad)))) return fail(rc);
   }
   if (cudaStreamSynchronize(c->stream) != cudaSuccess) return fail(MISAT_ERR_CUDA);
   *out = c;
@@ -604,7 +685,6 @@ int misat_route(misat_ctx* c, const misat_batch* b, misat_decisions* out) {
   ha.seed = c->seed;
   ha.keys = c->d_keys;
   ha.keys_cap = c->keys_cap;
-  ha.owner = c->d_owner;
   ha.work = c->work_ptr();
   ha.err = c->err_ptr();
   launch_block_hash(ha, c->num_sms, st);
@@ -626,7 +706,7 @@ int misat_route(misat_ctx* c, const misat_batch* b, misat_decisions* out) {
   pr.stats = c->stats_ptr() + 16;
   pr.stats_search = c->stats_ptr() + 22;
   pr.err = c->err_ptr();
-  pr.flat = getenv("MISAT_PROBE_FLAT") ? 1 : 0;
+  pr.gix = gix_or_null(c);
   launch_probe_first(pr, c->num_sms, st);
   c->mark(4);
   launch_probe_search(pr, c->num_sms, st);
@@ -718,6 +798,9 @@ int misat_commit(misat_ctx* c) {
     }
     int rc = ensure_capacity(c, sizes, add);
     if (rc) return rc;
+    int64_t add_all = 0;
+    for (int64_t x : add) add_all += x;
+    if ((rc = gix_ensure(c, sizes, add_all))) return rc;
     rc = maybe_rebuild_sessions(c, n);
     if (rc) return rc;
   }
@@ -728,16 +811,18 @@ int misat_commit(misat_ctx* c) {
     ia.desc = c->d_desc;
     ia.n_inst = c->W;
     ia.n = n;
-    ia.n_slots = c->last_ntok / 16;
+    ia.units = c->d_units;
+    ia.n_units = c->d_units_n;
+    ia.units_cap = c->units_cap;
     ia.nb = c->rq.nb;
     ia.kbase = c->rq.kbase;
     ia.inst = c->rq.inst;
     ia.keys = c->d_keys;
-    ia.owner = c->d_owner;
     ia.seq = c->seq + 1;
     ia.size = c->size_ptr();
     ia.new_keys = c->stats_ptr() + 18;
     ia.err = c->err_ptr();
+    ia.gix = gix_or_null(c);
     launch_insert(ia, c->num_sms, st);
     c->mark(9);
     SessUpdateArgs sa{n, c->rq, c->sess, c->d_prot, c->err_ptr()};
@@ -791,6 +876,10 @@ int misat_complete(misat_ctx* c, int32_t n, const uint64_t* session, const uint8
 
 int misat_reset_instance(misat_ctx* c, int32_t w) {
   if (!c || w < 0 || w >= c->W) return MISAT_ERR_INVALID_ARG;
+  if (c->use_gix) {
+    launch_gix_clear_table(c->h_desc[w], w, c->gix, c->err_ptr(), c->stream);
+    CK(cudaGetLastError());
+  }
   CK(cudaMemsetAsync(c->h_desc[w].tab, 0, ((size_t)1 << c->h_desc[w].log2nb) * sizeof(Bucket), c->stream));
   CK(cudaMemsetAsync(c->size_ptr() + w, 0, 8, c->stream));
   return MISAT_OK;
@@ -837,6 +926,7 @@ int misat_load_entries(misat_ctx* c, int32_t w, const misat_entry* entries, int6
   for (int x = 0; x < c->W; ++x) sizes[x] = c->h_size(x);
   add[w] = n;
   if ((rc = ensure_capacity(c, sizes, add))) return rc;
+  if ((rc = gix_ensure(c, sizes, n))) return rc;
   misat_entry* de = nullptr;
   if (n > 0) {
     if (cudaMalloc(&de, (size_t)n * sizeof(misat_entry)) != cudaSuccess) {
@@ -844,7 +934,7 @@ int misat_load_entries(misat_ctx* c, int32_t w, const misat_entry* entries, int6
       return MISAT_ERR_OOM;
     }
     CK(cudaMemcpyAsync(de, entries, (size_t)n * sizeof(misat_entry), cudaMemcpyHostToDevice, c->stream));
-    EntryInsertArgs a{c->h_desc[w], n, de, c->size_ptr() + w, c->err_ptr()};
+    EntryInsertArgs a{c->h_desc[w], n, de, c->size_ptr() + w, c->err_ptr(), w, gix_or_null(c)};
     launch_insert_entries(a, c->stream);
     CK(cudaGetLastError());
   }
@@ -879,6 +969,9 @@ int misat_load_chains(misat_ctx* c, int32_t n_chains, const int64_t* tok_off, co
   std::vector<int64_t> sizes(c->W);
   for (int x = 0; x < c->W; ++x) sizes[x] = c->h_size(x);
   if ((rc = ensure_capacity(c, sizes, add))) return rc;
+  int64_t add_all = 0;
+  for (int64_t x : add) add_all += x;
+  if ((rc = gix_ensure(c, sizes, add_all))) return rc;
   cudaStream_t st = c->stream;
   // stage: offsets, tokens, per-chain inst / tick / limit (reuse request scratch arrays)
   CK(cudaMemcpyAsync(c->d_stage_off, tok_off, (size_t)(n_chains + 1) * 8, cudaMemcpyHostToDevice, st));
@@ -904,7 +997,6 @@ int misat_load_chains(misat_ctx* c, int32_t n_chains, const int64_t* tok_off, co
   ha.seed = c->seed;
   ha.keys = c->d_keys;
   ha.keys_cap = c->keys_cap;
-  ha.owner = c->d_owner;
   ha.work = c->work_ptr();
   ha.err = c->err_ptr();
   launch_block_hash(ha, c->num_sms, st);
@@ -912,18 +1004,20 @@ int misat_load_chains(misat_ctx* c, int32_t n_chains, const int64_t* tok_off, co
   ia.desc = c->d_desc;
   ia.n_inst = c->W;
   ia.n = n_chains;
-  ia.n_slots = ntok / 16;
+  ia.units = c->d_units;
+  ia.n_units = c->d_units_n;
+  ia.units_cap = c->units_cap;
   ia.nb = c->rq.nb;
   ia.kbase = c->rq.kbase;
   ia.inst = c->rq.inst;
   ia.keys = c->d_keys;
-  ia.owner = c->d_owner;
   ia.meta_seq = c->rq.session;
   ia.meta_arr = reinterpret_cast<const uint32_t*>(c->d_out_hit);
   ia.max_blocks = c->rq.choice;
   ia.size = c->size_ptr();
   ia.new_keys = c->stats_ptr() + 21;
   ia.err = c->err_ptr();
+  ia.gix = gix_or_null(c);
   launch_insert(ia, c->num_sms, st);
   CK(cudaGetLastError());
   rc = load_common_evict(c);
@@ -1064,6 +1158,53 @@ int misat_stats(misat_ctx* c, misat_batch_stats* o) {
   return c->h_err();
 }
 
+int misat_global_info(misat_ctx* c, int32_t* mask_words, int64_t* slots, int64_t* claimed) {
+  if (!c) return MISAT_ERR_INVALID_ARG;
+  if (!c->use_gix) return MISAT_ERR_STATE;
+  int rc = read_meta(c);
+  if (rc) return rc;
+  if (mask_words) *mask_words = (int32_t)c->gix.mw;
+  if (slots) *slots = (int64_t)gix_slots(c);
+  if (claimed) *claimed = (int64_t)c->h_meta[c->ml.g_used];
+  return c->h_err();
+}
+
+int misat_global_dump(misat_ctx* c, uint64_t* keys, uint64_t* masks, int64_t cap, int64_t* n_out) {
+  if (!c || cap < 0 || !n_out || (cap > 0 && (!keys || !masks))) return MISAT_ERR_INVALID_ARG;
+  if (!c->use_gix) return MISAT_ERR_STATE;
+  const size_t slots = gix_slots(c), mw = c->gix.mw;
+  std::vector<unsigned long long> hk(slots), hm(slots * mw);
+  CK(cudaMemcpyAsync(hk.data(), c->gix.keys, slots * 8, cudaMemcpyDeviceToHost, c->stream));
+  CK(cudaMemcpyAsync(hm.data(), c->gix.masks, slots * mw * 8, cudaMemcpyDeviceToHost, c->stream));
+  int rc = read_meta(c);
+  if (rc) return rc;
+  int64_t n = 0;
+  for (size_t i = 0; i < slots; ++i) {
+    if (hk[i] == kEmpty) continue;
+    bool any = false;
+    for (size_t j = 0; j < mw; ++j) any |= hm[i * mw + j] != 0;
+    if (!any) continue;
+    if (n < cap) {
+      keys[n] = hk[i];
+      for (size_t j = 0; j < mw; ++j) masks[n * mw + j] = hm[i * mw + j];
+    }
+    ++n;
+  }
+  *n_out = n;
+  return c->h_err();
+}
+
+int misat_global_rebuild(misat_ctx* c) {
+  if (!c) return MISAT_ERR_INVALID_ARG;
+  if (!c->use_gix) return MISAT_ERR_STATE;
+  int rc = read_meta(c);
+  if (rc) return rc;
+  if (c->h_err()) return c->h_err();
+  int64_t live = 0;
+  for (int w = 0; w < c->W; ++w) live += c->h_size(w);
+  return gix_rebuild(c, live);
+}
+
 int misat_set_timing(misat_ctx* c, int enable) {
   if (!c) return MISAT_ERR_INVALID_ARG;
   if (enable && !c->ev[0])
@@ -1106,6 +1247,11 @@ struct misat_checkpoint {
   std::deque<int64_t> hist_blocks[3], hist_res[3];
   uint32_t rho[3] = {0, 0, 0};
   uint64_t seq = 0;
+  // global prefix index copy (NULL when the context has none)
+  unsigned long long* gkeys = nullptr;
+  unsigned long long* gmasks = nullptr;
+  uint32_t g_log2 = 0;
+  uint64_t g_used = 0;
 };
 
 extern "C" {
@@ -1118,6 +1264,8 @@ int misat_checkpoint_free(misat_checkpoint* k) {
   cudaFree(k->backlog);
   cudaFree(k->tokcost);
   cudaFree(k->contraction);
+  cudaFree(k->gkeys);
+  cudaFree(k->gmasks);
   delete k;
   return MISAT_OK;
 }
@@ -1149,6 +1297,10 @@ int misat_checkpoint_save(misat_ctx* c, misat_checkpoint** out) {
                cudaMalloc(&k->backlog, c->W * 8) != cudaSuccess || cudaMalloc(&k->tokcost, c->W * 8) != cudaSuccess ||
                cudaMalloc(&k->contraction, c->W * 4) != cudaSuccess))
     oom = true;
+  if (!oom && c->use_gix &&
+      (cudaMalloc(&k->gkeys, gix_slots(c) * 8) != cudaSuccess ||
+       cudaMalloc(&k->gmasks, gix_slots(c) * c->gix.mw * 8) != cudaSuccess))
+    oom = true;
   if (oom) {
     cudaGetLastError();
     misat_checkpoint_free(k);
@@ -1159,6 +1311,12 @@ int misat_checkpoint_save(misat_ctx* c, misat_checkpoint** out) {
   CK(cudaMemcpyAsync(k->backlog, c->d_backlog, c->W * 8, cudaMemcpyDeviceToDevice, st));
   CK(cudaMemcpyAsync(k->tokcost, c->d_tokcost, c->W * 8, cudaMemcpyDeviceToDevice, st));
   CK(cudaMemcpyAsync(k->contraction, c->d_contraction, c->W * 4, cudaMemcpyDeviceToDevice, st));
+  if (c->use_gix) {
+    CK(cudaMemcpyAsync(k->gkeys, c->gix.keys, gix_slots(c) * 8, cudaMemcpyDeviceToDevice, st));
+    CK(cudaMemcpyAsync(k->gmasks, c->gix.masks, gix_slots(c) * c->gix.mw * 8, cudaMemcpyDeviceToDevice, st));
+    k->g_log2 = c->gix.log2nb;
+    k->g_used = c->h_meta[c->ml.g_used];
+  }
   CK(cudaStreamSynchronize(st));
   k->sess_log2 = c->sess.log2n;
   k->sess_used = c->h_meta[c->ml.sess_used];
@@ -1216,6 +1374,17 @@ int misat_checkpoint_restore(misat_ctx* c, const misat_checkpoint* k) {
   CK(cudaMemcpyAsync(c->d_backlog, k->backlog, c->W * 8, cudaMemcpyDeviceToDevice, st));
   CK(cudaMemcpyAsync(c->d_tokcost, k->tokcost, c->W * 8, cudaMemcpyDeviceToDevice, st));
   CK(cudaMemcpyAsync(c->d_contraction, k->contraction, c->W * 4, cudaMemcpyDeviceToDevice, st));
+  if (c->use_gix) {
+    if (!k->gkeys) return MISAT_ERR_INVALID_ARG;
+    if (c->gix.log2nb != k->g_log2) {
+      int rc = gix_alloc(c, k->g_log2);
+      if (rc) return rc;
+    }
+    CK(cudaMemcpyAsync(c->gix.keys, k->gkeys, gix_slots(c) * 8, cudaMemcpyDeviceToDevice, st));
+    CK(cudaMemcpyAsync(c->gix.masks, k->gmasks, gix_slots(c) * c->gix.mw * 8, cudaMemcpyDeviceToDevice, st));
+    c->h_meta[c->ml.g_used] = k->g_used;
+    CK(cudaMemcpyAsync(c->d_meta + c->ml.g_used, c->h_meta + c->ml.g_used, 8, cudaMemcpyHostToDevice, st));
+  }
   // sizes and the session-slot counter live in the counters block
   for (int w = 0; w < c->W; ++w) reinterpret_cast<long long*>(c->h_meta + c->ml.size)[w] = k->size[w];
   c->h_meta[c->ml.sess_used] = k->sess_used;

@@ -17,16 +17,17 @@ namespace misat {
 namespace {
 constexpr unsigned kFull = 0xffffffffu;
 
-// Find-or-claim `key` in an instance table and merge `meta`.  Returns 1 if the key was
-// new, 0 if it existed, -1 if no free slot was found within the table.
-__device__ int table_insert(const InstDesc& d, uint64_t key, uint64_t meta) {
+// Find-or-claim `key` in an instance table and merge `meta`, starting at bucket `b` whose
+// four keys the caller has already read into k[] (possibly stale: keys are only ever
+// added while inserts run, so a stale read can only miss a claim, which the CAS catches).
+// Returns 1 if the key was new, 0 if it existed, -1 if no free slot was found.
+__device__ __forceinline__ int table_insert_at(const InstDesc& d, uint64_t key, uint64_t meta, uint32_t b,
+                                               unsigned long long k[4]) {
   const uint32_t mask = (1u << d.log2nb) - 1;
-  uint32_t b = home_bucket(key, d.log2nb);
   for (uint32_t it = 0; it <= mask; ++it) {
     Bucket* B = d.tab + b;
     for (int tries = 0; tries < 2 * kSlots; ++tries) {
-      unsigned long long k[4];
-      ld_bucket_keys_cg(B, k);
+      if (it | tries) ld_bucket_keys_cg(B, k);
       int s = -1;
 #pragma unroll
       for (int i = 0; i < 4; ++i)
@@ -41,13 +42,9 @@ __device__ int table_insert(const InstDesc& d, uint64_t key, uint64_t meta) {
         if (k[i] == kEmpty) e = i;
       if (e < 0) break;  // bucket full without the key: next bucket
       const unsigned long long old = atomicCAS(&B->key[e], kEmpty, (unsigned long long)key);
-      if (old == kEmpty) {
+      if (old == kEmpty || old == key) {
         atomicMax(&B->meta[e], (unsigned long long)meta);
-        return 1;
-      }
-      if (old == key) {
-        atomicMax(&B->meta[e], (unsigned long long)meta);
-        return 0;
+        return old == kEmpty ? 1 : 0;
       }
       // the slot went to another key: re-read this bucket
     }
@@ -56,86 +53,160 @@ __device__ int table_insert(const InstDesc& d, uint64_t key, uint64_t meta) {
   return -1;
 }
 
+__device__ __forceinline__ int table_insert(const InstDesc& d, uint64_t key, uint64_t meta) {
+  const uint32_t b = home_bucket(key, d.log2nb);
+  unsigned long long k[4];
+  ld_bucket_keys_cg(d.tab + b, k);
+  return table_insert_at(d, key, meta, b, k);
+}
+
 }  // namespace
 
 // ---------------------------------------------------------------------------
-// Insert: one thread per key slot of the batch; the owning request comes from the owner
-// map the hash kernel wrote next to the keys.
-__global__ void __launch_bounds__(256) k4_insert(InsertArgs a) {
+// Insert.  Work is listed first: every request with an instance contributes one unit per
+// kUnitBlocks of its blocks, so that the insert kernel touches only admitted keys and a
+// long prompt is spread over many warps.  A warp then inserts one unit: lane l takes blocks
+// l, l+32, l+64, l+96 of it and issues all four home-bucket reads before the first atomic;
+// a key already present costs one fire-and-forget atomicMax on its meta, a new one a CAS.
+// The order of the units is free: the final key set and metas do not depend on it.
+constexpr int kIns = 4;
+constexpr int kUnitBlocks = 32 * kIns;
+constexpr int kInsThreads = 256;
+
+__global__ void __launch_bounds__(256) k4_units(InsertArgs a) {
+  const int r = blockIdx.x * blockDim.x + threadIdx.x;
+  const int lane = threadIdx.x & 31;
+  int u = 0;
+  if (r < a.n && *a.err == 0 && a.inst[r] >= 0) {
+    int c = a.nb[r];
+    if (a.max_blocks && a.max_blocks[r] < c) c = a.max_blocks[r];
+    u = (c + kUnitBlocks - 1) / kUnitBlocks;
+  }
+  int incl = u;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const int t = __shfl_up_sync(kFull, incl, o);
+    if (lane >= o) incl += t;
+  }
+  const int tot = __shfl_sync(kFull, incl, 31);
+  if (tot == 0) return;
+  unsigned base = 0;
+  if (lane == 31) base = atomicAdd(a.n_units, (unsigned)tot);
+  base = __shfl_sync(kFull, base, 31) + (unsigned)(incl - u);
+  for (int i = 0; i < u; ++i) {
+    if ((int64_t)base + i < a.units_cap)
+      a.units[base + i] = make_int2(r, i);
+    else
+      set_error(a.err, MISAT_ERR_TABLE_FULL);
+  }
+}
+
+__global__ void __launch_bounds__(kInsThreads, 3) k4_insert(InsertArgs a) {
   __shared__ unsigned s_new[kMaxW];  // new keys per instance, flushed once per CTA
   if (block_error(a.err)) return;
   for (int i = threadIdx.x; i < a.n_inst; i += blockDim.x) s_new[i] = 0;
   __syncthreads();
-  constexpr int kPer = 4;  // independent key slots per thread per iteration
   const int lane = threadIdx.x & 31;
   unsigned long long nnew = 0;
-  const int64_t stride = (int64_t)gridDim.x * blockDim.x * kPer;
-  // a warp covers 32*kPer consecutive slots per iteration; lane handles base + lane + 32 k
-  const int64_t start = ((int64_t)blockIdx.x * blockDim.x + (threadIdx.x & ~31)) * kPer;
-  for (int64_t base = start; base < a.n_slots; base += stride) {
-    int r[kPer], w[kPer];
+  long long gclaim = 0;
+  const int64_t n_units = min((int64_t)__ldcg(a.n_units), a.units_cap);
+  const int64_t warps = (int64_t)gridDim.x * (blockDim.x >> 5);
+  for (int64_t u = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); u < n_units; u += warps) {
+    const int2 un = __ldg(a.units + u);
+    const int r = un.x;
+    const int w = __ldg(a.inst + r);
+    int c = __ldg(a.nb + r);
+    if (a.max_blocks) c = min(c, __ldg(a.max_blocks + r));
+    const int64_t kb = __ldg(a.kbase + r);
+    const uint64_t mseq = a.meta_seq ? __ldg(a.meta_seq + r) : a.seq;
+    const uint64_t marr = a.meta_seq ? __ldg(a.meta_arr + r) : (uint64_t)r;
+    const InstDesc d = a.desc[w];
+    const int j0 = un.y * kUnitBlocks + lane;
+    uint64_t key[kIns];
+    uint32_t hb[kIns];
+    unsigned long long kk[kIns][4];
 #pragma unroll
-    for (int k = 0; k < kPer; ++k) {
-      const int64_t q = base + lane + 32 * k;
-      r[k] = q < a.n_slots ? a.owner[q] : -1;
+    for (int k = 0; k < kIns; ++k) {
+      const int j = j0 + 32 * k;
+      key[k] = j < c ? __ldg(reinterpret_cast<const unsigned long long*>(a.keys) + kb + j) : 0;
     }
 #pragma unroll
-    for (int k = 0; k < kPer; ++k) {
-      w[k] = -1;
-      if (r[k] >= 0) {
-        w[k] = a.inst[r[k]];
-        const int64_t j = base + lane + 32 * k - a.kbase[r[k]];
-        if (w[k] >= 0 && a.max_blocks && j >= a.max_blocks[r[k]]) w[k] = -1;
-      }
+    for (int k = 0; k < kIns; ++k) {
+      hb[k] = home_bucket(key[k], d.log2nb);
+      if (j0 + 32 * k < c) ld_bucket_keys_cg(d.tab + hb[k], kk[k]);
     }
+    unsigned cnt = 0;
+    int isnew[kIns];
 #pragma unroll
-    for (int k = 0; k < kPer; ++k) {
-      const int64_t q = base + lane + 32 * k;
-      int isnew = 0;
-      if (w[k] >= 0) {
-        const int64_t j = q - a.kbase[r[k]];
-        const uint64_t meta = a.meta_seq ? pack_meta(a.meta_seq[r[k]], a.meta_arr[r[k]], (uint64_t)j)
-                                         : pack_meta(a.seq, (uint64_t)r[k], (uint64_t)j);
-        const int res = table_insert(a.desc[w[k]], a.keys[q], meta);
+    for (int k = 0; k < kIns; ++k) {
+      const int j = j0 + 32 * k;
+      isnew[k] = 0;
+      if (j < c) {
+        const int res = table_insert_at(d, key[k], pack_meta(mseq, marr, (uint64_t)j), hb[k], kk[k]);
         if (res < 0)
           set_error(a.err, MISAT_ERR_TABLE_FULL);
         else
-          isnew = res;
+          isnew[k] = res;
       }
-      // per-instance size increments, aggregated over the warp's lanes with the same instance
-      const unsigned peers = __match_any_sync(kFull, isnew ? w[k] : -1 - lane);
-      const unsigned newmask = __ballot_sync(kFull, isnew);
-      if (isnew && lane == __ffs(peers) - 1) {
-        const int c = __popc(peers & newmask);
-        atomicAdd(&s_new[w[k]], (unsigned)c);
-        nnew += c;
+      cnt += __popc(__ballot_sync(kFull, isnew[k]));
+    }
+    if (a.gix.keys) {
+      // a key new to instance w gets bit w in the global index
+#pragma unroll
+      for (int k = 0; k < kIns; ++k) {
+        if (!isnew[k]) continue;
+        const int g = gix_set(a.gix, key[k], w);
+        if (g < 0)
+          set_error(a.err, MISAT_ERR_TABLE_FULL);
+        else
+          gclaim += g;
       }
+    }
+    if (lane == 0 && cnt) {
+      atomicAdd(&s_new[w], cnt);
+      nnew += cnt;
     }
   }
   const long long tot = block_sum((long long)nnew);
   if (threadIdx.x == 0 && tot) atomicAdd(a.new_keys, (unsigned long long)tot);
+  if (a.gix.keys) {
+    const long long gt = block_sum(gclaim);
+    if (threadIdx.x == 0 && gt) atomicAdd(a.gix.used, (unsigned long long)gt);
+  }
   __syncthreads();
   for (int i = threadIdx.x; i < a.n_inst; i += blockDim.x)
     if (s_new[i]) atomic_add_i64(&a.size[i], (long long)s_new[i]);
 }
 
 void launch_insert(const InsertArgs& a, int num_sms, cudaStream_t st) {
-  if (a.n_slots <= 0 || a.n <= 0) return;
-  int64_t blocks = (a.n_slots + 1023) / 1024;
-  int grid = (int)(blocks < (int64_t)num_sms * 8 ? blocks : (int64_t)num_sms * 8);
-  k4_insert<<<grid, 256, 0, st>>>(a);
+  if (a.n <= 0) return;
+  cudaMemsetAsync(a.n_units, 0, sizeof(unsigned), st);
+  k4_units<<<(a.n + 255) / 256, 256, 0, st>>>(a);
+  k4_insert<<<num_sms * 3, kInsThreads, 0, st>>>(a);  // resident CTAs: 3 per SM
 }
 
 __global__ void __launch_bounds__(256) k4_insert_entries(EntryInsertArgs a) {
   if (block_error(a.err)) return;
-  long long nnew = 0;
+  long long nnew = 0, gclaim = 0;
   for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < a.n; i += (int64_t)gridDim.x * blockDim.x) {
     const misat_entry e = a.entries[i];
     const int res = table_insert(a.desc, e.key, e.meta);
-    if (res < 0)
+    if (res < 0) {
       set_error(a.err, MISAT_ERR_TABLE_FULL);
-    else
+    } else {
       nnew += res;
+      if (res && a.gix.keys) {
+        const int g = gix_set(a.gix, e.key, a.w);
+        if (g < 0)
+          set_error(a.err, MISAT_ERR_TABLE_FULL);
+        else
+          gclaim += g;
+      }
+    }
+  }
+  if (a.gix.keys) {
+    const long long gt = block_sum(gclaim);
+    if (threadIdx.x == 0 && gt) atomicAdd(a.gix.used, (unsigned long long)gt);
   }
   const long long tot = block_sum(nnew);
   if (threadIdx.x == 0 && tot) atomic_add_i64(a.size, tot);

@@ -380,8 +380,11 @@ __global__ void __launch_bounds__(kSelThreads) k4_evict_select(EvictArgs a) {
 }
 
 namespace {
-__device__ __forceinline__ void delete_slot(Bucket* tab, uint32_t* dmask, uint32_t sl) {
+// Delete slot sl of instance w's table; the global index (if any) loses bit w of its key.
+__device__ __forceinline__ void delete_slot(const GIndex& g, int w, Bucket* tab, uint32_t* dmask, uint32_t sl,
+                                            int32_t* err) {
   const uint32_t b = sl >> 2, s = sl & 3;
+  if (g.keys && gix_clear(g, tab[b].key[s], w) < 0) set_error(err, MISAT_ERR_INTERNAL);
   tab[b].key[s] = kEmpty;
   tab[b].meta[s] = 0;
   atomicOr(&dmask[b >> 3], 1u << ((b & 7) * 4 + s));
@@ -404,12 +407,12 @@ __global__ void __launch_bounds__(256) k4_evict_delete(EvictArgs a) {
   const unsigned stride = gridDim.x * blockDim.x;
   for (unsigned i = blockIdx.x * blockDim.x + threadIdx.x; i < nd + n; i += stride) {
     if (i < nd) {
-      delete_slot(tab, dmask, dsl[i]);
+      delete_slot(a.gix, w, tab, dmask, dsl[i], a.err);
       ++deleted;
     } else {
       const uint4 v = c0[i - nd];
       if (!le128(v_hi(v), v_lo(v), tm, tk)) continue;
-      delete_slot(tab, dmask, slots[i - nd]);
+      delete_slot(a.gix, w, tab, dmask, slots[i - nd], a.err);
       ++deleted;
     }
   }
@@ -545,6 +548,7 @@ __global__ void __launch_bounds__(256) k4_evict_compact(EvictArgs a) {
         if (k == kEmpty) continue;
         const unsigned long long m = B->meta[s];
         if (m == 0 || (act == 1 && le128(m, k, tm, tk))) {
+          if (a.gix.keys && gix_clear(a.gix, k, w) < 0) set_error(a.err, MISAT_ERR_INTERNAL);
           B->key[s] = kEmpty;
           B->meta[s] = 0;
           ++deleted;

@@ -90,9 +90,6 @@ __global__ void __launch_bounds__(256) k1_block_hash(HashArgs a) {
     const int64_t t1 = a.tok_off[r + 1];
     const int32_t nb = (int32_t)((t1 - t0) >> 4);
     const int64_t kb = t0 >> 4;
-    // key slots kb .. kb+nb-1 belong to r; at most one slot before the next request's
-    // first slot floor(t1/16) belongs to nobody (the owner map marks it -1)
-    if (lane == 0 && a.owner && kb + nb < (t1 >> 4) && kb + nb < a.keys_cap) a.owner[kb + nb] = -1;
     if (nb <= 0) continue;
     const int64_t q0 = t0 >> 2;
     const int off = (int)(t0 & 3);
@@ -154,10 +151,7 @@ __global__ void __launch_bounds__(256) k1_block_hash(HashArgs a) {
       uint64_t key = mix64(av ^ (uint64_t)(32 * c + lane + 1));
       key += key < 2 ? 2 : 0;
       const int64_t dst = kb + 32ll * c + lane;
-      if (lane < cnt && dst < a.keys_cap) {
-        a.keys[dst] = key;
-        if (a.owner) a.owner[dst] = r;
-      }
+      if (lane < cnt && dst < a.keys_cap) a.keys[dst] = key;
       carry = __shfl_sync(kFull, av, 31);
 #pragma unroll
       for (int i = 0; i < 4; ++i) v[i] = vn[i];

@@ -5,6 +5,7 @@
 #include <stdint.h>
 
 #include "common.cuh"
+#include "gindex.cuh"
 
 namespace misat {
 
@@ -16,7 +17,6 @@ struct HashArgs {
   int32_t n;
   uint64_t seed;
   uint64_t* keys;       // key of (r, j) at floor(tok_off[r]/16) + j
-  int32_t* owner;       // request owning each key slot, -1 for a slot of no request (may be NULL)
   int64_t keys_cap;
   unsigned* work;       // zeroed before the launch
   const int32_t* err;
@@ -71,7 +71,7 @@ struct ProbeArgs {
   unsigned long long* stats;         // phase 1: [0] probes, [1] bucket reads
   unsigned long long* stats_search;  // phase 2: [0] probes, [1] bucket reads
   int32_t* err;
-  int32_t flat;                      // 1: thread-per-pair phase 1 (comparison layout)
+  GIndex gix;                        // phase 1 reads the global index when gix.keys != NULL
 };
 void launch_probe_first(const ProbeArgs& a, int num_sms, cudaStream_t st);
 void launch_probe_search(const ProbeArgs& a, int num_sms, cudaStream_t st);
@@ -150,8 +150,9 @@ void launch_finalize(const FinalizeArgs& a, cudaStream_t st);
 struct InsertArgs {
   const InstDesc* desc;
   int32_t n;
-  int64_t n_slots;             // key slots to scan: floor(n_tokens / 16)
-  const int32_t* owner;        // request of each key slot (-1: none), written by the hash kernel
+  int2* units;                 // work list (request, unit): up to 128 blocks per unit
+  unsigned* n_units;           // units listed (zeroed by the launcher)
+  int64_t units_cap;
   const int32_t* nb;
   const int64_t* kbase;
   const int32_t* inst;         // instance per request (-1: skip)
@@ -164,6 +165,7 @@ struct InsertArgs {
   long long* size;             // [W] live entries
   unsigned long long* new_keys;
   int32_t* err;
+  GIndex gix;                  // mirrored when gix.keys != NULL
 };
 void launch_insert(const InsertArgs& a, int num_sms, cudaStream_t st);
 
@@ -173,6 +175,8 @@ struct EntryInsertArgs {
   const misat_entry* entries;
   long long* size;             // &size[w]
   int32_t* err;
+  int32_t w;
+  GIndex gix;
 };
 void launch_insert_entries(const EntryInsertArgs& a, cudaStream_t st);
 
@@ -214,6 +218,7 @@ struct EvictArgs {
   int32_t* active;             // [W] 1: delete entries <= theta, 2: marked entries only
   unsigned long long* evicted;
   int32_t* err;
+  GIndex gix;                  // deletions clear the instance's bit when gix.keys != NULL
 };
 void launch_evict(const EvictArgs& a, int chunks_per_inst, cudaStream_t st);
 void launch_compact_marked(const EvictArgs& a, cudaStream_t st);
@@ -241,5 +246,12 @@ struct SessRehashArgs {
   int32_t* err;
 };
 void launch_sess_rehash(const SessRehashArgs& a, cudaStream_t st);
+
+// ---- global prefix index maintenance ----
+// Rebuild: set bit w for every key of every instance table (index zeroed beforehand).
+void launch_gix_build(const InstDesc* desc, int32_t W, uint32_t max_log2nb, const GIndex& g, int32_t* err,
+                      cudaStream_t st);
+// Clear bit w of every key of instance w's table (before the table is reset).
+void launch_gix_clear_table(const InstDesc& d, int32_t w, const GIndex& g, int32_t* err, cudaStream_t st);
 
 }  // namespace misat

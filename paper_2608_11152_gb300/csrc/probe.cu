@@ -5,11 +5,11 @@
 // tick and eviction takes the deepest block of a tick first), so "block h-1 is
 // resident" is monotone in h and H is found by binary search.
 //
-// Phase 1 (k2_probe_first): one thread per (r, w) pair probes block 0.  A probe
-// reads one 32-byte sector (the four keys of the home bucket) and continues to
-// the next bucket only when the bucket is full without a match.  Most pairs miss
-// and finish after one sector.  Pairs with block 0 resident and at least two
-// blocks are appended to a compact hit list (warp-aggregated).
+// Phase 1 (k2_probe_first_group): every (r, w) pair probes block 0.  A probe reads
+// one 32-byte sector (the four keys of the home bucket) and continues to the next
+// bucket only when the bucket is full without a match.  Most pairs miss and finish
+// after one sector.  Pairs with block 0 resident and at least two blocks are
+// appended to a compact hit list (warp-aggregated).
 // Phase 2 (k2_probe_search): one thread per hit pair probes the last block
 // (fully cached prefixes finish there), then binary-searches [1, nb-1].
 #include "common.cuh"
@@ -44,63 +44,6 @@ __device__ __forceinline__ void block_add_stats(unsigned long long* stats, unsig
 }
 
 }  // namespace
-
-__global__ void __launch_bounds__(256) k2_probe_first(ProbeArgs a) {
-  __shared__ Bucket* s_tab[kMaxW];
-  __shared__ uint32_t s_lg[kMaxW];
-  if (block_error(a.err)) return;
-  for (int w = threadIdx.x; w < a.W; w += blockDim.x) {
-    s_tab[w] = a.desc[w].tab;
-    s_lg[w] = a.desc[w].log2nb;
-  }
-  __syncthreads();
-  const int64_t total = (int64_t)a.n * a.W;
-  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
-  unsigned long long probes = 0, reads = 0;
-  const int lane = threadIdx.x & 31;
-  // the loop trip count is uniform per warp so that ballots see every lane
-  const int64_t start = (int64_t)blockIdx.x * blockDim.x + (threadIdx.x & ~31);
-  for (int64_t base = start; base < total; base += stride) {
-    const int64_t p = base + lane;
-    bool hit_list = false;
-    int r = 0, w = 0;
-    if (p < total) {
-      r = (int)(p / a.W);
-      w = (int)(p - (int64_t)r * a.W);
-      const int32_t nb = a.nb[r];
-      uint16_t h = 0;
-      if (nb > 0) {
-        const uint64_t key = a.keys[a.kbase[r]];
-        InstDesc d;
-        d.tab = s_tab[w];
-        d.log2nb = s_lg[w];
-        uint32_t rd = 0;
-        const int res = table_contains(d, key, &rd);
-        probes += 1;
-        reads += rd;
-        if (res) {
-          h = 1;
-          hit_list = nb > 1;
-        }
-      }
-      a.H[p] = h;
-    }
-    const unsigned m = __ballot_sync(0xffffffffu, hit_list);
-    if (m) {
-      unsigned pos = 0;
-      const int leader = __ffs(m) - 1;
-      if (lane == leader) pos = atomicAdd(a.n_hits, (unsigned)__popc(m));
-      pos = __shfl_sync(0xffffffffu, pos, leader) + __popc(m & lanemask_lt());
-      if (hit_list) {
-        if ((int64_t)pos < a.hits_cap)
-          a.hits[pos] = make_int2(r, w);
-        else
-          set_error(a.err, MISAT_ERR_TABLE_FULL);
-      }
-    }
-  }
-  block_add_stats(a.stats, probes, reads);
-}
 
 // Phase 1, sub-warp layout: a group of S lanes (S = min(32, pow2 >= W)) owns one request;
 // its block-0 key is read once and broadcast, each lane probes instances w = lane, lane+S,
@@ -212,13 +155,88 @@ __global__ void __launch_bounds__(256) k2_probe_search(ProbeArgs a) {
   block_add_stats(a.stats_search, probes, reads);
 }
 
+// Phase 1 through the global index: a warp takes 32 requests, each lane looks up the
+// block-0 key of one of them (one lookup answers every instance), the masks go to shared
+// memory, and the warp then writes the 32 H rows (H = 1 where the bit is set) and the hit
+// pairs of requests with at least two blocks.
+__global__ void __launch_bounds__(256) k2_probe_first_gix(ProbeArgs a) {
+  extern __shared__ unsigned long long s_gm[];  // [warps][32][mw]
+  if (block_error(a.err)) return;
+  const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+  const uint32_t mw = a.gix.mw;
+  unsigned long long* sm = s_gm + (size_t)wid * 32 * mw;
+  unsigned long long probes = 0, reads = 0;
+  const int groups = (a.n + 31) >> 5;
+  const int wpb = blockDim.x >> 5;
+  for (int grp = blockIdx.x * wpb + wid; grp < groups; grp += gridDim.x * wpb) {
+    const int r = grp * 32 + lane;
+    int nb = 0;
+    int64_t slot = -1;
+    if (r < a.n) {
+      nb = a.nb[r];
+      if (nb > 0) {
+        uint32_t rd = 0;
+        slot = gix_find(a.gix, a.keys[a.kbase[r]], &rd);
+        probes += 1;
+        reads += rd;
+      }
+    }
+    int bits = 0;
+    for (uint32_t i = 0; i < mw; ++i) {
+      const unsigned long long m = slot >= 0 ? __ldg(a.gix.masks + (size_t)slot * mw + i) : 0ull;
+      sm[lane * mw + i] = m;
+      bits += __popcll(m);
+    }
+    // hit-list positions: one atomic per warp
+    const int nh = nb > 1 ? bits : 0;
+    int incl = nh;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int t = __shfl_up_sync(0xffffffffu, incl, o);
+      if (lane >= o) incl += t;
+    }
+    const int tot = __shfl_sync(0xffffffffu, incl, 31);
+    unsigned base = 0;
+    if (lane == 31 && tot) base = atomicAdd(a.n_hits, (unsigned)tot);
+    base = __shfl_sync(0xffffffffu, base, 31) + (unsigned)(incl - nh);
+    __syncwarp();
+    const int cnt = min(32, a.n - grp * 32);
+    for (int i = 0; i < cnt; ++i) {
+      const int ri = grp * 32 + i;
+      const bool list = __shfl_sync(0xffffffffu, nb, i) > 1;
+      unsigned pos = __shfl_sync(0xffffffffu, base, i);
+      const unsigned long long* mi = sm + i * mw;
+      uint16_t* row = a.H + (int64_t)ri * a.W;
+      for (int w0 = 0; w0 < a.W; w0 += 32) {
+        const int w = w0 + lane;
+        const bool bit = w < a.W && ((mi[w >> 6] >> (w & 63)) & 1ull);
+        if (w < a.W) row[w] = bit ? 1 : 0;
+        if (list) {
+          const unsigned bal = __ballot_sync(0xffffffffu, bit);
+          if (bit) {
+            const unsigned p = pos + __popc(bal & lanemask_lt());
+            if ((int64_t)p < a.hits_cap)
+              a.hits[p] = make_int2(ri, w);
+            else
+              set_error(a.err, MISAT_ERR_TABLE_FULL);
+          }
+          pos += __popc(bal);
+        }
+      }
+    }
+    __syncwarp();
+  }
+  block_add_stats(a.stats, probes, reads);
+}
+
 void launch_probe_first(const ProbeArgs& a, int num_sms, cudaStream_t st) {
   const int64_t total = (int64_t)a.n * a.W;
   if (total <= 0) return;
-  if (a.flat) {
-    int64_t blocks = (total + 255) / 256;
-    int grid = (int)(blocks < (int64_t)num_sms * 8 ? blocks : (int64_t)num_sms * 8);
-    k2_probe_first<<<grid, 256, 0, st>>>(a);
+  if (a.gix.keys) {
+    const int groups = (a.n + 31) / 32;
+    const int blocks = (groups + 7) / 8;
+    const int grid = blocks < num_sms * 8 ? blocks : num_sms * 8;
+    k2_probe_first_gix<<<grid, 256, 8 * 32 * a.gix.mw * sizeof(unsigned long long), st>>>(a);
     return;
   }
   int S = 1;

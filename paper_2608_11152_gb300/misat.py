@@ -26,7 +26,9 @@ _lib = C.CDLL(LIB_PATH)
 
 OK = 0
 ERR_INVALID_ARG, ERR_OOM, ERR_CUDA, ERR_STATE, ERR_TABLE_FULL, ERR_BATCH_TOO_LARGE = -1, -2, -3, -4, -5, -6
+ERR_INTERNAL = -7
 MODE_MISA_T, MODE_MISA, MODE_SESSION_ADMISSION, MODE_PLACEMENT_ONLY = 0, 1, 2, 3
+PREFIX_GLOBAL, PREFIX_PER_INSTANCE = 0, 1
 ADMIT_CONT, ADMIT_NEW, ADMIT_FOLLOW = 1, 2, 3
 HOLD_GLOBAL_CAP, HOLD_CLASS_CAP, HOLD_NO_ELIGIBLE, HOLD_PREFER_CACHE, HOLD_LEADER_HELD = 16, 17, 18, 19, 20
 
@@ -38,7 +40,7 @@ class misat_config(C.Structure):
                 ("rounds", C.c_int32), ("mode", C.c_int32), ("max_batch", C.c_int32), ("max_tokens", C.c_int64),
                 ("max_sessions", C.c_int32), ("hist_window", C.c_int32), ("min_obs", C.c_int32),
                 ("hold_delay_q", C.c_int64), ("prior_kbar_blocks", C.c_int64 * 3), ("prior_T_us", C.c_int64),
-                ("hash_seed", C.c_uint64), ("table_load", C.c_double)]
+                ("hash_seed", C.c_uint64), ("table_load", C.c_double), ("prefix_index", C.c_int32)]
 
 
 class misat_batch(C.Structure):
@@ -87,6 +89,9 @@ _SIG = {
     "misat_dump_counts": [_p, _p],
     "misat_dump_sessions": [_p, _p, _p, _p, _p, C.c_int64, C.POINTER(C.c_int64)],
     "misat_stats": [_p, C.POINTER(misat_batch_stats)],
+    "misat_global_info": [_p, C.POINTER(C.c_int32), C.POINTER(C.c_int64), C.POINTER(C.c_int64)],
+    "misat_global_dump": [_p, _p, _p, C.c_int64, C.POINTER(C.c_int64)],
+    "misat_global_rebuild": [_p],
     "misat_sync": [_p],
     "misat_checkpoint_save": [_p, C.POINTER(_p)],
     "misat_checkpoint_restore": [_p, _p],
@@ -151,7 +156,7 @@ class Router:
     def __init__(self, cap_blocks, *, max_batch, max_tokens, max_sessions=None, protected_frac_q16=58982,
                  rounds=4, mode=MODE_MISA_T, hold_delay_q=0, hist_window=256, min_obs=8,
                  prior_kbar=(64, 64, 64), prior_T_us=30_000_000, hash_seed=0x9E3779B97F4A7C15,
-                 table_load=0.75, stream=None):
+                 table_load=0.75, prefix_index=None, stream=None):
         import torch
 
         self._torch = torch
@@ -175,6 +180,8 @@ class Router:
         cfg.prior_T_us = int(prior_T_us)
         cfg.hash_seed = hash_seed
         cfg.table_load = table_load
+        cfg.prefix_index = PREFIX_GLOBAL if prefix_index is None else int(prefix_index)
+        self.prefix_index = cfg.prefix_index
         self.stream = stream if stream is not None else torch.cuda.current_stream()
         h = _p()
         _ck(_lib.misat_create(C.byref(cfg), _p(self.stream.cuda_stream), C.byref(h)), "misat_create")
@@ -324,6 +331,28 @@ class Router:
         s = misat_batch_stats()
         _ck(_lib.misat_stats(self._h, C.byref(s)), "misat_stats")
         return s
+
+    # ---- global prefix index (Sec. 4.5: block hash -> instances caching it)
+    def global_info(self):
+        """(mask words per key, slots, claimed slots) of the global prefix index."""
+        mw, slots, used = C.c_int32(0), C.c_int64(0), C.c_int64(0)
+        _ck(_lib.misat_global_info(self._h, C.byref(mw), C.byref(slots), C.byref(used)), "misat_global_info")
+        return mw.value, slots.value, used.value
+
+    def global_dump(self):
+        """Keys with a non-empty instance mask and their masks [n, mask words] (unordered)."""
+        mw = self.global_info()[0]
+        n = C.c_int64(0)
+        _ck(_lib.misat_global_dump(self._h, None, None, 0, C.byref(n)), "misat_global_dump")
+        cap = n.value + 16
+        keys = np.empty(cap, np.uint64)
+        masks = np.empty(cap * mw, np.uint64)
+        _ck(_lib.misat_global_dump(self._h, _nptr(keys), _nptr(masks), cap, C.byref(n)), "misat_global_dump")
+        k = n.value
+        return keys[:k], masks[: k * mw].reshape(k, mw)
+
+    def global_rebuild(self):
+        _ck(_lib.misat_global_rebuild(self._h), "misat_global_rebuild")
 
     def sync(self):
         _ck(_lib.misat_sync(self._h), "misat_sync")
