@@ -9,11 +9,18 @@
 // distance d), then a_j = carry G^{j+1} + s_j.
 //
 // Layout: one warp per request (dynamic work counter).  A chunk of 32 blocks is
-// 512 tokens = 2 KiB, read as four fully coalesced 512-byte warp loads of int4;
-// a prompt that does not start on a 16-byte boundary is realigned in registers
-// (funnel of the lane's int4 and its right neighbour's).  Lanes 4m..4m+3 hold the
-// four quarters of one block and combine their partial hashes with two xor
-// shuffles.  Keys are written coalesced at keys[floor(tok_off[r]/16) + j].
+// 512 tokens = 2 KiB, read as four fully coalesced 512-byte warp loads of int4
+// (the next chunk's loads are issued before the current one is hashed).  In
+// sub-row i of a chunk, lane 4m+q holds tokens 4q..4q+3 of block 8i+m.  A prompt
+// that does not start on a 16-byte boundary is realigned in registers: the
+// misalignment (0..3 words) is the same for the whole warp, so the chunk loop is
+// specialised on it and only the 1..3 words a lane needs from its right neighbour
+// are shuffled.  The four lanes of a block combine their partial XORs once per
+// chunk with a two-step reduce-scatter (lane 4m+q ends with block 8q+m), then one
+// shuffle moves block j to lane j for the scan.  Keys are written coalesced.
+//
+// The kernel is bound by integer issue (ten 64-bit mixes per block), so the
+// structure above is chosen to spend as few instructions as possible around them.
 #include <mutex>
 
 #include "common.cuh"
@@ -31,132 +38,156 @@ __host__ __device__ constexpr uint64_t gold_pow(int k) {
 
 constexpr unsigned kFull = 0xffffffffu;
 
-__device__ __forceinline__ int4 shfl_int4(int4 v, int src) {
-  int4 o;
-  o.x = __shfl_sync(kFull, v.x, src);
-  o.y = __shfl_sync(kFull, v.y, src);
-  o.z = __shfl_sync(kFull, v.z, src);
-  o.w = __shfl_sync(kFull, v.w, src);
-  return o;
-}
-
-__device__ __forceinline__ int4 shfl_down_int4(int4 v) {
-  int4 o;
-  o.x = __shfl_down_sync(kFull, v.x, 1);
-  o.y = __shfl_down_sync(kFull, v.y, 1);
-  o.z = __shfl_down_sync(kFull, v.z, 1);
-  o.w = __shfl_down_sync(kFull, v.w, 1);
-  return o;
-}
-
-// The four tokens at word offset `off` (0..3) of the 8-word window (cur, nxt).
-__device__ __forceinline__ int4 funnel(int4 cur, int4 nxt, int off) {
-  int4 t;
-  if (off == 1) {
-    t.x = cur.y; t.y = cur.z; t.z = cur.w; t.w = nxt.x;
-  } else if (off == 2) {
-    t.x = cur.z; t.y = cur.w; t.z = nxt.x; t.w = nxt.y;
-  } else {
-    t.x = cur.w; t.y = nxt.x; t.z = nxt.y; t.w = nxt.z;
-  }
-  return t;
-}
-
 __device__ __forceinline__ int4 load_tok4(const int4* base, int64_t idx, int64_t n_int4) {
   if (idx < n_int4) return ld_stream_v4(base + idx);
   return make_int4(0, 0, 0, 0);
+}
+
+// Per-lane constants of the chunk loop.
+struct LaneConst {
+  int lane;
+  int src;          // lane that holds block `lane` after the reduce-scatter
+  bool b0, b1;      // bits of the quarter index q = lane & 3
+  uint64_t pw;      // G^(lane+1): multiplier of the incoming carry for block `lane`
+  uint64_t addA;    // (2q+1) G: increment of the lane's first token pair
+  uint64_t addB;    // (2q+2) G: increment of its second pair
+};
+
+__device__ __forceinline__ LaneConst lane_const() {
+  LaneConst c;
+  c.lane = threadIdx.x & 31;
+  const int q = c.lane & 3;
+  c.src = 4 * (c.lane & 7) + (c.lane >> 3);
+  c.b0 = (q & 1) != 0;
+  c.b1 = (q & 2) != 0;
+  uint64_t pw = kGold;
+  for (int i = 0; i < c.lane; ++i) pw *= kGold;
+  c.pw = pw;
+  c.addA = (uint64_t)(2 * q + 1) * kGold;
+  c.addB = (uint64_t)(2 * q + 2) * kGold;
+  return c;
+}
+
+// The four tokens that start OFF words into `cur`, continued by `nxt`.
+template <int OFF>
+__device__ __forceinline__ int4 align_words(int4 cur, int4 nxt) {
+  if (OFF == 1) return make_int4(cur.y, cur.z, cur.w, nxt.x);
+  if (OFF == 2) return make_int4(cur.z, cur.w, nxt.x, nxt.y);
+  if (OFF == 3) return make_int4(cur.w, nxt.x, nxt.y, nxt.z);
+  return cur;
+}
+
+// The first OFF words of the int4 that follows this lane's `cur` in memory: lane l+1's
+// `cur`, or for lane 31 lane 0's `after` (the first int4 of the next sub-row).
+template <int OFF>
+__device__ __forceinline__ int4 next_words(int4 cur, int4 after, int lane) {
+  int4 nx = make_int4(0, 0, 0, 0);
+  const int src = (lane + 1) & 31;
+  const bool first = lane == 0;
+  if (OFF >= 1) nx.x = __shfl_sync(kFull, first ? after.x : cur.x, src);
+  if (OFF >= 2) nx.y = __shfl_sync(kFull, first ? after.y : cur.y, src);
+  if (OFF >= 3) nx.z = __shfl_sync(kFull, first ? after.z : cur.z, src);
+  return nx;
+}
+
+// Keys of one prompt of nb >= 1 full blocks whose first token is word OFF of int4 q0:
+// key j goes to out[j] for j < out_lim.
+template <int OFF>
+__device__ __forceinline__ void hash_chain(const int4* tok4, int64_t n_int4, int64_t q0, int32_t nb, uint64_t seed,
+                                           uint64_t* out, int64_t out_lim, const LaneConst& lc) {
+  const int lane = lc.lane;
+  uint64_t carry = seed;
+  const int n_chunks = (nb + 31) >> 5;
+  int4 v[4], ex = make_int4(0, 0, 0, 0);
+#pragma unroll
+  for (int i = 0; i < 4; ++i) v[i] = load_tok4(tok4, q0 + 32 * i + lane, n_int4);
+  if (OFF != 0 && lane == 0) ex = load_tok4(tok4, q0 + 128, n_int4);
+
+  for (int c = 0; c < n_chunks; ++c) {
+    // issue the next chunk's loads before this chunk is hashed
+    const bool more = (c + 1) < n_chunks;
+    const int64_t nbase = q0 + 128ll * (c + 1);
+    int4 vn[4], exn = make_int4(0, 0, 0, 0);
+#pragma unroll
+    for (int i = 0; i < 4; ++i) vn[i] = more ? load_tok4(tok4, nbase + 32 * i + lane, n_int4) : make_int4(0, 0, 0, 0);
+    if (OFF != 0 && more && lane == 0) exn = load_tok4(tok4, nbase + 128, n_int4);
+
+    // partial XOR of the lane's two pre-mixed token pairs, per sub-row
+    uint64_t p[4];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      int4 t = v[i];
+      if (OFF != 0) t = align_words<OFF>(v[i], next_words<OFF>(v[i], i < 3 ? v[i + 1] : ex, lane));
+      const uint64_t xa = (uint64_t)(uint32_t)t.x | ((uint64_t)(uint32_t)t.y << 32);
+      const uint64_t xb = (uint64_t)(uint32_t)t.z | ((uint64_t)(uint32_t)t.w << 32);
+      p[i] = mix64(xa + lc.addA) ^ mix64(xb + lc.addB);
+    }
+    // reduce-scatter over the quad: after the exchange with lane^1 a lane keeps the
+    // sub-rows with bit 0 = its q's bit 0, after lane^2 the sub-row i = q: block 8q + m
+    uint64_t k0 = lc.b0 ? p[1] : p[0], k1 = lc.b0 ? p[3] : p[2];
+    const uint64_t s0 = lc.b0 ? p[0] : p[1], s1 = lc.b0 ? p[2] : p[3];
+    k0 ^= __shfl_xor_sync(kFull, s0, 1);
+    k1 ^= __shfl_xor_sync(kFull, s1, 1);
+    uint64_t kq = lc.b1 ? k1 : k0;
+    const uint64_t sq = lc.b1 ? k0 : k1;
+    kq ^= __shfl_xor_sync(kFull, sq, 2);
+    // finishing mix, then block j moves to lane j
+    const uint64_t cmine = __shfl_sync(kFull, mix64(kq), lc.src);
+    const int cnt = min(32, nb - 32 * c);
+    uint64_t s = lane < cnt ? cmine : 0;
+    {
+      uint64_t t = __shfl_up_sync(kFull, s, 1);
+      if (lane >= 1) s += t * gold_pow(1);
+      t = __shfl_up_sync(kFull, s, 2);
+      if (lane >= 2) s += t * gold_pow(2);
+      t = __shfl_up_sync(kFull, s, 4);
+      if (lane >= 4) s += t * gold_pow(4);
+      t = __shfl_up_sync(kFull, s, 8);
+      if (lane >= 8) s += t * gold_pow(8);
+      t = __shfl_up_sync(kFull, s, 16);
+      if (lane >= 16) s += t * gold_pow(16);
+    }
+    const uint64_t av = carry * lc.pw + s;
+    uint64_t key = mix64(av ^ (uint64_t)(32 * c + lane + 1));
+    key += key < 2 ? 2 : 0;
+    const int64_t j = 32ll * c + lane;
+    if (lane < cnt && j < out_lim) out[j] = key;
+    carry = __shfl_sync(kFull, av, 31);
+#pragma unroll
+    for (int i = 0; i < 4; ++i) v[i] = vn[i];
+    ex = exn;
+  }
+}
+
+// One prompt: dispatch on its (warp-uniform) misalignment.
+__device__ __forceinline__ void hash_prompt(const int4* tok4, int64_t n_int4, int64_t t0, int32_t nb, uint64_t seed,
+                                            uint64_t* out, int64_t out_lim, const LaneConst& lc) {
+  const int64_t q0 = t0 >> 2;
+  switch ((int)(t0 & 3)) {
+    case 0: hash_chain<0>(tok4, n_int4, q0, nb, seed, out, out_lim, lc); break;
+    case 1: hash_chain<1>(tok4, n_int4, q0, nb, seed, out, out_lim, lc); break;
+    case 2: hash_chain<2>(tok4, n_int4, q0, nb, seed, out, out_lim, lc); break;
+    default: hash_chain<3>(tok4, n_int4, q0, nb, seed, out, out_lim, lc); break;
+  }
 }
 
 }  // namespace
 
 __global__ void __launch_bounds__(256) k1_block_hash(HashArgs a) {
   if (*a.err) return;
-  const int lane = threadIdx.x & 31;
-  const int q = lane & 3;
+  const LaneConst lc = lane_const();
   const int64_t n_int4 = (a.n_tokens + 3) >> 2;
   const int4* tok4 = reinterpret_cast<const int4*>(a.tokens);
-  // G^(lane+1): multiplier of the incoming carry for block `lane` of a chunk
-  uint64_t pw = kGold;
-  for (int i = 0; i < lane; ++i) pw *= kGold;
-  const uint64_t addA = (uint64_t)(2 * q + 1) * kGold;
-  const uint64_t addB = (uint64_t)(2 * q + 2) * kGold;
-
   while (true) {
     int r = 0;
-    if (lane == 0) r = (int)atomicAdd(a.work, 1u);
+    if (lc.lane == 0) r = (int)atomicAdd(a.work, 1u);
     r = __shfl_sync(kFull, r, 0);
     if (r >= a.n) break;
     const int64_t t0 = a.tok_off[r];
-    const int64_t t1 = a.tok_off[r + 1];
-    const int32_t nb = (int32_t)((t1 - t0) >> 4);
-    const int64_t kb = t0 >> 4;
+    const int32_t nb = (int32_t)((a.tok_off[r + 1] - t0) >> 4);
     if (nb <= 0) continue;
-    const int64_t q0 = t0 >> 2;
-    const int off = (int)(t0 & 3);
-    uint64_t carry = a.seed;
-    const int n_chunks = (nb + 31) >> 5;
-
-    int4 v[4], ex;
-#pragma unroll
-    for (int i = 0; i < 4; ++i) v[i] = load_tok4(tok4, q0 + 32 * i + lane, n_int4);
-    ex = (off != 0 && lane == 0) ? load_tok4(tok4, q0 + 128, n_int4) : make_int4(0, 0, 0, 0);
-
-    for (int c = 0; c < n_chunks; ++c) {
-      // prefetch the next chunk while this one is hashed
-      int4 vn[4], exn = make_int4(0, 0, 0, 0);
-      const bool more = (c + 1) < n_chunks;
-      const int64_t nbase = q0 + 128ll * (c + 1);
-#pragma unroll
-      for (int i = 0; i < 4; ++i) vn[i] = more ? load_tok4(tok4, nbase + 32 * i + lane, n_int4) : make_int4(0, 0, 0, 0);
-      if (more && off != 0 && lane == 0) exn = load_tok4(tok4, nbase + 128, n_int4);
-
-      // pre-mix XOR of block 8i + lane/4 after sub-iteration i (same in its 4 lanes); lane
-      // 4m + i' keeps the one of sub-iteration i' = lane % 4, i.e. block 8(lane%4) + lane/4
-      uint64_t pkeep = 0;
-#pragma unroll
-      for (int i = 0; i < 4; ++i) {
-        int4 t = v[i];
-        if (off != 0) {
-          int4 nxt = shfl_down_int4(v[i]);
-          int4 wrap = shfl_int4(i < 3 ? v[i + 1] : ex, 0);
-          if (lane == 31) nxt = wrap;
-          t = funnel(v[i], nxt, off);
-        }
-        // this lane holds tokens 4q..4q+3 of block 8i + lane/4 of the chunk
-        const uint64_t xa = (uint64_t)(uint32_t)t.x | ((uint64_t)(uint32_t)t.y << 32);
-        const uint64_t xb = (uint64_t)(uint32_t)t.z | ((uint64_t)(uint32_t)t.w << 32);
-        uint64_t p = mix64(xa + addA) ^ mix64(xb + addB);
-        p ^= __shfl_xor_sync(kFull, p, 1);
-        p ^= __shfl_xor_sync(kFull, p, 2);
-        if (q == i) pkeep = p;
-      }
-      // one finishing mix per lane, then block j moves to lane j (it sits on lane 4(j%8) + j/8)
-      const uint64_t cown = mix64(pkeep);
-      const uint64_t cmine = __shfl_sync(kFull, cown, 4 * (lane & 7) + (lane >> 3));
-      const int cnt = min(32, nb - 32 * c);
-      uint64_t s = lane < cnt ? cmine : 0;
-      {
-        uint64_t t = __shfl_up_sync(kFull, s, 1);
-        if (lane >= 1) s += t * gold_pow(1);
-        t = __shfl_up_sync(kFull, s, 2);
-        if (lane >= 2) s += t * gold_pow(2);
-        t = __shfl_up_sync(kFull, s, 4);
-        if (lane >= 4) s += t * gold_pow(4);
-        t = __shfl_up_sync(kFull, s, 8);
-        if (lane >= 8) s += t * gold_pow(8);
-        t = __shfl_up_sync(kFull, s, 16);
-        if (lane >= 16) s += t * gold_pow(16);
-      }
-      const uint64_t av = carry * pw + s;
-      uint64_t key = mix64(av ^ (uint64_t)(32 * c + lane + 1));
-      key += key < 2 ? 2 : 0;
-      const int64_t dst = kb + 32ll * c + lane;
-      if (lane < cnt && dst < a.keys_cap) a.keys[dst] = key;
-      carry = __shfl_sync(kFull, av, 31);
-#pragma unroll
-      for (int i = 0; i < 4; ++i) v[i] = vn[i];
-      ex = exn;
-    }
+    const int64_t kb = t0 >> 4;
+    hash_prompt(tok4, n_int4, t0, nb, a.seed, a.keys + kb, a.keys_cap - kb, lc);
   }
 }
 
@@ -254,65 +285,20 @@ __global__ void __launch_bounds__(256) k1na_hash(const int64_t* tok_off, const i
   if (scratch[1]) return;
   unsigned* work = reinterpret_cast<unsigned*>(scratch);
   const unsigned long long* off_r = scratch + 8;
-  const int lane = threadIdx.x & 31;
-  const int q = lane & 3;
+  const int64_t total = (int64_t)scratch[2];
+  const LaneConst lc = lane_const();
   const int64_t n_int4 = (n_tokens + 3) >> 2;
   const int4* tok4 = reinterpret_cast<const int4*>(tokens);
-  uint64_t pw = kGold;
-  for (int i = 0; i < lane; ++i) pw *= kGold;
-  const uint64_t addA = (uint64_t)(2 * q + 1) * kGold;
-  const uint64_t addB = (uint64_t)(2 * q + 2) * kGold;
   while (true) {
     int r = 0;
-    if (lane == 0) r = (int)atomicAdd(work, 1u);
+    if (lc.lane == 0) r = (int)atomicAdd(work, 1u);
     r = __shfl_sync(kFull, r, 0);
     if (r >= n) break;
     const int64_t t0 = tok_off[r];
     const int32_t nb = (int32_t)((tok_off[r + 1] - t0) >> 4);
     if (nb <= 0) continue;
     const int64_t kb = (int64_t)off_r[r];
-    const int64_t q0 = t0 >> 2;
-    const int off = (int)(t0 & 3);
-    uint64_t carry = seed;
-    const int n_chunks = (nb + 31) >> 5;
-    for (int c = 0; c < n_chunks; ++c) {
-      const int64_t base = q0 + 128ll * c;
-      int4 v[4];
-#pragma unroll
-      for (int i = 0; i < 4; ++i) v[i] = load_tok4(tok4, base + 32 * i + lane, n_int4);
-      const int4 ex = (off != 0 && lane == 0) ? load_tok4(tok4, base + 128, n_int4) : make_int4(0, 0, 0, 0);
-      uint64_t cmine = 0;
-#pragma unroll
-      for (int i = 0; i < 4; ++i) {
-        int4 t = v[i];
-        if (off != 0) {
-          int4 nxt = shfl_down_int4(v[i]);
-          const int4 wrap = shfl_int4(i < 3 ? v[i + 1] : ex, 0);
-          if (lane == 31) nxt = wrap;
-          t = funnel(v[i], nxt, off);
-        }
-        const uint64_t xa = (uint64_t)(uint32_t)t.x | ((uint64_t)(uint32_t)t.y << 32);
-        const uint64_t xb = (uint64_t)(uint32_t)t.z | ((uint64_t)(uint32_t)t.w << 32);
-        uint64_t p = mix64(xa + addA) ^ mix64(xb + addB);
-        p ^= __shfl_xor_sync(kFull, p, 1);
-        p ^= __shfl_xor_sync(kFull, p, 2);
-        const uint64_t cb = mix64(p);
-        const uint64_t got = __shfl_sync(kFull, cb, 4 * (lane & 7));
-        if ((lane >> 3) == i) cmine = got;
-      }
-      const int cnt = min(32, nb - 32 * c);
-      uint64_t s = lane < cnt ? cmine : 0;
-#pragma unroll
-      for (int d = 1; d < 32; d <<= 1) {
-        const uint64_t u = __shfl_up_sync(kFull, s, d);
-        if (lane >= d) s += u * gold_pow(d);
-      }
-      const uint64_t av = carry * pw + s;
-      uint64_t key = mix64(av ^ (uint64_t)(32 * c + lane + 1));
-      key += key < 2 ? 2 : 0;
-      if (lane < cnt) keys[kb + 32ll * c + lane] = key;
-      carry = __shfl_sync(kFull, av, 31);
-    }
+    hash_prompt(tok4, n_int4, t0, nb, seed, keys + kb, total - kb, lc);
   }
 }
 
