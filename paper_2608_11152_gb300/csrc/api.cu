@@ -115,8 +115,10 @@ struct misat_ctx {
   // global prefix index (MISAT_PREFIX_GLOBAL); its arrays are reallocated by rebuilds
   bool use_gix = false;
   GIndex gix{};
-  int2* d_units = nullptr;      // insert work list
+  int4* d_units = nullptr;      // insert work list (two int4 per unit)
   unsigned* d_units_n = nullptr;
+  ulonglong2* d_gnew = nullptr; // keys new to a table during a commit (global index pass)
+  unsigned* d_gnew_n = nullptr;
   int64_t units_cap = 0;
   int64_t keys_cap = 0;
   uint16_t* d_H = nullptr;
@@ -528,7 +530,7 @@ int misat_create(const misat_config* cfg, void* cuda_stream, misat_ctx** out) {
   const int bm_log2 = std::max(1, ceil_log2(2 * NB));
   const size_t n_tiles = (NB + kTileReq - 1) / kTileReq;
   if ((rc = dalloc_n(c, &c->d_meta, c->ml.words)) || (rc = dalloc_n(c, &c->d_keys, (size_t)c->keys_cap)) ||
-      (rc = dalloc_n(c, &c->d_units, (size_t)c->units_cap)) || (rc = dalloc_n(c, &c->d_units_n, 1)) ||
+      (rc = dalloc_n(c, &c->d_units, 2 * (size_t)c->units_cap)) || (rc = dalloc_n(c, &c->d_units_n, 1)) ||
       (rc = dalloc_n(c, &c->d_H, NB * Ws)) || (rc = dalloc_n(c, &c->d_hits, (size_t)c->hits_cap)) ||
       (rc = dalloc_n(c, &c->d_bm_key, (size_t)1 << bm_log2)) ||
       (rc = dalloc_n(c, &c->d_bm_val, (size_t)1 << bm_log2)) || (rc = dalloc_n(c, &c->d_tile, n_tiles * 3 * Ws)) ||
@@ -543,7 +545,8 @@ int misat_create(const misat_config* cfg, void* cuda_stream, misat_ctx** out) {
       (rc = dalloc_n(c, &c->ia.N_wb, 3 * Ws)) || (rc = dalloc_n(c, &c->ia.kbar_w, Ws)) ||
       (rc = dalloc_n(c, &c->ia.tot, Ws)) || (rc = dalloc_n(c, &c->ia.gh, Ws)) || (rc = dalloc_n(c, &c->ia.ch, 3 * Ws)) ||
       (rc = dalloc_n(c, &c->ia.delta, 3 * Ws)) || (rc = dalloc_n(c, &c->ia.backlog_k, Ws)) ||
-      (rc = dalloc_n(c, &c->ia.prefill, Ws)) || (rc = dalloc_n(c, &c->d_backlog, Ws)) ||
+      (rc = dalloc_n(c, &c->ia.prefill, Ws)) || (rc = dalloc_n(c, &c->ia.live, 2)) ||
+      (rc = dalloc_n(c, &c->d_backlog, Ws)) ||
       (rc = dalloc_n(c, &c->d_tokcost, Ws)) || (rc = dalloc_n(c, &c->d_contraction, Ws)) ||
       (rc = dalloc_n(c, &c->d_prot, 3 * Ws)) || (rc = dalloc_n(c, &c->d_theta, 2 * Ws)) ||
       (rc = dalloc_n(c, &c->d_active, Ws)) || (rc = dalloc_n(c, &c->d_onew, 1)) ||
@@ -587,6 +590,7 @@ int misat_create(const misat_config* cfg, void* cuda_stream, misat_ctx** out) {
     for (int w = 0; w < W; ++w) total_cap += c->cap[w];
     total_cap = std::min<int64_t>(total_cap, (int64_t)1 << 26);
     if ((rc = gix_alloc(c, buckets_log2_for(std::max<int64_t>(total_cap, 1024), kGixLoad)))) return fail(rc);
+    if ((rc = dalloc_n(c, &c->d_gnew, (size_t)c->keys_cap)) || (rc = dalloc_n(c, &c->d_gnew_n, 1))) return fail(rc);
   }
   if (cudaStreamSynchronize(c->stream) != cudaSuccess) return fail(MISAT_ERR_CUDA);
   *out = c;
@@ -823,6 +827,9 @@ int misat_commit(misat_ctx* c) {
     ia.new_keys = c->stats_ptr() + 18;
     ia.err = c->err_ptr();
     ia.gix = gix_or_null(c);
+    ia.gnew = c->d_gnew;
+    ia.n_gnew = c->d_gnew_n;
+    ia.gnew_cap = c->keys_cap;
     launch_insert(ia, c->num_sms, st);
     c->mark(9);
     SessUpdateArgs sa{n, c->rq, c->sess, c->d_prot, c->err_ptr()};
@@ -1018,6 +1025,9 @@ int misat_load_chains(misat_ctx* c, int32_t n_chains, const int64_t* tok_off, co
   ia.new_keys = c->stats_ptr() + 21;
   ia.err = c->err_ptr();
   ia.gix = gix_or_null(c);
+  ia.gnew = c->d_gnew;
+  ia.n_gnew = c->d_gnew_n;
+  ia.gnew_cap = c->keys_cap;
   launch_insert(ia, c->num_sms, st);
   CK(cudaGetLastError());
   rc = load_common_evict(c);

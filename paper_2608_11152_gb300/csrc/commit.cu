@@ -65,20 +65,54 @@ __device__ __forceinline__ int table_insert(const InstDesc& d, uint64_t key, uin
 // ---------------------------------------------------------------------------
 // Insert.  Work is listed first: every request with an instance contributes one unit per
 // kUnitBlocks of its blocks, so that the insert kernel touches only admitted keys and a
-// long prompt is spread over many warps.  A warp then inserts one unit: lane l takes blocks
-// l, l+32, l+64, l+96 of it and issues all four home-bucket reads before the first atomic;
-// a key already present costs one fire-and-forget atomicMax on its meta, a new one a CAS.
-// The order of the units is free: the final key set and metas do not depend on it.
+// long prompt is spread over many warps.  A unit is a self-contained 32-byte record
+// (pointer to its first key, the instance table, the tick of its request, first depth,
+// instance, table size, block count), so a warp reaches its keys in one dependent load
+// instead of walking request -> instance -> table descriptor.  A warp then inserts one unit:
+// lane l takes blocks l, l+32, l+64, l+96 of it and issues all four home-bucket reads
+// before the first atomic; a key already present costs one fire-and-forget atomicMax on
+// its meta, a new one a CAS.  While those are in flight the warp already loads its next
+// unit's record and keys (software pipelining over the warp's units).  The order of the
+// units is free: the final key set and metas do not depend on it.
 constexpr int kIns = 4;
 constexpr int kUnitBlocks = 32 * kIns;
 constexpr int kInsThreads = 256;
 
+struct UnitRec {
+  const unsigned long long* keys;  // key of block j0 (lane l, k: keys[l + 32k])
+  Bucket* tab;
+  uint64_t mhi;                    // seq << 36 | arrival << 16 of the request's tick
+  int32_t j0;                      // depth of the first block
+  int32_t w;
+  uint32_t log2nb;
+  int32_t cnt;                     // blocks in the unit, 1..kUnitBlocks
+};
+
+__device__ __forceinline__ UnitRec load_unit(const int4* units, int64_t u) {
+  const int4 x = __ldg(units + 2 * u), y = __ldg(units + 2 * u + 1);
+  UnitRec r;
+  r.keys = reinterpret_cast<const unsigned long long*>(((uint64_t)(uint32_t)x.y << 32) | (uint32_t)x.x);
+  r.tab = reinterpret_cast<Bucket*>(((uint64_t)(uint32_t)x.w << 32) | (uint32_t)x.z);
+  r.mhi = ((uint64_t)(uint32_t)y.y << 32) | (uint32_t)y.x;
+  r.j0 = y.z;
+  r.w = y.w & 0xffff;
+  r.log2nb = ((uint32_t)y.w >> 16) & 0xff;
+  r.cnt = (int32_t)((uint32_t)y.w >> 24) + 1;
+  return r;
+}
+
+__device__ __forceinline__ void load_unit_keys(const UnitRec& u, int lane, uint64_t key[kIns]) {
+#pragma unroll
+  for (int k = 0; k < kIns; ++k) key[k] = lane + 32 * k < u.cnt ? __ldg(u.keys + lane + 32 * k) : 0;
+}
+
 __global__ void __launch_bounds__(256) k4_units(InsertArgs a) {
   const int r = blockIdx.x * blockDim.x + threadIdx.x;
   const int lane = threadIdx.x & 31;
-  int u = 0;
+  int u = 0, c = 0, w = 0;
   if (r < a.n && *a.err == 0 && a.inst[r] >= 0) {
-    int c = a.nb[r];
+    w = a.inst[r];
+    c = a.nb[r];
     if (a.max_blocks && a.max_blocks[r] < c) c = a.max_blocks[r];
     u = (c + kUnitBlocks - 1) / kUnitBlocks;
   }
@@ -93,11 +127,27 @@ __global__ void __launch_bounds__(256) k4_units(InsertArgs a) {
   unsigned base = 0;
   if (lane == 31) base = atomicAdd(a.n_units, (unsigned)tot);
   base = __shfl_sync(kFull, base, 31) + (unsigned)(incl - u);
+  if (u == 0) return;
+  const InstDesc d = a.desc[w];
+  const uint64_t seq = a.meta_seq ? a.meta_seq[r] : a.seq;
+  const uint64_t arr = a.meta_seq ? (uint64_t)a.meta_arr[r] : (uint64_t)r;
+  const uint64_t mhi = pack_meta(seq, arr, 0);  // meta of depth j = mhi - j
+  const uint64_t kp = reinterpret_cast<uint64_t>(a.keys + a.kbase[r]);
+  const uint64_t tp = reinterpret_cast<uint64_t>(d.tab);
+  int4* units = reinterpret_cast<int4*>(a.units);
   for (int i = 0; i < u; ++i) {
-    if ((int64_t)base + i < a.units_cap)
-      a.units[base + i] = make_int2(r, i);
-    else
+    if ((int64_t)base + i >= a.units_cap) {
       set_error(a.err, MISAT_ERR_TABLE_FULL);
+      break;
+    }
+    const int j0 = i * kUnitBlocks;
+    const int cnt = min(kUnitBlocks, c - j0);
+    const uint64_t k0 = kp + 8ull * (uint64_t)j0;
+    units[2 * ((int64_t)base + i)] = make_int4((int)(uint32_t)k0, (int)(uint32_t)(k0 >> 32), (int)(uint32_t)tp,
+                                               (int)(uint32_t)(tp >> 32));
+    units[2 * ((int64_t)base + i) + 1] =
+        make_int4((int)(uint32_t)mhi, (int)(uint32_t)(mhi >> 32), j0,
+                  (int)((uint32_t)w | (d.log2nb << 16) | ((uint32_t)(cnt - 1) << 24)));
   }
 }
 
@@ -108,41 +158,41 @@ __global__ void __launch_bounds__(kInsThreads, 3) k4_insert(InsertArgs a) {
   __syncthreads();
   const int lane = threadIdx.x & 31;
   unsigned long long nnew = 0;
-  long long gclaim = 0;
+  const int4* units = reinterpret_cast<const int4*>(a.units);
   const int64_t n_units = min((int64_t)__ldcg(a.n_units), a.units_cap);
   const int64_t warps = (int64_t)gridDim.x * (blockDim.x >> 5);
-  for (int64_t u = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); u < n_units; u += warps) {
-    const int2 un = __ldg(a.units + u);
-    const int r = un.x;
-    const int w = __ldg(a.inst + r);
-    int c = __ldg(a.nb + r);
-    if (a.max_blocks) c = min(c, __ldg(a.max_blocks + r));
-    const int64_t kb = __ldg(a.kbase + r);
-    const uint64_t mseq = a.meta_seq ? __ldg(a.meta_seq + r) : a.seq;
-    const uint64_t marr = a.meta_seq ? __ldg(a.meta_arr + r) : (uint64_t)r;
-    const InstDesc d = a.desc[w];
-    const int j0 = un.y * kUnitBlocks + lane;
-    uint64_t key[kIns];
+  int64_t u = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+  UnitRec cur{};
+  uint64_t key[kIns];
+  if (u < n_units) {
+    cur = load_unit(units, u);
+    load_unit_keys(cur, lane, key);
+  }
+  for (; u < n_units; u += warps) {
+    // home-bucket reads of this unit's keys
     uint32_t hb[kIns];
     unsigned long long kk[kIns][4];
 #pragma unroll
     for (int k = 0; k < kIns; ++k) {
-      const int j = j0 + 32 * k;
-      key[k] = j < c ? __ldg(reinterpret_cast<const unsigned long long*>(a.keys) + kb + j) : 0;
+      hb[k] = home_bucket(key[k], cur.log2nb);
+      if (lane + 32 * k < cur.cnt) ld_bucket_keys_cg(cur.tab + hb[k], kk[k]);
     }
-#pragma unroll
-    for (int k = 0; k < kIns; ++k) {
-      hb[k] = home_bucket(key[k], d.log2nb);
-      if (j0 + 32 * k < c) ld_bucket_keys_cg(d.tab + hb[k], kk[k]);
+    // the next unit's record and keys, while the buckets are in flight
+    UnitRec nxt{};
+    uint64_t nkey[kIns] = {0, 0, 0, 0};
+    if (u + warps < n_units) {
+      nxt = load_unit(units, u + warps);
+      load_unit_keys(nxt, lane, nkey);
     }
+    const InstDesc d{cur.tab, cur.log2nb, 0, 0};
     unsigned cnt = 0;
     int isnew[kIns];
 #pragma unroll
     for (int k = 0; k < kIns; ++k) {
-      const int j = j0 + 32 * k;
+      const int j = lane + 32 * k;
       isnew[k] = 0;
-      if (j < c) {
-        const int res = table_insert_at(d, key[k], pack_meta(mseq, marr, (uint64_t)j), hb[k], kk[k]);
+      if (j < cur.cnt) {
+        const int res = table_insert_at(d, key[k], cur.mhi - (uint64_t)(cur.j0 + j), hb[k], kk[k]);
         if (res < 0)
           set_error(a.err, MISAT_ERR_TABLE_FULL);
         else
@@ -150,39 +200,63 @@ __global__ void __launch_bounds__(kInsThreads, 3) k4_insert(InsertArgs a) {
       }
       cnt += __popc(__ballot_sync(kFull, isnew[k]));
     }
-    if (a.gix.keys) {
-      // a key new to instance w gets bit w in the global index
+    if (a.gix.keys && cnt) {
+      // keys new to instance w are listed for the global-index pass (one slot range per warp)
+      unsigned base = 0;
+      if (lane == 0) base = atomicAdd(a.n_gnew, cnt);
+      base = __shfl_sync(kFull, base, 0);
 #pragma unroll
       for (int k = 0; k < kIns; ++k) {
-        if (!isnew[k]) continue;
-        const int g = gix_set(a.gix, key[k], w);
-        if (g < 0)
-          set_error(a.err, MISAT_ERR_TABLE_FULL);
-        else
-          gclaim += g;
+        const unsigned bal = __ballot_sync(kFull, isnew[k]);
+        if (isnew[k]) {
+          const unsigned pos = base + __popc(bal & lanemask_lt());
+          if ((int64_t)pos < a.gnew_cap)
+            a.gnew[pos] = make_ulonglong2((unsigned long long)key[k], (unsigned long long)cur.w);
+          else
+            set_error(a.err, MISAT_ERR_TABLE_FULL);
+        }
+        base += __popc(bal);
       }
     }
     if (lane == 0 && cnt) {
-      atomicAdd(&s_new[w], cnt);
+      atomicAdd(&s_new[cur.w], cnt);
       nnew += cnt;
     }
+    cur = nxt;
+#pragma unroll
+    for (int k = 0; k < kIns; ++k) key[k] = nkey[k];
   }
   const long long tot = block_sum((long long)nnew);
   if (threadIdx.x == 0 && tot) atomicAdd(a.new_keys, (unsigned long long)tot);
-  if (a.gix.keys) {
-    const long long gt = block_sum(gclaim);
-    if (threadIdx.x == 0 && gt) atomicAdd(a.gix.used, (unsigned long long)gt);
-  }
   __syncthreads();
   for (int i = threadIdx.x; i < a.n_inst; i += blockDim.x)
     if (s_new[i]) atomic_add_i64(&a.size[i], (long long)s_new[i]);
 }
 
+// Global index pass: bit w for every key new to instance w, one thread per listed key.
+__global__ void __launch_bounds__(256) k4_gix_insert(InsertArgs a) {
+  if (block_error(a.err)) return;
+  const int64_t n = min((int64_t)__ldcg(a.n_gnew), a.gnew_cap);
+  long long claimed = 0;
+  for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x) {
+    const ulonglong2 e = a.gnew[i];
+    const int g = gix_set(a.gix, e.x, (int)e.y);
+    if (g < 0)
+      set_error(a.err, MISAT_ERR_TABLE_FULL);
+    else
+      claimed += g;
+  }
+  const long long tot = block_sum(claimed);
+  if (threadIdx.x == 0 && tot) atomicAdd(a.gix.used, (unsigned long long)tot);
+}
+
 void launch_insert(const InsertArgs& a, int num_sms, cudaStream_t st) {
   if (a.n <= 0) return;
   cudaMemsetAsync(a.n_units, 0, sizeof(unsigned), st);
+  if (a.gix.keys) cudaMemsetAsync(a.n_gnew, 0, sizeof(unsigned), st);
   k4_units<<<(a.n + 255) / 256, 256, 0, st>>>(a);
   k4_insert<<<num_sms * 3, kInsThreads, 0, st>>>(a);  // resident CTAs: 3 per SM
+  if (a.gix.keys) k4_gix_insert<<<num_sms * 8, 256, 0, st>>>(a);
 }
 
 __global__ void __launch_bounds__(256) k4_insert_entries(EntryInsertArgs a) {

@@ -25,6 +25,7 @@ constexpr uint32_t kSessDead = 3;       // finished; slot reusable
 constexpr uint8_t kStUnresolved = 0;
 constexpr uint8_t kStResolved = 1;
 constexpr uint8_t kStFollower = 2;
+constexpr uint8_t kStHeld = 3;  // leader with no eligible instance: held for the rest of the batch
 
 // One bucket of an instance's resident-block table: four keys in one 32-byte
 // sector (what a probe reads) followed by their four metas (what a commit

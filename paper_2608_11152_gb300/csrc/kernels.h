@@ -33,7 +33,7 @@ struct ReqArrays {
   uint8_t* sst;         // session state at batch start (0 absent, 1 protected, 2 released)
   int32_t* sinst;       // protected / last instance
   int32_t* leader;      // first request of the session in the batch
-  uint8_t* status;      // kStUnresolved / kStResolved / kStFollower
+  uint8_t* status;      // kStUnresolved / kStResolved / kStFollower / kStHeld
   int32_t* choice;      // this round's choice of an unresolved leader needing headroom
   uint8_t* last_reason; // hold reason if it stays unresolved
   int32_t* inst;        // decision (internal copy)
@@ -54,6 +54,7 @@ struct InstArrays {
   int64_t* backlog_k;   // [W] in-batch backlog
   unsigned long long* prefill;  // [W] admitted prefill tokens of the current round
   long long* U;         // [W] upper bound of new keys of the pending commit
+  int32_t* live;        // [2]: [0] the current round runs, [1] ADMIT_CONT of the round
 };
 
 // ---- K2 ----
@@ -150,7 +151,7 @@ void launch_finalize(const FinalizeArgs& a, cudaStream_t st);
 struct InsertArgs {
   const InstDesc* desc;
   int32_t n;
-  int2* units;                 // work list (request, unit): up to 128 blocks per unit
+  int4* units;                 // work list: 32-byte unit records (2 int4), up to 128 blocks each
   unsigned* n_units;           // units listed (zeroed by the launcher)
   int64_t units_cap;
   const int32_t* nb;
@@ -166,6 +167,9 @@ struct InsertArgs {
   unsigned long long* new_keys;
   int32_t* err;
   GIndex gix;                  // mirrored when gix.keys != NULL
+  ulonglong2* gnew;            // keys new to an instance table, (key, instance), for the
+  unsigned* n_gnew;            //   global index pass (zeroed by the launcher)
+  int64_t gnew_cap;
 };
 void launch_insert(const InsertArgs& a, int num_sms, cudaStream_t st);
 

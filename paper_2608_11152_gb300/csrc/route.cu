@@ -113,6 +113,10 @@ void launch_prologue(const PrologueArgs& a, cudaStream_t st) {
 // K3a caps, one thread per instance (Sec. 4.1; Eqs. 9-10 MISA; Eqs. 11, 13 MISA-T).
 __global__ void __launch_bounds__(1024) k3_caps(CapsArgs a) {
   if (block_error(a.err)) return;
+  if (threadIdx.x == 0) {
+    a.ia.live[0] = 1;  // the first selection round always runs
+    a.ia.live[1] = 0;
+  }
   for (int w = threadIdx.x; w < a.W; w += blockDim.x) {
     int64_t N[3];
     int64_t sumN = 0, tot = 0;
@@ -176,103 +180,115 @@ __global__ void __launch_bounds__(1024) k3_caps(CapsArgs a) {
 
 void launch_caps(const CapsArgs& a, cudaStream_t st) { k3_caps<<<1, 1024, 0, st>>>(a); }
 
+// Whether the current selection round runs (block-uniform read of the round flag).
+__device__ __forceinline__ bool round_live(const RoundArgs& a) {
+  return *(volatile const int32_t*)a.ia.live != 0;
+}
+
 // ---------------------------------------------------------------------------
-// K3b score: one warp per unresolved leader.  Cost of Eq. (1) in fixed point,
-// cost = backlog_k[w] + (L_r - 16 H_rw) * tokcost[w]; eligibility of Eq. (6) with the
-// class cap of Sec. 4.2 (headroom at round start); argmin (cost, w) by warp shuffles.
-// A session protected on its choice is admitted here (ADMIT_CONT); a released session
-// may prefer to wait for its cached instance (Eq. 7).
+// K3b score: a group of G lanes per unresolved leader (G = 4..32 with W: each lane takes
+// 8-instance chunks of the H row, so a group reads its row as one coalesced segment).
+// Cost of Eq. (1) in fixed point, cost = backlog_k[w] + (L_r - 16 H_rw) * tokcost[w];
+// eligibility of Eq. (6) with the class cap of Sec. 4.2 (headroom at round start, as a
+// per-class byte map in shared memory); argmin (cost, w) and argmax (H, w) (ties to the
+// lower instance) by log2(G) shuffle steps inside the group.  A session protected on its
+// choice is admitted here (ADMIT_CONT); a released session may prefer to wait for its
+// cached instance (Eq. 7).
+template <int G>
 __global__ void __launch_bounds__(256) k3_score(RoundArgs a) {
   extern __shared__ unsigned char smem[];
   int64_t* s_bk = reinterpret_cast<int64_t*>(smem);
   int64_t* s_tc = s_bk + a.W;
   int32_t* s_gh = reinterpret_cast<int32_t*>(s_tc + a.W);
-  int32_t* s_ch = s_gh + a.W;  // [W*3]
-  if (block_error(a.err)) return;
+  int32_t* s_ch = s_gh + a.W;                                     // [W*3]
+  uint8_t* s_el = reinterpret_cast<uint8_t*>(s_ch + 3 * a.W);     // [3][W]: headroom on w
+  if (block_error(a.err) || !round_live(a)) return;
   for (int w = threadIdx.x; w < a.W; w += blockDim.x) {
     s_bk[w] = a.ia.backlog_k[w];
     s_tc[w] = a.tokcost[w];
-    s_gh[w] = a.ia.gh[w];
-    s_ch[w * 3 + 0] = a.ia.ch[w * 3 + 0];
-    s_ch[w * 3 + 1] = a.ia.ch[w * 3 + 1];
-    s_ch[w * 3 + 2] = a.ia.ch[w * 3 + 2];
+    const int32_t gh = a.ia.gh[w];
+    s_gh[w] = gh;
+#pragma unroll
+    for (int b = 0; b < 3; ++b) {
+      const int32_t ch = a.ia.ch[w * 3 + b];
+      s_ch[w * 3 + b] = ch;
+      s_el[b * a.W + w] = (gh > 0 && ch > 0) ? 1 : 0;
+    }
   }
   __syncthreads();
   const int lane = threadIdx.x & 31;
-  const int warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
-  const int nwarps = (gridDim.x * blockDim.x) >> 5;
-  // the next request's fields and first H values are loaded while this one is reduced
-  constexpr int kPre = 4;  // H values per lane prefetched (instances lane + 32 i, i < kPre)
-  struct Next {
-    uint8_t st, b, sst;
-    int sinst;
-    int32_t L;
-    uint16_t h[kPre];
-  };
-  auto fetch = [&](int rr, Next& x) {
-    x.st = rr < a.n ? a.rq.status[rr] : kStResolved;
-    if (x.st != kStUnresolved) return;
-    x.b = a.rq.cls[rr];
-    x.sst = a.rq.sst[rr];
-    x.sinst = a.rq.sinst[rr];
-    x.L = a.rq.L[rr];
-    const uint16_t* Hr = a.H + (int64_t)rr * a.W;
-#pragma unroll
-    for (int i = 0; i < kPre; ++i) x.h[i] = (lane + 32 * i < a.W) ? Hr[lane + 32 * i] : 0;
-  };
-  Next nx;
-  fetch(warp, nx);
-  for (int r = warp; r < a.n; r += nwarps) {
-    const Next cur = nx;
-    fetch(r + nwarps, nx);
-    if (cur.st != kStUnresolved) continue;
-    const int b = cur.b;
-    const uint8_t sst = cur.sst;
-    const int pw = sst == kSessProtected ? cur.sinst : -1;
-    const int64_t Lr = cur.L;
+  const int gl = lane & (G - 1);                 // lane within the group
+  const unsigned gmask = G == 32 ? kFull : (((1u << G) - 1) << (lane & ~(G - 1)));
+  const int64_t gid = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) / G;
+  const int64_t ngroups = ((int64_t)gridDim.x * blockDim.x) / G;
+  const int chunks = (a.W + 7) >> 3;
+  const bool row_vec = (a.W & 7) == 0;           // H rows 16-byte aligned
+  for (int64_t rr = gid; rr < a.n; rr += ngroups) {
+    const int r = (int)rr;
+    if (a.rq.status[r] != kStUnresolved) continue;  // uniform within the group
+    const int b = a.rq.cls[r];
+    const uint8_t sst = a.rq.sst[r];
+    const int pw = sst == kSessProtected ? a.rq.sinst[r] : -1;
+    const int64_t Lr = a.rq.L[r];
     const uint16_t* Hr = a.H + (int64_t)r * a.W;
+    const uint8_t* el = s_el + b * a.W;
     int64_t best_c = INT64_MAX;
     int best_w = INT32_MAX;
     int hmax = -1, whit = INT32_MAX;
-    auto visit = [&](int w, int h) {
-      const bool elig = (w == pw) || (s_gh[w] > 0 && s_ch[w * 3 + b] > 0);
-      if (elig) {
-        const int64_t cost = s_bk[w] + (Lr - 16 * (int64_t)h) * s_tc[w];
-        if (cost < best_c) {
-          best_c = cost;
-          best_w = w;
+    for (int ck = gl; ck < chunks; ck += G) {
+      const int w0 = ck * 8;
+      uint16_t h[8];
+      if (row_vec) {
+        const uint4 v = *reinterpret_cast<const uint4*>(Hr + w0);
+        h[0] = (uint16_t)v.x; h[1] = (uint16_t)(v.x >> 16);
+        h[2] = (uint16_t)v.y; h[3] = (uint16_t)(v.y >> 16);
+        h[4] = (uint16_t)v.z; h[5] = (uint16_t)(v.z >> 16);
+        h[6] = (uint16_t)v.w; h[7] = (uint16_t)(v.w >> 16);
+      } else {
+#pragma unroll
+        for (int i = 0; i < 8; ++i) h[i] = w0 + i < a.W ? Hr[w0 + i] : 0;
+      }
+#pragma unroll
+      for (int i = 0; i < 8; ++i) {
+        const int w = w0 + i;
+        if (w >= a.W) break;
+        if (w == pw || el[w]) {
+          const int64_t cost = s_bk[w] + (Lr - 16 * (int64_t)h[i]) * s_tc[w];
+          if (cost < best_c) {
+            best_c = cost;
+            best_w = w;
+          }
+        }
+        if ((int)h[i] > hmax) {
+          hmax = h[i];
+          whit = w;
         }
       }
-      if (h > hmax) {
-        hmax = h;
-        whit = w;
-      }
-    };
+    }
 #pragma unroll
-    for (int i = 0; i < kPre; ++i)
-      if (lane + 32 * i < a.W) visit(lane + 32 * i, cur.h[i]);
-    for (int w = lane + 32 * kPre; w < a.W; w += 32) visit(w, Hr[w]);
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
-      const int64_t oc = __shfl_xor_sync(kFull, best_c, o);
-      const int ow = __shfl_xor_sync(kFull, best_w, o);
+    for (int o = G / 2; o > 0; o >>= 1) {
+      const int64_t oc = __shfl_xor_sync(gmask, best_c, o, G);
+      const int ow = __shfl_xor_sync(gmask, best_w, o, G);
       if (oc < best_c || (oc == best_c && ow < best_w)) {
         best_c = oc;
         best_w = ow;
       }
-      const int oh = __shfl_xor_sync(kFull, hmax, o);
-      const int owh = __shfl_xor_sync(kFull, whit, o);
+      const int oh = __shfl_xor_sync(gmask, hmax, o, G);
+      const int owh = __shfl_xor_sync(gmask, whit, o, G);
       if (oh > hmax || (oh == hmax && owh < whit)) {
         hmax = oh;
         whit = owh;
       }
     }
-    if (lane == 0) {
+    if (gl == 0) {
       a.rq.hmax[r] = hmax < 0 ? 0 : hmax;
       int choice = -1;
       uint8_t reason = 0;
       if (best_w == INT32_MAX) {
+        // no instance has headroom: headroom only shrinks over the rounds and protection
+        // is fixed by the snapshot, so no later round can admit it
         reason = MISAT_HOLD_NO_ELIGIBLE;
+        a.rq.status[r] = kStHeld;
       } else {
         choice = best_w;
         if (sst == kSessReleased && hmax > 0) {
@@ -293,6 +309,7 @@ __global__ void __launch_bounds__(256) k3_score(RoundArgs a) {
         a.rq.reason[r] = MISAT_ADMIT_CONT;
         a.rq.choice[r] = -1;
         atomicAdd(&a.ia.prefill[choice], (unsigned long long)(Lr - 16 * (int64_t)Hr[choice]));
+        atomicAdd(&a.ia.live[1], 1);
       } else {
         a.rq.choice[r] = choice;
         if (choice < 0) a.rq.last_reason[r] = reason;
@@ -309,7 +326,7 @@ __global__ void __launch_bounds__(256) k3_score(RoundArgs a) {
 // and sum_b' min(c_{i,b'}, H_{w,b'}) < G_w -- exactly the sequential walk of Eq. (6).
 __global__ void __launch_bounds__(256) k4_tile_count(RoundArgs a) {
   extern __shared__ int32_t s_cnt[];
-  if (block_error(a.err)) return;
+  if (block_error(a.err) || !round_live(a)) return;
   const int nb = 3 * a.W;
   for (int k = threadIdx.x; k < nb; k += blockDim.x) s_cnt[k] = 0;
   __syncthreads();
@@ -331,7 +348,7 @@ __global__ void __launch_bounds__(256) k4_tile_count(RoundArgs a) {
 // scanned across warps, then each warp rewrites its stripe with running prefixes.
 __global__ void __launch_bounds__(1024) k4_tile_scan(RoundArgs a) {
   __shared__ int32_t s_sum[32][33];
-  if (block_error(a.err)) return;
+  if (block_error(a.err) || !round_live(a)) return;
   const int nb = 3 * a.W;
   const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
   const int col = blockIdx.x * 32 + lane;
@@ -364,56 +381,79 @@ __global__ void __launch_bounds__(1024) k4_tile_scan(RoundArgs a) {
 
 __global__ void __launch_bounds__(32) k4_admit(RoundArgs a) {
   extern __shared__ int32_t s_cnt[];
-  if (block_error(a.err)) return;
+  if (block_error(a.err) || !round_live(a)) return;
   const int nb = 3 * a.W;
   const int t = blockIdx.x;
   const int lane = threadIdx.x;
+  constexpr int kC = kTile / 32;  // chunks of 32 requests per tile
   for (int k = lane; k < nb; k += 32) s_cnt[k] = a.tile_counts[(int64_t)t * nb + k];
+  // every load of the tile is issued before the in-order walk: the choosers, then the
+  // headroom of their instances
+  bool need[kC];
+  int w[kC], b[kC], G[kC], h0[kC], h1[kC], h2[kC];
+#pragma unroll
+  for (int c = 0; c < kC; ++c) {
+    const int r = t * kTile + 32 * c + lane;
+    need[c] = false;
+    w[c] = -1;
+    b[c] = 0;
+    if (r < a.n && a.rq.status[r] == kStUnresolved) {
+      w[c] = a.rq.choice[r];
+      need[c] = w[c] >= 0;
+      b[c] = a.rq.cls[r];
+    }
+  }
+#pragma unroll
+  for (int c = 0; c < kC; ++c) {
+    if (need[c]) {
+      G[c] = a.ia.gh[w[c]];
+      h0[c] = a.ia.ch[w[c] * 3 + 0];
+      h1[c] = a.ia.ch[w[c] * 3 + 1];
+      h2[c] = a.ia.ch[w[c] * 3 + 2];
+    }
+  }
   __syncwarp();
   const uint32_t lt = lanemask_lt();
-  for (int c0 = 0; c0 < kTile; c0 += 32) {
-    const int r = t * kTile + c0 + lane;
-    bool need = false;
-    int w = -1, b = 0;
-    if (r < a.n && a.rq.status[r] == kStUnresolved) {
-      w = a.rq.choice[r];
-      need = w >= 0;
-      b = a.rq.cls[r];
-    }
-    const unsigned peers_w = __match_any_sync(kFull, need ? w : -1 - lane);
-    const unsigned m0 = __ballot_sync(kFull, need && b == 0);
-    const unsigned m1 = __ballot_sync(kFull, need && b == 1);
-    const unsigned m2 = __ballot_sync(kFull, need && b == 2);
-    if (need) {
-      const int c_0 = s_cnt[w * 3 + 0] + __popc(peers_w & m0 & lt);
-      const int c_1 = s_cnt[w * 3 + 1] + __popc(peers_w & m1 & lt);
-      const int c_2 = s_cnt[w * 3 + 2] + __popc(peers_w & m2 & lt);
-      const int h0 = a.ia.ch[w * 3 + 0], h1 = a.ia.ch[w * 3 + 1], h2 = a.ia.ch[w * 3 + 2];
-      const int G = a.ia.gh[w];
-      const int cb = b == 0 ? c_0 : (b == 1 ? c_1 : c_2);
-      const int hb = b == 0 ? h0 : (b == 1 ? h1 : h2);
-      const long long g = (long long)min(c_0, h0) + min(c_1, h1) + min(c_2, h2);
-      if (cb < hb && g < G) {
+#pragma unroll
+  for (int c = 0; c < kC; ++c) {
+    const int r = t * kTile + 32 * c + lane;
+    const unsigned peers_w = __match_any_sync(kFull, need[c] ? w[c] : -1 - lane);
+    const unsigned m0 = __ballot_sync(kFull, need[c] && b[c] == 0);
+    const unsigned m1 = __ballot_sync(kFull, need[c] && b[c] == 1);
+    const unsigned m2 = __ballot_sync(kFull, need[c] && b[c] == 2);
+    if (need[c]) {
+      const int wc = w[c], bc = b[c];
+      const int c_0 = s_cnt[wc * 3 + 0] + __popc(peers_w & m0 & lt);
+      const int c_1 = s_cnt[wc * 3 + 1] + __popc(peers_w & m1 & lt);
+      const int c_2 = s_cnt[wc * 3 + 2] + __popc(peers_w & m2 & lt);
+      const int cb = bc == 0 ? c_0 : (bc == 1 ? c_1 : c_2);
+      const int hb = bc == 0 ? h0[c] : (bc == 1 ? h1[c] : h2[c]);
+      const long long g = (long long)min(c_0, h0[c]) + min(c_1, h1[c]) + min(c_2, h2[c]);
+      if (cb < hb && g < G[c]) {
         a.rq.status[r] = kStResolved;
-        a.rq.inst[r] = w;
+        a.rq.inst[r] = wc;
         a.rq.reason[r] = MISAT_ADMIT_NEW;
-        atomicAdd(&a.ia.delta[w * 3 + b], 1);
-        atomicAdd(&a.ia.prefill[w], (unsigned long long)(a.rq.L[r] - 16 * (int64_t)a.H[(int64_t)r * a.W + w]));
+        atomicAdd(&a.ia.delta[wc * 3 + bc], 1);
+        atomicAdd(&a.ia.prefill[wc], (unsigned long long)(a.rq.L[r] - 16 * (int64_t)a.H[(int64_t)r * a.W + wc]));
       } else {
-        a.rq.last_reason[r] = g >= G ? MISAT_HOLD_GLOBAL_CAP : MISAT_HOLD_CLASS_CAP;
+        a.rq.last_reason[r] = g >= G[c] ? MISAT_HOLD_GLOBAL_CAP : MISAT_HOLD_CLASS_CAP;
       }
     }
     __syncwarp();
-    const unsigned peers_wb = __match_any_sync(kFull, need ? w * 3 + b : -1 - lane);
-    if (need && lane == __ffs(peers_wb) - 1) s_cnt[w * 3 + b] += __popc(peers_wb);
+    const unsigned peers_wb = __match_any_sync(kFull, need[c] ? w[c] * 3 + b[c] : -1 - lane);
+    if (need[c] && lane == __ffs(peers_wb) - 1) s_cnt[w[c] * 3 + b[c]] += __popc(peers_wb);
     __syncwarp();
   }
 }
 
 // End of a round: fold this round's admissions into the headroom, and add the admitted
-// prefill to the in-batch backlog d_w (saturating), so the next round sees the load.
+// prefill to the in-batch backlog d_w (saturating), so the next round sees the load.  A
+// round that admitted nobody leaves every input of the next round as it was (headroom,
+// backlog, statuses), so the next round would repeat it exactly: the remaining rounds
+// are then skipped.
 __global__ void __launch_bounds__(1024) k4_round_end(RoundArgs a) {
-  if (block_error(a.err)) return;
+  if (block_error(a.err) || !round_live(a)) return;
+  int admitted = 0;
   for (int w = threadIdx.x; w < a.W; w += blockDim.x) {
     int32_t sum = 0;
     for (int b = 0; b < 3; ++b) {
@@ -423,19 +463,33 @@ __global__ void __launch_bounds__(1024) k4_round_end(RoundArgs a) {
       sum += d;
     }
     a.ia.gh[w] -= sum;
+    admitted |= sum;
     const unsigned long long tok = a.ia.prefill[w];
     a.ia.prefill[w] = 0;
     const __int128 v = (__int128)a.ia.backlog_k[w] + (__int128)a.tokcost[w] * (__int128)tok;
     a.ia.backlog_k[w] = v > kBacklogMax ? kBacklogMax : (int64_t)v;
   }
+  const int any = __syncthreads_or(admitted != 0);
+  if (threadIdx.x == 0) {
+    if (!any && a.ia.live[1] == 0) a.ia.live[0] = 0;
+    a.ia.live[1] = 0;
+  }
 }
 
 void launch_round(const RoundArgs& a, int num_sms, cudaStream_t st) {
-  const size_t score_smem = (size_t)a.W * (8 + 8 + 4 + 12);
-  int score_grid = (a.n + 7) / 8;
-  if (score_grid > num_sms * 8) score_grid = num_sms * 8;
+  const size_t score_smem = (size_t)a.W * (8 + 8 + 4 + 12 + 3);
+  int G = 4;
+  while (G < 32 && G * 16 < a.W) G <<= 1;  // about two 8-instance chunks per lane
+  const int64_t threads = (int64_t)a.n * G;
+  int64_t score_grid = (threads + 255) / 256;
+  if (score_grid > (int64_t)num_sms * 8) score_grid = (int64_t)num_sms * 8;
   if (score_grid < 1) score_grid = 1;
-  k3_score<<<score_grid, 256, score_smem, st>>>(a);
+  switch (G) {
+    case 4: k3_score<4><<<(int)score_grid, 256, score_smem, st>>>(a); break;
+    case 8: k3_score<8><<<(int)score_grid, 256, score_smem, st>>>(a); break;
+    case 16: k3_score<16><<<(int)score_grid, 256, score_smem, st>>>(a); break;
+    default: k3_score<32><<<(int)score_grid, 256, score_smem, st>>>(a); break;
+  }
   const size_t cnt_smem = (size_t)a.W * 3 * sizeof(int32_t);
   k4_tile_count<<<a.n_tiles, 128, cnt_smem, st>>>(a);
   k4_tile_scan<<<(3 * a.W + 31) / 32, 1024, 0, st>>>(a);
@@ -461,7 +515,7 @@ __global__ void __launch_bounds__(256) k4_finalize(FinalizeArgs a) {
     if (stv == kStFollower) {
       w = a.rq.inst[a.rq.leader[r]];
       reason = w >= 0 ? MISAT_ADMIT_FOLLOW : MISAT_HOLD_LEADER_HELD;
-    } else if (stv == kStUnresolved) {
+    } else if (stv == kStUnresolved || stv == kStHeld) {
       w = -1;
       reason = a.rq.last_reason[r];
     } else {
@@ -480,7 +534,7 @@ __global__ void __launch_bounds__(256) k4_finalize(FinalizeArgs a) {
     if (stv == kStFollower) {
       a.rq.inst[r] = w;
       a.rq.reason[r] = reason;
-    } else if (stv == kStUnresolved) {
+    } else if (stv == kStUnresolved || stv == kStHeld) {
       a.rq.reason[r] = reason;
     }
     a.out_inst[r] = w;
