@@ -10,7 +10,12 @@ instances x 262,144 KV blocks filled to 95% (33.5M resident block hashes), batch
 Every timed step starts from the same router state (a device checkpoint restored
 before the step, outside the step's CUDA events), so the K steps do identical work.
 
-  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl gb300|reference]
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl gb300|reference] [--config 1..5]
+
+--config selects another of the five synthetic workloads (1: 4 x 2,048 blocks, 64 requests;
+2: 16 x 65,536, 4,096 requests; 3: 32 x 131,072, 16,384 RLVR-heavy; 4: 64 x 262,144,
+9,216 with long agentic sessions; 5, the default: the throughput stress above, whose
+--n and --fill span its sweep).
 
 Under torchrun (N > 1) every rank runs an independent replica (the path does not
 shard across GPUs in this build): weak scaling, value = all ranks' requests / max time.
@@ -19,6 +24,7 @@ shard across GPUs in this build): weak scaling, value = all ranks' requests / ma
 from __future__ import annotations
 
 import argparse
+import hashlib
 import json
 import os
 import statistics
@@ -47,12 +53,13 @@ CLOCK_QUERY = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.ac
                "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
 
 
-def kernels_per_step(rounds):
+def kernels_per_step(rounds, global_index):
     """Kernels one route+commit launches.  Route: prologue, leaders, hash, caps, probe first,
-    probe search, 5 per selection round (score, tile count, tile scan, admit, round end),
-    finalize.  Commit: insert work list, insert, sessions, and the five eviction kernels
-    (estimate, collect, select, delete, shift)."""
-    return 7 + 5 * rounds + 8
+    probe search, 5 per selection round (score, tile count, tile scan, admit, round end;
+    rounds after one that admitted nobody still launch and exit at once), finalize.
+    Commit: insert work list, insert, the global-index pass (global layout only), sessions,
+    and the five eviction kernels (estimate, collect, select, delete, shift)."""
+    return 7 + 5 * rounds + 8 + (1 if global_index else 0)
 
 
 def parse_args():
@@ -68,7 +75,41 @@ def parse_args():
     ap.add_argument("--instances", type=int, default=128, help="fewer only for small profiling captures")
     ap.add_argument("--prefix-index", default="global", choices=["global", "per-instance"],
                     help="block-0 probe through the global key->instance-mask index or per instance table")
+    ap.add_argument("--config", type=int, default=5, choices=[1, 2, 3, 4, 5],
+                    help="workload: 1-4 the smaller mixed configurations, 5 the throughput stress sweep")
     return ap.parse_args()
+
+
+L2_FLUSH_BYTES = 256 << 20  # twice the 129 MB L2
+
+HASH_SOURCES = ("paper_2608_11152_gb300/csrc/hash.cu", "paper_2608_11152_gb300/csrc/common.cuh")
+HASH_PROFILE = os.path.join(ROOT, "profiles", "k1_block_hash_stress_n65536.md")
+
+
+def hash_sources_sha256():
+    h = hashlib.sha256()
+    for f in HASH_SOURCES:
+        with open(os.path.join(ROOT, f), "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()
+
+
+def profiled_traffic(batch_tokens):
+    """DRAM bytes per launch of the block-hash kernel from the committed ncu summary, if that
+    capture was taken on the same batch with the kernel's current sources; else None."""
+    try:
+        fields = {}
+        for line in open(HASH_PROFILE):
+            if ":" in line and line.startswith("- `"):
+                k, v = line[3:].split("`:", 1)
+                fields[k.strip()] = v.strip().strip("`")
+        if fields.get("sources_sha256") != hash_sources_sha256():
+            return None
+        if int(fields["batch_tokens"]) != int(batch_tokens):
+            return None
+        return int(fields["traffic_bytes_per_launch"])
+    except Exception:
+        return None
 
 
 def peaks():
@@ -82,17 +123,32 @@ def peaks():
 def workload(args):
     from paper_2608_11152_gb300 import workload as wl
 
-    return wl.config5(n=args.n, fill=args.fill, instances=args.instances)
+    if args.config == 5:
+        return wl.config5(n=args.n, fill=args.fill, instances=args.instances)
+    return {1: wl.config1, 2: wl.config2, 3: wl.config3, 4: wl.config4}[args.config]()
+
+
+CONFIG_NAMES = {
+    1: "tiny mixed batch: 4 instances x 2048 blocks, 64 requests 50/25/25",
+    2: "medium mixed batch: 16 instances x 65536 blocks, 4096 requests 40/30/30",
+    3: "RLVR-heavy long tail: 32 instances x 131072 blocks, 16384 requests 70/15/15, fan-out 16",
+    4: "agentic-heavy long sessions: 64 instances x 262144 blocks, 1024 sessions + 8192 RLVR/RLHF, 20/20/60",
+}
 
 
 def workload_config(args, sc):
-    return {"workload": f"throughput stress: {sc.W} instances x {int(sc.cap_blocks[0])} blocks, "
-                        f"fill {int(round(args.fill * 100))}%, {args.n} requests/batch 40/30/30 RLVR/RLHF/agentic",
-            "instances": int(sc.W), "cap_blocks": int(sc.cap_blocks[0]), "fill": args.fill,
-            "batch_requests": int(args.n), "batch_tokens": int(sc.batch.n_tokens), "block_tokens": 16,
+    if args.config == 5:
+        name = (f"throughput stress: {sc.W} instances x {int(sc.cap_blocks[0])} blocks, "
+                f"fill {int(round(args.fill * 100))}%, {args.n} requests/batch 40/30/30 RLVR/RLHF/agentic")
+    else:
+        name = CONFIG_NAMES[args.config]
+    return {"workload": name,
+            "instances": int(sc.W), "cap_blocks": int(sc.cap_blocks[0]), "fill": args.fill if args.config == 5 else None,
+            "batch_requests": int(sc.batch.n), "batch_tokens": int(sc.batch.n_tokens), "block_tokens": 16,
             "rounds": int(sc.rounds), "mode": "MISA-T", "prefix_index": args.prefix_index,
-            "l2": "inputs larger than L2 (tokens %.2f GB, tables %.2f GB) and a state restore of the "
-                  "tables between steps" % (sc.batch.n_tokens * 4 / 1e9, sc.W * 2 * int(sc.cap_blocks[0]) * 16 / 1e9)}
+            "l2": ("L2 flushed before every timed step (a %d MB write, outside the step's events) after the "
+                   "state restore; tokens %.3f GB, tables %.3f GB" % (L2_FLUSH_BYTES >> 20, sc.batch.n_tokens * 4 / 1e9,
+                                                                    sc.W * 2 * int(sc.cap_blocks[0]) * 16 / 1e9))}
 
 
 class ClockSampler:
@@ -236,22 +292,26 @@ def run_gb300(args):
     db = r.device_batch(sc.batch)
     out = r.alloc_decisions(sc.batch.n)
     stream = r.stream
-    r.set_timing(True)
     log("checkpoint saved, batch resident")
 
     def step():
         r.route(db, out)
         r.commit()
 
+    flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device="cuda")
+
+    def flush_l2():
+        with torch.cuda.stream(stream):
+            flush.fill_(1)
+
     for i in range(args.warmup):
         r.checkpoint_restore(ckpt)
+        flush_l2()
         step()
-        log(f"warm-up step {i}: " + ", ".join(f"{k} {v:.3f}" for k, v in r.phase_times().items()))
     torch.cuda.synchronize()
     K = args.steps
     starts = [torch.cuda.Event(enable_timing=True) for _ in range(K)]
     ends = [torch.cuda.Event(enable_timing=True) for _ in range(K)]
-    phase_tot = {p: 0.0 for p in misat.PHASES}
     sampler = ClockSampler(local)
     sampler.start()
     time.sleep(0.3)
@@ -261,13 +321,13 @@ def run_gb300(args):
     t_wall = time.perf_counter()
     for k in range(K):
         r.checkpoint_restore(ckpt)
+        flush_l2()
         torch.cuda.nvtx.range_push("misat_step")
         starts[k].record(stream)
         step()
         ends[k].record(stream)
         torch.cuda.nvtx.range_pop()
-        for p, v in r.phase_times().items():  # waits for the step (outside its events)
-            phase_tot[p] += v
+        ends[k].synchronize()
     torch.cuda.synchronize()
     if dist:
         dist.barrier()
@@ -276,6 +336,21 @@ def run_gb300(args):
     step_ms = [starts[k].elapsed_time(ends[k]) for k in range(K)]
     total_ms = float(sum(step_ms))
     log(f"timed steps done: {total_ms / K:.3f} ms/step (wall {wall:.2f} s for {K} steps incl. restores)")
+    # per-phase device times (for the roofline and the phase breakdown) come from separate
+    # steps with the library's phase events on: the events are kept out of the timed steps
+    KP = max(1, min(K, 10))
+    phase_tot = {p: 0.0 for p in misat.PHASES}
+    r.set_timing(True)
+    for k in range(KP):
+        r.checkpoint_restore(ckpt)
+        flush_l2()
+        step()
+        for p, v in r.phase_times().items():
+            phase_tot[p] += v
+    r.set_timing(False)
+    r.checkpoint_restore(ckpt)
+    step()  # leaves the statistics of one plain step
+    torch.cuda.synchronize()
     st = r.stats()
     r.sync()
     if dist:
@@ -306,6 +381,7 @@ def run_gb300(args):
     e2e_ms = 0.0
     for k in range(args.e2e_steps):
         r.checkpoint_restore(ckpt)
+        flush_l2()
         torch.cuda.synchronize()
         e0 = torch.cuda.Event(enable_timing=True)
         e1 = torch.cuda.Event(enable_timing=True)
@@ -346,7 +422,7 @@ def run_gb300(args):
                 "amortized_rebuild_ms_per_step": round(rb_ms / steps_between, 4)}
         log(f"global index: {gidx}")
     ab = algorithmic_bytes(sc, st, mask_words=gidx["mask_words"] if gidx else None)
-    phase_ms = {p: phase_tot[p] / K for p in phase_tot}
+    phase_ms = {p: phase_tot[p] / KP for p in phase_tot}
     dom = max(phase_ms, key=lambda p: phase_ms[p])
 
     def roof(kind):
@@ -360,6 +436,8 @@ def run_gb300(args):
                 "ms_per_launch": round(ms, 4), "peak_kind": peak_kind}
 
     kernels = {k: roof(k) for k in ("hash", "probe_first", "probe_search")}
+    if kernels["hash"] is not None:
+        kernels["hash"]["traffic"] = profiled_traffic(sc.batch.n_tokens)
     dom_roof = roof(dom)
     if dom_roof is None:
         dom_roof = {"bound": "hbm", "achieved": None, "peak": peak, "unit": "GB/s", "frac": None, "traffic": None,
@@ -375,7 +453,7 @@ def run_gb300(args):
         "config": workload_config(args, sc),
         "probes_per_s": round(world * st.probes * K / (total_ms / 1e3), 1),
         "e2e": {"value": round(e2e, 1), "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
-        "gpu_launches": kernels_per_step(sc.rounds) * K,
+        "gpu_launches": kernels_per_step(sc.rounds, pidx == misat.PREFIX_GLOBAL) * K,
         "roofline": dom_roof,
         "kernels": kernels,
         "prefix_index": args.prefix_index,

@@ -1,6 +1,7 @@
 // C ABI of the MISA-T routing library: context, orchestration of the kernels, class
 // histories (host), table growth and state dumps.  See include/misat.h.
 #include <algorithm>
+#include <array>
 #include <cstdlib>
 #include <cstring>
 #include <deque>
@@ -141,6 +142,13 @@ struct misat_ctx {
   uint8_t* d_out_reason = nullptr;
   int32_t* d_out_hit = nullptr;
   std::vector<void*> owned;  // fixed allocations freed in destroy
+  // launch sequences replayed as CUDA graphs (captured on a private stream, which never
+  // runs work, and launched on the context's stream)
+  cudaStream_t cap_stream = nullptr;
+  struct GraphCache {
+    cudaGraphExec_t exec = nullptr;
+    std::array<uint64_t, 4> key{};
+  } g_rounds, g_evict;
   // phase timing: events 0..7 bracket the route phases, 8..11 the commit phases
   bool timing = false;
   cudaEvent_t ev[12] = {};
@@ -167,6 +175,39 @@ namespace {
   do {                                           \
     if ((x) != cudaSuccess) return MISAT_ERR_CUDA; \
   } while (0)
+
+// Launch a fixed sequence through a cached CUDA graph: `launch(stream)` enqueues the
+// sequence; it is captured once per key (the values its kernel arguments depend on) and
+// replayed with one graph launch.  When the context's stream is itself being captured by
+// the caller, or capture is unavailable, the sequence is launched directly.
+template <class F>
+int run_graph(misat_ctx* c, misat_ctx::GraphCache& gc, const std::array<uint64_t, 4>& key, F&& launch) {
+  cudaStream_t st = c->stream;
+  cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+  if (!c->cap_stream || cudaStreamIsCapturing(st, &cs) != cudaSuccess || cs != cudaStreamCaptureStatusNone) {
+    cudaGetLastError();
+    launch(st);
+    return cudaGetLastError() == cudaSuccess ? MISAT_OK : MISAT_ERR_CUDA;
+  }
+  if (!gc.exec || gc.key != key) {
+    if (gc.exec) cudaGraphExecDestroy(gc.exec);
+    gc.exec = nullptr;
+    cudaGraph_t g = nullptr;
+    CK(cudaStreamBeginCapture(c->cap_stream, cudaStreamCaptureModeThreadLocal));
+    launch(c->cap_stream);
+    const cudaError_t e = cudaStreamEndCapture(c->cap_stream, &g);
+    if (e != cudaSuccess || !g) return MISAT_ERR_CUDA;
+    const cudaError_t ei = cudaGraphInstantiate(&gc.exec, g, 0);
+    cudaGraphDestroy(g);
+    if (ei != cudaSuccess) {
+      gc.exec = nullptr;
+      return MISAT_ERR_CUDA;
+    }
+    gc.key = key;
+  }
+  CK(cudaGraphLaunch(gc.exec, st));
+  return MISAT_OK;
+}
 
 int dalloc(misat_ctx* c, void** p, size_t bytes) {
   *p = nullptr;
@@ -428,9 +469,9 @@ int evict_all(misat_ctx* c, unsigned long long* evicted_counter) {
   uint32_t maxlg = 1;
   for (auto& d : c->h_desc) maxlg = std::max(maxlg, d.log2nb);
   const int chunks = (int)std::min<uint64_t>(256, std::max<uint64_t>(1, ((uint64_t)1 << maxlg) / (4 * 256)));
-  launch_evict(ev, chunks, c->stream);
-  CK(cudaGetLastError());
-  return MISAT_OK;
+  const std::array<uint64_t, 4> key{(uint64_t)chunks, reinterpret_cast<uint64_t>(ev.gix.keys),
+                                    (uint64_t)ev.gix.log2nb, reinterpret_cast<uint64_t>(evicted_counter)};
+  return run_graph(c, c->g_evict, key, [&](cudaStream_t s) { launch_evict(ev, chunks, s); });
 }
 
 }  // namespace
@@ -454,6 +495,9 @@ const char* misat_strerror(int code) {
 int misat_destroy(misat_ctx* c) {
   if (!c) return MISAT_ERR_INVALID_ARG;
   cudaStreamSynchronize(c->stream);
+  if (c->g_rounds.exec) cudaGraphExecDestroy(c->g_rounds.exec);
+  if (c->g_evict.exec) cudaGraphExecDestroy(c->g_evict.exec);
+  if (c->cap_stream) cudaStreamDestroy(c->cap_stream);
   for (size_t w = 0; w < c->h_desc.size(); ++w) {
     cudaFree(c->h_desc[w].tab);
     if (w < c->h_bufs.size()) free_bufs(c->h_bufs[w]);
@@ -520,6 +564,10 @@ int misat_create(const misat_config* cfg, void* cuda_stream, misat_ctx** out) {
   c->table_load = cfg->table_load;
   c->ml.init(W);
   if (cudaEventCreateWithFlags(&c->ev_meta, cudaEventDisableTiming) != cudaSuccess) return fail(MISAT_ERR_CUDA);
+  if (cudaStreamCreateWithFlags(&c->cap_stream, cudaStreamNonBlocking) != cudaSuccess) {
+    cudaGetLastError();
+    c->cap_stream = nullptr;  // sequences are then launched directly
+  }
   if (cudaMallocHost(&c->h_meta, c->ml.words * 8) != cudaSuccess) return fail(MISAT_ERR_OOM);
   std::memset(c->h_meta, 0, c->ml.words * 8);
 
@@ -729,7 +777,13 @@ int misat_route(misat_ctx* c, const misat_batch* b, misat_decisions* out) {
   ra.tile_counts = c->d_tile;
   ra.n_tiles = (n + kTileReq - 1) / kTileReq;
   ra.err = c->err_ptr();
-  for (int k = 0; k < c->rounds; ++k) launch_round(ra, c->num_sms, st);
+  {
+    const std::array<uint64_t, 4> key{(uint64_t)n, 0, 0, 0};
+    const int rc = run_graph(c, c->g_rounds, key, [&](cudaStream_t s) {
+      for (int k = 0; k < c->rounds; ++k) launch_round(ra, c->num_sms, s);
+    });
+    if (rc) return rc;
+  }
   c->mark(6);
 
   FinalizeArgs fa{};
