@@ -194,7 +194,7 @@ __device__ __forceinline__ bool round_live(const RoundArgs& a) {
 // lower instance) by log2(G) shuffle steps inside the group.  A session protected on its
 // choice is admitted here (ADMIT_CONT); a released session may prefer to wait for its
 // cached instance (Eq. 7).
-template <int G>
+template <int G, int CPL>
 __global__ void __launch_bounds__(256) k3_score(RoundArgs a) {
   extern __shared__ unsigned char smem[];
   int64_t* s_bk = reinterpret_cast<int64_t*>(smem);
@@ -218,102 +218,144 @@ __global__ void __launch_bounds__(256) k3_score(RoundArgs a) {
   __syncthreads();
   const int lane = threadIdx.x & 31;
   const int gl = lane & (G - 1);                 // lane within the group
-  const unsigned gmask = G == 32 ? kFull : (((1u << G) - 1) << (lane & ~(G - 1)));
+  const int g0 = lane & ~(G - 1);                // first lane of the group in the warp
+  const unsigned gmask = G == 32 ? kFull : (((1u << G) - 1) << g0);
   const int64_t gid = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) / G;
   const int64_t ngroups = ((int64_t)gridDim.x * blockDim.x) / G;
   const int chunks = (a.W + 7) >> 3;
   const bool row_vec = (a.W & 7) == 0;           // H rows 16-byte aligned
-  for (int64_t rr = gid; rr < a.n; rr += ngroups) {
-    const int r = (int)rr;
-    if (a.rq.status[r] != kStUnresolved) continue;  // uniform within the group
-    const int b = a.rq.cls[r];
-    const uint8_t sst = a.rq.sst[r];
-    const int pw = sst == kSessProtected ? a.rq.sinst[r] : -1;
-    const int64_t Lr = a.rq.L[r];
+  // a group owns requests gid + k * ngroups; they are taken G at a time: lane k of the
+  // group loads request k's status and fields, so the group learns which of its requests
+  // are unresolved in one round trip, and each request's H chunks are loaded while the
+  // previous request is reduced
+  auto load_h = [&](int r, uint4 (&hv)[CPL]) {
     const uint16_t* Hr = a.H + (int64_t)r * a.W;
-    const uint8_t* el = s_el + b * a.W;
-    int64_t best_c = INT64_MAX;
-    int best_w = INT32_MAX;
-    int hmax = -1, whit = INT32_MAX;
-    for (int ck = gl; ck < chunks; ck += G) {
-      const int w0 = ck * 8;
-      uint16_t h[8];
-      if (row_vec) {
-        const uint4 v = *reinterpret_cast<const uint4*>(Hr + w0);
-        h[0] = (uint16_t)v.x; h[1] = (uint16_t)(v.x >> 16);
-        h[2] = (uint16_t)v.y; h[3] = (uint16_t)(v.y >> 16);
-        h[4] = (uint16_t)v.z; h[5] = (uint16_t)(v.z >> 16);
-        h[6] = (uint16_t)v.w; h[7] = (uint16_t)(v.w >> 16);
-      } else {
 #pragma unroll
-        for (int i = 0; i < 8; ++i) h[i] = w0 + i < a.W ? Hr[w0 + i] : 0;
+    for (int c = 0; c < CPL; ++c) {
+      const int ck = gl + G * c;
+      hv[c] = make_uint4(0, 0, 0, 0);
+      if (ck < chunks) {
+        if (row_vec) {
+          hv[c] = *reinterpret_cast<const uint4*>(Hr + ck * 8);
+        } else {
+          uint32_t t[4] = {0, 0, 0, 0};
+          for (int i = 0; i < 8; ++i)
+            if (ck * 8 + i < a.W) t[i >> 1] |= (uint32_t)Hr[ck * 8 + i] << (16 * (i & 1));
+          hv[c] = make_uint4(t[0], t[1], t[2], t[3]);
+        }
       }
+    }
+  };
+  for (int64_t base = gid; base < a.n; base += ngroups * G) {
+    const int64_t rk = base + (int64_t)gl * ngroups;
+    uint8_t st = kStResolved, kb = 0, ksst = 0;
+    int ksinst = -1, kL = 0;
+    if (rk < a.n) {
+      st = a.rq.status[rk];
+      if (st == kStUnresolved) {
+        kb = a.rq.cls[rk];
+        ksst = a.rq.sst[rk];
+        ksinst = a.rq.sinst[rk];
+        kL = a.rq.L[rk];
+      }
+    }
+    unsigned todo = (__ballot_sync(gmask, st == kStUnresolved) >> g0) & (G == 32 ? kFull : ((1u << G) - 1));
+    if (!todo) continue;
+    int k = __ffs(todo) - 1;
+    uint4 hv[CPL];
+    load_h((int)(base + (int64_t)k * ngroups), hv);
+    while (true) {
+      todo &= todo - 1;
+      const int knext = todo ? __ffs(todo) - 1 : -1;
+      uint4 hn[CPL];
+      if (knext >= 0) load_h((int)(base + (int64_t)knext * ngroups), hn);
+      const int r = (int)(base + (int64_t)k * ngroups);
+      const int b = __shfl_sync(gmask, (int)kb, g0 + k);
+      const uint8_t sst = (uint8_t)__shfl_sync(gmask, (int)ksst, g0 + k);
+      const int sinst = __shfl_sync(gmask, ksinst, g0 + k);
+      const int64_t Lr = __shfl_sync(gmask, kL, g0 + k);
+      const int pw = sst == kSessProtected ? sinst : -1;
+      const uint8_t* el = s_el + b * a.W;
+      int64_t best_c = INT64_MAX;
+      int best_w = INT32_MAX;
+      int hmax = -1, whit = INT32_MAX;
 #pragma unroll
-      for (int i = 0; i < 8; ++i) {
-        const int w = w0 + i;
-        if (w >= a.W) break;
-        if (w == pw || el[w]) {
-          const int64_t cost = s_bk[w] + (Lr - 16 * (int64_t)h[i]) * s_tc[w];
-          if (cost < best_c) {
-            best_c = cost;
-            best_w = w;
+      for (int c = 0; c < CPL; ++c) {
+        const int ck = gl + G * c;
+        if (ck >= chunks) break;
+        const uint32_t hw[4] = {hv[c].x, hv[c].y, hv[c].z, hv[c].w};
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+          const int w = ck * 8 + i;
+          if (w >= a.W) break;
+          const int h = (int)((hw[i >> 1] >> (16 * (i & 1))) & 0xffffu);
+          if (w == pw || el[w]) {
+            const int64_t cost = s_bk[w] + (Lr - 16 * (int64_t)h) * s_tc[w];
+            if (cost < best_c) {
+              best_c = cost;
+              best_w = w;
+            }
+          }
+          if (h > hmax) {
+            hmax = h;
+            whit = w;
           }
         }
-        if ((int)h[i] > hmax) {
-          hmax = h[i];
-          whit = w;
+      }
+#pragma unroll
+      for (int o = G / 2; o > 0; o >>= 1) {
+        const int64_t oc = __shfl_xor_sync(gmask, best_c, o, G);
+        const int ow = __shfl_xor_sync(gmask, best_w, o, G);
+        if (oc < best_c || (oc == best_c && ow < best_w)) {
+          best_c = oc;
+          best_w = ow;
+        }
+        const int oh = __shfl_xor_sync(gmask, hmax, o, G);
+        const int owh = __shfl_xor_sync(gmask, whit, o, G);
+        if (oh > hmax || (oh == hmax && owh < whit)) {
+          hmax = oh;
+          whit = owh;
         }
       }
-    }
-#pragma unroll
-    for (int o = G / 2; o > 0; o >>= 1) {
-      const int64_t oc = __shfl_xor_sync(gmask, best_c, o, G);
-      const int ow = __shfl_xor_sync(gmask, best_w, o, G);
-      if (oc < best_c || (oc == best_c && ow < best_w)) {
-        best_c = oc;
-        best_w = ow;
-      }
-      const int oh = __shfl_xor_sync(gmask, hmax, o, G);
-      const int owh = __shfl_xor_sync(gmask, whit, o, G);
-      if (oh > hmax || (oh == hmax && owh < whit)) {
-        hmax = oh;
-        whit = owh;
-      }
-    }
-    if (gl == 0) {
-      a.rq.hmax[r] = hmax < 0 ? 0 : hmax;
-      int choice = -1;
-      uint8_t reason = 0;
-      if (best_w == INT32_MAX) {
-        // no instance has headroom: headroom only shrinks over the rounds and protection
-        // is fixed by the snapshot, so no later round can admit it
-        reason = MISAT_HOLD_NO_ELIGIBLE;
-        a.rq.status[r] = kStHeld;
-      } else {
-        choice = best_w;
-        if (sst == kSessReleased && hmax > 0) {
-          const bool elig_hit = s_gh[whit] > 0 && s_ch[whit * 3 + b] > 0;
-          if (!elig_hit) {
-            const int64_t lhs = a.hold_delay_q + s_bk[whit] - s_bk[best_w];
-            const int64_t rhs = 16 * (int64_t)hmax * s_tc[whit];
-            if (lhs < rhs) {
-              choice = -1;
-              reason = MISAT_HOLD_PREFER_CACHE;
+      if (gl == 0) {
+        a.rq.hmax[r] = hmax < 0 ? 0 : hmax;
+        int choice = -1;
+        uint8_t reason = 0;
+        if (best_w == INT32_MAX) {
+          // no instance has headroom: headroom only shrinks over the rounds and protection
+          // is fixed by the snapshot, so no later round can admit it
+          reason = MISAT_HOLD_NO_ELIGIBLE;
+          a.rq.status[r] = kStHeld;
+        } else {
+          choice = best_w;
+          if (sst == kSessReleased && hmax > 0) {
+            const bool elig_hit = s_gh[whit] > 0 && s_ch[whit * 3 + b] > 0;
+            if (!elig_hit) {
+              const int64_t lhs = a.hold_delay_q + s_bk[whit] - s_bk[best_w];
+              const int64_t rhs = 16 * (int64_t)hmax * s_tc[whit];
+              if (lhs < rhs) {
+                choice = -1;
+                reason = MISAT_HOLD_PREFER_CACHE;
+              }
             }
           }
         }
+        if (choice >= 0 && choice == pw) {
+          a.rq.status[r] = kStResolved;
+          a.rq.inst[r] = choice;
+          a.rq.reason[r] = MISAT_ADMIT_CONT;
+          a.rq.choice[r] = -1;
+          atomicAdd(&a.ia.prefill[choice], (unsigned long long)(Lr - 16 * (int64_t)a.H[(int64_t)r * a.W + choice]));
+          atomicAdd(&a.ia.live[1], 1);
+        } else {
+          a.rq.choice[r] = choice;
+          if (choice < 0) a.rq.last_reason[r] = reason;
+        }
       }
-      if (choice >= 0 && choice == pw) {
-        a.rq.status[r] = kStResolved;
-        a.rq.inst[r] = choice;
-        a.rq.reason[r] = MISAT_ADMIT_CONT;
-        a.rq.choice[r] = -1;
-        atomicAdd(&a.ia.prefill[choice], (unsigned long long)(Lr - 16 * (int64_t)Hr[choice]));
-        atomicAdd(&a.ia.live[1], 1);
-      } else {
-        a.rq.choice[r] = choice;
-        if (choice < 0) a.rq.last_reason[r] = reason;
-      }
+      if (knext < 0) break;
+      k = knext;
+#pragma unroll
+      for (int c = 0; c < CPL; ++c) hv[c] = hn[c];
     }
   }
 }
@@ -484,11 +526,11 @@ void launch_round(const RoundArgs& a, int num_sms, cudaStream_t st) {
   int64_t score_grid = (threads + 255) / 256;
   if (score_grid > (int64_t)num_sms * 8) score_grid = (int64_t)num_sms * 8;
   if (score_grid < 1) score_grid = 1;
-  switch (G) {
-    case 4: k3_score<4><<<(int)score_grid, 256, score_smem, st>>>(a); break;
-    case 8: k3_score<8><<<(int)score_grid, 256, score_smem, st>>>(a); break;
-    case 16: k3_score<16><<<(int)score_grid, 256, score_smem, st>>>(a); break;
-    default: k3_score<32><<<(int)score_grid, 256, score_smem, st>>>(a); break;
+  switch (G) {  // CPL: 8-instance chunks per lane, ceil(ceil(W/8) / G)
+    case 4: k3_score<4, 2><<<(int)score_grid, 256, score_smem, st>>>(a); break;
+    case 8: k3_score<8, 2><<<(int)score_grid, 256, score_smem, st>>>(a); break;
+    case 16: k3_score<16, 2><<<(int)score_grid, 256, score_smem, st>>>(a); break;
+    default: k3_score<32, 4><<<(int)score_grid, 256, score_smem, st>>>(a); break;
   }
   const size_t cnt_smem = (size_t)a.W * 3 * sizeof(int32_t);
   k4_tile_count<<<a.n_tiles, 128, cnt_smem, st>>>(a);
