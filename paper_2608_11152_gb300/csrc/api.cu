@@ -106,6 +106,8 @@ struct misat_ctx {
   int32_t* d_prot = nullptr;
   unsigned long long* d_theta = nullptr;
   int32_t* d_active = nullptr;
+  int32_t* d_act = nullptr;      // instances over capacity in the current eviction
+  unsigned* d_nact = nullptr;
   int32_t* d_onew = nullptr;
   InstArrays ia{};
   // sessions
@@ -457,6 +459,8 @@ EvictArgs evict_args(misat_ctx* c, unsigned long long* evicted_counter) {
   ev.thr_hi = c->d_thr + c->W;
   ev.theta = c->d_theta;
   ev.active = c->d_active;
+  ev.act = c->d_act;
+  ev.n_act = c->d_nact;
   ev.evicted = evicted_counter;
   ev.err = c->err_ptr();
   ev.gix = gix_or_null(c);
@@ -471,7 +475,7 @@ int evict_all(misat_ctx* c, unsigned long long* evicted_counter) {
   const int chunks = (int)std::min<uint64_t>(256, std::max<uint64_t>(1, ((uint64_t)1 << maxlg) / (4 * 256)));
   const std::array<uint64_t, 4> key{(uint64_t)chunks, reinterpret_cast<uint64_t>(ev.gix.keys),
                                     (uint64_t)ev.gix.log2nb, reinterpret_cast<uint64_t>(evicted_counter)};
-  return run_graph(c, c->g_evict, key, [&](cudaStream_t s) { launch_evict(ev, chunks, s); });
+  return run_graph(c, c->g_evict, key, [&](cudaStream_t s) { launch_evict(ev, chunks, c->num_sms, s); });
 }
 
 }  // namespace
@@ -598,6 +602,7 @@ int misat_create(const misat_config* cfg, void* cuda_stream, misat_ctx** out) {
       (rc = dalloc_n(c, &c->d_tokcost, Ws)) || (rc = dalloc_n(c, &c->d_contraction, Ws)) ||
       (rc = dalloc_n(c, &c->d_prot, 3 * Ws)) || (rc = dalloc_n(c, &c->d_theta, 2 * Ws)) ||
       (rc = dalloc_n(c, &c->d_active, Ws)) || (rc = dalloc_n(c, &c->d_onew, 1)) ||
+      (rc = dalloc_n(c, &c->d_act, Ws)) || (rc = dalloc_n(c, &c->d_nact, 1)) ||
       (rc = dalloc_n(c, &c->d_desc, Ws)) || (rc = dalloc_n(c, &c->d_bitmap, Ws)) || (rc = dalloc_n(c, &c->d_ca, Ws)) ||
       (rc = dalloc_n(c, &c->d_cb, Ws)) || (rc = dalloc_n(c, &c->d_cc, Ws)) || (rc = dalloc_n(c, &c->d_slots, Ws)) ||
       (rc = dalloc_n(c, &c->d_dmask, Ws)) || (rc = dalloc_n(c, &c->d_ncand, Ws)) ||

@@ -110,6 +110,7 @@ __global__ void __launch_bounds__(kSelThreads) k4_evict_estimate(EvictArgs a) {
     a.active[w] = E > 0 ? 1 : 0;
     a.n_d[w] = 0;
     a.n_cand[w] = 0;
+    if (E > 0) a.act[atomicAdd(a.n_act, 1u)] = w;  // the streaming passes visit only these
   }
   if (E <= 0) return;
   const InstDesc d = a.desc[w];
@@ -191,12 +192,9 @@ __global__ void __launch_bounds__(kSelThreads) k4_evict_estimate(EvictArgs a) {
   }
 }
 
-// Streaming pass over the instance's metas (grid.x CTAs per instance).
-__global__ void __launch_bounds__(256) k4_evict_collect(EvictArgs a) {
+// Streaming pass over the instance's metas: chunk `cidx` of `chunks` of instance w.
+__device__ __forceinline__ void collect_chunk(const EvictArgs& a, int w, uint32_t cidx, uint32_t chunks) {
   __shared__ unsigned s_wd[8], s_wu[8], s_bd, s_bu;
-  const int w = a.only_w ? *a.only_w : blockIdx.y;
-  if (block_error(a.err)) return;
-  if (a.active[w] != 1) return;
   const InstDesc d = a.desc[w];
   const uint32_t NB = 1u << d.log2nb;
   const unsigned long long lo = a.thr_lo[w], hi = a.thr_hi[w];
@@ -206,8 +204,8 @@ __global__ void __launch_bounds__(256) k4_evict_collect(EvictArgs a) {
   uint4* u = a.cand_a[w];
   uint32_t* usl = a.slots[w];
   const int lane = threadIdx.x & 31;
-  const uint32_t stride = gridDim.x * blockDim.x;
-  for (uint32_t b0 = blockIdx.x * blockDim.x; b0 < NB; b0 += stride) {
+  const uint32_t stride = chunks * blockDim.x;
+  for (uint32_t b0 = cidx * blockDim.x; b0 < NB; b0 += stride) {
     const uint32_t b = b0 + threadIdx.x;
     unsigned long long m[4] = {0, 0, 0, 0};
     bool full = false;
@@ -275,6 +273,14 @@ __global__ void __launch_bounds__(256) k4_evict_collect(EvictArgs a) {
     if (lane == 0 && b < NB) bitmap[b >> 5] = bits;
     if ((lane & 7) == 0 && b < NB) dmask[b >> 3] = 0;
   }
+}
+
+// Work items (active instance, chunk), taken by a grid of resident CTAs: instances within
+// capacity cost nothing (their list entries are never made).
+__global__ void __launch_bounds__(256) k4_evict_collect(EvictArgs a, uint32_t chunks) {
+  if (block_error(a.err)) return;
+  const uint32_t items = *(volatile const unsigned*)a.n_act * chunks;
+  for (uint32_t it = blockIdx.x; it < items; it += gridDim.x) collect_chunk(a, a.act[it / chunks], it % chunks, chunks);
 }
 
 __global__ void __launch_bounds__(kSelThreads) k4_evict_select(EvictArgs a) {
@@ -392,10 +398,7 @@ __device__ __forceinline__ void delete_slot(const GIndex& g, int w, Bucket* tab,
 }  // namespace
 
 // Delete D and the candidates at or below theta; record them in the deleted-slot masks.
-__global__ void __launch_bounds__(256) k4_evict_delete(EvictArgs a) {
-  const int w = a.only_w ? *a.only_w : blockIdx.y;
-  if (block_error(a.err)) return;
-  if (a.active[w] != 1) return;
+__device__ __forceinline__ void delete_chunk(const EvictArgs& a, int w, uint32_t cidx, uint32_t chunks) {
   const unsigned nd = a.n_d[w], n = a.n_cand[w];
   const uint32_t* dsl = a.dslots[w];
   const uint4* c0 = a.cand_a[w];
@@ -404,8 +407,8 @@ __global__ void __launch_bounds__(256) k4_evict_delete(EvictArgs a) {
   Bucket* tab = a.desc[w].tab;
   const unsigned long long tm = a.theta[2 * w], tk = a.theta[2 * w + 1];
   long long deleted = 0;
-  const unsigned stride = gridDim.x * blockDim.x;
-  for (unsigned i = blockIdx.x * blockDim.x + threadIdx.x; i < nd + n; i += stride) {
+  const unsigned stride = chunks * blockDim.x;
+  for (unsigned i = cidx * blockDim.x + threadIdx.x; i < nd + n; i += stride) {
     if (i < nd) {
       delete_slot(a.gix, w, tab, dmask, dsl[i], a.err);
       ++deleted;
@@ -423,12 +426,15 @@ __global__ void __launch_bounds__(256) k4_evict_delete(EvictArgs a) {
   }
 }
 
+__global__ void __launch_bounds__(256) k4_evict_delete(EvictArgs a, uint32_t chunks) {
+  if (block_error(a.err)) return;
+  const uint32_t items = *(volatile const unsigned*)a.n_act * chunks;
+  for (uint32_t it = blockIdx.x; it < items; it += gridDim.x) delete_chunk(a, a.act[it / chunks], it % chunks, chunks);
+}
+
 // Refill the holes of every run of full buckets that lost an entry.  The thread of the
 // run's first deleted slot (lowest bucket, then lowest slot) owns the run.
-__global__ void __launch_bounds__(256) k4_evict_shift(EvictArgs a) {
-  const int w = a.only_w ? *a.only_w : blockIdx.y;
-  if (block_error(a.err)) return;
-  if (a.active[w] != 1) return;
+__device__ __forceinline__ void shift_chunk(const EvictArgs& a, int w, uint32_t cidx, uint32_t chunks) {
   const unsigned nd = a.n_d[w], n = a.n_cand[w];
   const uint32_t* dsl = a.dslots[w];
   const uint4* c0 = a.cand_a[w];
@@ -438,8 +444,8 @@ __global__ void __launch_bounds__(256) k4_evict_shift(EvictArgs a) {
   const InstDesc d = a.desc[w];
   const uint32_t NB = 1u << d.log2nb, mask = NB - 1;
   const unsigned long long tm = a.theta[2 * w], tk = a.theta[2 * w + 1];
-  const unsigned stride = gridDim.x * blockDim.x;
-  for (unsigned i = blockIdx.x * blockDim.x + threadIdx.x; i < nd + n; i += stride) {
+  const unsigned stride = chunks * blockDim.x;
+  for (unsigned i = cidx * blockDim.x + threadIdx.x; i < nd + n; i += stride) {
     uint32_t sl;
     if (i < nd) {
       sl = dsl[i];
@@ -500,13 +506,23 @@ __global__ void __launch_bounds__(256) k4_evict_shift(EvictArgs a) {
   }
 }
 
-void launch_evict(const EvictArgs& a, int chunks_per_inst, cudaStream_t st) {
+__global__ void __launch_bounds__(256) k4_evict_shift(EvictArgs a, uint32_t chunks) {
+  if (block_error(a.err)) return;
+  const uint32_t items = *(volatile const unsigned*)a.n_act * chunks;
+  for (uint32_t it = blockIdx.x; it < items; it += gridDim.x) shift_chunk(a, a.act[it / chunks], it % chunks, chunks);
+}
+
+void launch_evict(const EvictArgs& a, int chunks_per_inst, int num_sms, cudaStream_t st) {
   const int W = a.only_w ? 1 : a.W;
+  // streaming passes: resident CTAs over (active instance, chunk) items
+  const int64_t items = (int64_t)W * chunks_per_inst;
+  const int grid = (int)(items < (int64_t)num_sms * 8 ? items : (int64_t)num_sms * 8);
+  cudaMemsetAsync(a.n_act, 0, sizeof(unsigned), st);
   k4_evict_estimate<<<W, kSelThreads, 0, st>>>(a);
-  k4_evict_collect<<<dim3(chunks_per_inst, W), 256, 0, st>>>(a);
+  k4_evict_collect<<<grid, 256, 0, st>>>(a, (uint32_t)chunks_per_inst);
   k4_evict_select<<<W, kSelThreads, 0, st>>>(a);
-  k4_evict_delete<<<dim3(chunks_per_inst, W), 256, 0, st>>>(a);
-  k4_evict_shift<<<dim3(chunks_per_inst, W), 256, 0, st>>>(a);
+  k4_evict_delete<<<grid, 256, 0, st>>>(a, (uint32_t)chunks_per_inst);
+  k4_evict_shift<<<grid, 256, 0, st>>>(a, (uint32_t)chunks_per_inst);
 }
 
 // Compaction of one instance table: delete entries with meta == 0 (marked) or

@@ -223,8 +223,10 @@ struct EvictArgs {
   unsigned long long* evicted;
   int32_t* err;
   GIndex gix;                  // deletions clear the instance's bit when gix.keys != NULL
+  int32_t* act;                // [W] instances over capacity (listed by the estimate pass)
+  unsigned* n_act;             // entries in act (zeroed by the launcher)
 };
-void launch_evict(const EvictArgs& a, int chunks_per_inst, cudaStream_t st);
+void launch_evict(const EvictArgs& a, int chunks_per_inst, int num_sms, cudaStream_t st);
 void launch_compact_marked(const EvictArgs& a, cudaStream_t st);
 
 struct MarkArgs {
