@@ -62,6 +62,23 @@ def kernels_per_step(rounds, global_index):
     return 7 + 5 * rounds + 8 + (1 if global_index else 0)
 
 
+def max_over_ranks(ms, dist, device):
+    """The largest of every rank's time (ms); the time itself on a single process.  Each rank
+    runs an independent replica, so the job takes as long as its slowest rank."""
+    if dist is None:
+        return float(ms)
+    import torch
+
+    t = torch.tensor([float(ms)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def whole_job_rate(units_per_rank, world, steps, max_ms):
+    """Units per second of the whole job: all ranks' units over the slowest rank's time."""
+    return world * units_per_rank * steps / max(max_ms / 1e3, 1e-12)
+
+
 def PHASE_KERNELS(rounds, global_index):
     """Kernel launches per phase of one route+commit (see kernels_per_step)."""
     return {"prologue": 2, "hash": 1, "caps": 1, "probe_first": 1, "probe_search": 1, "rounds": 5 * rounds,
@@ -359,12 +376,9 @@ def run_gb300(args):
     torch.cuda.synchronize()
     st = r.stats()
     r.sync()
-    if dist:
-        t = torch.tensor([total_ms], device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        total_ms = float(t.item())
+    total_ms = max_over_ranks(total_ms, dist, "cuda")
     n = sc.batch.n
-    value = world * n * K / (total_ms / 1e3)
+    value = whole_job_rate(n, world, K, total_ms)
 
     # end to end through the public host API: H2D of the batch from pinned memory, route, commit,
     # D2H of the decisions, every step
@@ -397,11 +411,8 @@ def run_gb300(args):
         e1.record(stream)
         e1.synchronize()
         e2e_ms += e0.elapsed_time(e1)
-    if dist:
-        t = torch.tensor([e2e_ms], device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        e2e_ms = float(t.item())
-    e2e = world * n * args.e2e_steps / max(e2e_ms / 1e3, 1e-9)
+    e2e_ms = max_over_ranks(e2e_ms, dist, "cuda")
+    e2e = whole_job_rate(n, world, args.e2e_steps, e2e_ms)
     log(f"e2e done: {e2e_ms / max(1, args.e2e_steps):.3f} ms/step")
     h2d = int(b.cls.nbytes + b.session.nbytes + b.tok_off.nbytes + b.tokens.nbytes)
     d2h = int(n * (4 + 1 + 4))
