@@ -307,6 +307,56 @@ int misat_phase_times(misat_ctx* ctx, float* ms_out);
 int misat_block_hash_noalloc(const int64_t* tok_off, const int32_t* tokens, int32_t n, int64_t n_tokens,
                              uint64_t hash_seed, uint64_t* keys_out, int64_t keys_cap, void* cuda_stream);
 
+/* ---- overload pressure controller (host only; Sec. 4.1) ----
+ * The operational cap K_w stays at or below its base floor(C_w / kbar_w).  A confirmed
+ * decline of instance w's prefix-cache hit rate relative to its recent healthy windows, or
+ * a persistent waiting queue, contracts the cap; it recovers gradually afterwards.  Per
+ * observation window and instance:
+ *   h_w   = floor(10^6 * hit_tokens / query_tokens) (none when query_tokens = 0)
+ *   h*_w  = the largest h of the last ref_windows healthy windows (once min_ref exist)
+ *   G_w   = max(0, h*_w - h_w)                         (the paper's hit-rate gap)
+ *   hit signal   G_w > gap_ppm and h_w <= the previous window's h (slope check)
+ *   queue signal waiting > queue_thresh
+ *   after `confirm` consecutive signalling windows, each further signalling window adds
+ *   max(1, floor(k_base * G_w / 10^6)) (hit) or max(1, floor(k_base / 8)) (queue),
+ *   whichever is larger; each run of recover_after windows without a signal removes 1;
+ *   the contraction stays within [0, floor(k_base * max_contraction_pct / 100)].
+ *   A window is healthy (joins the reference) when observed, G_w <= gap_ppm and no queue
+ *   signal.
+ * The paper gives the signals, not their thresholds: every number in the configuration is
+ * this library's choice (misat_overload_default_config).  The output is the
+ * cap_contraction argument of misat_set_instance_state.  No CUDA call is made. */
+typedef struct misat_overload misat_overload;
+typedef struct misat_overload_config {
+  int32_t ref_windows;         /* healthy windows kept for h*, 1..64 (8) */
+  int32_t min_ref;             /* healthy windows before G_w is evaluated, 1..ref_windows (3) */
+  int32_t gap_ppm;             /* hit-rate gap that signals degradation, 0..10^6 (100000) */
+  int32_t confirm;             /* consecutive signalling windows before a contraction, 1..1000 (2) */
+  int64_t queue_thresh;        /* waiting requests above which the queue signals, >= 0 (64) */
+  int32_t recover_after;       /* windows without a signal per recovery step, 1..1000 (2) */
+  int32_t max_contraction_pct; /* largest contraction in percent of the base cap, 0..100 (50) */
+} misat_overload_config;
+
+void misat_overload_default_config(misat_overload_config* cfg);
+/* W instances, 1..1024.  Errors: INVALID_ARG (a field out of range), OOM. */
+int misat_overload_create(int32_t n_instances, const misat_overload_config* cfg, misat_overload** out);
+int misat_overload_destroy(misat_overload* ov);
+/* One observation window, host arrays [W]: hit_tokens and query_tokens of the window's
+ * admitted requests (0 <= hit <= query <= 2^40), waiting requests, the base cap
+ * floor(C_w / kbar_w) (0..2^31); writes the new contraction per instance to
+ * contraction_out (may be NULL).  Errors: INVALID_ARG (state unchanged). */
+int misat_overload_observe(misat_overload* ov, const int64_t* hit_tokens, const int64_t* query_tokens,
+                           const int64_t* waiting, const int64_t* k_base, int32_t* contraction_out);
+
+/* ---- grouped-rollout recheck delays (host only; Sec. 4.1: the recheck delay of a held
+ * request decreases as more siblings of its prompt group become visible) ----
+ * Host arrays [n]: prompt group (0 = none) and held flag of each request the scheduler
+ * currently sees.  delay_out = 0 for a request not held, base_delay_us without a group, and
+ * max(min_delay_us, floor(base_delay_us / v)) with v = requests of its group in the list.
+ * The 1/v law is this library's choice (the paper gives none).  Errors: INVALID_ARG. */
+int misat_recheck_delays(int32_t n, const uint64_t* group, const uint8_t* held, int64_t base_delay_us,
+                         int64_t min_delay_us, int64_t* delay_out);
+
 /* Wait for the stream and return the sticky device error (0 if none), then clear it and
  * drop any pending route.  A batch rejected on the device changes no persistent state;
  * after TABLE_FULL during a commit the index of the affected instance may hold part of

@@ -65,6 +65,11 @@ class misat_batch_stats(C.Structure):
                 ("new_keys", C.c_int64), ("evicted", C.c_int64), ("seq", C.c_int64)]
 
 
+class misat_overload_config(C.Structure):
+    _fields_ = [("ref_windows", C.c_int32), ("min_ref", C.c_int32), ("gap_ppm", C.c_int32), ("confirm", C.c_int32),
+                ("queue_thresh", C.c_int64), ("recover_after", C.c_int32), ("max_contraction_pct", C.c_int32)]
+
+
 PHASES = ("prologue", "hash", "caps", "probe_first", "probe_search", "rounds", "finalize", "insert",
           "sessions", "evict")
 
@@ -99,6 +104,10 @@ _SIG = {
     "misat_set_timing": [_p, C.c_int],
     "misat_phase_times": [_p, _p],
     "misat_block_hash_noalloc": [_p, _p, C.c_int32, C.c_int64, C.c_uint64, _p, C.c_int64, _p],
+    "misat_overload_create": [C.c_int32, C.POINTER(misat_overload_config), C.POINTER(_p)],
+    "misat_overload_destroy": [_p],
+    "misat_overload_observe": [_p, _p, _p, _p, _p, _p],
+    "misat_recheck_delays": [C.c_int32, _p, _p, C.c_int64, C.c_int64, _p],
 }
 NOALLOC_MAX_REQUESTS = 65536
 
@@ -119,7 +128,9 @@ for _name, _args in _SIG.items():
 _lib.misat_strerror.argtypes = [C.c_int]
 _lib.misat_strerror.restype = C.c_char_p
 
-EXPORTS = sorted(list(_SIG) + ["misat_strerror"])
+_lib.misat_overload_default_config.argtypes = [C.POINTER(misat_overload_config)]
+_lib.misat_overload_default_config.restype = None
+EXPORTS = sorted(list(_SIG) + ["misat_strerror", "misat_overload_default_config"])
 
 
 class MisatError(RuntimeError):
@@ -391,3 +402,60 @@ class Checkpoint:
             self.free()
         except Exception:
             pass
+
+
+def _np_ptr(a):
+    return _p(a.ctypes.data)
+
+
+def overload_default_config() -> dict:
+    """The library's default overload-controller thresholds (misat_overload_default_config)."""
+    c = misat_overload_config()
+    _lib.misat_overload_default_config(C.byref(c))
+    return {f: getattr(c, f) for f, _ in misat_overload_config._fields_}
+
+
+class OverloadController:
+    """Per-instance overload pressure (Sec. 4.1) on the host: one observe() per window returns
+    the cap contraction to pass to Router.set_instance_state (misat_overload_*)."""
+
+    def __init__(self, n_instances: int, **cfg):
+        conf = overload_default_config()
+        conf.update(cfg)
+        c = misat_overload_config(**conf)
+        self.W = int(n_instances)
+        h = _p()
+        _ck(_lib.misat_overload_create(self.W, C.byref(c), C.byref(h)), "misat_overload_create")
+        self._h = h
+
+    def observe(self, hit_tokens, query_tokens, waiting, k_base) -> np.ndarray:
+        arrs = [np.ascontiguousarray(x, dtype=np.int64) for x in (hit_tokens, query_tokens, waiting, k_base)]
+        for x in arrs:
+            if x.shape != (self.W,):
+                raise ValueError("observe: every array must have one entry per instance")
+        out = np.zeros(self.W, dtype=np.int32)
+        _ck(_lib.misat_overload_observe(self._h, *[_np_ptr(x) for x in arrs], _np_ptr(out)), "misat_overload_observe")
+        return out
+
+    def close(self):
+        if self._h:
+            _lib.misat_overload_destroy(self._h)
+            self._h = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+
+def recheck_delays(group, held, base_delay_us: int, min_delay_us: int) -> np.ndarray:
+    """Recheck delay per request of the scheduler's current view (misat_recheck_delays)."""
+    g = np.ascontiguousarray(group, dtype=np.uint64)
+    h = np.ascontiguousarray(held, dtype=np.uint8)
+    if g.shape != h.shape or g.ndim != 1:
+        raise ValueError("recheck_delays: group and held must be 1-d arrays of one length")
+    out = np.zeros(g.shape[0], dtype=np.int64)
+    _ck(_lib.misat_recheck_delays(int(g.shape[0]), _np_ptr(g), _np_ptr(h), int(base_delay_us), int(min_delay_us),
+                                  _np_ptr(out)), "misat_recheck_delays")
+    return out
