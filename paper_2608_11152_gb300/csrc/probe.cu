@@ -10,8 +10,8 @@
 // bucket only when the bucket is full without a match.  Most pairs miss and finish
 // after one sector.  Pairs with block 0 resident and at least two blocks are
 // appended to a compact hit list (warp-aggregated).
-// Phase 2 (k2_probe_search): one thread per hit pair probes the last block
-// (fully cached prefixes finish there), then binary-searches [1, nb-1].
+// Phase 2 (k2_probe_search): a group of 16 lanes per hit pair searches [1, nb] with 16
+// parallel lookups per step (monotone predicate under prefix closure).
 #include "common.cuh"
 #include "kernels.h"
 
@@ -121,36 +121,57 @@ __global__ void __launch_bounds__(256) k2_probe_first_group(ProbeArgs a) {
   block_add_stats(a.stats, probes, reads);
 }
 
+// Phase 2: a group of kSG lanes per hit pair.  H is the largest h in [1, nb] with block h-1
+// resident, and residency is prefix-closed, so "block h-1 resident" holds exactly for
+// h <= H.  Each step the lanes test kSG points spread over the current interval [lo, hi]
+// (the last one at hi) with one table lookup each; the points that hold form a prefix, so
+// one ballot leaves an interval kSG times shorter: about log_kSG(nb) dependent lookups per
+// pair instead of log_2(nb).  Points that repeat (short intervals) are tested once.
+constexpr int kSG = 16;
+
 __global__ void __launch_bounds__(256) k2_probe_search(ProbeArgs a) {
   if (block_error(a.err)) return;
   const unsigned nh = *a.n_hits;
   const unsigned lim = (int64_t)nh < a.hits_cap ? nh : (unsigned)a.hits_cap;
+  const int lane = threadIdx.x & 31;
+  const int gl = lane & (kSG - 1);
+  const int g0 = lane & ~(kSG - 1);
+  const unsigned gmask = ((1u << kSG) - 1) << g0;
   unsigned long long probes = 0, reads = 0;
-  for (unsigned i = blockIdx.x * blockDim.x + threadIdx.x; i < lim; i += gridDim.x * blockDim.x) {
+  const unsigned groups = (gridDim.x * blockDim.x) / kSG;
+  for (unsigned i = (blockIdx.x * blockDim.x + threadIdx.x) / kSG; i < lim; i += groups) {
     const int2 pr = a.hits[i];
     const int r = pr.x, w = pr.y;
     const int32_t nb = a.nb[r];
     const uint64_t* k = a.keys + a.kbase[r];
     const InstDesc d = a.desc[w];
+    int32_t lo = 1, hi = nb;  // H in [lo, hi]; block 0 is resident
     uint32_t rd = 0;
-    int32_t h;
-    probes += 1;
-    if (table_contains(d, k[nb - 1], &rd)) {
-      h = nb;
-    } else {
-      int32_t lo = 1, hi = nb - 1;  // H in [lo, hi]: block 0 resident, block nb-1 not
-      while (lo < hi) {
-        const int32_t mid = (lo + hi + 1) >> 1;
+    while (lo < hi) {
+      const int64_t span = hi - lo;
+      // point of lane gl: lo + ceil((gl + 1) * span / kSG), increasing, the last one = hi
+      const int32_t h = lo + (int32_t)(((int64_t)(gl + 1) * span + kSG - 1) / kSG);
+      const int32_t hprev = gl == 0 ? lo : lo + (int32_t)(((int64_t)gl * span + kSG - 1) / kSG);
+      bool res = false;
+      if (h != hprev) {
         probes += 1;
-        if (table_contains(d, k[mid - 1], &rd))
-          lo = mid;
-        else
-          hi = mid - 1;
+        res = table_contains(d, k[h - 1], &rd) != 0;
       }
-      h = lo;
+      // repeated points take the answer of the lane that tested them
+      const unsigned tested = __ballot_sync(gmask, h != hprev) >> g0;
+      const unsigned yes = __ballot_sync(gmask, res) >> g0;
+      // lanes in increasing point order: the largest tested point that holds, and the
+      // smallest tested point that does not
+      const int last_yes = yes ? 31 - __clz(yes) : -1;
+      const unsigned no = tested & ~yes;
+      const int first_no = no ? __ffs(no) - 1 : kSG;
+      const int32_t nlo = last_yes >= 0 ? __shfl_sync(gmask, h, g0 + last_yes) : lo;
+      const int32_t nhi = first_no < kSG ? __shfl_sync(gmask, h, g0 + first_no) - 1 : hi;
+      lo = nlo;
+      hi = nhi;
     }
+    if (gl == 0) a.H[(int64_t)r * a.W + w] = (uint16_t)lo;
     reads += rd;
-    a.H[(int64_t)r * a.W + w] = (uint16_t)h;
   }
   block_add_stats(a.stats_search, probes, reads);
 }
@@ -256,7 +277,7 @@ void launch_probe_first(const ProbeArgs& a, int num_sms, cudaStream_t st) {
 
 void launch_probe_search(const ProbeArgs& a, int num_sms, cudaStream_t st) {
   if ((int64_t)a.n * a.W <= 0) return;
-  k2_probe_search<<<num_sms * 4, 256, 0, st>>>(a);
+  k2_probe_search<<<num_sms * 8, 256, 0, st>>>(a);
 }
 
 }  // namespace misat
