@@ -96,6 +96,7 @@ def parse_args():
     ap.add_argument("--e2e-steps", type=int, default=5)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--instances", type=int, default=128, help="fewer only for small profiling captures")
+    ap.add_argument("--cap", type=int, default=262144, help="blocks per instance; smaller only for profiling captures")
     ap.add_argument("--prefix-index", default="global", choices=["global", "per-instance"],
                     help="block-0 probe through the global key->instance-mask index or per instance table")
     ap.add_argument("--config", type=int, default=5, choices=[1, 2, 3, 4, 5],
@@ -147,7 +148,7 @@ def workload(args):
     from paper_2608_11152_gb300 import workload as wl
 
     if args.config == 5:
-        return wl.config5(n=args.n, fill=args.fill, instances=args.instances)
+        return wl.config5(n=args.n, fill=args.fill, instances=args.instances, cap=args.cap)
     return {1: wl.config1, 2: wl.config2, 3: wl.config3, 4: wl.config4}[args.config]()
 
 

@@ -197,15 +197,18 @@ __device__ __forceinline__ bool round_live(const RoundArgs& a) {
 template <int G, int CPL>
 __global__ void __launch_bounds__(256) k3_score(RoundArgs a) {
   extern __shared__ unsigned char smem[];
+  // backlog and token cost per instance, stored at w + w/8: the 8 lanes of a group read
+  // instances 8 apart, which this padding puts in 8 distinct bank pairs
+  const int wpad = a.W + (a.W >> 3) + 1;
   int64_t* s_bk = reinterpret_cast<int64_t*>(smem);
-  int64_t* s_tc = s_bk + a.W;
-  int32_t* s_gh = reinterpret_cast<int32_t*>(s_tc + a.W);
+  int64_t* s_tc = s_bk + wpad;
+  int32_t* s_gh = reinterpret_cast<int32_t*>(s_tc + wpad);
   int32_t* s_ch = s_gh + a.W;                                     // [W*3]
   uint8_t* s_el = reinterpret_cast<uint8_t*>(s_ch + 3 * a.W);     // [3][W]: headroom on w
   if (block_error(a.err) || !round_live(a)) return;
   for (int w = threadIdx.x; w < a.W; w += blockDim.x) {
-    s_bk[w] = a.ia.backlog_k[w];
-    s_tc[w] = a.tokcost[w];
+    s_bk[w + (w >> 3)] = a.ia.backlog_k[w];
+    s_tc[w + (w >> 3)] = a.tokcost[w];
     const int32_t gh = a.ia.gh[w];
     s_gh[w] = gh;
 #pragma unroll
@@ -290,7 +293,7 @@ __global__ void __launch_bounds__(256) k3_score(RoundArgs a) {
           if (w >= a.W) break;
           const int h = (int)((hw[i >> 1] >> (16 * (i & 1))) & 0xffffu);
           if (w == pw || el[w]) {
-            const int64_t cost = s_bk[w] + (Lr - 16 * (int64_t)h) * s_tc[w];
+            const int64_t cost = s_bk[w + (w >> 3)] + (Lr - 16 * (int64_t)h) * s_tc[w + (w >> 3)];
             if (cost < best_c) {
               best_c = cost;
               best_w = w;
@@ -331,8 +334,8 @@ __global__ void __launch_bounds__(256) k3_score(RoundArgs a) {
           if (sst == kSessReleased && hmax > 0) {
             const bool elig_hit = s_gh[whit] > 0 && s_ch[whit * 3 + b] > 0;
             if (!elig_hit) {
-              const int64_t lhs = a.hold_delay_q + s_bk[whit] - s_bk[best_w];
-              const int64_t rhs = 16 * (int64_t)hmax * s_tc[whit];
+              const int64_t lhs = a.hold_delay_q + s_bk[whit + (whit >> 3)] - s_bk[best_w + (best_w >> 3)];
+              const int64_t rhs = 16 * (int64_t)hmax * s_tc[whit + (whit >> 3)];
               if (lhs < rhs) {
                 choice = -1;
                 reason = MISAT_HOLD_PREFER_CACHE;
@@ -428,7 +431,13 @@ __global__ void __launch_bounds__(32) k4_admit(RoundArgs a) {
   const int t = blockIdx.x;
   const int lane = threadIdx.x;
   constexpr int kC = kTile / 32;  // chunks of 32 requests per tile
-  for (int k = lane; k < nb; k += 32) s_cnt[k] = a.tile_counts[(int64_t)t * nb + k];
+  if ((nb & 3) == 0) {  // rows start on 16-byte boundaries
+    const int4* src = reinterpret_cast<const int4*>(a.tile_counts + (int64_t)t * nb);
+    int4* dst = reinterpret_cast<int4*>(s_cnt);
+    for (int k = lane; k < (nb >> 2); k += 32) dst[k] = src[k];
+  } else {
+    for (int k = lane; k < nb; k += 32) s_cnt[k] = a.tile_counts[(int64_t)t * nb + k];
+  }
   // every load of the tile is issued before the in-order walk: the choosers, then the
   // headroom of their instances
   bool need[kC];
@@ -519,7 +528,7 @@ __global__ void __launch_bounds__(1024) k4_round_end(RoundArgs a) {
 }
 
 void launch_round(const RoundArgs& a, int num_sms, cudaStream_t st) {
-  const size_t score_smem = (size_t)a.W * (8 + 8 + 4 + 12 + 3);
+  const size_t score_smem = (size_t)16 * (a.W + (a.W >> 3) + 1) + (size_t)a.W * (4 + 12 + 3);
   int G = 4;
   while (G < 32 && G * 16 < a.W) G <<= 1;  // about two 8-instance chunks per lane
   const int64_t threads = (int64_t)a.n * G;
