@@ -150,7 +150,11 @@ struct misat_ctx {
   struct GraphCache {
     cudaGraphExec_t exec = nullptr;
     std::array<uint64_t, 4> key{};
-  } g_rounds, g_evict;
+  } g_rounds, g_evict, g_evict_apply;
+  // the commit's global-index pass runs on a side stream, beside the session update and
+  // the read-only half of the eviction, and joins before the deletions
+  cudaStream_t side_stream = nullptr;
+  cudaEvent_t ev_fork = nullptr, ev_join = nullptr;
   // phase timing: events 0..7 bracket the route phases, 8..11 the commit phases
   bool timing = false;
   cudaEvent_t ev[12] = {};
@@ -467,7 +471,9 @@ EvictArgs evict_args(misat_ctx* c, unsigned long long* evicted_counter) {
   return ev;
 }
 
-int evict_all(misat_ctx* c, unsigned long long* evicted_counter) {
+// Eviction of every instance above capacity; `join` (may be NULL) is waited for between the
+// read-only half and the deletions.
+int evict_all(misat_ctx* c, unsigned long long* evicted_counter, cudaEvent_t join = nullptr) {
   const EvictArgs ev = evict_args(c, evicted_counter);
   // streaming CTAs per instance: about 4 buckets per thread, at most 256 CTAs of 256
   uint32_t maxlg = 1;
@@ -475,7 +481,10 @@ int evict_all(misat_ctx* c, unsigned long long* evicted_counter) {
   const int chunks = (int)std::min<uint64_t>(256, std::max<uint64_t>(1, ((uint64_t)1 << maxlg) / (4 * 256)));
   const std::array<uint64_t, 4> key{(uint64_t)chunks, reinterpret_cast<uint64_t>(ev.gix.keys),
                                     (uint64_t)ev.gix.log2nb, reinterpret_cast<uint64_t>(evicted_counter)};
-  return run_graph(c, c->g_evict, key, [&](cudaStream_t s) { launch_evict(ev, chunks, c->num_sms, s); });
+  int rc = run_graph(c, c->g_evict, key, [&](cudaStream_t s) { launch_evict_select(ev, chunks, c->num_sms, s); });
+  if (rc) return rc;
+  if (join) CK(cudaStreamWaitEvent(c->stream, join, 0));
+  return run_graph(c, c->g_evict_apply, key, [&](cudaStream_t s) { launch_evict_apply(ev, chunks, c->num_sms, s); });
 }
 
 }  // namespace
@@ -501,7 +510,14 @@ int misat_destroy(misat_ctx* c) {
   cudaStreamSynchronize(c->stream);
   if (c->g_rounds.exec) cudaGraphExecDestroy(c->g_rounds.exec);
   if (c->g_evict.exec) cudaGraphExecDestroy(c->g_evict.exec);
+  if (c->g_evict_apply.exec) cudaGraphExecDestroy(c->g_evict_apply.exec);
   if (c->cap_stream) cudaStreamDestroy(c->cap_stream);
+  if (c->side_stream) {
+    cudaStreamSynchronize(c->side_stream);
+    cudaStreamDestroy(c->side_stream);
+  }
+  if (c->ev_fork) cudaEventDestroy(c->ev_fork);
+  if (c->ev_join) cudaEventDestroy(c->ev_join);
   for (size_t w = 0; w < c->h_desc.size(); ++w) {
     cudaFree(c->h_desc[w].tab);
     if (w < c->h_bufs.size()) free_bufs(c->h_bufs[w]);
@@ -572,6 +588,13 @@ int misat_create(const misat_config* cfg, void* cuda_stream, misat_ctx** out) {
     cudaGetLastError();
     c->cap_stream = nullptr;  // sequences are then launched directly
   }
+  if (cudaStreamCreateWithFlags(&c->side_stream, cudaStreamNonBlocking) != cudaSuccess ||
+      cudaEventCreateWithFlags(&c->ev_fork, cudaEventDisableTiming) != cudaSuccess ||
+      cudaEventCreateWithFlags(&c->ev_join, cudaEventDisableTiming) != cudaSuccess) {
+    cudaGetLastError();
+    if (c->side_stream) cudaStreamDestroy(c->side_stream);
+    c->side_stream = nullptr;  // the global-index pass then runs on the context's stream
+  }
   if (cudaMallocHost(&c->h_meta, c->ml.words * 8) != cudaSuccess) return fail(MISAT_ERR_OOM);
   std::memset(c->h_meta, 0, c->ml.words * 8);
 
@@ -592,7 +615,7 @@ int misat_create(const misat_config* cfg, void* cuda_stream, misat_ctx** out) {
       (rc = dalloc_n(c, &c->rq.leader, NB)) || (rc = dalloc_n(c, &c->rq.status, NB)) ||
       (rc = dalloc_n(c, &c->rq.choice, NB)) || (rc = dalloc_n(c, &c->rq.last_reason, NB)) ||
       (rc = dalloc_n(c, &c->rq.inst, NB)) || (rc = dalloc_n(c, &c->rq.reason, NB)) ||
-      (rc = dalloc_n(c, &c->rq.hmax, NB)) ||
+      (rc = dalloc_n(c, &c->rq.hbest, NB)) ||
       (rc = dalloc_n(c, &c->ia.K_w, Ws)) || (rc = dalloc_n(c, &c->ia.K_wb, 3 * Ws)) ||
       (rc = dalloc_n(c, &c->ia.N_wb, 3 * Ws)) || (rc = dalloc_n(c, &c->ia.kbar_w, Ws)) ||
       (rc = dalloc_n(c, &c->ia.tot, Ws)) || (rc = dalloc_n(c, &c->ia.gh, Ws)) || (rc = dalloc_n(c, &c->ia.ch, 3 * Ws)) ||
@@ -758,6 +781,7 @@ int misat_route(misat_ctx* c, const misat_batch* b, misat_decisions* out) {
   pr.keys = c->d_keys;
   pr.H = c->d_H;
   pr.hits = c->d_hits;
+  pr.hbest = c->rq.hbest;
   pr.n_hits = c->nhits_ptr();
   pr.hits_cap = c->hits_cap;
   pr.stats = c->stats_ptr() + 16;
@@ -889,12 +913,24 @@ int misat_commit(misat_ctx* c) {
     ia.gnew = c->d_gnew;
     ia.n_gnew = c->d_gnew_n;
     ia.gnew_cap = c->keys_cap;
-    launch_insert(ia, c->num_sms, st);
+    launch_insert_tables(ia, c->num_sms, st);
     c->mark(9);
+    cudaEvent_t join = nullptr;
+    if (ia.gix.keys) {
+      if (c->side_stream) {
+        CK(cudaEventRecord(c->ev_fork, st));
+        CK(cudaStreamWaitEvent(c->side_stream, c->ev_fork, 0));
+        launch_insert_gix(ia, c->num_sms * 4, c->side_stream);
+        CK(cudaEventRecord(c->ev_join, c->side_stream));
+        join = c->ev_join;
+      } else {
+        launch_insert_gix(ia, c->num_sms * 8, st);
+      }
+    }
     SessUpdateArgs sa{n, c->rq, c->sess, c->d_prot, c->err_ptr()};
     launch_session_update(sa, st);
     c->mark(10);
-    int rc = evict_all(c, c->stats_ptr() + 19);
+    int rc = evict_all(c, c->stats_ptr() + 19, join);
     if (rc) return rc;
   } else {
     c->mark(9);

@@ -250,13 +250,22 @@ __global__ void __launch_bounds__(256) k4_gix_insert(InsertArgs a) {
   if (threadIdx.x == 0 && tot) atomicAdd(a.gix.used, (unsigned long long)tot);
 }
 
-void launch_insert(const InsertArgs& a, int num_sms, cudaStream_t st) {
+void launch_insert_tables(const InsertArgs& a, int num_sms, cudaStream_t st) {
   if (a.n <= 0) return;
   cudaMemsetAsync(a.n_units, 0, sizeof(unsigned), st);
   if (a.gix.keys) cudaMemsetAsync(a.n_gnew, 0, sizeof(unsigned), st);
   k4_units<<<(a.n + 255) / 256, 256, 0, st>>>(a);
   k4_insert<<<num_sms * 3, kInsThreads, 0, st>>>(a);  // resident CTAs: 3 per SM
-  if (a.gix.keys) k4_gix_insert<<<num_sms * 8, 256, 0, st>>>(a);
+}
+
+void launch_insert_gix(const InsertArgs& a, int ctas, cudaStream_t st) {
+  if (a.n <= 0 || !a.gix.keys) return;
+  k4_gix_insert<<<ctas, 256, 0, st>>>(a);
+}
+
+void launch_insert(const InsertArgs& a, int num_sms, cudaStream_t st) {
+  launch_insert_tables(a, num_sms, st);
+  launch_insert_gix(a, num_sms * 8, st);
 }
 
 __global__ void __launch_bounds__(256) k4_insert_entries(EntryInsertArgs a) {

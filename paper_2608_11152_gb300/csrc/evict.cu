@@ -512,17 +512,31 @@ __global__ void __launch_bounds__(256) k4_evict_shift(EvictArgs a, uint32_t chun
   for (uint32_t it = blockIdx.x; it < items; it += gridDim.x) shift_chunk(a, a.act[it / chunks], it % chunks, chunks);
 }
 
-void launch_evict(const EvictArgs& a, int chunks_per_inst, int num_sms, cudaStream_t st) {
-  const int W = a.only_w ? 1 : a.W;
+namespace {
+int stream_grid(const EvictArgs& a, int chunks_per_inst, int num_sms) {
   // streaming passes: resident CTAs over (active instance, chunk) items
-  const int64_t items = (int64_t)W * chunks_per_inst;
-  const int grid = (int)(items < (int64_t)num_sms * 8 ? items : (int64_t)num_sms * 8);
+  const int64_t items = (int64_t)(a.only_w ? 1 : a.W) * chunks_per_inst;
+  return (int)(items < (int64_t)num_sms * 8 ? items : (int64_t)num_sms * 8);
+}
+}  // namespace
+
+void launch_evict_select(const EvictArgs& a, int chunks_per_inst, int num_sms, cudaStream_t st) {
+  const int W = a.only_w ? 1 : a.W;
   cudaMemsetAsync(a.n_act, 0, sizeof(unsigned), st);
   k4_evict_estimate<<<W, kSelThreads, 0, st>>>(a);
-  k4_evict_collect<<<grid, 256, 0, st>>>(a, (uint32_t)chunks_per_inst);
+  k4_evict_collect<<<stream_grid(a, chunks_per_inst, num_sms), 256, 0, st>>>(a, (uint32_t)chunks_per_inst);
   k4_evict_select<<<W, kSelThreads, 0, st>>>(a);
+}
+
+void launch_evict_apply(const EvictArgs& a, int chunks_per_inst, int num_sms, cudaStream_t st) {
+  const int grid = stream_grid(a, chunks_per_inst, num_sms);
   k4_evict_delete<<<grid, 256, 0, st>>>(a, (uint32_t)chunks_per_inst);
   k4_evict_shift<<<grid, 256, 0, st>>>(a, (uint32_t)chunks_per_inst);
+}
+
+void launch_evict(const EvictArgs& a, int chunks_per_inst, int num_sms, cudaStream_t st) {
+  launch_evict_select(a, chunks_per_inst, num_sms, st);
+  launch_evict_apply(a, chunks_per_inst, num_sms, st);
 }
 
 // Compaction of one instance table: delete entries with meta == 0 (marked) or

@@ -38,7 +38,8 @@ struct ReqArrays {
   uint8_t* last_reason; // hold reason if it stays unresolved
   int32_t* inst;        // decision (internal copy)
   uint8_t* reason;      // reason (internal copy)
-  int32_t* hmax;        // max over instances of H_rw (set by the score kernel for leaders)
+  uint32_t* hbest;      // max over instances of (H_rw << 16 | 65535 - w): the largest H and,
+                        // among instances with it, the lowest index (set by the probe kernels)
 };
 
 // ---- per-instance round state ----
@@ -67,6 +68,7 @@ struct ProbeArgs {
   const uint64_t* keys;
   uint16_t* H;                 // [n*W]
   int2* hits;                  // (r, w) pairs with block 0 resident and nb >= 2
+  uint32_t* hbest;             // [n] packed best (H, instance) per request, see ReqArrays
   unsigned* n_hits;
   int64_t hits_cap;
   unsigned long long* stats;         // phase 1: [0] probes, [1] bucket reads
@@ -171,7 +173,9 @@ struct InsertArgs {
   unsigned* n_gnew;            //   global index pass (zeroed by the launcher)
   int64_t gnew_cap;
 };
-void launch_insert(const InsertArgs& a, int num_sms, cudaStream_t st);
+void launch_insert(const InsertArgs& a, int num_sms, cudaStream_t st);  // tables, then global index
+void launch_insert_tables(const InsertArgs& a, int num_sms, cudaStream_t st);
+void launch_insert_gix(const InsertArgs& a, int ctas, cudaStream_t st);
 
 struct EntryInsertArgs {
   InstDesc desc;
@@ -227,6 +231,10 @@ struct EvictArgs {
   unsigned* n_act;             // entries in act (zeroed by the launcher)
 };
 void launch_evict(const EvictArgs& a, int chunks_per_inst, int num_sms, cudaStream_t st);
+// the two halves: select (estimate, collect, select; reads the tables only) and apply
+// (delete, shift; also clears global-index bits)
+void launch_evict_select(const EvictArgs& a, int chunks_per_inst, int num_sms, cudaStream_t st);
+void launch_evict_apply(const EvictArgs& a, int chunks_per_inst, int num_sms, cudaStream_t st);
 void launch_compact_marked(const EvictArgs& a, cudaStream_t st);
 
 struct MarkArgs {

@@ -75,6 +75,7 @@ __global__ void __launch_bounds__(256) k2_probe_first_group(ProbeArgs a) {
       nb = a.nb[r];
       if (nb > 0) key = a.keys[a.kbase[r]];
     }
+    int wmin = INT32_MAX;  // lowest instance holding block 0
     for (int w0 = 0; w0 < a.W; w0 += S * kIlp) {
       int res[kIlp];
       uint32_t rd[kIlp];
@@ -94,6 +95,7 @@ __global__ void __launch_bounds__(256) k2_probe_first_group(ProbeArgs a) {
       for (int i = 0; i < kIlp; ++i) {
         const int w = w0 + i * S + sub;
         const bool valid = live && w < a.W;
+        if (valid && res[i]) wmin = min(wmin, w);
         if (valid) {
           a.H[(int64_t)r * a.W + w] = (uint16_t)res[i];
           if (nb > 0) {
@@ -117,6 +119,9 @@ __global__ void __launch_bounds__(256) k2_probe_first_group(ProbeArgs a) {
         }
       }
     }
+#pragma unroll
+    for (int o = S / 2; o > 0; o >>= 1) wmin = min(wmin, __shfl_xor_sync(0xffffffffu, wmin, o, S));
+    if (live && sub == 0) a.hbest[r] = wmin < a.W ? (1u << 16) | (65535u - (uint32_t)wmin) : 65535u;
   }
   block_add_stats(a.stats, probes, reads);
 }
@@ -170,7 +175,10 @@ __global__ void __launch_bounds__(256) k2_probe_search(ProbeArgs a) {
       lo = nlo;
       hi = nhi;
     }
-    if (gl == 0) a.H[(int64_t)r * a.W + w] = (uint16_t)lo;
+    if (gl == 0) {
+      a.H[(int64_t)r * a.W + w] = (uint16_t)lo;
+      atomicMax(a.hbest + r, ((uint32_t)lo << 16) | (65535u - (uint32_t)w));
+    }
     reads += rd;
   }
   block_add_stats(a.stats_search, probes, reads);
@@ -202,12 +210,14 @@ __global__ void __launch_bounds__(256) k2_probe_first_gix(ProbeArgs a) {
         reads += rd;
       }
     }
-    int bits = 0;
+    int bits = 0, wmin = INT32_MAX;
     for (uint32_t i = 0; i < mw; ++i) {
       const unsigned long long m = slot >= 0 ? __ldg(a.gix.masks + (size_t)slot * mw + i) : 0ull;
       sm[lane * mw + i] = m;
       bits += __popcll(m);
+      if (m && wmin == INT32_MAX) wmin = 64 * (int)i + __ffsll((long long)m) - 1;
     }
+    if (r < a.n) a.hbest[r] = wmin < a.W ? (1u << 16) | (65535u - (uint32_t)wmin) : 65535u;
     // hit-list positions: one atomic per warp
     const int nh = nb > 1 ? bits : 0;
     int incl = nh;

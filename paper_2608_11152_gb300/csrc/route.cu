@@ -253,6 +253,7 @@ __global__ void __launch_bounds__(256) k3_score(RoundArgs a) {
     const int64_t rk = base + (int64_t)gl * ngroups;
     uint8_t st = kStResolved, kb = 0, ksst = 0;
     int ksinst = -1, kL = 0;
+    uint32_t khb = 0;
     if (rk < a.n) {
       st = a.rq.status[rk];
       if (st == kStUnresolved) {
@@ -260,6 +261,7 @@ __global__ void __launch_bounds__(256) k3_score(RoundArgs a) {
         ksst = a.rq.sst[rk];
         ksinst = a.rq.sinst[rk];
         kL = a.rq.L[rk];
+        khb = a.rq.hbest[rk];
       }
     }
     unsigned todo = (__ballot_sync(gmask, st == kStUnresolved) >> g0) & (G == 32 ? kFull : ((1u << G) - 1));
@@ -277,11 +279,12 @@ __global__ void __launch_bounds__(256) k3_score(RoundArgs a) {
       const uint8_t sst = (uint8_t)__shfl_sync(gmask, (int)ksst, g0 + k);
       const int sinst = __shfl_sync(gmask, ksinst, g0 + k);
       const int64_t Lr = __shfl_sync(gmask, kL, g0 + k);
+      const uint32_t hb = __shfl_sync(gmask, khb, g0 + k);
+      const int hmax = (int)(hb >> 16), whit = 65535 - (int)(hb & 0xffffu);  // max H, lowest such w
       const int pw = sst == kSessProtected ? sinst : -1;
       const uint8_t* el = s_el + b * a.W;
       int64_t best_c = INT64_MAX;
       int best_w = INT32_MAX;
-      int hmax = -1, whit = INT32_MAX;
 #pragma unroll
       for (int c = 0; c < CPL; ++c) {
         const int ck = gl + G * c;
@@ -299,10 +302,6 @@ __global__ void __launch_bounds__(256) k3_score(RoundArgs a) {
               best_w = w;
             }
           }
-          if (h > hmax) {
-            hmax = h;
-            whit = w;
-          }
         }
       }
 #pragma unroll
@@ -313,15 +312,8 @@ __global__ void __launch_bounds__(256) k3_score(RoundArgs a) {
           best_c = oc;
           best_w = ow;
         }
-        const int oh = __shfl_xor_sync(gmask, hmax, o, G);
-        const int owh = __shfl_xor_sync(gmask, whit, o, G);
-        if (oh > hmax || (oh == hmax && owh < whit)) {
-          hmax = oh;
-          whit = owh;
-        }
       }
       if (gl == 0) {
-        a.rq.hmax[r] = hmax < 0 ? 0 : hmax;
         int choice = -1;
         uint8_t reason = 0;
         if (best_w == INT32_MAX) {
@@ -559,12 +551,14 @@ __global__ void __launch_bounds__(256) k4_finalize(FinalizeArgs a) {
   if (threadIdx.x < 16) s_st[threadIdx.x] = 0;
   __syncthreads();
   const int r = blockIdx.x * blockDim.x + threadIdx.x;
+  const int lane = threadIdx.x & 31;
+  int w = -1, hb = 0, b = 0, ri = -1, L = 0;
   if (r < a.n) {
-    int w;
     uint8_t reason;
     const uint8_t stv = a.rq.status[r];
+    const int ld = a.rq.leader[r];
     if (stv == kStFollower) {
-      w = a.rq.inst[a.rq.leader[r]];
+      w = a.rq.inst[ld];
       reason = w >= 0 ? MISAT_ADMIT_FOLLOW : MISAT_HOLD_LEADER_HELD;
     } else if (stv == kStUnresolved || stv == kStHeld) {
       w = -1;
@@ -573,15 +567,7 @@ __global__ void __launch_bounds__(256) k4_finalize(FinalizeArgs a) {
       w = a.rq.inst[r];
       reason = a.rq.reason[r];
     }
-    const uint16_t* Hr = a.H + (int64_t)r * a.W;
-    int hb = 0;
-    if (w >= 0) {
-      hb = Hr[w];
-    } else if (stv != kStFollower) {
-      hb = a.rq.hmax[r];  // every leader was scored at least once
-    } else {
-      for (int x = 0; x < a.W; ++x) hb = Hr[x] > hb ? Hr[x] : hb;
-    }
+    hb = w >= 0 ? (int)a.H[(int64_t)r * a.W + w] : (int)(a.rq.hbest[r] >> 16);  // HOLD: max over instances
     if (stv == kStFollower) {
       a.rq.inst[r] = w;
       a.rq.reason[r] = reason;
@@ -591,17 +577,28 @@ __global__ void __launch_bounds__(256) k4_finalize(FinalizeArgs a) {
     a.out_inst[r] = w;
     a.out_reason[r] = reason;
     a.out_hit[r] = hb;
-    const int ri = reason < 16 ? reason - 1 : 3 + (reason - 16);
-    atomicAdd(&s_st[ri], 1ull);
-    const int b = a.rq.cls[r];
+    ri = reason < 16 ? reason - 1 : 3 + (reason - 16);
+    b = a.rq.cls[r];
     if (w >= 0) {
-      atomicAdd(&s_st[8 + b], 1ull);
-      atomicAdd(&s_st[14], (unsigned long long)(16 * hb));
-      atomicAdd(&s_st[15], (unsigned long long)a.rq.L[r]);
+      L = a.rq.L[r];
       atomic_add_i64(&a.U[w], (long long)(a.rq.nb[r] - hb));
-    } else {
-      atomicAdd(&s_st[11 + b], 1ull);
     }
+  }
+  // statistics: warp ballots and sums, one shared-memory add per warp and counter
+  unsigned c[16];
+#pragma unroll
+  for (int v = 0; v < 8; ++v) c[v] = __popc(__ballot_sync(0xffffffffu, ri == v));
+#pragma unroll
+  for (int v = 0; v < 3; ++v) {
+    c[8 + v] = __popc(__ballot_sync(0xffffffffu, ri >= 0 && w >= 0 && b == v));
+    c[11 + v] = __popc(__ballot_sync(0xffffffffu, ri >= 0 && w < 0 && b == v));
+  }
+  c[14] = __reduce_add_sync(0xffffffffu, w >= 0 ? (unsigned)(16 * hb) : 0u);
+  c[15] = __reduce_add_sync(0xffffffffu, w >= 0 ? (unsigned)L : 0u);
+  if (lane == 0) {
+#pragma unroll
+    for (int v = 0; v < 16; ++v)
+      if (c[v]) atomicAdd(&s_st[v], (unsigned long long)c[v]);
   }
   __syncthreads();
   if (threadIdx.x < 16 && s_st[threadIdx.x]) atomicAdd(&a.stats[threadIdx.x], s_st[threadIdx.x]);
