@@ -96,7 +96,19 @@ __global__ void __launch_bounds__(256) k0_leaders(PrologueArgs a) {
     }
     a.rq.leader[r] = ld;
     a.rq.status[r] = ld == r ? kStUnresolved : kStFollower;
-    if (ld == r && a.rq.sst[r] != kSessProtected) atomicAdd(&s_cand[a.rq.cls[r]], 1ull);
+  }
+  {
+    // candidate sessions by class: warp ballots, one shared add per warp and class
+    const bool cand = r < a.n && a.rq.leader[r] == r && a.rq.sst[r] != kSessProtected;
+    const int b = cand ? a.rq.cls[r] : -1;
+    const unsigned c0 = __popc(__ballot_sync(0xffffffffu, b == 0));
+    const unsigned c1 = __popc(__ballot_sync(0xffffffffu, b == 1));
+    const unsigned c2 = __popc(__ballot_sync(0xffffffffu, b == 2));
+    if ((threadIdx.x & 31) == 0) {
+      if (c0) atomicAdd(&s_cand[0], (unsigned long long)c0);
+      if (c1) atomicAdd(&s_cand[1], (unsigned long long)c1);
+      if (c2) atomicAdd(&s_cand[2], (unsigned long long)c2);
+    }
   }
   __syncthreads();
   if (threadIdx.x < 3 && s_cand[threadIdx.x]) atomicAdd((unsigned long long*)&a.cand[threadIdx.x], s_cand[threadIdx.x]);
