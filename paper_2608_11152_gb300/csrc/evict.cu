@@ -366,9 +366,20 @@ __global__ void __launch_bounds__(kSelThreads) k4_evict_select(EvictArgs a) {
     Erem -= bl;
     if (tid == 0) s_cnt = 0;
     __syncthreads();
-    for (unsigned i = tid; i < cnt; i += kSelThreads) {
-      const uint4 v = cur[i];
-      if (digit128(v_hi(v), v_lo(v), shift) == (uint32_t)t) nxt[atomicAdd(&s_cnt, 1u)] = v;
+    for (unsigned i0 = 0; i0 < cnt; i0 += kSelThreads) {
+      // keep the target bin: one shared add per warp, positions by ballot rank
+      const unsigned i = i0 + tid;
+      uint4 v = make_uint4(0, 0, 0, 0);
+      bool keep = false;
+      if (i < cnt) {
+        v = cur[i];
+        keep = digit128(v_hi(v), v_lo(v), shift) == (uint32_t)t;
+      }
+      const unsigned bal = __ballot_sync(kFull, keep);
+      unsigned base = 0;
+      if ((tid & 31) == 0 && bal) base = atomicAdd(&s_cnt, (unsigned)__popc(bal));
+      base = __shfl_sync(kFull, base, 0);
+      if (keep) nxt[base + __popc(bal & lanemask_lt())] = v;
     }
     __syncthreads();
     cnt = s_cnt;

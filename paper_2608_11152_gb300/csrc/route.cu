@@ -380,12 +380,17 @@ __global__ void __launch_bounds__(256) k4_tile_count(RoundArgs a) {
   for (int k = threadIdx.x; k < nb; k += blockDim.x) s_cnt[k] = 0;
   __syncthreads();
   const int t = blockIdx.x;
-  for (int i = threadIdx.x; i < kTile; i += blockDim.x) {
+  for (int i0 = 0; i0 < kTile; i0 += blockDim.x) {
+    // choosers herd to the same (instance, class): one shared add per group of equal keys
+    const int i = i0 + (int)threadIdx.x;
     const int r = t * kTile + i;
-    if (r < a.n && a.rq.status[r] == kStUnresolved) {
+    int key = -1;
+    if (i < kTile && r < a.n && a.rq.status[r] == kStUnresolved) {
       const int c = a.rq.choice[r];
-      if (c >= 0) atomicAdd(&s_cnt[c * 3 + a.rq.cls[r]], 1);
+      if (c >= 0) key = c * 3 + a.rq.cls[r];
     }
+    const unsigned peers = __match_any_sync(kFull, key);
+    if (key >= 0 && (int)(threadIdx.x & 31) == __ffs(peers) - 1) atomicAdd(&s_cnt[key], __popc(peers));
   }
   __syncthreads();
   int32_t* out = a.tile_counts + (int64_t)t * nb;
