@@ -192,9 +192,14 @@ __global__ void __launch_bounds__(kSelThreads) k4_evict_estimate(EvictArgs a) {
   }
 }
 
-// Streaming pass over the instance's metas: chunk `cidx` of `chunks` of instance w.
+// Streaming pass over the instance's metas: chunk `cidx` of `chunks` of instance w, a range
+// of whole 32-bucket bitmap words.  A CTA takes 4 x blockDim buckets at a time: each thread
+// loads the metas of four buckets (all loads in flight together), keeps only which slots
+// are certainly evicted (meta < lo) or candidates (lo <= meta <= hi) as bit masks, writes
+// the fullness bitmap words and clears the deleted-slot masks; the list entries are
+// reserved with one CTA-wide scan per step, and only candidates re-read their meta and key.
 __device__ __forceinline__ void collect_chunk(const EvictArgs& a, int w, uint32_t cidx, uint32_t chunks) {
-  __shared__ unsigned s_wd[8], s_wu[8], s_bd, s_bu;
+  __shared__ unsigned s_wd[32], s_wu[32], s_bd, s_bu;
   const InstDesc d = a.desc[w];
   const uint32_t NB = 1u << d.log2nb;
   const unsigned long long lo = a.thr_lo[w], hi = a.thr_hi[w];
@@ -204,27 +209,41 @@ __device__ __forceinline__ void collect_chunk(const EvictArgs& a, int w, uint32_
   uint4* u = a.cand_a[w];
   uint32_t* usl = a.slots[w];
   const int lane = threadIdx.x & 31;
-  const uint32_t stride = chunks * blockDim.x;
-  for (uint32_t b0 = cidx * blockDim.x; b0 < NB; b0 += stride) {
-    const uint32_t b = b0 + threadIdx.x;
-    unsigned long long m[4] = {0, 0, 0, 0};
-    bool full = false;
-    if (b < NB) {
-      const ulonglong2* mp = reinterpret_cast<const ulonglong2*>(d.tab[b].meta);
-      const ulonglong2 m01 = __ldcg(mp), m23 = __ldcg(mp + 1);
-      m[0] = m01.x;
-      m[1] = m01.y;
-      m[2] = m23.x;
-      m[3] = m23.y;
-      full = m[0] && m[1] && m[2] && m[3];
-    }
-    int nd = 0, nu = 0;
+  const int wid = threadIdx.x >> 5;
+  const uint32_t words = (NB + 31) >> 5;
+  const uint32_t b_beg = (uint32_t)(((uint64_t)words * cidx / chunks) << 5);
+  const uint32_t b_end = min(NB, (uint32_t)(((uint64_t)words * (cidx + 1) / chunks) << 5));
+  for (uint32_t base = b_beg; base < b_end; base += 4 * blockDim.x) {
+    ulonglong2 m01[4], m23[4];
 #pragma unroll
-    for (int s = 0; s < 4; ++s) {
-      if (!m[s]) continue;
-      if (m[s] < lo) ++nd;
-      else if (m[s] <= hi) ++nu;
+    for (int k = 0; k < 4; ++k) {
+      const uint32_t b = base + k * blockDim.x + threadIdx.x;
+      if (b < b_end) {
+        const ulonglong2* mp = reinterpret_cast<const ulonglong2*>(d.tab[b].meta);
+        m01[k] = __ldcg(mp);
+        m23[k] = __ldcg(mp + 1);
+      } else {
+        m01[k] = make_ulonglong2(0, 0);
+        m23[k] = make_ulonglong2(0, 0);
+      }
     }
+    unsigned dm = 0, um = 0;  // bit 4k + s: slot s of this thread's k-th bucket
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      const uint32_t b = base + k * blockDim.x + threadIdx.x;
+      const unsigned long long m[4] = {m01[k].x, m01[k].y, m23[k].x, m23[k].y};
+      const bool full = m[0] && m[1] && m[2] && m[3];
+      const unsigned bits = __ballot_sync(kFull, full);
+      if (lane == 0 && b < b_end) bitmap[b >> 5] = bits;
+      if ((lane & 7) == 0 && b < b_end) dmask[b >> 3] = 0;
+#pragma unroll
+      for (int sl = 0; sl < 4; ++sl) {
+        if (!m[sl]) continue;
+        if (m[sl] < lo) dm |= 1u << (4 * k + sl);
+        else if (m[sl] <= hi) um |= 1u << (4 * k + sl);
+      }
+    }
+    const int nd = __popc(dm), nu = __popc(um);
     // CTA-wide reservation in both lists: warp scans, then one atomic pair per CTA
     int id = nd, iu = nu;
 #pragma unroll
@@ -235,7 +254,6 @@ __device__ __forceinline__ void collect_chunk(const EvictArgs& a, int w, uint32_
         iu += vu;
       }
     }
-    const int wid = threadIdx.x >> 5;
     if (lane == 31) {
       s_wd[wid] = id;
       s_wu[wid] = iu;
@@ -256,22 +274,24 @@ __device__ __forceinline__ void collect_chunk(const EvictArgs& a, int w, uint32_
     __syncthreads();
     unsigned bd = s_bd + s_wd[wid] + (unsigned)(id - nd);
     unsigned bu = s_bu + s_wu[wid] + (unsigned)(iu - nu);
-    __syncthreads();  // the shared offsets are rewritten by the next iteration
-#pragma unroll
-    for (int s = 0; s < 4; ++s) {
-      if (!m[s]) continue;
-      if (m[s] < lo) {
-        dsl[bd++] = b * 4 + s;
-      } else if (m[s] <= hi) {
-        const unsigned long long key = __ldcg(&d.tab[b].key[s]);
-        u[bu] = make_uint4((uint32_t)m[s], (uint32_t)(m[s] >> 32), (uint32_t)key, (uint32_t)(key >> 32));
-        usl[bu] = b * 4 + s;
-        ++bu;
-      }
+    __syncthreads();  // the shared offsets are rewritten by the next step
+    while (dm) {
+      const int bit = __ffs(dm) - 1;
+      dm &= dm - 1;
+      const uint32_t b = base + (bit >> 2) * blockDim.x + threadIdx.x;
+      dsl[bd++] = b * 4 + (bit & 3);
     }
-    const unsigned bits = __ballot_sync(kFull, full);
-    if (lane == 0 && b < NB) bitmap[b >> 5] = bits;
-    if ((lane & 7) == 0 && b < NB) dmask[b >> 3] = 0;
+    while (um) {
+      const int bit = __ffs(um) - 1;
+      um &= um - 1;
+      const uint32_t b = base + (bit >> 2) * blockDim.x + threadIdx.x;
+      const int sl = bit & 3;
+      const unsigned long long x = __ldcg(&d.tab[b].meta[sl]);
+      const unsigned long long key = __ldcg(&d.tab[b].key[sl]);
+      u[bu] = make_uint4((uint32_t)x, (uint32_t)(x >> 32), (uint32_t)key, (uint32_t)(key >> 32));
+      usl[bu] = b * 4 + sl;
+      ++bu;
+    }
   }
 }
 
