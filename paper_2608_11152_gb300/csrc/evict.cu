@@ -560,9 +560,13 @@ void launch_evict_select(const EvictArgs& a, int chunks_per_inst, int num_sms, c
 }
 
 void launch_evict_apply(const EvictArgs& a, int chunks_per_inst, int num_sms, cudaStream_t st) {
-  const int grid = stream_grid(a, chunks_per_inst, num_sms);
-  k4_evict_delete<<<grid, 256, 0, st>>>(a, (uint32_t)chunks_per_inst);
-  k4_evict_shift<<<grid, 256, 0, st>>>(a, (uint32_t)chunks_per_inst);
+  // the eviction lists (about E entries per instance) are split into fewer, larger pieces
+  // than the tables: each piece then holds several entries per thread
+  (void)chunks_per_inst;
+  constexpr int kListChunks = 32;
+  const int grid = stream_grid(a, kListChunks, num_sms);
+  k4_evict_delete<<<grid, 256, 0, st>>>(a, (uint32_t)kListChunks);
+  k4_evict_shift<<<grid, 256, 0, st>>>(a, (uint32_t)kListChunks);
 }
 
 void launch_evict(const EvictArgs& a, int chunks_per_inst, int num_sms, cudaStream_t st) {
