@@ -149,8 +149,9 @@ struct misat_ctx {
   cudaStream_t cap_stream = nullptr;
   struct GraphCache {
     cudaGraphExec_t exec = nullptr;
-    std::array<uint64_t, 4> key{};
-  } g_rounds, g_evict, g_evict_apply;
+    std::vector<uint64_t> key;
+  } g_evict, g_evict_apply, g_route;
+  int64_t* d_params = nullptr;  // [9] per-route class parameters (caps)
   // the commit's global-index pass runs on a side stream, beside the session update and
   // the read-only half of the eviction, and joins before the deletions
   cudaStream_t side_stream = nullptr;
@@ -161,6 +162,9 @@ struct misat_ctx {
 
   void mark(int i) {
     if (timing) cudaEventRecord(ev[i], stream);
+  }
+  void mark(int i, cudaStream_t s) {
+    if (timing) cudaEventRecord(ev[i], s);
   }
 
   long long* size_ptr() { return reinterpret_cast<long long*>(d_meta + ml.size); }
@@ -187,7 +191,7 @@ namespace {
 // replayed with one graph launch.  When the context's stream is itself being captured by
 // the caller, or capture is unavailable, the sequence is launched directly.
 template <class F>
-int run_graph(misat_ctx* c, misat_ctx::GraphCache& gc, const std::array<uint64_t, 4>& key, F&& launch) {
+int run_graph(misat_ctx* c, misat_ctx::GraphCache& gc, const std::vector<uint64_t>& key, F&& launch) {
   cudaStream_t st = c->stream;
   cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
   if (!c->cap_stream || cudaStreamIsCapturing(st, &cs) != cudaSuccess || cs != cudaStreamCaptureStatusNone) {
@@ -479,13 +483,127 @@ int evict_all(misat_ctx* c, unsigned long long* evicted_counter, cudaEvent_t joi
   uint32_t maxlg = 1;
   for (auto& d : c->h_desc) maxlg = std::max(maxlg, d.log2nb);
   const int chunks = (int)std::min<uint64_t>(256, std::max<uint64_t>(1, ((uint64_t)1 << maxlg) / (4 * 256)));
-  const std::array<uint64_t, 4> key{(uint64_t)chunks, reinterpret_cast<uint64_t>(ev.gix.keys),
-                                    (uint64_t)ev.gix.log2nb, reinterpret_cast<uint64_t>(evicted_counter)};
+  const std::vector<uint64_t> key{(uint64_t)chunks, reinterpret_cast<uint64_t>(ev.gix.keys),
+                                  (uint64_t)ev.gix.log2nb, reinterpret_cast<uint64_t>(evicted_counter)};
   int rc = run_graph(c, c->g_evict, key, [&](cudaStream_t s) { launch_evict_select(ev, chunks, c->num_sms, s); });
   if (rc) return rc;
   if (join) CK(cudaStreamWaitEvent(c->stream, join, 0));
   return run_graph(c, c->g_evict_apply, key, [&](cudaStream_t s) { launch_evict_apply(ev, chunks, c->num_sms, s); });
 }
+
+CapsArgs caps_args(misat_ctx* c) {
+  CapsArgs ca{};
+  ca.W = c->W;
+  ca.desc = c->d_desc;
+  ca.prot = c->d_prot;
+  ca.cand = c->cand_ptr();
+  ca.params = c->d_params;
+  ca.pf_q16 = c->pf_q16;
+  ca.mode = c->mode;
+  ca.contraction = c->d_contraction;
+  ca.backlog = c->d_backlog;
+  ca.ia = c->ia;
+  ca.err = c->err_ptr();
+  return ca;
+}
+
+// The device work of one route (n > 0), enqueued on stream st: counters reset, prologue,
+// block hash, caps, probes, selection rounds, finalize.  Captured into the route graph, or
+// launched directly while the caller captures the context's stream.
+void enqueue_route(misat_ctx* c, const misat_batch* b, misat_decisions* out, cudaStream_t st) {
+  const int32_t n = b->n;
+  // reset the per-batch counters: stats, U, cand, work, n_hits (size and sess_used persist)
+  cudaMemsetAsync(c->d_meta + c->ml.stats, 0, 32 * 8, st);
+  cudaMemsetAsync(c->d_meta + c->ml.U, 0, c->W * 8, st);
+  cudaMemsetAsync(c->d_meta + c->ml.cand, 0, 5 * 8, st);
+  const int bm_log2 = std::max(1, ceil_log2(2 * (uint64_t)n));
+  cudaMemsetAsync(c->d_bm_key, 0, ((size_t)1 << bm_log2) * 8, st);
+  cudaMemsetAsync(c->d_bm_val, 0x7f, ((size_t)1 << bm_log2) * 4, st);
+
+  c->mark(0, st);
+  PrologueArgs pa{};
+  pa.n = n;
+  pa.n_tokens = b->n_tokens;
+  pa.cls = b->cls;
+  pa.session = b->session;
+  pa.tok_off = b->tok_off;
+  pa.rq = c->rq;
+  pa.st = c->sess;
+  pa.bm_key = c->d_bm_key;
+  pa.bm_val = c->d_bm_val;
+  pa.bm_log2 = (uint32_t)bm_log2;
+  pa.cand = c->cand_ptr();
+  pa.err = c->err_ptr();
+  launch_prologue(pa, st);
+  c->mark(1, st);
+
+  HashArgs ha{};
+  ha.tok_off = b->tok_off;
+  ha.tokens = b->tokens;
+  ha.n_tokens = b->n_tokens;
+  ha.n = n;
+  ha.seed = c->seed;
+  ha.keys = c->d_keys;
+  ha.keys_cap = c->keys_cap;
+  ha.work = c->work_ptr();
+  ha.err = c->err_ptr();
+  launch_block_hash(ha, c->num_sms, st);
+  c->mark(2, st);
+  launch_caps(caps_args(c), st);
+  c->mark(3, st);
+
+  ProbeArgs pr{};
+  pr.desc = c->d_desc;
+  pr.W = c->W;
+  pr.n = n;
+  pr.nb = c->rq.nb;
+  pr.kbase = c->rq.kbase;
+  pr.keys = c->d_keys;
+  pr.H = c->d_H;
+  pr.hits = c->d_hits;
+  pr.hbest = c->rq.hbest;
+  pr.n_hits = c->nhits_ptr();
+  pr.hits_cap = c->hits_cap;
+  pr.stats = c->stats_ptr() + 16;
+  pr.stats_search = c->stats_ptr() + 22;
+  pr.err = c->err_ptr();
+  pr.gix = gix_or_null(c);
+  launch_probe_first(pr, c->num_sms, st);
+  c->mark(4, st);
+  launch_probe_search(pr, c->num_sms, st);
+  c->mark(5, st);
+  if (b->out_H)
+    cudaMemcpyAsync(b->out_H, c->d_H, (size_t)n * c->W * sizeof(uint16_t), cudaMemcpyDeviceToDevice, st);
+
+  RoundArgs ra{};
+  ra.n = n;
+  ra.W = c->W;
+  ra.rq = c->rq;
+  ra.ia = c->ia;
+  ra.H = c->d_H;
+  ra.tokcost = c->d_tokcost;
+  ra.hold_delay_q = c->hold_delay_q;
+  ra.tile_counts = c->d_tile;
+  ra.n_tiles = (n + kTileReq - 1) / kTileReq;
+  ra.err = c->err_ptr();
+  for (int k = 0; k < c->rounds; ++k) launch_round(ra, c->num_sms, st);
+  c->mark(6, st);
+
+  FinalizeArgs fa{};
+  fa.n = n;
+  fa.W = c->W;
+  fa.rq = c->rq;
+  fa.H = c->d_H;
+  fa.out_inst = out->inst;
+  fa.out_reason = out->reason;
+  fa.out_hit = out->hit_blocks;
+  fa.U = c->U_ptr();
+  fa.stats = c->stats_ptr();
+  fa.err = c->err_ptr();
+  launch_finalize(fa, st);
+  c->mark(7, st);
+}
+
 
 }  // namespace
 
@@ -508,9 +626,9 @@ const char* misat_strerror(int code) {
 int misat_destroy(misat_ctx* c) {
   if (!c) return MISAT_ERR_INVALID_ARG;
   cudaStreamSynchronize(c->stream);
-  if (c->g_rounds.exec) cudaGraphExecDestroy(c->g_rounds.exec);
   if (c->g_evict.exec) cudaGraphExecDestroy(c->g_evict.exec);
   if (c->g_evict_apply.exec) cudaGraphExecDestroy(c->g_evict_apply.exec);
+  if (c->g_route.exec) cudaGraphExecDestroy(c->g_route.exec);
   if (c->cap_stream) cudaStreamDestroy(c->cap_stream);
   if (c->side_stream) {
     cudaStreamSynchronize(c->side_stream);
@@ -620,7 +738,7 @@ int misat_create(const misat_config* cfg, void* cuda_stream, misat_ctx** out) {
       (rc = dalloc_n(c, &c->ia.N_wb, 3 * Ws)) || (rc = dalloc_n(c, &c->ia.kbar_w, Ws)) ||
       (rc = dalloc_n(c, &c->ia.tot, Ws)) || (rc = dalloc_n(c, &c->ia.gh, Ws)) || (rc = dalloc_n(c, &c->ia.ch, 3 * Ws)) ||
       (rc = dalloc_n(c, &c->ia.delta, 3 * Ws)) || (rc = dalloc_n(c, &c->ia.backlog_k, Ws)) ||
-      (rc = dalloc_n(c, &c->ia.prefill, Ws)) || (rc = dalloc_n(c, &c->ia.live, 2)) ||
+      (rc = dalloc_n(c, &c->ia.prefill, Ws)) || (rc = dalloc_n(c, &c->ia.live, 2)) || (rc = dalloc_n(c, &c->d_params, 9)) ||
       (rc = dalloc_n(c, &c->d_backlog, Ws)) ||
       (rc = dalloc_n(c, &c->d_tokcost, Ws)) || (rc = dalloc_n(c, &c->d_contraction, Ws)) ||
       (rc = dalloc_n(c, &c->d_prot, 3 * Ws)) || (rc = dalloc_n(c, &c->d_theta, 2 * Ws)) ||
@@ -706,129 +824,52 @@ int misat_route(misat_ctx* c, const misat_batch* b, misat_decisions* out) {
   cudaStream_t st = c->stream;
   c->routed = false;
   estimate_classes(c);
-  // reset the per-batch counters: stats, U, cand, work, n_hits (size and sess_used persist)
-  CK(cudaMemsetAsync(c->d_meta + c->ml.stats, 0, 32 * 8, st));
-  CK(cudaMemsetAsync(c->d_meta + c->ml.U, 0, c->W * 8, st));
-  CK(cudaMemsetAsync(c->d_meta + c->ml.cand, 0, 5 * 8, st));
   c->last_n = n;
   c->last_ntok = b->n_tokens;
-  CapsArgs ca{};
-  ca.W = c->W;
-  ca.desc = c->d_desc;
-  ca.prot = c->d_prot;
-  ca.cand = c->cand_ptr();
+  RouteParams prm{};
   for (int i = 0; i < 3; ++i) {
-    ca.kbar_b[i] = c->kbar_b[i];
-    ca.T_b[i] = c->T_b[i];
-    ca.rho[i] = c->rho[i];
+    prm.v[i] = c->kbar_b[i];
+    prm.v[3 + i] = c->T_b[i];
+    prm.v[6 + i] = (int64_t)c->rho[i];
   }
-  ca.pf_q16 = c->pf_q16;
-  ca.mode = c->mode;
-  ca.contraction = c->d_contraction;
-  ca.backlog = c->d_backlog;
-  ca.ia = c->ia;
-  ca.err = c->err_ptr();
+  launch_route_params(prm, c->d_params, st);
+  CK(cudaGetLastError());
   if (n == 0) {
     // the caps of an empty batch are still defined (no candidate sessions)
-    launch_caps(ca, st);
+    CK(cudaMemsetAsync(c->d_meta + c->ml.stats, 0, 32 * 8, st));
+    CK(cudaMemsetAsync(c->d_meta + c->ml.U, 0, c->W * 8, st));
+    CK(cudaMemsetAsync(c->d_meta + c->ml.cand, 0, 5 * 8, st));
+    launch_caps(caps_args(c), st);
     CK(cudaGetLastError());
     CK(enqueue_meta(c));
     c->routed = true;
     return MISAT_OK;
   }
-  const int bm_log2 = std::max(1, ceil_log2(2 * (uint64_t)n));
-  CK(cudaMemsetAsync(c->d_bm_key, 0, ((size_t)1 << bm_log2) * 8, st));
-  CK(cudaMemsetAsync(c->d_bm_val, 0x7f, ((size_t)1 << bm_log2) * 4, st));
-
-  c->mark(0);
-  PrologueArgs pa{};
-  pa.n = n;
-  pa.n_tokens = b->n_tokens;
-  pa.cls = b->cls;
-  pa.session = b->session;
-  pa.tok_off = b->tok_off;
-  pa.rq = c->rq;
-  pa.st = c->sess;
-  pa.bm_key = c->d_bm_key;
-  pa.bm_val = c->d_bm_val;
-  pa.bm_log2 = (uint32_t)bm_log2;
-  pa.cand = c->cand_ptr();
-  pa.err = c->err_ptr();
-  launch_prologue(pa, st);
-  c->mark(1);
-
-  HashArgs ha{};
-  ha.tok_off = b->tok_off;
-  ha.tokens = b->tokens;
-  ha.n_tokens = b->n_tokens;
-  ha.n = n;
-  ha.seed = c->seed;
-  ha.keys = c->d_keys;
-  ha.keys_cap = c->keys_cap;
-  ha.work = c->work_ptr();
-  ha.err = c->err_ptr();
-  launch_block_hash(ha, c->num_sms, st);
-  c->mark(2);
-  launch_caps(ca, st);
-  c->mark(3);
-
-  ProbeArgs pr{};
-  pr.desc = c->d_desc;
-  pr.W = c->W;
-  pr.n = n;
-  pr.nb = c->rq.nb;
-  pr.kbase = c->rq.kbase;
-  pr.keys = c->d_keys;
-  pr.H = c->d_H;
-  pr.hits = c->d_hits;
-  pr.hbest = c->rq.hbest;
-  pr.n_hits = c->nhits_ptr();
-  pr.hits_cap = c->hits_cap;
-  pr.stats = c->stats_ptr() + 16;
-  pr.stats_search = c->stats_ptr() + 22;
-  pr.err = c->err_ptr();
-  pr.gix = gix_or_null(c);
-  launch_probe_first(pr, c->num_sms, st);
-  c->mark(4);
-  launch_probe_search(pr, c->num_sms, st);
-  c->mark(5);
-  if (b->out_H)
-    CK(cudaMemcpyAsync(b->out_H, c->d_H, (size_t)n * c->W * sizeof(uint16_t), cudaMemcpyDeviceToDevice, st));
-
-  RoundArgs ra{};
-  ra.n = n;
-  ra.W = c->W;
-  ra.rq = c->rq;
-  ra.ia = c->ia;
-  ra.H = c->d_H;
-  ra.tokcost = c->d_tokcost;
-  ra.hold_delay_q = c->hold_delay_q;
-  ra.tile_counts = c->d_tile;
-  ra.n_tiles = (n + kTileReq - 1) / kTileReq;
-  ra.err = c->err_ptr();
-  {
-    const std::array<uint64_t, 4> key{(uint64_t)n, 0, 0, 0};
-    const int rc = run_graph(c, c->g_rounds, key, [&](cudaStream_t s) {
-      for (int k = 0; k < c->rounds; ++k) launch_round(ra, c->num_sms, s);
-    });
+  // the device work of a route depends on the batch only through these values: it is
+  // replayed as one CUDA graph while they repeat
+  const std::vector<uint64_t> key{(uint64_t)n,
+                                  (uint64_t)b->n_tokens,
+                                  reinterpret_cast<uint64_t>(b->cls),
+                                  reinterpret_cast<uint64_t>(b->session),
+                                  reinterpret_cast<uint64_t>(b->tok_off),
+                                  reinterpret_cast<uint64_t>(b->tokens),
+                                  reinterpret_cast<uint64_t>(b->out_H),
+                                  reinterpret_cast<uint64_t>(out->inst),
+                                  reinterpret_cast<uint64_t>(out->reason),
+                                  reinterpret_cast<uint64_t>(out->hit_blocks),
+                                  reinterpret_cast<uint64_t>(c->sess.slots),
+                                  (uint64_t)c->sess.log2n,
+                                  reinterpret_cast<uint64_t>(c->gix.keys),
+                                  reinterpret_cast<uint64_t>(c->gix.masks),
+                                  (uint64_t)c->gix.log2nb};
+  if (c->timing) {
+    // phase events bracket the kernels directly (events recorded inside a graph do not time)
+    enqueue_route(c, b, out, st);
+    CK(cudaGetLastError());
+  } else {
+    const int rc = run_graph(c, c->g_route, key, [&](cudaStream_t s) { enqueue_route(c, b, out, s); });
     if (rc) return rc;
   }
-  c->mark(6);
-
-  FinalizeArgs fa{};
-  fa.n = n;
-  fa.W = c->W;
-  fa.rq = c->rq;
-  fa.H = c->d_H;
-  fa.out_inst = out->inst;
-  fa.out_reason = out->reason;
-  fa.out_hit = out->hit_blocks;
-  fa.U = c->U_ptr();
-  fa.stats = c->stats_ptr();
-  fa.err = c->err_ptr();
-  launch_finalize(fa, st);
-  c->mark(7);
-  CK(cudaGetLastError());
   CK(enqueue_meta(c));
   c->routed = true;
   return MISAT_OK;

@@ -107,9 +107,7 @@ struct CapsArgs {
   const InstDesc* desc;
   const int32_t* prot;         // [W*3]
   const long long* cand;       // [3]
-  int64_t kbar_b[3];
-  int64_t T_b[3];
-  uint32_t rho[3];
+  const int64_t* params;       // [9] device: kbar_b[3], T_b[3], rho_ppm[3] of this route
   int32_t pf_q16;
   int32_t mode;
   const int32_t* contraction;  // [W]
@@ -118,6 +116,12 @@ struct CapsArgs {
   const int32_t* err;
 };
 void launch_caps(const CapsArgs& a, cudaStream_t st);
+// Writes the host's per-route class parameters (footprints, residencies, mixture) to the
+// device (kernel arguments are taken at launch, so the host array may change right after).
+struct RouteParams {
+  int64_t v[9];
+};
+void launch_route_params(const RouteParams& p, int64_t* dst, cudaStream_t st);
 
 constexpr int kAdmitTile = 128;  // requests per admission tile
 

@@ -125,6 +125,14 @@ void launch_prologue(const PrologueArgs& a, cudaStream_t st) {
 // K3a caps, one thread per instance (Sec. 4.1; Eqs. 9-10 MISA; Eqs. 11, 13 MISA-T).
 __global__ void __launch_bounds__(1024) k3_caps(CapsArgs a) {
   if (block_error(a.err)) return;
+  int64_t kbar_b[3], T_b[3];
+  uint32_t rho[3];
+#pragma unroll
+  for (int b = 0; b < 3; ++b) {
+    kbar_b[b] = a.params[b];
+    T_b[b] = a.params[3 + b];
+    rho[b] = (uint32_t)a.params[6 + b];
+  }
   if (threadIdx.x == 0) {
     a.ia.live[0] = 1;  // the first selection round always runs
     a.ia.live[1] = 0;
@@ -143,11 +151,11 @@ __global__ void __launch_bounds__(1024) k3_caps(CapsArgs a) {
     int64_t kw;
     if (sumN > 0) {
       __int128 num = 0;
-      for (int b = 0; b < 3; ++b) num += (__int128)N[b] * a.kbar_b[b];
+      for (int b = 0; b < 3; ++b) num += (__int128)N[b] * kbar_b[b];
       kw = (int64_t)((num + sumN - 1) / sumN);
     } else {
-      kw = a.kbar_b[0] < a.kbar_b[1] ? a.kbar_b[0] : a.kbar_b[1];
-      kw = kw < a.kbar_b[2] ? kw : a.kbar_b[2];
+      kw = kbar_b[0] < kbar_b[1] ? kbar_b[0] : kbar_b[1];
+      kw = kw < kbar_b[2] ? kw : kbar_b[2];
     }
     const int64_t Cw = (int64_t)(((__int128)a.desc[w].cap * a.pf_q16) >> 16);
     int64_t Kw = Cw / kw - a.contraction[w];
@@ -159,8 +167,8 @@ __global__ void __launch_bounds__(1024) k3_caps(CapsArgs a) {
     } else {
       unsigned __int128 R[3], sumR = 0;
       for (int b = 0; b < 3; ++b) {
-        R[b] = (unsigned __int128)N[b] * (unsigned __int128)a.kbar_b[b];
-        if (a.mode == MISAT_MODE_MISA_T) R[b] *= (unsigned __int128)a.T_b[b];
+        R[b] = (unsigned __int128)N[b] * (unsigned __int128)kbar_b[b];
+        if (a.mode == MISAT_MODE_MISA_T) R[b] *= (unsigned __int128)T_b[b];
         sumR += R[b];
       }
       for (int b = 0; b < 3; ++b) {
@@ -168,8 +176,8 @@ __global__ void __launch_bounds__(1024) k3_caps(CapsArgs a) {
         if (sumR > 0)
           M = (int64_t)(((unsigned __int128)Cw * R[b]) / sumR);
         else
-          M = (int64_t)(((__int128)Cw * a.rho[b]) / 1000000);
-        const int64_t k = M / a.kbar_b[b];
+          M = (int64_t)(((__int128)Cw * rho[b]) / 1000000);
+        const int64_t k = M / kbar_b[b];
         Kwb[b] = k < 1 ? 1 : k;
       }
     }
@@ -191,6 +199,12 @@ __global__ void __launch_bounds__(1024) k3_caps(CapsArgs a) {
 }
 
 void launch_caps(const CapsArgs& a, cudaStream_t st) { k3_caps<<<1, 1024, 0, st>>>(a); }
+
+__global__ void k_route_params(RouteParams p, int64_t* dst) {
+  if (threadIdx.x < 9) dst[threadIdx.x] = p.v[threadIdx.x];
+}
+
+void launch_route_params(const RouteParams& p, int64_t* dst, cudaStream_t st) { k_route_params<<<1, 32, 0, st>>>(p, dst); }
 
 // Whether the current selection round runs (block-uniform read of the round flag).
 __device__ __forceinline__ bool round_live(const RoundArgs& a) {
