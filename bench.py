@@ -54,12 +54,13 @@ CLOCK_QUERY = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.ac
 
 
 def kernels_per_step(rounds, global_index):
-    """Kernels one route+commit launches.  Route: prologue, leaders, hash, caps, probe first,
-    probe search, 5 per selection round (score, tile count, tile scan, admit, round end;
-    rounds after one that admitted nobody still launch and exit at once), finalize.
+    """Kernels one route+commit launches.  Route: class parameters, prologue, leaders, hash,
+    caps, probe first, probe search, 5 per selection round (score, tile count, tile scan,
+    admit, round end; rounds after one that admitted nobody still launch and exit at once),
+    finalize.
     Commit: insert work list, insert, the global-index pass (global layout only), sessions,
     and the five eviction kernels (estimate, collect, select, delete, shift)."""
-    return 7 + 5 * rounds + 8 + (1 if global_index else 0)
+    return 8 + 5 * rounds + 8 + (1 if global_index else 0)
 
 
 def max_over_ranks(ms, dist, device):
