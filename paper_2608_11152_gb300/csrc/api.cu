@@ -149,7 +149,8 @@ struct misat_ctx {
   cudaStream_t cap_stream = nullptr;
   struct GraphCache {
     cudaGraphExec_t exec = nullptr;
-    std::vector<uint64_t> key;
+    std::vector<uint64_t> key;      // key of exec
+    std::vector<uint64_t> pending;  // key seen once (captured when it comes again)
   } g_evict, g_evict_apply, g_route;
   int64_t* d_params = nullptr;  // [9] per-route class parameters (caps)
   // the commit's global-index pass runs on a side stream, beside the session update and
@@ -200,6 +201,13 @@ int run_graph(misat_ctx* c, misat_ctx::GraphCache& gc, const std::vector<uint64_
     return cudaGetLastError() == cudaSuccess ? MISAT_OK : MISAT_ERR_CUDA;
   }
   if (!gc.exec || gc.key != key) {
+    // a sequence is captured only when its key repeats: a caller that changes buffers on
+    // every call is served by direct launches instead of a capture per call
+    if (gc.pending != key) {
+      gc.pending = key;
+      launch(st);
+      return cudaGetLastError() == cudaSuccess ? MISAT_OK : MISAT_ERR_CUDA;
+    }
     if (gc.exec) cudaGraphExecDestroy(gc.exec);
     gc.exec = nullptr;
     cudaGraph_t g = nullptr;

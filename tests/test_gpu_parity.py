@@ -326,3 +326,37 @@ def test_checkpoint_restore_replays_identically():
     ck.free()
     o2.close()
     r.close()
+
+
+def test_route_graph_capture_and_replay_match_the_oracle():
+    """The route is launched directly the first time a set of buffers is seen, captured the
+    second time and replayed from then on; with phase timing on it is launched directly.  All
+    of these give the oracle's decisions (the same batch routed repeatedly before its commit
+    replaces the pending route on both sides)."""
+    import torch
+
+    sc = wl.config2()
+    r = make_router(sc)
+    o = make_oracle(sc)
+    try:
+        for i, (b, comp) in enumerate(list(sc.warm) + [(sc.batch, None)]):
+            db = r.device_batch(b)
+            out = r.alloc_decisions(b.n)
+            oi, orr, oh = o.route(b.cls, b.session, b.tok_off, b.tokens)
+            for rep in range(4):
+                r.set_timing(rep == 3)
+                r.route(db, out)
+                torch.cuda.synchronize()
+                assert_equal(f"inst batch {i} call {rep}", out["inst"][: b.n].cpu().numpy(), oi)
+                assert_equal(f"reason batch {i} call {rep}", out["reason"][: b.n].cpu().numpy(), orr)
+                assert_equal(f"hit batch {i} call {rep}", out["hit_blocks"][: b.n].cpu().numpy(), oh)
+            r.set_timing(False)
+            r.commit()
+            o.commit()
+            compare_state(r, o, sc.W, index=(i == len(sc.warm)))
+            if comp is not None:
+                r.complete(comp.session, comp.cls, comp.total_blocks, comp.residency_us, comp.done)
+                o.complete(comp.session, comp.cls, comp.total_blocks, comp.residency_us, comp.done)
+        r.sync()
+    finally:
+        r.close()
