@@ -119,9 +119,10 @@ def hash_sources_sha256():
     return h.hexdigest()
 
 
-def profiled_traffic(batch_tokens):
-    """DRAM bytes per launch of the block-hash kernel from the committed ncu summary, if that
-    capture was taken on the same batch with the kernel's current sources; else None."""
+def profiled_hash_fields(batch_tokens):
+    """Figures of the block-hash kernel from the committed ncu summary (DRAM bytes per launch,
+    ALU pipe occupancy), if that capture was taken on the same batch with the kernel's current
+    sources; else {}."""
     try:
         fields = {}
         for line in open(HASH_PROFILE):
@@ -129,12 +130,18 @@ def profiled_traffic(batch_tokens):
                 k, v = line[3:].split("`:", 1)
                 fields[k.strip()] = v.strip().strip("`")
         if fields.get("sources_sha256") != hash_sources_sha256():
-            return None
+            return {}
         if int(fields["batch_tokens"]) != int(batch_tokens):
-            return None
-        return int(fields["traffic_bytes_per_launch"])
+            return {}
+        return fields
     except Exception:
-        return None
+        return {}
+
+
+def profiled_traffic(batch_tokens):
+    """DRAM bytes per launch of the block-hash kernel (see profiled_hash_fields), or None."""
+    f = profiled_hash_fields(batch_tokens)
+    return int(f["traffic_bytes_per_launch"]) if "traffic_bytes_per_launch" in f else None
 
 
 def peaks():
@@ -459,6 +466,10 @@ def run_gb300(args):
     kernels = {k: roof(k) for k in ("hash", "probe_first", "probe_search")}
     if kernels["hash"] is not None:
         kernels["hash"]["traffic"] = profiled_traffic(sc.batch.n_tokens)
+        hf = profiled_hash_fields(sc.batch.n_tokens)
+        if "alu_pipe_active_frac" in hf:
+            # the kernel's actual limiter: integer ALU issue (ncu sm__pipe_alu_cycles_active)
+            kernels["hash"]["alu_pipe_active_frac_ncu"] = float(hf["alu_pipe_active_frac"])
     dom_roof = dict(kernels[dom]) if kernels.get(dom) else roof(dom)
     if dom_roof is None:
         dom_roof = {"bound": "hbm", "achieved": None, "peak": peak, "unit": "GB/s", "frac": None, "traffic": None,
