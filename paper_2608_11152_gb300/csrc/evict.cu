@@ -485,19 +485,35 @@ __device__ __forceinline__ void shift_chunk(const EvictArgs& a, int w, uint32_t 
       if (!le128(v_hi(v), v_lo(v), tm, tk)) continue;
       sl = slots[i - nd];
     }
+    // the bitmap and deleted-mask words last read (runs are short: mostly one word each)
+    uint32_t fw_i = 0xffffffffu, fw = 0, dw_i = 0xffffffffu, dw = 0;
+    auto is_full = [&](uint32_t b) {
+      if ((b >> 5) != fw_i) {
+        fw_i = b >> 5;
+        fw = full[fw_i];
+      }
+      return (fw >> (b & 31)) & 1u;
+    };
+    auto dmask_at = [&](uint32_t b) {
+      if ((b >> 3) != dw_i) {
+        dw_i = b >> 3;
+        dw = dmask[dw_i];
+      }
+      return (dw >> ((b & 7) * 4)) & 0xFu;
+    };
     const uint32_t x = sl >> 2, sx = sl & 3;
     // a hole in the last (not full) bucket of a run needs no refill
-    if (!bit_of(full, x)) continue;
+    if (!is_full(x)) continue;
     // my deletion must be the lowest deleted slot of bucket x (the masks are not modified
     // by this kernel, unlike the buckets)
-    if ((uint32_t)(__ffs(dmask_of(dmask, x)) - 1) != sx) continue;
+    if ((uint32_t)(__ffs(dmask_at(x)) - 1) != sx) continue;
     // run start: walk back over full buckets; no earlier bucket of the run may hold a deletion
     uint32_t s0 = x, len = 0;
     bool lead = true;
-    while (bit_of(full, (s0 - 1) & mask) && len < NB) {
+    while (is_full((s0 - 1) & mask) && len < NB) {
       s0 = (s0 - 1) & mask;
       ++len;
-      if (dmask_of(dmask, s0)) {
+      if (dmask_at(s0)) {
         lead = false;
         break;
       }
@@ -505,33 +521,48 @@ __device__ __forceinline__ void shift_chunk(const EvictArgs& a, int w, uint32_t 
     if (!lead) continue;
     // run end: the first bucket after x that was not full
     uint32_t e = x, rl = 0;
-    while (bit_of(full, e) && rl < NB) {
+    while (is_full(e) && rl < NB) {
       e = (e + 1) & mask;
       ++rl;
     }
     const uint32_t runlen = ((e - s0) & mask);  // buckets s0 .. e-1 are full, e ends the run
     for (uint32_t ii = 0; ii < runlen; ++ii) {
       Bucket* X = d.tab + ((s0 + ii) & mask);
+      unsigned long long xk[4];
+      {
+        const ulonglong2* p = reinterpret_cast<const ulonglong2*>(X->key);
+        const ulonglong2 u0 = p[0], u1 = p[1];
+        xk[0] = u0.x;
+        xk[1] = u0.y;
+        xk[2] = u1.x;
+        xk[3] = u1.y;
+      }
+      bool stop = false;
+#pragma unroll
       for (int s = 0; s < 4; ++s) {
-        if (X->key[s] != kEmpty) continue;
+        if (stop || xk[s] != kEmpty) continue;
         bool moved = false;
         for (uint32_t j = ii + 1; j <= runlen && !moved; ++j) {
           Bucket* Y = d.tab + ((s0 + j) & mask);
+          const ulonglong2* p = reinterpret_cast<const ulonglong2*>(Y->key);
+          const ulonglong2 u0 = p[0], u1 = p[1];
+          const unsigned long long yk[4] = {u0.x, u0.y, u1.x, u1.y};
+#pragma unroll
           for (int t = 0; t < 4; ++t) {
-            const unsigned long long k = Y->key[t];
-            if (k == kEmpty) continue;
+            const unsigned long long k = yk[t];
+            if (moved || k == kEmpty) continue;
             const uint32_t rel = (home_bucket(k, d.log2nb) - s0) & mask;
             if (rel <= ii) {
               X->key[s] = k;
               X->meta[s] = Y->meta[t];
               Y->key[t] = kEmpty;
               Y->meta[t] = 0;
+              xk[s] = k;
               moved = true;
-              break;
             }
           }
         }
-        if (!moved) break;  // no later entry of the run can move into this bucket
+        if (!moved) stop = true;  // no later entry of the run can move into this bucket
       }
     }
   }
