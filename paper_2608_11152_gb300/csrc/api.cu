@@ -151,6 +151,7 @@ struct misat_ctx {
     cudaGraphExec_t exec = nullptr;
     std::vector<uint64_t> key;      // key of exec
     std::vector<uint64_t> pending;  // key seen once (captured when it comes again)
+    bool failed = false;            // a capture or instantiation failed: launch directly
   } g_evict, g_evict_apply, g_route;
   int64_t* d_params = nullptr;  // [9] per-route class parameters (caps)
   // the commit's global-index pass runs on a side stream, beside the session update and
@@ -195,7 +196,8 @@ template <class F>
 int run_graph(misat_ctx* c, misat_ctx::GraphCache& gc, const std::vector<uint64_t>& key, F&& launch) {
   cudaStream_t st = c->stream;
   cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
-  if (!c->cap_stream || cudaStreamIsCapturing(st, &cs) != cudaSuccess || cs != cudaStreamCaptureStatusNone) {
+  if (gc.failed || !c->cap_stream || cudaStreamIsCapturing(st, &cs) != cudaSuccess ||
+      cs != cudaStreamCaptureStatusNone) {
     cudaGetLastError();
     launch(st);
     return cudaGetLastError() == cudaSuccess ? MISAT_OK : MISAT_ERR_CUDA;
@@ -211,15 +213,20 @@ int run_graph(misat_ctx* c, misat_ctx::GraphCache& gc, const std::vector<uint64_
     if (gc.exec) cudaGraphExecDestroy(gc.exec);
     gc.exec = nullptr;
     cudaGraph_t g = nullptr;
-    CK(cudaStreamBeginCapture(c->cap_stream, cudaStreamCaptureModeThreadLocal));
-    launch(c->cap_stream);
-    const cudaError_t e = cudaStreamEndCapture(c->cap_stream, &g);
-    if (e != cudaSuccess || !g) return MISAT_ERR_CUDA;
-    const cudaError_t ei = cudaGraphInstantiate(&gc.exec, g, 0);
-    cudaGraphDestroy(g);
-    if (ei != cudaSuccess) {
+    cudaError_t e = cudaStreamBeginCapture(c->cap_stream, cudaStreamCaptureModeThreadLocal);
+    if (e == cudaSuccess) {
+      launch(c->cap_stream);
+      e = cudaStreamEndCapture(c->cap_stream, &g);
+    }
+    if (e == cudaSuccess && g) e = cudaGraphInstantiate(&gc.exec, g, 0);
+    if (g) cudaGraphDestroy(g);
+    if (e != cudaSuccess || !gc.exec) {
+      // nothing was launched by the failed capture: run the sequence directly, now and later
+      cudaGetLastError();
       gc.exec = nullptr;
-      return MISAT_ERR_CUDA;
+      gc.failed = true;
+      launch(st);
+      return cudaGetLastError() == cudaSuccess ? MISAT_OK : MISAT_ERR_CUDA;
     }
     gc.key = key;
   }
