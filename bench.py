@@ -407,7 +407,27 @@ def run_gb300(args):
     r.route_host(hb, hout)
     r.commit()
     torch.cuda.synchronize()
+    # the host link itself: one plain pinned-to-device copy of the token array
+    link_gbs = None
+    if b.n_tokens:
+        dtok = torch.empty(b.n_tokens, dtype=torch.int32, device="cuda")
+        ttok = pin["tokens"]
+        dtok.copy_(ttok, non_blocking=True)
+        best = None
+        for _ in range(3):
+            l0, l1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            l0.record(stream)
+            with torch.cuda.stream(stream):
+                dtok.copy_(ttok, non_blocking=True)
+            l1.record(stream)
+            l1.synchronize()
+            t = l0.elapsed_time(l1)
+            best = t if best is None else min(best, t)
+        link_gbs = round(b.tokens.nbytes / (best / 1e3) / 1e9, 1)
+        del dtok
+        log(f"host link: {link_gbs} GB/s host to device (pinned, best of 3)")
     e2e_ms = 0.0
+    e2e_each = []
     for k in range(args.e2e_steps):
         r.checkpoint_restore(ckpt)
         flush_l2()
@@ -420,9 +440,39 @@ def run_gb300(args):
         e1.record(stream)
         e1.synchronize()
         e2e_ms += e0.elapsed_time(e1)
+        e2e_each.append(round(e0.elapsed_time(e1), 3))
     e2e_ms = max_over_ranks(e2e_ms, dist, "cuda")
-    e2e = whole_job_rate(n, world, args.e2e_steps, e2e_ms)
-    log(f"e2e done: {e2e_ms / max(1, args.e2e_steps):.3f} ms/step")
+    e2e_seq = whole_job_rate(n, world, args.e2e_steps, e2e_ms)
+    log(f"e2e (one call per step, copy then route) done: {e2e_ms / max(1, args.e2e_steps):.3f} ms/step {e2e_each}")
+
+    # end to end, pipelined: the batch of step k+1 is copied (library copy stream) while step k
+    # is routed and committed; every step's copy and its decisions' read-back are inside the
+    # timed region, and so is the state restore that lets each step repeat the same batch
+    # (host wall clock, the device idle at both ends)
+    KE = args.e2e_steps
+    e2e_pipe = None
+    def pipelined(steps):
+        r.checkpoint_restore(ckpt)
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        r.stage_host(hb, 0)
+        for k in range(steps):
+            if k > 0:
+                r.checkpoint_restore(ckpt)
+            if k + 1 < steps:
+                r.stage_host(hb, (k + 1) % 2)
+            r.route_staged(k % 2, hout)
+            r.commit()
+        torch.cuda.synchronize()
+        return (time.perf_counter() - t0) * 1e3
+
+    if KE > 0:
+        pipelined(4)  # untimed: each slot's route graph is captured on its second use
+        pipe_ms = pipelined(KE)
+        pipe_ms = max_over_ranks(pipe_ms, dist, "cuda")
+        e2e_pipe = whole_job_rate(n, world, KE, pipe_ms)
+        log(f"e2e pipelined done: {pipe_ms / KE:.3f} ms/step")
+    e2e = e2e_pipe if e2e_pipe is not None else e2e_seq
     h2d = int(b.cls.nbytes + b.session.nbytes + b.tok_off.nbytes + b.tokens.nbytes)
     d2h = int(n * (4 + 1 + 4))
 
@@ -486,7 +536,11 @@ def run_gb300(args):
         "scaling": "weak", "vs_baseline": None, "dtype": "u64", "data": "synthetic (seeded, shaped after the paper's workloads)",
         "config": workload_config(args, sc),
         "probes_per_s": round(world * st.probes * K / (total_ms / 1e3), 1),
-        "e2e": {"value": round(e2e, 1), "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
+        "e2e": {"value": round(e2e, 1), "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
+                "api": "misat_stage_host + misat_route_staged + misat_commit (copy of step k+1 overlaps step k)",
+                "timer": "host wall clock over all steps, device idle at both ends; state restore inside",
+                "sequential_value": round(e2e_seq, 1), "host_link_h2d_gbs": link_gbs,
+                "sequential_api": "misat_route_host + misat_commit (copy, route, read-back; CUDA events)"},
         "gpu_launches": kernels_per_step(sc.rounds, pidx == misat.PREFIX_GLOBAL) * K,
         "roofline": dom_roof,
         "kernels": kernels,

@@ -178,6 +178,33 @@ int misat_route(misat_ctx* ctx, const misat_batch* batch, misat_decisions* out);
  * back.  out_H must be NULL.  [sync] */
 int misat_route_host(misat_ctx* ctx, const misat_batch* host_batch, misat_decisions* host_out);
 
+/* Pipelined host path: the copy of the next batch overlaps the routing of the current one.
+ * Not in the paper, which routes requests one at a time; this is the batch ingestion of a
+ * router whose requests arrive in host memory, where the host link (not the GPU) bounds the
+ * end-to-end rate.
+ *
+ * misat_stage_host copies a HOST batch (pinned memory, or the copies are not asynchronous)
+ * into staging slot 0 or 1 on a library copy stream and returns at once.  The copies start
+ * after the last route from that slot has finished reading it.  The host arrays must stay
+ * unchanged until misat_route_staged of that slot has returned.  out_H must be NULL.  The
+ * first call allocates both slots (2 x (4 max_tokens + 17 max_batch) bytes of device memory)
+ * and the copy stream.  [async]  Errors: INVALID_ARG, BATCH_TOO_LARGE, STATE (the slot holds
+ * a batch not yet routed), OOM, CUDA.
+ *
+ * misat_route_staged routes the batch of `slot` on the context's stream once its copies are
+ * done, exactly as misat_route would route it, and copies the decisions to the HOST arrays
+ * of host_out ([n] each).  Returns when they are there.  A staged batch is routed once; the
+ * slot is then free for the next misat_stage_host.  Not for use while the caller captures
+ * the context's stream.  [sync]  Errors: as misat_route, STATE (nothing staged in the slot).
+ *
+ * Typical loop: stage(0, batch 0); for k: stage((k+1)%2, batch k+1); route_staged(k%2);
+ * commit.  The GPU's copy engine takes host-to-device copies in order, so a host copy that
+ * another call enqueues on the context's stream (misat_set_instance_state, misat_complete,
+ * misat_load_*) while a staged batch is being copied starts after that batch's copy;
+ * misat_route_staged and misat_commit make no host-to-device copy. */
+int misat_stage_host(misat_ctx* ctx, const misat_batch* host_batch, int32_t slot);
+int misat_route_staged(misat_ctx* ctx, int32_t slot, misat_decisions* host_out);
+
 /* Apply the pending route: insert every admitted request's blocks into its instance's
  * index (tick = commit number and arrival index, depth = block index, max-merge), make
  * newly admitted sessions protected on their instance (a rebound session leaves its old

@@ -143,15 +143,39 @@ struct misat_ctx {
   int32_t* d_out_inst = nullptr;
   uint8_t* d_out_reason = nullptr;
   int32_t* d_out_hit = nullptr;
+  // pipelined host path (misat_stage_host / misat_route_staged): two device slots, filled on
+  // a copy stream while the context's stream routes the other one; allocated on first use
+  struct StageSlot {
+    int32_t* tok = nullptr;
+    int64_t* off = nullptr;
+    uint8_t* cls = nullptr;
+    uint64_t* ses = nullptr;
+    int32_t n = 0;
+    int64_t n_tokens = 0;
+    bool staged = false;
+    cudaEvent_t ev_copied = nullptr;  // the slot's H2D copies are done
+    cudaEvent_t ev_free = nullptr;    // the last route that read the slot is done
+  } slot[2];
+  cudaStream_t copy_stream = nullptr;
   std::vector<void*> owned;  // fixed allocations freed in destroy
   // launch sequences replayed as CUDA graphs (captured on a private stream, which never
   // runs work, and launched on the context's stream)
   cudaStream_t cap_stream = nullptr;
   struct GraphCache {
-    cudaGraphExec_t exec = nullptr;
-    std::vector<uint64_t> key;      // key of exec
-    std::vector<uint64_t> pending;  // key seen once (captured when it comes again)
-    bool failed = false;            // a capture or instantiation failed: launch directly
+    static constexpr size_t kEntries = 4;  // execs kept (least recently used dropped first)
+    struct Entry {
+      std::vector<uint64_t> key;
+      cudaGraphExec_t exec = nullptr;
+    };
+    std::vector<Entry> entries;                   // most recently used last
+    std::vector<std::vector<uint64_t>> pending;   // keys seen once (captured when they come again)
+    bool failed = false;                          // a capture or instantiation failed: launch directly
+    void clear() {
+      for (auto& e : entries)
+        if (e.exec) cudaGraphExecDestroy(e.exec);
+      entries.clear();
+      pending.clear();
+    }
   } g_evict, g_evict_apply, g_route;
   int64_t* d_params = nullptr;  // [9] per-route class parameters (caps)
   // the commit's global-index pass runs on a side stream, beside the session update and
@@ -202,35 +226,57 @@ int run_graph(misat_ctx* c, misat_ctx::GraphCache& gc, const std::vector<uint64_
     launch(st);
     return cudaGetLastError() == cudaSuccess ? MISAT_OK : MISAT_ERR_CUDA;
   }
-  if (!gc.exec || gc.key != key) {
-    // a sequence is captured only when its key repeats: a caller that changes buffers on
-    // every call is served by direct launches instead of a capture per call
-    if (gc.pending != key) {
-      gc.pending = key;
-      launch(st);
-      return cudaGetLastError() == cudaSuccess ? MISAT_OK : MISAT_ERR_CUDA;
-    }
-    if (gc.exec) cudaGraphExecDestroy(gc.exec);
-    gc.exec = nullptr;
-    cudaGraph_t g = nullptr;
-    cudaError_t e = cudaStreamBeginCapture(c->cap_stream, cudaStreamCaptureModeThreadLocal);
-    if (e == cudaSuccess) {
-      launch(c->cap_stream);
-      e = cudaStreamEndCapture(c->cap_stream, &g);
-    }
-    if (e == cudaSuccess && g) e = cudaGraphInstantiate(&gc.exec, g, 0);
-    if (g) cudaGraphDestroy(g);
-    if (e != cudaSuccess || !gc.exec) {
-      // nothing was launched by the failed capture: run the sequence directly, now and later
-      cudaGetLastError();
-      gc.exec = nullptr;
-      gc.failed = true;
-      launch(st);
-      return cudaGetLastError() == cudaSuccess ? MISAT_OK : MISAT_ERR_CUDA;
-    }
-    gc.key = key;
+  for (size_t i = 0; i < gc.entries.size(); ++i) {
+    if (gc.entries[i].key != key) continue;
+    // replay; the entry becomes the most recently used
+    misat_ctx::GraphCache::Entry hit = std::move(gc.entries[i]);
+    gc.entries.erase(gc.entries.begin() + i);
+    gc.entries.push_back(std::move(hit));
+    CK(cudaGraphLaunch(gc.entries.back().exec, st));
+    return MISAT_OK;
   }
-  CK(cudaGraphLaunch(gc.exec, st));
+  // a sequence is captured only when its key repeats: a caller that changes buffers on every
+  // call is served by direct launches instead of a capture per call.  A few keys are
+  // remembered, so that callers alternating between buffer sets (double-buffered staging)
+  // are replayed from graphs too.
+  bool seen = false;
+  for (size_t i = 0; i < gc.pending.size(); ++i)
+    if (gc.pending[i] == key) {
+      gc.pending.erase(gc.pending.begin() + i);
+      seen = true;
+      break;
+    }
+  if (!seen) {
+    if (gc.pending.size() >= misat_ctx::GraphCache::kEntries) gc.pending.erase(gc.pending.begin());
+    gc.pending.push_back(key);
+    launch(st);
+    return cudaGetLastError() == cudaSuccess ? MISAT_OK : MISAT_ERR_CUDA;
+  }
+  cudaGraphExec_t exec = nullptr;
+  cudaGraph_t g = nullptr;
+  cudaError_t e = cudaStreamBeginCapture(c->cap_stream, cudaStreamCaptureModeThreadLocal);
+  if (e == cudaSuccess) {
+    launch(c->cap_stream);
+    e = cudaStreamEndCapture(c->cap_stream, &g);
+  }
+  if (e == cudaSuccess && g) e = cudaGraphInstantiate(&exec, g, 0);
+  if (g) cudaGraphDestroy(g);
+  if (e != cudaSuccess || !exec) {
+    // nothing was launched by the failed capture: run the sequence directly, now and later
+    cudaGetLastError();
+    if (exec) cudaGraphExecDestroy(exec);
+    gc.clear();
+    gc.failed = true;
+    launch(st);
+    return cudaGetLastError() == cudaSuccess ? MISAT_OK : MISAT_ERR_CUDA;
+  }
+  if (gc.entries.size() >= misat_ctx::GraphCache::kEntries) {
+    // the stream may still run the oldest exec: destroying it is deferred by CUDA until then
+    cudaGraphExecDestroy(gc.entries.front().exec);
+    gc.entries.erase(gc.entries.begin());
+  }
+  gc.entries.push_back({key, exec});
+  CK(cudaGraphLaunch(exec, st));
   return MISAT_OK;
 }
 
@@ -641,13 +687,21 @@ const char* misat_strerror(int code) {
 int misat_destroy(misat_ctx* c) {
   if (!c) return MISAT_ERR_INVALID_ARG;
   cudaStreamSynchronize(c->stream);
-  if (c->g_evict.exec) cudaGraphExecDestroy(c->g_evict.exec);
-  if (c->g_evict_apply.exec) cudaGraphExecDestroy(c->g_evict_apply.exec);
-  if (c->g_route.exec) cudaGraphExecDestroy(c->g_route.exec);
+  c->g_evict.clear();
+  c->g_evict_apply.clear();
+  c->g_route.clear();
   if (c->cap_stream) cudaStreamDestroy(c->cap_stream);
   if (c->side_stream) {
     cudaStreamSynchronize(c->side_stream);
     cudaStreamDestroy(c->side_stream);
+  }
+  if (c->copy_stream) {
+    cudaStreamSynchronize(c->copy_stream);
+    cudaStreamDestroy(c->copy_stream);
+  }
+  for (auto& sl : c->slot) {
+    if (sl.ev_copied) cudaEventDestroy(sl.ev_copied);
+    if (sl.ev_free) cudaEventDestroy(sl.ev_free);
   }
   if (c->ev_fork) cudaEventDestroy(c->ev_fork);
   if (c->ev_join) cudaEventDestroy(c->ev_join);
@@ -915,6 +969,87 @@ int misat_route_host(misat_ctx* c, const misat_batch* hb, misat_decisions* ho) {
   db.out_H = nullptr;
   misat_decisions dd{c->d_out_inst, c->d_out_reason, c->d_out_hit};
   int rc = misat_route(c, &db, &dd);
+  if (rc) return rc;
+  if (n > 0) {
+    CK(cudaMemcpyAsync(ho->inst, c->d_out_inst, (size_t)n * 4, cudaMemcpyDeviceToHost, st));
+    CK(cudaMemcpyAsync(ho->reason, c->d_out_reason, (size_t)n, cudaMemcpyDeviceToHost, st));
+    CK(cudaMemcpyAsync(ho->hit_blocks, c->d_out_hit, (size_t)n * 4, cudaMemcpyDeviceToHost, st));
+  }
+  CK(cudaStreamSynchronize(st));
+  return MISAT_OK;
+}
+
+namespace {
+
+// The staging slots of the pipelined host path, their events and the copy stream.
+int ensure_staging(misat_ctx* c) {
+  if (c->copy_stream) return MISAT_OK;
+  const size_t NB = (size_t)c->max_batch;
+  for (auto& sl : c->slot) {
+    int rc;
+    if ((!sl.tok && (rc = dalloc_n(c, &sl.tok, (size_t)c->max_tokens + 8))) ||
+        (!sl.off && (rc = dalloc_n(c, &sl.off, NB + 1))) || (!sl.cls && (rc = dalloc_n(c, &sl.cls, NB))) ||
+        (!sl.ses && (rc = dalloc_n(c, &sl.ses, NB))))
+      return rc;
+    if (!sl.ev_copied) CK(cudaEventCreateWithFlags(&sl.ev_copied, cudaEventDisableTiming));
+    if (!sl.ev_free) CK(cudaEventCreateWithFlags(&sl.ev_free, cudaEventDisableTiming));
+  }
+  CK(cudaStreamCreateWithFlags(&c->copy_stream, cudaStreamNonBlocking));
+  return MISAT_OK;
+}
+
+}  // namespace
+
+int misat_stage_host(misat_ctx* c, const misat_batch* hb, int32_t slot) {
+  if (!c || !hb || hb->out_H || slot < 0 || slot > 1) return MISAT_ERR_INVALID_ARG;
+  const int32_t n = hb->n;
+  if (n < 0 || hb->n_tokens < 0) return MISAT_ERR_INVALID_ARG;
+  if (n > c->max_batch || hb->n_tokens > c->max_tokens) return MISAT_ERR_BATCH_TOO_LARGE;
+  if (n > 0 && (!hb->cls || !hb->session || !hb->tok_off)) return MISAT_ERR_INVALID_ARG;
+  if (hb->n_tokens > 0 && !hb->tokens) return MISAT_ERR_INVALID_ARG;
+  misat_ctx::StageSlot& sl = c->slot[slot];
+  if (sl.staged) return MISAT_ERR_STATE;  // staged and not yet routed
+  int rc = ensure_staging(c);
+  if (rc) return rc;
+  cudaStream_t cs = c->copy_stream;
+  // the slot's buffers are overwritten only after the route that last read them
+  CK(cudaStreamWaitEvent(cs, sl.ev_free, 0));
+  if (n > 0) {
+    CK(cudaMemcpyAsync(sl.off, hb->tok_off, (size_t)(n + 1) * 8, cudaMemcpyHostToDevice, cs));
+    CK(cudaMemcpyAsync(sl.cls, hb->cls, (size_t)n, cudaMemcpyHostToDevice, cs));
+    CK(cudaMemcpyAsync(sl.ses, hb->session, (size_t)n * 8, cudaMemcpyHostToDevice, cs));
+    if (hb->n_tokens > 0)
+      CK(cudaMemcpyAsync(sl.tok, hb->tokens, (size_t)hb->n_tokens * 4, cudaMemcpyHostToDevice, cs));
+  }
+  CK(cudaEventRecord(sl.ev_copied, cs));
+  sl.n = n;
+  sl.n_tokens = hb->n_tokens;
+  sl.staged = true;
+  return MISAT_OK;
+}
+
+int misat_route_staged(misat_ctx* c, int32_t slot, misat_decisions* ho) {
+  if (!c || !ho || slot < 0 || slot > 1) return MISAT_ERR_INVALID_ARG;
+  misat_ctx::StageSlot& sl = c->slot[slot];
+  if (!sl.staged) return MISAT_ERR_STATE;
+  const int32_t n = sl.n;
+  if (n > 0 && (!ho->inst || !ho->reason || !ho->hit_blocks)) return MISAT_ERR_INVALID_ARG;
+  cudaStream_t st = c->stream;
+  CK(cudaStreamWaitEvent(st, sl.ev_copied, 0));
+  misat_batch db{};
+  db.n = n;
+  db.n_tokens = sl.n_tokens;
+  db.cls = sl.cls;
+  db.session = sl.ses;
+  db.group = nullptr;
+  db.tok_off = sl.off;
+  db.tokens = sl.tok;
+  db.out_H = nullptr;
+  misat_decisions dd{c->d_out_inst, c->d_out_reason, c->d_out_hit};
+  const int rc = misat_route(c, &db, &dd);
+  // the slot is free again once the work enqueued so far has run (also after a failed route)
+  sl.staged = false;
+  CK(cudaEventRecord(sl.ev_free, st));
   if (rc) return rc;
   if (n > 0) {
     CK(cudaMemcpyAsync(ho->inst, c->d_out_inst, (size_t)n * 4, cudaMemcpyDeviceToHost, st));
@@ -1413,6 +1548,10 @@ struct misat_checkpoint {
   unsigned long long* gmasks = nullptr;
   uint32_t g_log2 = 0;
   uint64_t g_used = 0;
+  // device copy of the counters restored with the state: [W] sizes, sessions used, global
+  // slots claimed (restored device to device: a host-to-device copy on the context's stream
+  // would queue behind a staged batch copy in flight on the copy engine)
+  unsigned long long* counters = nullptr;
 };
 
 extern "C" {
@@ -1427,6 +1566,7 @@ int misat_checkpoint_free(misat_checkpoint* k) {
   cudaFree(k->contraction);
   cudaFree(k->gkeys);
   cudaFree(k->gmasks);
+  cudaFree(k->counters);
   delete k;
   return MISAT_OK;
 }
@@ -1456,7 +1596,8 @@ int misat_checkpoint_save(misat_ctx* c, misat_checkpoint** out) {
   const size_t sbytes = ((size_t)1 << c->sess.log2n) * sizeof(SessSlot);
   if (!oom && (cudaMalloc(&k->sess, sbytes) != cudaSuccess || cudaMalloc(&k->prot, c->W * 12) != cudaSuccess ||
                cudaMalloc(&k->backlog, c->W * 8) != cudaSuccess || cudaMalloc(&k->tokcost, c->W * 8) != cudaSuccess ||
-               cudaMalloc(&k->contraction, c->W * 4) != cudaSuccess))
+               cudaMalloc(&k->contraction, c->W * 4) != cudaSuccess ||
+               cudaMalloc(&k->counters, (c->W + 2) * 8) != cudaSuccess))
     oom = true;
   if (!oom && c->use_gix &&
       (cudaMalloc(&k->gkeys, gix_slots(c) * 8) != cudaSuccess ||
@@ -1472,6 +1613,8 @@ int misat_checkpoint_save(misat_ctx* c, misat_checkpoint** out) {
   CK(cudaMemcpyAsync(k->backlog, c->d_backlog, c->W * 8, cudaMemcpyDeviceToDevice, st));
   CK(cudaMemcpyAsync(k->tokcost, c->d_tokcost, c->W * 8, cudaMemcpyDeviceToDevice, st));
   CK(cudaMemcpyAsync(k->contraction, c->d_contraction, c->W * 4, cudaMemcpyDeviceToDevice, st));
+  CK(cudaMemcpyAsync(k->counters, c->d_meta + c->ml.size, (c->W + 1) * 8, cudaMemcpyDeviceToDevice, st));
+  CK(cudaMemcpyAsync(k->counters + c->W + 1, c->d_meta + c->ml.g_used, 8, cudaMemcpyDeviceToDevice, st));
   if (c->use_gix) {
     CK(cudaMemcpyAsync(k->gkeys, c->gix.keys, gix_slots(c) * 8, cudaMemcpyDeviceToDevice, st));
     CK(cudaMemcpyAsync(k->gmasks, c->gix.masks, gix_slots(c) * c->gix.mw * 8, cudaMemcpyDeviceToDevice, st));
@@ -1544,12 +1687,12 @@ int misat_checkpoint_restore(misat_ctx* c, const misat_checkpoint* k) {
     CK(cudaMemcpyAsync(c->gix.keys, k->gkeys, gix_slots(c) * 8, cudaMemcpyDeviceToDevice, st));
     CK(cudaMemcpyAsync(c->gix.masks, k->gmasks, gix_slots(c) * c->gix.mw * 8, cudaMemcpyDeviceToDevice, st));
     c->h_meta[c->ml.g_used] = k->g_used;
-    CK(cudaMemcpyAsync(c->d_meta + c->ml.g_used, c->h_meta + c->ml.g_used, 8, cudaMemcpyHostToDevice, st));
+    CK(cudaMemcpyAsync(c->d_meta + c->ml.g_used, k->counters + c->W + 1, 8, cudaMemcpyDeviceToDevice, st));
   }
-  // sizes and the session-slot counter live in the counters block
+  // sizes and the session-slot counter live in the counters block (host mirror and device)
   for (int w = 0; w < c->W; ++w) reinterpret_cast<long long*>(c->h_meta + c->ml.size)[w] = k->size[w];
   c->h_meta[c->ml.sess_used] = k->sess_used;
-  CK(cudaMemcpyAsync(c->d_meta + c->ml.size, c->h_meta + c->ml.size, (c->W + 1) * 8, cudaMemcpyHostToDevice, st));
+  CK(cudaMemcpyAsync(c->d_meta + c->ml.size, k->counters, (c->W + 1) * 8, cudaMemcpyDeviceToDevice, st));
   for (int b = 0; b < 3; ++b) {
     c->hist_blocks[b] = k->hist_blocks[b];
     c->hist_res[b] = k->hist_res[b];

@@ -185,18 +185,22 @@ __global__ void __launch_bounds__(256) k2_probe_search(ProbeArgs a) {
 }
 
 // Phase 1 through the global index: a warp takes 32 requests, each lane looks up the
-// block-0 key of one of them (one lookup answers every instance), the masks go to shared
-// memory, and the warp then writes the 32 H rows (H = 1 where the bit is set) and the hit
-// pairs of requests with at least two blocks.
+// block-0 key of one of them (one lookup answers every instance) and the masks go to shared
+// memory.  The warp's 32 H rows are one contiguous run of 32W u16 (64W bytes, 16-byte
+// aligned), written as 16-byte stores of eight entries (H = 1 where the bit is set) spread
+// over the lanes; each set bit of a request with at least two blocks also becomes a hit
+// pair, at its request's base (one atomic per warp) plus the rank of the bit in the mask.
 __global__ void __launch_bounds__(256) k2_probe_first_gix(ProbeArgs a) {
-  extern __shared__ unsigned long long s_gm[];  // [warps][32][mw]
+  extern __shared__ unsigned long long s_gm[];  // [warps][32][mw] masks, then [warps][32] (nb, base)
   if (block_error(a.err)) return;
   const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+  const int wpb = blockDim.x >> 5;
   const uint32_t mw = a.gix.mw;
   unsigned long long* sm = s_gm + (size_t)wid * 32 * mw;
+  int2* s_nbb = reinterpret_cast<int2*>(s_gm + (size_t)wpb * 32 * mw) + wid * 32;
   unsigned long long probes = 0, reads = 0;
   const int groups = (a.n + 31) >> 5;
-  const int wpb = blockDim.x >> 5;
+  const int W = a.W;
   for (int grp = blockIdx.x * wpb + wid; grp < groups; grp += gridDim.x * wpb) {
     const int r = grp * 32 + lane;
     int nb = 0;
@@ -217,7 +221,7 @@ __global__ void __launch_bounds__(256) k2_probe_first_gix(ProbeArgs a) {
       bits += __popcll(m);
       if (m && wmin == INT32_MAX) wmin = 64 * (int)i + __ffsll((long long)m) - 1;
     }
-    if (r < a.n) a.hbest[r] = wmin < a.W ? (1u << 16) | (65535u - (uint32_t)wmin) : 65535u;
+    if (r < a.n) a.hbest[r] = wmin < W ? (1u << 16) | (65535u - (uint32_t)wmin) : 65535u;
     // hit-list positions: one atomic per warp
     const int nh = nb > 1 ? bits : 0;
     int incl = nh;
@@ -230,29 +234,50 @@ __global__ void __launch_bounds__(256) k2_probe_first_gix(ProbeArgs a) {
     unsigned base = 0;
     if (lane == 31 && tot) base = atomicAdd(a.n_hits, (unsigned)tot);
     base = __shfl_sync(0xffffffffu, base, 31) + (unsigned)(incl - nh);
+    s_nbb[lane] = make_int2(nb, (int)base);
     __syncwarp();
+    // the group's rows: elements e = i*W + w of a run of cnt*W entries
     const int cnt = min(32, a.n - grp * 32);
-    for (int i = 0; i < cnt; ++i) {
-      const int ri = grp * 32 + i;
-      const bool list = __shfl_sync(0xffffffffu, nb, i) > 1;
-      unsigned pos = __shfl_sync(0xffffffffu, base, i);
-      const unsigned long long* mi = sm + i * mw;
-      uint16_t* row = a.H + (int64_t)ri * a.W;
-      for (int w0 = 0; w0 < a.W; w0 += 32) {
-        const int w = w0 + lane;
-        const bool bit = w < a.W && ((mi[w >> 6] >> (w & 63)) & 1ull);
-        if (w < a.W) row[w] = bit ? 1 : 0;
-        if (list) {
-          const unsigned bal = __ballot_sync(0xffffffffu, bit);
-          if (bit) {
-            const unsigned p = pos + __popc(bal & lanemask_lt());
+    const int64_t run = (int64_t)cnt * W;
+    uint16_t* rows = a.H + (int64_t)grp * 32 * W;
+    const int64_t n8 = (run + 7) >> 3;
+    for (int64_t c8 = lane; c8 < n8; c8 += 32) {
+      const int64_t e0 = c8 << 3;
+      int i = (int)(e0 / W);
+      int w = (int)(e0 - (int64_t)i * W);
+      uint32_t packed[4] = {0u, 0u, 0u, 0u};
+      const int ne = run - e0 < 8 ? (int)(run - e0) : 8;
+#pragma unroll
+      for (int k = 0; k < 8; ++k) {
+        if (k >= ne) break;
+        const unsigned long long* mi = sm + i * mw;
+        const uint32_t wd = (uint32_t)w >> 6;
+        const unsigned long long m = mi[wd];
+        const unsigned long long below = m & ((1ull << (w & 63)) - 1ull);
+        if ((m >> (w & 63)) & 1ull) {
+          packed[k >> 1] |= 1u << (16 * (k & 1));
+          const int2 q = s_nbb[i];
+          if (q.x > 1) {
+            unsigned rank = (unsigned)__popcll(below);
+            for (uint32_t j = 0; j < wd; ++j) rank += (unsigned)__popcll(mi[j]);
+            const unsigned p = (unsigned)q.y + rank;
             if ((int64_t)p < a.hits_cap)
-              a.hits[p] = make_int2(ri, w);
+              a.hits[p] = make_int2(grp * 32 + i, w);
             else
               set_error(a.err, MISAT_ERR_TABLE_FULL);
           }
-          pos += __popc(bal);
         }
+        if (++w == W) {
+          w = 0;
+          ++i;
+        }
+      }
+      if (ne == 8) {
+        *reinterpret_cast<uint4*>(rows + e0) = make_uint4(packed[0], packed[1], packed[2], packed[3]);
+      } else {
+#pragma unroll
+        for (int k = 0; k < 8; ++k)
+          if (k < ne) rows[e0 + k] = (uint16_t)((packed[k >> 1] >> (16 * (k & 1))) & 0xffffu);
       }
     }
     __syncwarp();
@@ -267,7 +292,7 @@ void launch_probe_first(const ProbeArgs& a, int num_sms, cudaStream_t st) {
     const int groups = (a.n + 31) / 32;
     const int blocks = (groups + 7) / 8;
     const int grid = blocks < num_sms * 8 ? blocks : num_sms * 8;
-    k2_probe_first_gix<<<grid, 256, 8 * 32 * a.gix.mw * sizeof(unsigned long long), st>>>(a);
+    k2_probe_first_gix<<<grid, 256, 8 * 32 * (a.gix.mw * sizeof(unsigned long long) + sizeof(int2)), st>>>(a);
     return;
   }
   int S = 1;

@@ -81,6 +81,8 @@ _SIG = {
     "misat_set_instance_state": [_p, _p, _p, _p],
     "misat_route": [_p, C.POINTER(misat_batch), C.POINTER(misat_decisions)],
     "misat_route_host": [_p, C.POINTER(misat_batch), C.POINTER(misat_decisions)],
+    "misat_stage_host": [_p, C.POINTER(misat_batch), C.c_int32],
+    "misat_route_staged": [_p, C.c_int32, C.POINTER(misat_decisions)],
     "misat_commit": [_p],
     "misat_complete": [_p, C.c_int32, _p, _p, _p, _p, _p],
     "misat_evict": [_p, C.c_int32, _p, C.c_int64],
@@ -260,6 +262,30 @@ class Router:
         b = misat_batch(n, batch.n_tokens, _nptr(cls), _nptr(ses), None, _nptr(off), _nptr(tok), None)
         d = misat_decisions(_nptr(out["inst"]), _nptr(out["reason"]), _nptr(out["hit_blocks"]))
         _ck(_lib.misat_route_host(self._h, C.byref(b), C.byref(d)), "misat_route_host")
+        return out
+
+    def stage_host(self, batch, slot):
+        """Start the copy of a host batch (numpy arrays, pinned for asynchrony) into staging
+        slot 0 or 1; returns at once.  The arrays are kept referenced until the slot is routed."""
+        cls, ses, off, tok = batch.cls, batch.session, batch.tok_off, batch.tokens
+        b = misat_batch(batch.n, batch.n_tokens, _nptr(cls), _nptr(ses), None, _nptr(off), _nptr(tok), None)
+        _ck(_lib.misat_stage_host(self._h, C.byref(b), int(slot)), "misat_stage_host")
+        if not hasattr(self, "_staged"):
+            self._staged = {}
+        self._staged[int(slot)] = (batch.n, cls, ses, off, tok)
+
+    def route_staged(self, slot, out=None):
+        """Route the batch staged in `slot`; returns numpy decisions (written into `out` if given)."""
+        n = self._staged[int(slot)][0] if getattr(self, "_staged", None) and int(slot) in self._staged else 0
+        if out is None:
+            out = dict(inst=np.empty(max(1, n), np.int32), reason=np.empty(max(1, n), np.uint8),
+                       hit_blocks=np.empty(max(1, n), np.int32))
+        d = misat_decisions(_nptr(out["inst"]), _nptr(out["reason"]), _nptr(out["hit_blocks"]))
+        try:
+            _ck(_lib.misat_route_staged(self._h, int(slot), C.byref(d)), "misat_route_staged")
+        finally:
+            if getattr(self, "_staged", None):
+                self._staged.pop(int(slot), None)
         return out
 
     def commit(self):

@@ -242,6 +242,90 @@ def test_route_host_matches_device_route():
     r2.close()
 
 
+def _pinned_batch(b):
+    def pin(a):
+        t = torch.from_numpy(np.ascontiguousarray(a)).pin_memory()
+        return t.numpy()
+
+    return wl.Batch(cls=pin(b.cls), session=pin(b.session.view(np.int64)).view(np.uint64), group=b.group,
+                    tok_off=pin(b.tok_off), tokens=pin(b.tokens))
+
+
+@pytest.mark.parametrize("cfg", [1, 2])
+def test_pipelined_host_staging_matches_the_oracle(cfg):
+    """Batch k+1 is staged (copy stream) before batch k is routed from the other slot; every
+    decision and the index after every commit equal the oracle's."""
+    sc = {1: wl.config1, 2: wl.config2}[cfg]()
+    r, o = make_router(sc), make_oracle(sc)
+    steps = list(sc.warm) + [(sc.batch, None)]
+    pinned = [_pinned_batch(b) for b, _ in steps]
+    r.stage_host(pinned[0], 0)
+    for k, (b, comp) in enumerate(steps):
+        if k + 1 < len(steps):
+            r.stage_host(pinned[k + 1], (k + 1) % 2)
+        got = r.route_staged(k % 2)
+        oi, orr, oh = o.route(b.cls, b.session, b.tok_off, b.tokens)
+        assert_equal("inst", got["inst"][: b.n], oi)
+        assert_equal("reason", got["reason"][: b.n], orr)
+        assert_equal("hit_blocks", got["hit_blocks"][: b.n], oh)
+        r.commit()
+        o.commit()
+        compare_state(r, o, sc.W)
+        if comp is not None:
+            for x in (r, o):
+                x.complete(comp.session, comp.cls, comp.total_blocks, comp.residency_us, comp.done)
+    r.sync()
+    r.close()
+
+
+def test_pipelined_staging_slot_states_and_graph_replay():
+    """A slot holds one batch until it is routed; routing an empty slot is refused.  The same
+    batch routed from alternating slots after a state restore (graphs captured per slot and
+    replayed) gives the same decisions every time."""
+    from paper_2608_11152_gb300 import misat
+
+    sc = wl.config2()
+    r = make_router(sc)
+    for b, comp in sc.warm:
+        r.route_host(b)
+        r.commit()
+        if comp is not None:
+            r.complete(comp.session, comp.cls, comp.total_blocks, comp.residency_us, comp.done)
+    pb = _pinned_batch(sc.batch)
+    with pytest.raises(misat.MisatError) as e:
+        r.route_staged(0)
+    assert e.value.code == misat.ERR_STATE
+    r.stage_host(pb, 0)
+    with pytest.raises(misat.MisatError) as e:
+        r.stage_host(pb, 0)
+    assert e.value.code == misat.ERR_STATE
+    with pytest.raises(misat.MisatError) as e:
+        r.stage_host(pb, 2)
+    assert e.value.code == misat.ERR_INVALID_ARG
+    ckpt = r.checkpoint_save()
+    ref = r.route_host(sc.batch)
+    ref = {k: v[: sc.batch.n].copy() for k, v in ref.items()}
+
+    def slot(k):  # 1, 0, 1, 0, ...
+        return (k + 1) % 2
+
+    first = r.route_staged(0)  # the batch staged above, routed from the same state
+    for name in ("inst", "reason", "hit_blocks"):
+        assert_equal(name, first[name][: sc.batch.n], ref[name])
+    r.stage_host(pb, slot(0))
+    for k in range(6):
+        r.checkpoint_restore(ckpt)
+        if k + 1 < 6:
+            r.stage_host(pb, slot(k + 1))
+        got = r.route_staged(slot(k))
+        for name in ("inst", "reason", "hit_blocks"):
+            assert_equal(f"{name} (route {k})", got[name][: sc.batch.n], ref[name])
+    r.commit()
+    r.sync()
+    ckpt.free()
+    r.close()
+
+
 def test_external_evict_reset_and_load_chains():
     sc = wl.small_random(18, W=3, cap=200, n=20, n_warm=2)
     r, o = run_parity(sc)
