@@ -241,6 +241,42 @@ __global__ void __launch_bounds__(256) k2_probe_first_gix(ProbeArgs a) {
     const int64_t run = (int64_t)cnt * W;
     uint16_t* rows = a.H + (int64_t)grp * 32 * W;
     const int64_t n8 = (run + 7) >> 3;
+    if ((W & 7) == 0) {
+      // eight entries of one row per chunk: one mask byte gives them all
+      const int cpr = W >> 3;  // chunks per row
+      for (int c8 = lane; c8 < (int)n8; c8 += 32) {
+        const int i = c8 / cpr;
+        const int w0 = (c8 - i * cpr) << 3;
+        const unsigned long long* mi = sm + i * mw;
+        const uint32_t b8 = (uint32_t)(mi[w0 >> 6] >> (w0 & 63)) & 0xffu;
+        uint4 v;
+        v.x = (b8 & 1u) | (((b8 >> 1) & 1u) << 16);
+        v.y = ((b8 >> 2) & 1u) | (((b8 >> 3) & 1u) << 16);
+        v.z = ((b8 >> 4) & 1u) | (((b8 >> 5) & 1u) << 16);
+        v.w = ((b8 >> 6) & 1u) | (((b8 >> 7) & 1u) << 16);
+        *reinterpret_cast<uint4*>(rows + ((int64_t)c8 << 3)) = v;
+        if (b8) {
+          const int2 q = s_nbb[i];
+          if (q.x > 1) {
+            // rank of the chunk's first entry among the row's set bits
+            unsigned rank = (unsigned)__popcll(mi[w0 >> 6] & ((1ull << (w0 & 63)) - 1ull));
+            for (int j = 0; j < (w0 >> 6); ++j) rank += (unsigned)__popcll(mi[j]);
+            uint32_t rest = b8;
+            while (rest) {
+              const int bit = __ffs(rest) - 1;
+              rest &= rest - 1;
+              const unsigned p = (unsigned)q.y + rank++;
+              if ((int64_t)p < a.hits_cap)
+                a.hits[p] = make_int2(grp * 32 + i, w0 + bit);
+              else
+                set_error(a.err, MISAT_ERR_TABLE_FULL);
+            }
+          }
+        }
+      }
+      __syncwarp();
+      continue;
+    }
     for (int64_t c8 = lane; c8 < n8; c8 += 32) {
       const int64_t e0 = c8 << 3;
       int i = (int)(e0 / W);

@@ -215,34 +215,34 @@ __device__ __forceinline__ bool round_live(const RoundArgs& a) {
 // K3b score: a group of G lanes per unresolved leader (G = 4..32 with W: each lane takes
 // 8-instance chunks of the H row, so a group reads its row as one coalesced segment).
 // Cost of Eq. (1) in fixed point, cost = backlog_k[w] + (L_r - 16 H_rw) * tokcost[w];
-// eligibility of Eq. (6) with the class cap of Sec. 4.2 (headroom at round start, as a
-// per-class byte map in shared memory); argmin (cost, w) and argmax (H, w) (ties to the
-// lower instance) by log2(G) shuffle steps inside the group.  A session protected on its
-// choice is admitted here (ADMIT_CONT); a released session may prefer to wait for its
+// eligibility of Eq. (6) with the class cap of Sec. 4.2 (headroom at round start) is folded
+// into a per-class backlog: an instance without headroom for class b carries a sentinel
+// backlog above every eligible cost, so the scan over instances has no branch.  Bounds:
+// backlog_k <= 2^61 and (L_r - 16 H_rw) * tokcost < 2^20 * 2^32 + 1, so eligible costs stay
+// below 2^62 = sentinel, and sentinel costs below 2^63.  argmin (cost, w) (ties to the lower
+// instance) by log2(G) shuffle steps inside the group; the instance a session is protected
+// on is eligible without headroom and is compared after the scan.  A session protected on
+// its choice is admitted here (ADMIT_CONT); a released session may prefer to wait for its
 // cached instance (Eq. 7).
+constexpr int64_t kCostSentinel = (int64_t)1 << 62;
+
 template <int G, int CPL>
-__global__ void __launch_bounds__(256) k3_score(RoundArgs a) {
+__global__ void __launch_bounds__(256, 4) k3_score(RoundArgs a) {
   extern __shared__ unsigned char smem[];
-  // backlog and token cost per instance, stored at w + w/8: the 8 lanes of a group read
-  // instances 8 apart, which this padding puts in 8 distinct bank pairs
+  // per-class backlog (sentinel without headroom) and token cost per instance, stored at
+  // w + w/8: the lanes of a group read instances 8 apart, which this padding puts in
+  // distinct bank pairs
   const int wpad = a.W + (a.W >> 3) + 1;
-  int64_t* s_bk = reinterpret_cast<int64_t*>(smem);
-  int64_t* s_tc = s_bk + wpad;
-  int32_t* s_gh = reinterpret_cast<int32_t*>(s_tc + wpad);
-  int32_t* s_ch = s_gh + a.W;                                     // [W*3]
-  uint8_t* s_el = reinterpret_cast<uint8_t*>(s_ch + 3 * a.W);     // [3][W]: headroom on w
+  int64_t* s_bkc = reinterpret_cast<int64_t*>(smem);  // [3][wpad]
+  int64_t* s_tc = s_bkc + 3 * wpad;
   if (block_error(a.err) || !round_live(a)) return;
   for (int w = threadIdx.x; w < a.W; w += blockDim.x) {
-    s_bk[w + (w >> 3)] = a.ia.backlog_k[w];
-    s_tc[w + (w >> 3)] = a.tokcost[w];
+    const int wp = w + (w >> 3);
+    const int64_t bk = a.ia.backlog_k[w];
+    s_tc[wp] = a.tokcost[w];
     const int32_t gh = a.ia.gh[w];
-    s_gh[w] = gh;
 #pragma unroll
-    for (int b = 0; b < 3; ++b) {
-      const int32_t ch = a.ia.ch[w * 3 + b];
-      s_ch[w * 3 + b] = ch;
-      s_el[b * a.W + w] = (gh > 0 && ch > 0) ? 1 : 0;
-    }
+    for (int b = 0; b < 3; ++b) s_bkc[b * wpad + wp] = (gh > 0 && a.ia.ch[w * 3 + b] > 0) ? bk : kCostSentinel;
   }
   __syncthreads();
   const int lane = threadIdx.x & 31;
@@ -308,7 +308,7 @@ __global__ void __launch_bounds__(256) k3_score(RoundArgs a) {
       const uint32_t hb = __shfl_sync(gmask, khb, g0 + k);
       const int hmax = (int)(hb >> 16), whit = 65535 - (int)(hb & 0xffffu);  // max H, lowest such w
       const int pw = sst == kSessProtected ? sinst : -1;
-      const uint8_t* el = s_el + b * a.W;
+      const int64_t* bkc = s_bkc + b * wpad;
       int64_t best_c = INT64_MAX;
       int best_w = INT32_MAX;
 #pragma unroll
@@ -320,13 +320,13 @@ __global__ void __launch_bounds__(256) k3_score(RoundArgs a) {
         for (int i = 0; i < 8; ++i) {
           const int w = ck * 8 + i;
           if (w >= a.W) break;
-          const int h = (int)((hw[i >> 1] >> (16 * (i & 1))) & 0xffffu);
-          if (w == pw || el[w]) {
-            const int64_t cost = s_bk[w + (w >> 3)] + (Lr - 16 * (int64_t)h) * s_tc[w + (w >> 3)];
-            if (cost < best_c) {
-              best_c = cost;
-              best_w = w;
-            }
+          const uint32_t h = (hw[i >> 1] >> (16 * (i & 1))) & 0xffffu;
+          const uint32_t cold = (uint32_t)Lr - 16u * h;  // L_r - 16 H_rw >= 0, < 2^20
+          const int wp = w + (w >> 3);
+          const int64_t cost = bkc[wp] + (int64_t)((uint64_t)cold * (uint64_t)s_tc[wp]);
+          if (cost < best_c) {
+            best_c = cost;
+            best_w = w;
           }
         }
       }
@@ -340,6 +340,16 @@ __global__ void __launch_bounds__(256) k3_score(RoundArgs a) {
         }
       }
       if (gl == 0) {
+        if (best_c >= kCostSentinel) best_w = INT32_MAX;  // no instance with headroom
+        if (pw >= 0 && bkc[pw + (pw >> 3)] >= kCostSentinel) {
+          // protected on pw: eligible there without headroom, at its real cost
+          const int64_t hp = a.H[(int64_t)r * a.W + pw];
+          const int64_t cpw = a.ia.backlog_k[pw] + (Lr - 16 * hp) * s_tc[pw + (pw >> 3)];
+          if (best_w == INT32_MAX || cpw < best_c || (cpw == best_c && pw < best_w)) {
+            best_c = cpw;
+            best_w = pw;
+          }
+        }
         int choice = -1;
         uint8_t reason = 0;
         if (best_w == INT32_MAX) {
@@ -350,9 +360,9 @@ __global__ void __launch_bounds__(256) k3_score(RoundArgs a) {
         } else {
           choice = best_w;
           if (sst == kSessReleased && hmax > 0) {
-            const bool elig_hit = s_gh[whit] > 0 && s_ch[whit * 3 + b] > 0;
+            const bool elig_hit = bkc[whit + (whit >> 3)] < kCostSentinel;
             if (!elig_hit) {
-              const int64_t lhs = a.hold_delay_q + s_bk[whit + (whit >> 3)] - s_bk[best_w + (best_w >> 3)];
+              const int64_t lhs = a.hold_delay_q + a.ia.backlog_k[whit] - a.ia.backlog_k[best_w];
               const int64_t rhs = 16 * (int64_t)hmax * s_tc[whit + (whit >> 3)];
               if (lhs < rhs) {
                 choice = -1;
@@ -551,7 +561,7 @@ __global__ void __launch_bounds__(1024) k4_round_end(RoundArgs a) {
 }
 
 void launch_round(const RoundArgs& a, int num_sms, cudaStream_t st) {
-  const size_t score_smem = (size_t)16 * (a.W + (a.W >> 3) + 1) + (size_t)a.W * (4 + 12 + 3);
+  const size_t score_smem = (size_t)32 * (a.W + (a.W >> 3) + 1);
   int G = 4;
   while (G < 32 && G * 16 < a.W) G <<= 1;  // about two 8-instance chunks per lane
   const int64_t threads = (int64_t)a.n * G;
