@@ -94,7 +94,7 @@ def parse_args():
     ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
     ap.add_argument("--n", type=int, default=65536, help="requests per batch")
     ap.add_argument("--fill", type=float, default=0.95, help="resident fraction of the KV block capacity")
-    ap.add_argument("--e2e-steps", type=int, default=5)
+    ap.add_argument("--e2e-steps", type=int, default=10)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--instances", type=int, default=128, help="fewer only for small profiling captures")
     ap.add_argument("--cap", type=int, default=262144, help="blocks per instance; smaller only for profiling captures")
