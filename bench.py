@@ -55,12 +55,12 @@ CLOCK_QUERY = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.ac
 
 def kernels_per_step(rounds, global_index):
     """Kernels one route+commit launches.  Route: class parameters, prologue, leaders, hash,
-    caps, probe first, probe search, 5 per selection round (score, tile count, tile scan,
-    admit, round end; rounds after one that admitted nobody still launch and exit at once),
-    finalize.
+    caps, probe first, probe search, 4 per selection round (score, tile count, tile scan,
+    admit, whose last tile also ends the round; rounds after one that admitted nobody still
+    launch and exit at once), finalize.
     Commit: insert work list, insert, the global-index pass (global layout only), sessions,
     and the five eviction kernels (estimate, collect, select, delete, shift)."""
-    return 8 + 5 * rounds + 8 + (1 if global_index else 0)
+    return 8 + 4 * rounds + 8 + (1 if global_index else 0)
 
 
 def max_over_ranks(ms, dist, device):
@@ -82,7 +82,7 @@ def whole_job_rate(units_per_rank, world, steps, max_ms):
 
 def PHASE_KERNELS(rounds, global_index):
     """Kernel launches per phase of one route+commit (see kernels_per_step)."""
-    return {"prologue": 2, "hash": 1, "caps": 1, "probe_first": 1, "probe_search": 1, "rounds": 5 * rounds,
+    return {"prologue": 2, "hash": 1, "caps": 1, "probe_first": 1, "probe_search": 1, "rounds": 4 * rounds,
             "finalize": 1, "insert": 3 if global_index else 2, "sessions": 1, "evict": 5}
 
 

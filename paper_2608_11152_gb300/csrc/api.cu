@@ -807,7 +807,7 @@ int misat_create(const misat_config* cfg, void* cuda_stream, misat_ctx** out) {
       (rc = dalloc_n(c, &c->ia.N_wb, 3 * Ws)) || (rc = dalloc_n(c, &c->ia.kbar_w, Ws)) ||
       (rc = dalloc_n(c, &c->ia.tot, Ws)) || (rc = dalloc_n(c, &c->ia.gh, Ws)) || (rc = dalloc_n(c, &c->ia.ch, 3 * Ws)) ||
       (rc = dalloc_n(c, &c->ia.delta, 3 * Ws)) || (rc = dalloc_n(c, &c->ia.backlog_k, Ws)) ||
-      (rc = dalloc_n(c, &c->ia.prefill, Ws)) || (rc = dalloc_n(c, &c->ia.live, 2)) || (rc = dalloc_n(c, &c->d_params, 9)) ||
+      (rc = dalloc_n(c, &c->ia.prefill, Ws)) || (rc = dalloc_n(c, &c->ia.live, 3)) || (rc = dalloc_n(c, &c->d_params, 9)) ||
       (rc = dalloc_n(c, &c->d_backlog, Ws)) ||
       (rc = dalloc_n(c, &c->d_tokcost, Ws)) || (rc = dalloc_n(c, &c->d_contraction, Ws)) ||
       (rc = dalloc_n(c, &c->d_prot, 3 * Ws)) || (rc = dalloc_n(c, &c->d_theta, 2 * Ws)) ||

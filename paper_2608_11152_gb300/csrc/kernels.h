@@ -55,7 +55,8 @@ struct InstArrays {
   int64_t* backlog_k;   // [W] in-batch backlog
   unsigned long long* prefill;  // [W] admitted prefill tokens of the current round
   long long* U;         // [W] upper bound of new keys of the pending commit
-  int32_t* live;        // [2]: [0] the current round runs, [1] ADMIT_CONT of the round
+  int32_t* live;        // [3]: [0] the current round runs, [1] ADMIT_CONT of the round,
+                        //      [2] admission tiles finished in the round
 };
 
 // ---- K2 ----

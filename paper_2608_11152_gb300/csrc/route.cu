@@ -136,6 +136,7 @@ __global__ void __launch_bounds__(1024) k3_caps(CapsArgs a) {
   if (threadIdx.x == 0) {
     a.ia.live[0] = 1;  // the first selection round always runs
     a.ia.live[1] = 0;
+    a.ia.live[2] = 0;
   }
   for (int w = threadIdx.x; w < a.W; w += blockDim.x) {
     int64_t N[3];
@@ -457,6 +458,59 @@ __global__ void __launch_bounds__(1024) k4_tile_scan(RoundArgs a) {
     }
 }
 
+// End of a selection round (one warp, after every tile's admissions): admissions leave the
+// headroom of their (instance, class), the admitted prefill joins the instance backlog
+// (saturating at 2^61), and a round that admitted nobody (no ADMIT_NEW, no ADMIT_CONT) ends
+// the rounds: its successors would see the same inputs.
+__device__ __forceinline__ void round_fold(const RoundArgs& a, int lane) {
+  constexpr int kF = 4;  // instances per lane per pass, all of their loads issued together
+  int admitted = 0;
+  for (int w0 = 0; w0 < a.W; w0 += 32 * kF) {
+    int32_t d[kF][3], ch[kF][3], gh[kF];
+    unsigned long long tok[kF];
+    int64_t bk[kF], tc[kF];
+#pragma unroll
+    for (int f = 0; f < kF; ++f) {
+      const int w = w0 + 32 * f + lane;
+      if (w < a.W) {
+#pragma unroll
+        for (int b = 0; b < 3; ++b) {
+          d[f][b] = __ldcg(&a.ia.delta[w * 3 + b]);
+          ch[f][b] = a.ia.ch[w * 3 + b];
+        }
+        gh[f] = a.ia.gh[w];
+        tok[f] = __ldcg(&a.ia.prefill[w]);
+        bk[f] = a.ia.backlog_k[w];
+        tc[f] = a.tokcost[w];
+      }
+    }
+#pragma unroll
+    for (int f = 0; f < kF; ++f) {
+      const int w = w0 + 32 * f + lane;
+      if (w < a.W) {
+        int32_t sum = 0;
+#pragma unroll
+        for (int b = 0; b < 3; ++b) {
+          a.ia.ch[w * 3 + b] = ch[f][b] - d[f][b];
+          a.ia.delta[w * 3 + b] = 0;
+          sum += d[f][b];
+        }
+        a.ia.gh[w] = gh[f] - sum;
+        admitted |= sum;
+        a.ia.prefill[w] = 0;
+        const __int128 v = (__int128)bk[f] + (__int128)tc[f] * (__int128)tok[f];
+        a.ia.backlog_k[w] = v > kBacklogMax ? kBacklogMax : (int64_t)v;
+      }
+    }
+  }
+  const bool any = __any_sync(kFull, admitted != 0);
+  if (lane == 0) {
+    if (!any && *(volatile int32_t*)&a.ia.live[1] == 0) a.ia.live[0] = 0;
+    a.ia.live[1] = 0;
+    a.ia.live[2] = 0;  // the next round's tile tickets
+  }
+}
+
 __global__ void __launch_bounds__(32) k4_admit(RoundArgs a) {
   extern __shared__ int32_t s_cnt[];
   if (block_error(a.err) || !round_live(a)) return;
@@ -528,6 +582,15 @@ __global__ void __launch_bounds__(32) k4_admit(RoundArgs a) {
     if (need[c] && lane == __ffs(peers_wb) - 1) s_cnt[w[c] * 3 + b[c]] += __popc(peers_wb);
     __syncwarp();
   }
+  // the last tile to finish folds the round's admissions into headroom and backlog (its
+  // ticket comes after every other tile's admissions, which the fences make visible)
+  __threadfence();
+  unsigned ticket = 0;
+  if (lane == 0) ticket = atomicAdd(reinterpret_cast<unsigned*>(&a.ia.live[2]), 1u);
+  ticket = __shfl_sync(kFull, ticket, 0);
+  if (ticket != gridDim.x - 1) return;
+  __threadfence();
+  round_fold(a, lane);
 }
 
 // End of a round: fold this round's admissions into the headroom, and add the admitted
@@ -535,30 +598,6 @@ __global__ void __launch_bounds__(32) k4_admit(RoundArgs a) {
 // round that admitted nobody leaves every input of the next round as it was (headroom,
 // backlog, statuses), so the next round would repeat it exactly: the remaining rounds
 // are then skipped.
-__global__ void __launch_bounds__(1024) k4_round_end(RoundArgs a) {
-  if (block_error(a.err) || !round_live(a)) return;
-  int admitted = 0;
-  for (int w = threadIdx.x; w < a.W; w += blockDim.x) {
-    int32_t sum = 0;
-    for (int b = 0; b < 3; ++b) {
-      const int32_t d = a.ia.delta[w * 3 + b];
-      a.ia.ch[w * 3 + b] -= d;
-      a.ia.delta[w * 3 + b] = 0;
-      sum += d;
-    }
-    a.ia.gh[w] -= sum;
-    admitted |= sum;
-    const unsigned long long tok = a.ia.prefill[w];
-    a.ia.prefill[w] = 0;
-    const __int128 v = (__int128)a.ia.backlog_k[w] + (__int128)a.tokcost[w] * (__int128)tok;
-    a.ia.backlog_k[w] = v > kBacklogMax ? kBacklogMax : (int64_t)v;
-  }
-  const int any = __syncthreads_or(admitted != 0);
-  if (threadIdx.x == 0) {
-    if (!any && a.ia.live[1] == 0) a.ia.live[0] = 0;
-    a.ia.live[1] = 0;
-  }
-}
 
 void launch_round(const RoundArgs& a, int num_sms, cudaStream_t st) {
   const size_t score_smem = (size_t)32 * (a.W + (a.W >> 3) + 1);
@@ -577,8 +616,7 @@ void launch_round(const RoundArgs& a, int num_sms, cudaStream_t st) {
   const size_t cnt_smem = (size_t)a.W * 3 * sizeof(int32_t);
   k4_tile_count<<<a.n_tiles, 128, cnt_smem, st>>>(a);
   k4_tile_scan<<<(3 * a.W + 31) / 32, 1024, 0, st>>>(a);
-  k4_admit<<<a.n_tiles, 32, cnt_smem, st>>>(a);
-  k4_round_end<<<1, 1024, 0, st>>>(a);
+  k4_admit<<<a.n_tiles, 32, cnt_smem, st>>>(a);  // its last tile also ends the round
 }
 
 // ---------------------------------------------------------------------------
