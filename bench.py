@@ -451,6 +451,8 @@ def run_gb300(args):
     # (host wall clock, the device idle at both ends)
     KE = args.e2e_steps
     e2e_pipe = None
+    pipe_runs = []
+
     def pipelined(steps):
         r.checkpoint_restore(ckpt)
         torch.cuda.synchronize()
@@ -468,7 +470,11 @@ def run_gb300(args):
 
     if KE > 0:
         pipelined(4)  # untimed: each slot's route graph is captured on its second use
-        pipe_ms = pipelined(KE)
+        # three runs of KE steps; the median is reported (the host link is shared with the
+        # machine's other tenants, and one stall inside a run moves its mean)
+        pipe_runs = [pipelined(KE) for _ in range(3)]
+        pipe_ms = sorted(pipe_runs)[1]
+        log(f"e2e pipelined runs: {[round(x / KE, 3) for x in pipe_runs]} ms/step")
         pipe_ms = max_over_ranks(pipe_ms, dist, "cuda")
         e2e_pipe = whole_job_rate(n, world, KE, pipe_ms)
         log(f"e2e pipelined done: {pipe_ms / KE:.3f} ms/step")
@@ -538,7 +544,8 @@ def run_gb300(args):
         "probes_per_s": round(world * st.probes * K / (total_ms / 1e3), 1),
         "e2e": {"value": round(e2e, 1), "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
                 "api": "misat_stage_host + misat_route_staged + misat_commit (copy of step k+1 overlaps step k)",
-                "timer": "host wall clock over all steps, device idle at both ends; state restore inside",
+                "timer": "host wall clock over all steps, device idle at both ends; state restore inside; median of 3 runs",
+                "runs_ms_per_step": [round(x / KE, 3) for x in pipe_runs] if KE > 0 else None,
                 "sequential_value": round(e2e_seq, 1), "host_link_h2d_gbs": link_gbs,
                 "sequential_api": "misat_route_host + misat_commit (copy, route, read-back; CUDA events)"},
         "gpu_launches": kernels_per_step(sc.rounds, pidx == misat.PREFIX_GLOBAL) * K,

@@ -5,6 +5,7 @@
 #include <cstdlib>
 #include <cstring>
 #include <deque>
+#include <memory>
 #include <new>
 #include <unordered_set>
 #include <vector>
@@ -1636,11 +1637,56 @@ int misat_checkpoint_save(misat_ctx* c, misat_checkpoint** out) {
   return MISAT_OK;
 }
 
+namespace {
+
+// Device-to-device copies of a restore, gathered into copy lists and run by one kernel per
+// list (the SMs, not a copy engine, move the bytes).
+struct RestoreCopies {
+  misat_ctx* c;
+  cudaStream_t st;
+  CopyList* l;
+  int add(void* dst, const void* src, uint64_t bytes) {
+    if (bytes == 0) return MISAT_OK;
+    if (l->n == kMaxCopies) {
+      const int rc = flush();
+      if (rc) return rc;
+    }
+    const uintptr_t a = reinterpret_cast<uintptr_t>(dst) | reinterpret_cast<uintptr_t>(src);
+    const uint32_t lg = (a & 15) == 0 ? 4 : (a & 7) == 0 ? 3 : (a & 3) == 0 ? 2 : 0;
+    CopyItem& it = l->item[l->n++];
+    it.dst = dst;
+    it.src = src;
+    it.bytes = bytes;
+    it.start = l->units;
+    it.lg = lg;
+    it.pad = 0;
+    l->units += (bytes + (1ull << lg) - 1) >> lg;
+    return MISAT_OK;
+  }
+  int flush() {
+    launch_copy_list(*l, c->num_sms, st);
+    CK(cudaGetLastError());
+    l->n = 0;
+    l->units = 0;
+    return MISAT_OK;
+  }
+};
+
+}  // namespace
+
 int misat_checkpoint_restore(misat_ctx* c, const misat_checkpoint* k) {
   if (!c || !k || k->W != c->W) return MISAT_ERR_INVALID_ARG;
   cudaStream_t st = c->stream;
   // the counters block is mirrored in pinned host memory: let pending copies land first
   CK(cudaStreamSynchronize(st));
+  std::unique_ptr<CopyList> list(new (std::nothrow) CopyList());
+  if (!list) return MISAT_ERR_OOM;
+  RestoreCopies cp{c, st, list.get()};
+  int crc = MISAT_OK;
+#define ADD_COPY(dst, src, bytes)                 \
+  do {                                            \
+    if ((crc = cp.add((dst), (src), (bytes)))) return crc; \
+  } while (0)
   for (int w = 0; w < c->W; ++w) {
     if (c->h_desc[w].log2nb > k->desc[w].log2nb) {
       // the table grew after the save: keep the larger table and re-insert the saved
@@ -1658,8 +1704,7 @@ int misat_checkpoint_restore(misat_ctx* c, const misat_checkpoint* k) {
       if (rc) return rc;
       if ((rc = swap_instance(c, w, nd, nb))) return rc;
     }
-    CK(cudaMemcpyAsync(c->h_desc[w].tab, k->desc[w].tab, ((size_t)1 << k->desc[w].log2nb) * sizeof(Bucket),
-                       cudaMemcpyDeviceToDevice, st));
+    ADD_COPY(c->h_desc[w].tab, k->desc[w].tab, ((size_t)1 << k->desc[w].log2nb) * sizeof(Bucket));
   }
   if (c->sess.log2n != k->sess_log2) {
     CK(cudaStreamSynchronize(st));
@@ -1672,27 +1717,28 @@ int misat_checkpoint_restore(misat_ctx* c, const misat_checkpoint* k) {
     c->sess.slots = ns;
     c->sess.log2n = k->sess_log2;
   }
-  CK(cudaMemcpyAsync(c->sess.slots, k->sess, ((size_t)1 << k->sess_log2) * sizeof(SessSlot),
-                     cudaMemcpyDeviceToDevice, st));
-  CK(cudaMemcpyAsync(c->d_prot, k->prot, c->W * 12, cudaMemcpyDeviceToDevice, st));
-  CK(cudaMemcpyAsync(c->d_backlog, k->backlog, c->W * 8, cudaMemcpyDeviceToDevice, st));
-  CK(cudaMemcpyAsync(c->d_tokcost, k->tokcost, c->W * 8, cudaMemcpyDeviceToDevice, st));
-  CK(cudaMemcpyAsync(c->d_contraction, k->contraction, c->W * 4, cudaMemcpyDeviceToDevice, st));
+  ADD_COPY(c->sess.slots, k->sess, ((size_t)1 << k->sess_log2) * sizeof(SessSlot));
+  ADD_COPY(c->d_prot, k->prot, c->W * 12);
+  ADD_COPY(c->d_backlog, k->backlog, c->W * 8);
+  ADD_COPY(c->d_tokcost, k->tokcost, c->W * 8);
+  ADD_COPY(c->d_contraction, k->contraction, c->W * 4);
   if (c->use_gix) {
     if (!k->gkeys) return MISAT_ERR_INVALID_ARG;
     if (c->gix.log2nb != k->g_log2) {
       int rc = gix_alloc(c, k->g_log2);
       if (rc) return rc;
     }
-    CK(cudaMemcpyAsync(c->gix.keys, k->gkeys, gix_slots(c) * 8, cudaMemcpyDeviceToDevice, st));
-    CK(cudaMemcpyAsync(c->gix.masks, k->gmasks, gix_slots(c) * c->gix.mw * 8, cudaMemcpyDeviceToDevice, st));
+    ADD_COPY(c->gix.keys, k->gkeys, gix_slots(c) * 8);
+    ADD_COPY(c->gix.masks, k->gmasks, gix_slots(c) * c->gix.mw * 8);
     c->h_meta[c->ml.g_used] = k->g_used;
-    CK(cudaMemcpyAsync(c->d_meta + c->ml.g_used, k->counters + c->W + 1, 8, cudaMemcpyDeviceToDevice, st));
+    ADD_COPY(c->d_meta + c->ml.g_used, k->counters + c->W + 1, 8);
   }
   // sizes and the session-slot counter live in the counters block (host mirror and device)
   for (int w = 0; w < c->W; ++w) reinterpret_cast<long long*>(c->h_meta + c->ml.size)[w] = k->size[w];
   c->h_meta[c->ml.sess_used] = k->sess_used;
-  CK(cudaMemcpyAsync(c->d_meta + c->ml.size, k->counters, (c->W + 1) * 8, cudaMemcpyDeviceToDevice, st));
+  ADD_COPY(c->d_meta + c->ml.size, k->counters, (c->W + 1) * 8);
+#undef ADD_COPY
+  if ((crc = cp.flush())) return crc;
   for (int b = 0; b < 3; ++b) {
     c->hist_blocks[b] = k->hist_blocks[b];
     c->hist_res[b] = k->hist_res[b];

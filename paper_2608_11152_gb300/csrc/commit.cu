@@ -427,6 +427,48 @@ void launch_mark_evict(const MarkArgs& a, int32_t w, const EvictArgs& ev, cudaSt
 }
 
 // Growth: re-insert every entry of `from` into the empty, larger table `to`.
+// Copy list: CTAs take spans of kSpan units of the flattened list; the item holding a span's
+// first unit is found by a (uniform) binary search, later items by stepping forward.
+__global__ void __launch_bounds__(256) k_copy_list(const __grid_constant__ CopyList L) {
+  constexpr uint64_t kSpan = 256 * 16;
+  for (uint64_t s0 = (uint64_t)blockIdx.x * kSpan; s0 < L.units; s0 += (uint64_t)gridDim.x * kSpan) {
+    int lo = 0, hi = L.n - 1;
+    while (lo < hi) {
+      const int mid = (lo + hi + 1) >> 1;
+      if (L.item[mid].start <= s0)
+        lo = mid;
+      else
+        hi = mid - 1;
+    }
+    int i = lo;
+    const uint64_t s1 = min(s0 + kSpan, L.units);
+    for (uint64_t u = s0 + threadIdx.x; u < s1; u += blockDim.x) {
+      while (i < L.n - 1 && u >= L.item[i].start + ((L.item[i].bytes + (1ull << L.item[i].lg) - 1) >> L.item[i].lg)) ++i;
+      const CopyItem& it = L.item[i];
+      const uint64_t off = (u - it.start) << it.lg;
+      char* d = static_cast<char*>(it.dst) + off;
+      const char* sp = static_cast<const char*>(it.src) + off;
+      if (off + (1ull << it.lg) <= it.bytes) {
+        switch (it.lg) {
+          case 4: *reinterpret_cast<int4*>(d) = *reinterpret_cast<const int4*>(sp); break;
+          case 3: *reinterpret_cast<unsigned long long*>(d) = *reinterpret_cast<const unsigned long long*>(sp); break;
+          case 2: *reinterpret_cast<unsigned*>(d) = *reinterpret_cast<const unsigned*>(sp); break;
+          default: *d = *sp; break;
+        }
+      } else {
+        for (uint64_t b = off; b < it.bytes; ++b) static_cast<char*>(it.dst)[b] = static_cast<const char*>(it.src)[b];
+      }
+    }
+  }
+}
+
+void launch_copy_list(const CopyList& l, int num_sms, cudaStream_t st) {
+  if (l.n <= 0 || l.units == 0) return;
+  const uint64_t spans = (l.units + 256 * 16 - 1) / (256 * 16);
+  const int grid = (int)(spans < (uint64_t)num_sms * 8 ? spans : (uint64_t)num_sms * 8);
+  k_copy_list<<<grid, 256, 0, st>>>(l);
+}
+
 __global__ void __launch_bounds__(256) k_rehash(RehashArgs a) {
   const uint32_t NB = 1u << a.from.log2nb;
   for (uint32_t b = blockIdx.x * blockDim.x + threadIdx.x; b < NB; b += gridDim.x * blockDim.x) {

@@ -26,7 +26,6 @@ namespace {
 constexpr unsigned kFull = 0xffffffffu;
 constexpr int kSelThreads = 1024;
 constexpr int kBins = 4096;
-constexpr int kSamples = 4096;  // 4 slots of up to 1024 sampled buckets
 
 __device__ __forceinline__ bool le128(uint64_t ma, uint64_t ka, uint64_t mb, uint64_t kb) {
   return ma < mb || (ma == mb && ka <= kb);
@@ -88,9 +87,6 @@ __device__ __forceinline__ uint32_t digit128(uint64_t hi, uint64_t lo, int shift
   return (uint32_t)v & (kBins - 1);
 }
 
-__device__ __forceinline__ bool bit_of(const uint32_t* bm, uint32_t b) { return (bm[b >> 5] >> (b & 31)) & 1u; }
-// deleted-slot mask of bucket b (4 bits per bucket, 8 buckets per word)
-__device__ __forceinline__ uint32_t dmask_of(const uint32_t* dm, uint32_t b) { return (dm[b >> 3] >> ((b & 7) * 4)) & 0xFu; }
 }  // namespace
 
 

@@ -259,6 +259,27 @@ struct RehashArgs {
 };
 void launch_rehash(const RehashArgs& a, cudaStream_t st);
 
+// Device-to-device copies of a checkpoint restore, done by one kernel on the SMs (a
+// cudaMemcpyAsync between device buffers may be given to a copy engine, where it waits
+// behind a host-to-device copy in flight).  The list travels as the kernel's parameter block,
+// so the launch itself copies nothing from the host.
+constexpr int kMaxCopies = 768;  // the list fits the 32 KB kernel parameter space
+struct CopyItem {
+  void* dst;
+  const void* src;
+  uint64_t bytes;
+  uint64_t start;  // first unit of this item in the flattened list
+  uint32_t lg;     // log2 of the unit size in bytes (4, 3, 2 or 0: both pointers aligned to it)
+  uint32_t pad;
+};
+struct CopyList {
+  int32_t n;
+  int32_t pad;
+  uint64_t units;  // total units
+  CopyItem item[kMaxCopies];
+};
+void launch_copy_list(const CopyList& l, int num_sms, cudaStream_t st);
+
 struct SessRehashArgs {
   SessTable from;
   SessTable to;

@@ -444,3 +444,41 @@ def test_route_graph_capture_and_replay_match_the_oracle():
         r.sync()
     finally:
         r.close()
+
+
+def test_route_graph_cache_rotation_over_more_buffer_sets_than_it_keeps():
+    """Six copies of one batch, each routed twice in a row (launched directly, then captured)
+    and visited in rotation, so that the cache (four graphs) drops the least recently used
+    graphs and captures them again; then the last four copies in rotation (replayed).  Every
+    route before the commit gives the oracle's decisions."""
+    import torch
+
+    sc = wl.config1()
+    r = make_router(sc)
+    o = make_oracle(sc)
+    try:
+        for b, comp in sc.warm:
+            route_both(r, o, b, sc.W, check_H=False, check_keys=False)
+            r.commit()
+            o.commit()
+            if comp is not None:
+                r.complete(comp.session, comp.cls, comp.total_blocks, comp.residency_us, comp.done)
+                o.complete(comp.session, comp.cls, comp.total_blocks, comp.residency_us, comp.done)
+        b = sc.batch
+        oi, orr, oh = o.route(b.cls, b.session, b.tok_off, b.tokens)
+        copies = [(r.device_batch(b), r.alloc_decisions(b.n)) for _ in range(6)]
+        order = [j for _ in range(3) for j in range(6) for _ in range(2)] + [2, 3, 4, 5] * 3
+        for step, j in enumerate(order):
+            db, out = copies[j]
+            out["inst"].fill_(-7)
+            r.route(db, out)
+            torch.cuda.synchronize()
+            assert_equal(f"inst copy {j} step {step}", out["inst"][: b.n].cpu().numpy(), oi)
+            assert_equal(f"reason copy {j} step {step}", out["reason"][: b.n].cpu().numpy(), orr)
+            assert_equal(f"hit copy {j} step {step}", out["hit_blocks"][: b.n].cpu().numpy(), oh)
+        r.commit()
+        o.commit()
+        compare_state(r, o, sc.W)
+        r.sync()
+    finally:
+        r.close()
