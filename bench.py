@@ -48,7 +48,7 @@ def log(msg):
 
 METRIC = "routed requests/s (route+commit)"
 UNIT = "requests/s"
-CLOCK_QUERY = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+CLOCK_QUERY = ("timestamp,index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
                "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
                "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
 
@@ -89,7 +89,7 @@ def PHASE_KERNELS(rounds, global_index):
 def parse_args():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=30)
+    ap.add_argument("--steps", type=int, default=300)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
     ap.add_argument("--n", type=int, default=65536, help="requests per batch")
@@ -184,7 +184,8 @@ def workload_config(args, sc):
 
 
 class ClockSampler:
-    """nvidia-smi clocks and throttle reasons sampled every 100 ms while active."""
+    """nvidia-smi clocks and throttle reasons sampled every 20 ms while active; the summary
+    keeps the samples taken inside the timed region (mark() brackets it)."""
 
     def __init__(self, index):
         self.index = index
@@ -195,10 +196,14 @@ class ClockSampler:
     def start(self):
         try:
             self.p = subprocess.Popen(["nvidia-smi", f"--id={self.index}", f"--query-gpu={CLOCK_QUERY}",
-                                       "--format=csv,noheader,nounits", "-lms", "100"], stdout=self.f,
+                                       "--format=csv,noheader,nounits", "-lms", "20"], stdout=self.f,
                                       stderr=subprocess.DEVNULL)
         except Exception:
             self.p = None
+
+    def mark(self, t0, t1):
+        """Host wall-clock bounds (time.time()) of the timed region."""
+        self.t0, self.t1 = t0, t1
 
     def stop(self):
         if self.p is not None:
@@ -209,22 +214,48 @@ class ClockSampler:
                 self.p.kill()
         self.f.flush()
 
+    @staticmethod
+    def parse(lines):
+        """(epoch seconds, fields after the timestamp) of every well-formed sample line."""
+        import datetime
+
+        out = []
+        for line in lines:
+            parts = [x.strip() for x in line.split(",")]
+            if len(parts) < 10 or not parts[2].replace(".", "").isdigit():
+                continue
+            try:
+                ts = datetime.datetime.strptime(parts[0], "%Y/%m/%d %H:%M:%S.%f").timestamp()
+            except ValueError:
+                continue
+            out.append((ts, parts[1:]))
+        return out
+
     def summary(self):
-        rows = []
         try:
-            for line in open(self.f.name):
-                parts = [x.strip() for x in line.split(",")]
-                if len(parts) >= 9 and parts[1].replace(".", "").isdigit():
-                    rows.append(parts)
+            samples = self.parse(open(self.f.name))
         except Exception:
-            pass
-        if not rows:
+            samples = []
+        return self.summarize(samples, self.t0, self.t1)
+
+    @staticmethod
+    def summarize(samples, t0, t1):
+        if not samples:
             return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no nvidia-smi samples"], "samples": 0}
+        window = "timed region"
+        rows = [r for ts, r in samples if t0 is not None and t0 - 0.01 <= ts <= t1 + 0.01]
+        if not rows:
+            # the region was shorter than the sampling period: the samples nearest to it
+            window = "nearest samples (timed region shorter than the sampling period)"
+            mid = 0.5 * (t0 + t1) if t0 is not None else samples[-1][0]
+            near = sorted(samples, key=lambda x: abs(x[0] - mid))[:3]
+            rows = [r for _, r in near]
         sm = [float(r[1]) for r in rows]
         names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
         reasons = sorted({names[i] for r in rows for i in range(4) if r[5 + i].lower().startswith("active")})
         return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(float(r[2]) for r in rows),
-                "reasons": reasons, "samples": len(rows), "power_w_max": max(float(r[3]) for r in rows)}
+                "reasons": reasons, "samples": len(rows), "window": window,
+                "power_w_max": max(float(r[3]) for r in rows)}
 
 
 def setup_router(sc, torch, prefix_index):
@@ -351,6 +382,7 @@ def run_gb300(args):
         dist.barrier()
     torch.cuda.synchronize()
     t_wall = time.perf_counter()
+    t_epoch0 = time.time()
     for k in range(K):
         r.checkpoint_restore(ckpt)
         flush_l2()
@@ -364,6 +396,8 @@ def run_gb300(args):
     if dist:
         dist.barrier()
     wall = time.perf_counter() - t_wall
+    sampler.mark(t_epoch0, time.time())
+    time.sleep(0.05)
     sampler.stop()
     step_ms = [starts[k].elapsed_time(ends[k]) for k in range(K)]
     total_ms = float(sum(step_ms))
