@@ -105,10 +105,46 @@ def test_parity_config5_reduced():
 
 def test_parity_config5_full_size():
     """The benchmark workload itself: 128 x 262,144 blocks at 95% fill, 65,536 requests,
-    in the launch configuration the benchmark times."""
+    in the launch configuration the benchmark times: the measured batch is routed as the
+    benchmark routes it (same buffers every call, so the route is launched directly, then
+    captured, then replayed from its CUDA graph) and every one of those routes must give the
+    oracle's decisions; then the commit and every instance's index are compared."""
+    import torch
+
     sc = wl.config5(n=65536, fill=0.95)
-    r, o = run_parity(sc, index_every_step=False, check_keys=True)
-    r.close()
+    r = make_router(sc)
+    o = make_oracle(sc)
+    try:
+        for f in sc.fillers:
+            r.load_entries(f.w, f.keys, f.metas)
+            o.load_entries(f.w, f.keys, f.metas)
+        for b, comp in sc.warm:
+            route_both(r, o, b, sc.W, check_H=False, check_keys=False)
+            r.commit()
+            o.commit()
+            if comp is not None:
+                for x in (r, o):
+                    x.complete(comp.session, comp.cls, comp.total_blocks, comp.residency_us, comp.done)
+        b = sc.batch
+        route_both(r, o, b, sc.W, check_H=True, check_keys=True)  # H and keys against the oracle
+        oi, orr, oh = o.route(b.cls, b.session, b.tok_off, b.tokens)
+        db, out = r.device_batch(b), r.alloc_decisions(b.n)
+        for rep in range(3):
+            out["inst"].fill_(-7)
+            r.route(db, out)
+            torch.cuda.synchronize()
+            assert_equal(f"inst (bench call {rep})", out["inst"][: b.n].cpu().numpy(), oi)
+            assert_equal(f"reason (bench call {rep})", out["reason"][: b.n].cpu().numpy(), orr)
+            assert_equal(f"hit blocks (bench call {rep})", out["hit_blocks"][: b.n].cpu().numpy(), oh)
+        r.commit()
+        o.commit()
+        compare_state(r, o, sc.W, index=True)
+        s, os_ = r.stats(), o.stats()
+        assert s.new_keys == os_[21] and s.evicted == os_[22]
+        assert o.check_invariants() == 0
+        r.sync()
+    finally:
+        r.close()
 
 
 # ------------------------------------------------------------------ edge cases
