@@ -112,10 +112,17 @@ HASH_PROFILE = os.path.join(ROOT, "profiles", "k1_block_hash_stress_n65536.md")
 
 
 def hash_sources_sha256():
+    """sha256 of the block-hash kernel's sources with comments and blank space removed (a
+    comment edit does not make the committed ncu figures stale; a code edit does)."""
+    import re
+
     h = hashlib.sha256()
     for f in HASH_SOURCES:
-        with open(os.path.join(ROOT, f), "rb") as fh:
-            h.update(fh.read())
+        with open(os.path.join(ROOT, f)) as fh:
+            text = fh.read()
+        text = re.sub(r"/\*.*?\*/", " ", text, flags=re.S)
+        text = re.sub(r"//[^\n]*", " ", text)
+        h.update(" ".join(text.split()).encode())
     return h.hexdigest()
 
 

@@ -7,9 +7,9 @@
  * places the request on an inference instance, or holds it for re-evaluation.
  * This library computes that decision for a whole batch on one GPU:
  *
- *   1. chained 16-token block hashes of every prompt (Sec. 4.5),
+ *   1. chained 16-token block hashes of every prompt (Sec. 4.4),
  *   2. the longest cached prefix H_rw of every request on every instance's
- *      resident-block index, held as GPU open-addressing hash tables (Sec. 4.5),
+ *      resident-block index, held as GPU open-addressing hash tables (Sec. 4.4),
  *   3. caps K_w and K_wb (Sec. 4.1, Eqs. 9-13), eligibility (Eq. 6), prefill
  *      cost (Eq. 1) and the hold-vs-cold rule (Eq. 7), argmin placement,
  *   4. arrival-order admission under the global and class caps (Eq. 6, Sec. 4.2),
@@ -57,7 +57,7 @@ extern "C" {
 #define MISAT_PREFIX_GLOBAL 0       /* key -> instance bitmask, one lookup per request (default) */
 #define MISAT_PREFIX_PER_INSTANCE 1 /* one lookup per (request, instance) pair */
 
-/* ---- policy modes (Sec. 5.2 ablation variants) ---- */
+/* ---- policy modes (Sec. 5.1: the policies the evaluation compares) ---- */
 #define MISAT_MODE_MISA_T 0            /* block-time quota, Eqs. (11),(13) (default) */
 #define MISAT_MODE_MISA 1              /* spatial quota, Eqs. (9)-(10) */
 #define MISAT_MODE_SESSION_ADMISSION 2 /* global cap only (class-agnostic) */
@@ -208,7 +208,7 @@ int misat_route_staged(misat_ctx* ctx, int32_t slot, misat_decisions* host_out);
 /* Apply the pending route: insert every admitted request's blocks into its instance's
  * index (tick = commit number and arrival index, depth = block index, max-merge), make
  * newly admitted sessions protected on their instance (a rebound session leaves its old
- * instance), then evict each instance down to Cap_w (Sec. 4.1, Sec. 4.5).  Waits for the
+ * instance), then evict each instance down to Cap_w (Sec. 4.1, Sec. 4.4).  Waits for the
  * route's small summary, then enqueues.  Errors: STATE (no pending route). */
 int misat_commit(misat_ctx* ctx);
 
@@ -217,12 +217,12 @@ int misat_commit(misat_ctx* ctx);
  *              bounded histories (Sec. 4.1, Sec. 4.3) and the session leaves the
  *              protected set and is forgotten;
  *   done == 0: protection is released but the session is remembered; its next
- *              request is a continuation that must reacquire admission (Eq. 7).
+ *              request is a continuation that must be admitted again (Eq. 7).
  * Unknown sessions only update the histories.  [async] */
 int misat_complete(misat_ctx* ctx, int32_t n, const uint64_t* session, const uint8_t* cls,
                    const int32_t* total_blocks, const int64_t* residency_us, const uint8_t* done);
 
-/* Engine removal events (Sec. 4.5): remove the listed keys (host array) from instance
+/* Engine removal events (Sec. 4.4): remove the listed keys (host array) from instance
  * w's index.  The removed set must be suffix-closed (no remaining block may lose its
  * parent).  [sync] */
 int misat_evict(misat_ctx* ctx, int32_t w, const uint64_t* keys, int64_t n);
@@ -269,7 +269,7 @@ int misat_dump_sessions(misat_ctx* ctx, uint64_t* ids, int32_t* state, int32_t* 
 /* Statistics of the last route / commit.  [sync] */
 int misat_stats(misat_ctx* ctx, misat_batch_stats* host_out);
 
-/* Global prefix index (Sec. 4.5: the router maps every prefix block hash to the set of
+/* Global prefix index (Sec. 4.4: the router maps every prefix block hash to the set of
  * instances that currently cache it).  With MISAT_PREFIX_GLOBAL the library keeps, next to
  * the per-instance tables, one table key -> W-bit instance mask that mirrors them exactly;
  * the block-0 probe of a request reads one mask instead of W tables.

@@ -9,12 +9,12 @@
 //
 // Paper passages followed (section / equation):
 //   Sec. 3.2 Eq. (1)   prefill-cost placement  c = d_w + (L_r - H_rw) / mu_w
-//   Sec. 4.5           H_rw = longest matching prompt-block hash on instance w;
+//   Sec. 4.4           H_rw = longest matching prompt-block hash on instance w;
 //                      eviction / reset removes hashes
 //   Sec. 4.1 Eq. (6)   Admit(r,w): continuation admitted, new session only with
 //                      headroom |O_w|+|P_w| < K_w, otherwise HOLD
-//   Sec. 4.1 Eq. (7)   hold-vs-cold rule for a continuation that must reacquire
-//                      admission
+//   Sec. 4.1 Eq. (7)   hold-vs-cold rule for a continuation that must be admitted
+//                      again
 //   Sec. 4.1           K_w^base = floor(C_w / kbar_w), operational K_w <= K_w^base
 //   Sec. 4.2 Eqs. (9)-(10)  MISA spatial quota and class cap
 //   Sec. 4.3 Eqs. (11),(13) MISA-T block-time quota and class cap
@@ -71,7 +71,7 @@ constexpr int64_t TOKCOST_MAX = (int64_t)1 << 32;
 constexpr int64_t MAX_PROMPT_TOKENS = (int64_t)1 << 20;
 constexpr int BLOCK = 16;  // tokens per KV block
 
-// ---- block hash (reading: the engine's block hash is not specified, Sec. 4.5) ----
+// ---- block hash (reading: the engine's block hash is not specified, Sec. 4.4) ----
 // SplitMix64 finaliser (Steele, Lea & Flood 2014), golden-ratio increment G.
 constexpr uint64_t G = 0x9e3779b97f4a7c15ULL;
 
@@ -186,7 +186,7 @@ int insert_block(Oracle& o, int w, uint64_t key, uint64_t meta, uint64_t parent)
 
 // Evict down to capacity: remove the smallest (meta, key) pairs, i.e. least
 // recently committed first, deepest block first among equal ticks, key as the
-// last tie-break (reading: eviction policy unspecified, Sec. 4.5).
+// last tie-break (reading: eviction policy unspecified, Sec. 4.4).
 int64_t evict_to_cap(Oracle& o, int w) {
   int64_t sz = index_size(o, w);
   if (sz <= o.cap[w]) return 0;
@@ -223,7 +223,7 @@ int64_t estimate_T(const Oracle& o, int b) {
 void instance_caps(const Oracle& o, int w, const int64_t N[3], const int64_t kb[3],
                    const int64_t Tb[3], int64_t* Kw_out, int64_t Kwb_out[3],
                    int64_t* kbar_w_out) {
-  // conservative reference length: demand-weighted mean footprint, rounded up
+  // reference footprint of the instance: demand-weighted mean footprint, rounded up
   int64_t sumN = N[0] + N[1] + N[2];
   int64_t kw;
   if (sumN > 0) {
@@ -385,7 +385,7 @@ int oracle_route(void* h, int32_t n, const uint8_t* cls, const uint64_t* session
     o->keys[r] = hash_prompt(tokens + tok_off[r], o->L[r], o->hash_seed);
   }
 
-  // H_rw: number of leading blocks of r resident on w, by linear scan (Sec. 4.5)
+  // H_rw: number of leading blocks of r resident on w, by linear scan (Sec. 4.4)
   o->H.assign((size_t)n * W, 0);
   int64_t lookups = 0;
   for (int r = 0; r < n; ++r) {
@@ -488,7 +488,7 @@ int oracle_route(void* h, int32_t n, const uint8_t* cls, const uint64_t* session
         last_reason[r] = HOLD_NO_ELIGIBLE;
         continue;
       }
-      // Eq. (7): a continuation that must reacquire admission may prefer to wait
+      // Eq. (7): a continuation that must be admitted again may prefer to wait
       if (st_state[r] == SESS_RELEASED) {
         int wh = 0;
         for (int w = 1; w < W; ++w)
@@ -691,7 +691,7 @@ int oracle_commit(void* h) {
 
 // Completion events: done=1 finishes the session (histories, leaves the
 // protected set, forgotten); done=0 releases its protection but remembers it
-// (a later request is a continuation that must reacquire admission, Eq. 7).
+// (a later request is a continuation that must be admitted again, Eq. 7).
 int oracle_complete(void* h, int32_t n, const uint64_t* session, const uint8_t* cls,
                     const int32_t* total_blocks, const int64_t* residency_us,
                     const uint8_t* done) {
@@ -721,7 +721,7 @@ int oracle_complete(void* h, int32_t n, const uint64_t* session, const uint8_t* 
   return OK;
 }
 
-// Engine removal events (Sec. 4.5): remove the listed keys of instance w.
+// Engine removal events (Sec. 4.4): remove the listed keys of instance w.
 int oracle_evict(void* h, int32_t w, const uint64_t* keys, int64_t n) {
   Oracle* o = (Oracle*)h;
   if (w < 0 || w >= o->W || n < 0) return ERR_INVALID_ARG;

@@ -4,7 +4,7 @@
 // Index tables are bucketed linear-probing hash sets (4 keys per 32-byte sector).
 // Insert claims only empty slots with a CAS, so two threads inserting the same new
 // key always meet in the same slot (no duplicates) and an existing key is found by
-// every later inserter; the tick is merged with atomicMax (Sec. 4.5 reading: LRU).
+// every later inserter; the tick is merged with atomicMax (Sec. 4.4 reading: LRU).
 // Eviction never leaves tombstones: the exact eviction threshold theta (the E-th
 // smallest (meta, key)) is found by a per-instance radix select, then every run of
 // full buckets is compacted by one thread with backward shifts, so lookups keep
@@ -345,7 +345,7 @@ void launch_session_update(const SessUpdateArgs& a, cudaStream_t st) {
 }
 
 // Completion events (distinct sessions): leave the protected set; done -> dead slot,
-// otherwise released (a later request must reacquire admission, Eq. 7).
+// otherwise released (a later request must be admitted again, Eq. 7).
 __global__ void __launch_bounds__(256) k_complete(CompleteArgs a) {
   const int i = blockIdx.x * blockDim.x + threadIdx.x;
   if (i >= a.n) return;
@@ -373,7 +373,7 @@ void launch_complete(const CompleteArgs& a, cudaStream_t st) {
   k_complete<<<(a.n + 255) / 256, 256, 0, st>>>(a);
 }
 
-// External removal (Sec. 4.5 engine events): mark listed keys (meta = 0), rebuild the
+// External removal (Sec. 4.4 engine events): mark listed keys (meta = 0), rebuild the
 // fullness bitmap from the keys, then compact with theta inactive.
 __global__ void __launch_bounds__(256) k_mark(MarkArgs a) {
   long long cnt = 0;

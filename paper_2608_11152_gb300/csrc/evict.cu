@@ -1,6 +1,6 @@
 // Eviction down to capacity (K4c): after a commit's inserts, each instance whose index
 // holds E = size - Cap_w > 0 entries too many loses its E smallest (meta, key): the
-// least recently committed blocks, deepest first among equal ticks (Sec. 4.5 reading:
+// least recently committed blocks, deepest first among equal ticks (Sec. 4.4 reading:
 // LRU; the commit-tick order keeps every index prefix-closed).
 //
 // Admissions concentrate on few instances (every cold request of a round prefers the

@@ -1,5 +1,5 @@
 // Global prefix index maintenance outside the commit path: rebuild from the instance
-// tables, and the clear that precedes an instance reset (Sec. 4.5: a cache reset removes
+// tables, and the clear that precedes an instance reset (Sec. 4.4: a cache reset removes
 // the instance from every hash it held).
 #include <algorithm>
 

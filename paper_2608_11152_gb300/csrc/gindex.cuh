@@ -1,5 +1,5 @@
 // Global prefix index: block key -> bitmask of the instances whose table holds the key
-// (Sec. 4.5: the router keeps, for every prefix hash, the set of instances caching it).
+// (Sec. 4.4: the router keeps, for every prefix hash, the set of instances caching it).
 //
 // The per-instance tables stay the source of truth (they carry the eviction order); the
 // global index mirrors their key sets exactly: a key enters instance w's table <=> bit w

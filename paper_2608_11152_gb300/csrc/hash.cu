@@ -1,4 +1,4 @@
-// K1: chained 16-token block hash (Sec. 4.5: the router's prefix index is keyed by
+// K1: chained 16-token block hash (Sec. 4.4: the router's prefix index is keyed by
 // block hashes of the engine's prefix cache).
 //
 // Key of block j of a prompt:  c_j = mix64(XOR_i mix64(x_i + (i+1)G)) over the

@@ -1,5 +1,6 @@
 // K2: longest cached prefix H_rw of every request on every instance (Sec. 3.2, Eq. 1;
-// Sec. 4.5: "the longest matching prompt-block hash determines the reusable prefix").
+// Sec. 4.4: the reusable prefix on an instance is the longest run of the prompt's block
+// hashes that the instance caches).
 //
 // Every instance index is prefix-closed (a commit writes whole prefixes with one
 // tick and eviction takes the deepest block of a tick first), so "block h-1 is

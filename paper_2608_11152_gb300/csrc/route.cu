@@ -148,7 +148,7 @@ __global__ void __launch_bounds__(1024) k3_caps(CapsArgs a) {
       tot += p;
       a.ia.N_wb[w * 3 + b] = N[b];
     }
-    // conservative reference length kbar_w: demand-weighted class footprint, rounded up
+    // reference footprint kbar_w: demand-weighted class footprint, rounded up
     int64_t kw;
     if (sumN > 0) {
       __int128 num = 0;

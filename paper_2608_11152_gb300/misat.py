@@ -369,7 +369,7 @@ class Router:
         _ck(_lib.misat_stats(self._h, C.byref(s)), "misat_stats")
         return s
 
-    # ---- global prefix index (Sec. 4.5: block hash -> instances caching it)
+    # ---- global prefix index (Sec. 4.4: block hash -> instances caching it)
     def global_info(self):
         """(mask words per key, slots, claimed slots) of the global prefix index."""
         mw, slots, used = C.c_int32(0), C.c_int64(0), C.c_int64(0)

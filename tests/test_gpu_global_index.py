@@ -1,4 +1,4 @@
-"""Global prefix index (Sec. 4.5: the router maps each prefix block hash to the set of
+"""Global prefix index (Sec. 4.4: the router maps each prefix block hash to the set of
 instances that cache it) against the oracle's per-instance indexes.
 
 The CUDA path keeps a key -> instance-bitmask table next to the per-instance tables and

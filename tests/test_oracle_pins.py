@@ -335,7 +335,7 @@ def test_prefer_cache_rule_eq7():
         inst, reason, _ = o.route(b1.cls, b1.session, b1.tok_off, b1.tokens)
         assert inst[0] == 0 and reason[0] == oracle.ADMIT_NEW
         o.commit()
-        o.complete([77], [2], [0], [0], [0])              # released: must reacquire admission
+        o.complete([77], [2], [0], [0], [0])              # released: must be admitted again
         # another session now fills instance 0's single slot
         b2 = _batch([0], [88], [16], seed=5)
         o.route(b2.cls, b2.session, b2.tok_off, b2.tokens)
