@@ -205,6 +205,38 @@ int misat_route_host(misat_ctx* ctx, const misat_batch* host_batch, misat_decisi
 int misat_stage_host(misat_ctx* ctx, const misat_batch* host_batch, int32_t slot);
 int misat_route_staged(misat_ctx* ctx, int32_t slot, misat_decisions* host_out);
 
+/* A batch whose prompts are sent as extensions of earlier prompts of the same batch (HOST
+ * pointers).  An agentic turn re-sends its session's whole history, and the samples of an
+ * RL prompt group share one prompt; with this layout each request carries only the tokens
+ * that follow the prompt of an earlier request it extends, so far fewer bytes cross the
+ * host link.  No counterpart in the paper: it is an input encoding; the routing decision is
+ * the one of the full batch.
+ *   base[r]    -1, or an earlier request (0 <= base[r] < r) whose whole prompt is the start
+ *              of r's prompt; chains of bases at most MISAT_DELTA_MAX_DEPTH long
+ *   delta_off  [n+1] CSR offsets into delta_tokens, delta_off[0] = 0, non-decreasing
+ *   delta_tokens  request r's prompt = prompt(base[r]) followed by
+ *              delta_tokens[delta_off[r] .. delta_off[r+1]) */
+#define MISAT_DELTA_MAX_DEPTH 64
+typedef struct misat_batch_delta {
+  int32_t n;
+  const uint8_t* cls;
+  const uint64_t* session;
+  const int32_t* base;
+  const int64_t* delta_off;
+  const int32_t* delta_tokens;
+} misat_batch_delta;
+
+/* misat_stage_host for a delta-encoded batch: copies cls, session, bases and delta tokens
+ * into staging slot 0 or 1 on the copy stream, then rebuilds the slot's full token array on
+ * the GPU (on the same stream), so that misat_route_staged routes exactly the batch the
+ * bases and deltas describe.  The full offsets are computed on the host; full prompts must
+ * stay below 2^20 tokens and their total within max_tokens.  The first delta call also
+ * allocates the slots' delta buffers (4 max_tokens + 12 max_batch bytes of device memory
+ * each, and 8 max_batch bytes of pinned host memory).  Host arrays as for misat_stage_host.
+ * [async]  Errors: INVALID_ARG (a base out of range, a chain deeper than
+ * MISAT_DELTA_MAX_DEPTH, offsets out of order), BATCH_TOO_LARGE, STATE, OOM, CUDA. */
+int misat_stage_host_delta(misat_ctx* ctx, const misat_batch_delta* host_batch, int32_t slot);
+
 /* Apply the pending route: insert every admitted request's blocks into its instance's
  * index (tick = commit number and arrival index, depth = block index, max-merge), make
  * newly admitted sessions protected on their instance (a rebound session leaves its old

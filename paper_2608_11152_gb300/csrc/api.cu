@@ -156,7 +156,14 @@ struct misat_ctx {
     bool staged = false;
     cudaEvent_t ev_copied = nullptr;  // the slot's H2D copies are done
     cudaEvent_t ev_free = nullptr;    // the last route that read the slot is done
+    // delta-encoded batches (misat_stage_host_delta), allocated on first use
+    int32_t* dbase = nullptr;
+    int64_t* doff = nullptr;
+    int32_t* dtok = nullptr;
+    int64_t* h_off = nullptr;  // pinned: full offsets computed on the host
   } slot[2];
+  std::vector<int64_t> delta_len;  // host scratch of misat_stage_host_delta
+  std::vector<uint8_t> delta_depth;
   cudaStream_t copy_stream = nullptr;
   std::vector<void*> owned;  // fixed allocations freed in destroy
   // launch sequences replayed as CUDA graphs (captured on a private stream, which never
@@ -703,6 +710,7 @@ int misat_destroy(misat_ctx* c) {
   for (auto& sl : c->slot) {
     if (sl.ev_copied) cudaEventDestroy(sl.ev_copied);
     if (sl.ev_free) cudaEventDestroy(sl.ev_free);
+    if (sl.h_off) cudaFreeHost(sl.h_off);
   }
   if (c->ev_fork) cudaEventDestroy(c->ev_fork);
   if (c->ev_join) cudaEventDestroy(c->ev_join);
@@ -1025,6 +1033,83 @@ int misat_stage_host(misat_ctx* c, const misat_batch* hb, int32_t slot) {
   CK(cudaEventRecord(sl.ev_copied, cs));
   sl.n = n;
   sl.n_tokens = hb->n_tokens;
+  sl.staged = true;
+  return MISAT_OK;
+}
+
+namespace {
+
+// Device and pinned host buffers of the delta-encoded staging path (first use).
+int ensure_delta_staging(misat_ctx* c) {
+  const size_t NB = (size_t)c->max_batch;
+  for (auto& sl : c->slot) {
+    int rc;
+    if ((!sl.dbase && (rc = dalloc_n(c, &sl.dbase, NB))) || (!sl.doff && (rc = dalloc_n(c, &sl.doff, NB + 1))) ||
+        (!sl.dtok && (rc = dalloc_n(c, &sl.dtok, (size_t)c->max_tokens + 8))))
+      return rc;
+    if (!sl.h_off) {
+      if (cudaMallocHost(&sl.h_off, (NB + 1) * sizeof(int64_t)) != cudaSuccess) {
+        cudaGetLastError();
+        sl.h_off = nullptr;
+        return MISAT_ERR_OOM;
+      }
+    }
+  }
+  return MISAT_OK;
+}
+
+}  // namespace
+
+int misat_stage_host_delta(misat_ctx* c, const misat_batch_delta* hb, int32_t slot) {
+  if (!c || !hb || slot < 0 || slot > 1) return MISAT_ERR_INVALID_ARG;
+  const int32_t n = hb->n;
+  if (n < 0) return MISAT_ERR_INVALID_ARG;
+  if (n > c->max_batch) return MISAT_ERR_BATCH_TOO_LARGE;
+  if (n > 0 && (!hb->cls || !hb->session || !hb->base || !hb->delta_off)) return MISAT_ERR_INVALID_ARG;
+  misat_ctx::StageSlot& sl = c->slot[slot];
+  if (sl.staged) return MISAT_ERR_STATE;
+  const int64_t nd = n > 0 ? hb->delta_off[n] : 0;
+  if (n > 0 && hb->delta_off[0] != 0) return MISAT_ERR_INVALID_ARG;
+  if (nd < 0 || nd > c->max_tokens) return MISAT_ERR_BATCH_TOO_LARGE;
+  if (nd > 0 && !hb->delta_tokens) return MISAT_ERR_INVALID_ARG;
+  int rc = ensure_staging(c);
+  if (rc) return rc;
+  if ((rc = ensure_delta_staging(c))) return rc;
+  // full lengths and offsets: prompt(r) = prompt(base[r]) ++ delta(r), written to the slot's
+  // pinned buffer once the copy of the slot's previous batch has read it
+  CK(cudaEventSynchronize(sl.ev_copied));
+  c->delta_len.resize((size_t)n);
+  c->delta_depth.resize((size_t)n);
+  int64_t* off = sl.h_off;
+  off[0] = 0;
+  for (int32_t r = 0; r < n; ++r) {
+    const int32_t b = hb->base[r];
+    const int64_t d = hb->delta_off[r + 1] - hb->delta_off[r];
+    if (b < -1 || b >= r || d < 0) return MISAT_ERR_INVALID_ARG;
+    const int64_t L = (b >= 0 ? c->delta_len[b] : 0) + d;
+    const int depth = (b >= 0 ? c->delta_depth[b] : 0) + 1;
+    if (depth > MISAT_DELTA_MAX_DEPTH || L >= ((int64_t)1 << 20)) return MISAT_ERR_INVALID_ARG;
+    c->delta_len[r] = L;
+    c->delta_depth[r] = (uint8_t)depth;
+    off[r + 1] = off[r] + L;
+    if (off[r + 1] > c->max_tokens) return MISAT_ERR_BATCH_TOO_LARGE;
+  }
+  cudaStream_t cs = c->copy_stream;
+  CK(cudaStreamWaitEvent(cs, sl.ev_free, 0));
+  if (n > 0) {
+    CK(cudaMemcpyAsync(sl.off, off, (size_t)(n + 1) * 8, cudaMemcpyHostToDevice, cs));
+    CK(cudaMemcpyAsync(sl.cls, hb->cls, (size_t)n, cudaMemcpyHostToDevice, cs));
+    CK(cudaMemcpyAsync(sl.ses, hb->session, (size_t)n * 8, cudaMemcpyHostToDevice, cs));
+    CK(cudaMemcpyAsync(sl.dbase, hb->base, (size_t)n * 4, cudaMemcpyHostToDevice, cs));
+    CK(cudaMemcpyAsync(sl.doff, hb->delta_off, (size_t)(n + 1) * 8, cudaMemcpyHostToDevice, cs));
+    if (nd > 0) CK(cudaMemcpyAsync(sl.dtok, hb->delta_tokens, (size_t)nd * 4, cudaMemcpyHostToDevice, cs));
+    DeltaArgs da{n, sl.dbase, sl.doff, sl.dtok, sl.off, sl.tok};
+    launch_delta_expand(da, c->num_sms, cs);
+    CK(cudaGetLastError());
+  }
+  CK(cudaEventRecord(sl.ev_copied, cs));
+  sl.n = n;
+  sl.n_tokens = n > 0 ? off[n] : 0;
   sl.staged = true;
   return MISAT_OK;
 }

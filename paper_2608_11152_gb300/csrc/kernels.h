@@ -280,6 +280,18 @@ struct CopyList {
 };
 void launch_copy_list(const CopyList& l, int num_sms, cudaStream_t st);
 
+// ---- delta-encoded host batches (misat_stage_host_delta) ----
+constexpr int kDeltaMaxDepth = MISAT_DELTA_MAX_DEPTH;
+struct DeltaArgs {
+  int32_t n;
+  const int32_t* base;     // [n] base request or -1
+  const int64_t* doff;     // [n+1] offsets of the deltas
+  const int32_t* dtok;     // delta tokens
+  const int64_t* tok_off;  // [n+1] full offsets (computed on the host)
+  int32_t* tokens;         // full tokens (output)
+};
+void launch_delta_expand(const DeltaArgs& a, int num_sms, cudaStream_t st);
+
 struct SessRehashArgs {
   SessTable from;
   SessTable to;

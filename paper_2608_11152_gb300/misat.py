@@ -48,6 +48,11 @@ class misat_batch(C.Structure):
                 ("tok_off", _p), ("tokens", _p), ("out_H", _p)]
 
 
+class misat_batch_delta(C.Structure):
+    _fields_ = [("n", C.c_int32), ("cls", _p), ("session", _p), ("base", _p), ("delta_off", _p),
+                ("delta_tokens", _p)]
+
+
 class misat_decisions(C.Structure):
     _fields_ = [("inst", _p), ("reason", _p), ("hit_blocks", _p)]
 
@@ -83,6 +88,7 @@ _SIG = {
     "misat_route_host": [_p, C.POINTER(misat_batch), C.POINTER(misat_decisions)],
     "misat_stage_host": [_p, C.POINTER(misat_batch), C.c_int32],
     "misat_route_staged": [_p, C.c_int32, C.POINTER(misat_decisions)],
+    "misat_stage_host_delta": [_p, C.POINTER(misat_batch_delta), C.c_int32],
     "misat_commit": [_p],
     "misat_complete": [_p, C.c_int32, _p, _p, _p, _p, _p],
     "misat_evict": [_p, C.c_int32, _p, C.c_int64],
@@ -273,6 +279,16 @@ class Router:
         if not hasattr(self, "_staged"):
             self._staged = {}
         self._staged[int(slot)] = (batch.n, cls, ses, off, tok)
+
+    def stage_host_delta(self, enc, slot):
+        """stage_host for a delta-encoded batch (workload.DeltaBatch: numpy arrays, pinned for
+        asynchrony); the arrays are kept referenced until the slot is routed."""
+        b = misat_batch_delta(enc.n, _nptr(enc.cls), _nptr(enc.session), _nptr(enc.base), _nptr(enc.delta_off),
+                              _nptr(enc.delta_tokens))
+        _ck(_lib.misat_stage_host_delta(self._h, C.byref(b), int(slot)), "misat_stage_host_delta")
+        if not hasattr(self, "_staged"):
+            self._staged = {}
+        self._staged[int(slot)] = (enc.n, enc.cls, enc.session, enc.base, enc.delta_off, enc.delta_tokens)
 
     def route_staged(self, slot, out=None):
         """Route the batch staged in `slot`; returns numpy decisions (written into `out` if given)."""

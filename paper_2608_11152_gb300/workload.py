@@ -79,6 +79,75 @@ class Batch:
 
 
 @dataclass
+class DeltaBatch:
+    """A batch whose prompts extend earlier prompts of the batch (the host layout of
+    misat_stage_host_delta): prompt(r) = prompt(base[r]) ++ delta_tokens[delta_off[r]:delta_off[r+1]]."""
+    cls: np.ndarray           # uint8 [n]
+    session: np.ndarray       # uint64 [n]
+    base: np.ndarray          # int32 [n], -1 or an earlier request
+    delta_off: np.ndarray     # int64 [n+1]
+    delta_tokens: np.ndarray  # int32
+
+    @property
+    def n(self) -> int:
+        return int(len(self.cls))
+
+
+DELTA_MAX_DEPTH = 64
+
+
+def encode_delta(b: Batch) -> DeltaBatch:
+    """Delta layout of a batch: a request's base is the latest earlier request of its session,
+    else the first earlier request of its prompt group, whose whole prompt starts its own
+    (checked token by token); chains stay within DELTA_MAX_DEPTH."""
+    n = b.n
+    base = np.full(n, -1, np.int32)
+    depth = np.zeros(n, np.int32)
+    last_of_session = {}
+    first_of_group = {}
+    parts, off = [], np.zeros(n + 1, np.int64)
+    for r in range(n):
+        t = b.tokens[b.tok_off[r]:b.tok_off[r + 1]]
+        cands = []
+        s = int(b.session[r])
+        if s in last_of_session:
+            cands.append(last_of_session[s])
+        g = int(b.group[r]) if b.group is not None else 0
+        if g and g in first_of_group:
+            cands.append(first_of_group[g])
+        for c in cands:
+            pt = b.tokens[b.tok_off[c]:b.tok_off[c + 1]]
+            if len(pt) <= len(t) and depth[c] < DELTA_MAX_DEPTH and np.array_equal(pt, t[:len(pt)]):
+                base[r] = c
+                depth[r] = depth[c] + 1
+                t = t[len(pt):]
+                break
+        else:
+            depth[r] = 1
+        parts.append(t)
+        off[r + 1] = off[r] + len(t)
+        last_of_session[s] = r
+        if g and g not in first_of_group:
+            first_of_group[g] = r
+    tok = np.concatenate(parts).astype(np.int32) if parts else np.zeros(0, np.int32)
+    return DeltaBatch(cls=b.cls.copy(), session=b.session.copy(), base=base, delta_off=off, delta_tokens=tok)
+
+
+def decode_delta(d: DeltaBatch) -> tuple:
+    """(tok_off, tokens) of the full batch a delta layout describes."""
+    n = d.n
+    full = []
+    off = np.zeros(n + 1, np.int64)
+    for r in range(n):
+        own = d.delta_tokens[d.delta_off[r]:d.delta_off[r + 1]]
+        t = np.concatenate([full[d.base[r]], own]) if d.base[r] >= 0 else own
+        full.append(t)
+        off[r + 1] = off[r] + len(t)
+    tok = np.concatenate(full).astype(np.int32) if full else np.zeros(0, np.int32)
+    return off, tok
+
+
+@dataclass
 class Completion:
     session: np.ndarray       # uint64
     cls: np.ndarray           # uint8

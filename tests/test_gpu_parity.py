@@ -314,6 +314,81 @@ def test_pipelined_host_staging_matches_the_oracle(cfg):
     r.close()
 
 
+def _pinned_delta(d):
+    def pin(a):
+        return torch.from_numpy(np.ascontiguousarray(a)).pin_memory().numpy()
+
+    return wl.DeltaBatch(cls=pin(d.cls), session=pin(d.session.view(np.int64)).view(np.uint64), base=pin(d.base),
+                         delta_off=pin(d.delta_off), delta_tokens=pin(d.delta_tokens))
+
+
+@pytest.mark.parametrize("cfg", [1, 2, 3])
+def test_delta_staging_matches_the_oracle(cfg):
+    """Batches sent in the delta layout (each prompt as an extension of an earlier prompt of
+    the batch), rebuilt on the GPU and routed through the pipelined slots: every decision,
+    every block key and the state after every commit equal the oracle's on the full batch."""
+    sc = {1: wl.config1, 2: wl.config2, 3: wl.config3}[cfg]()
+    r, o = make_router(sc), make_oracle(sc)
+    steps = list(sc.warm) + [(sc.batch, None)]
+    encs = [_pinned_delta(wl.encode_delta(b)) for b, _ in steps]
+    r.stage_host_delta(encs[0], 0)
+    for k, (b, comp) in enumerate(steps):
+        if k + 1 < len(steps):
+            r.stage_host_delta(encs[k + 1], (k + 1) % 2)
+        got = r.route_staged(k % 2)
+        oi, orr, oh = o.route(b.cls, b.session, b.tok_off, b.tokens)
+        assert_equal("inst", got["inst"][: b.n], oi)
+        assert_equal("reason", got["reason"][: b.n], orr)
+        assert_equal("hit_blocks", got["hit_blocks"][: b.n], oh)
+        cap = b.n_tokens // 16 + 1
+        assert_equal("keys", r.dump_keys(cap), o.keys(cap))
+        r.commit()
+        o.commit()
+        compare_state(r, o, sc.W)
+        if comp is not None:
+            for x in (r, o):
+                x.complete(comp.session, comp.cls, comp.total_blocks, comp.residency_us, comp.done)
+    r.sync()
+    r.close()
+
+
+def test_delta_staging_rejects_malformed_layouts():
+    """A base that is not an earlier request, a chain deeper than the limit and offsets that
+    do not start at zero are refused before anything is copied; the slot stays free."""
+    from paper_2608_11152_gb300 import misat
+
+    sc = wl.config1()
+    r = make_router(sc, max_batch=128)
+    b = sc.warm[0][0]
+    good = wl.encode_delta(b)
+
+    def variant(**kw):
+        f = dict(cls=good.cls, session=good.session, base=good.base.copy(), delta_off=good.delta_off.copy(),
+                 delta_tokens=good.delta_tokens)
+        f.update(kw)
+        return wl.DeltaBatch(**f)
+
+    bad_base = good.base.copy()
+    bad_base[3] = 3
+    deep = 70
+    chain = wl.DeltaBatch(cls=np.zeros(deep, np.uint8), session=np.arange(1, deep + 1, dtype=np.uint64),
+                          base=np.arange(-1, deep - 1, dtype=np.int32), delta_off=np.arange(0, 16 * deep + 1, 16,
+                                                                                            dtype=np.int64),
+                          delta_tokens=np.ones(16 * deep, np.int32))
+    shifted = good.delta_off.copy() + 1
+    for enc in (variant(base=bad_base), chain, variant(delta_off=shifted)):
+        with pytest.raises(misat.MisatError) as e:
+            r.stage_host_delta(enc, 0)
+        assert e.value.code == misat.ERR_INVALID_ARG
+    r.stage_host_delta(good, 0)  # the slot is still free
+    got = r.route_staged(0)
+    ref = r.route_host(b)
+    for k in ("inst", "reason", "hit_blocks"):
+        assert_equal(k, got[k][: b.n], ref[k][: b.n])
+    r.sync()
+    r.close()
+
+
 def test_pipelined_staging_slot_states_and_graph_replay():
     """A slot holds one batch until it is routed; routing an empty slot is refused.  The same
     batch routed from alternating slots after a state restore (graphs captured per slot and

@@ -17,7 +17,8 @@ def _declared():
 def test_header_declares_the_boundary():
     names = _declared()
     for must in ("misat_create", "misat_destroy", "misat_set_mixture", "misat_set_instance_state", "misat_route",
-                 "misat_route_host", "misat_stage_host", "misat_route_staged", "misat_commit", "misat_complete",
+                 "misat_route_host", "misat_stage_host", "misat_route_staged", "misat_stage_host_delta",
+                 "misat_commit", "misat_complete",
                  "misat_evict", "misat_reset_instance",
                  "misat_load_chains", "misat_load_entries", "misat_dump_index", "misat_stats", "misat_sync",
                  "misat_strerror"):
