@@ -28,3 +28,14 @@ def test_reasons_and_a_region_shorter_than_the_sampling_period():
     assert s["window"].startswith("nearest samples")
     assert "sw_power_cap" in s["reasons"]
     assert bench.ClockSampler.summarize([], t0, t0 + 1)["samples"] == 0
+
+
+def test_launch_count_claim_matches_the_committed_launch_list():
+    """gpu_launches (kernels per step x steps) against the ncu launch list of the stress step
+    (two steps captured): the per-step count the benchmark claims is the one ncu saw."""
+    import os
+    import re
+
+    path = os.path.join(os.path.dirname(bench.__file__), "profiles", "launches_route_commit_cfg5_n65536_fill95.md")
+    totals = [int(m.group(1)) for m in re.finditer(r"\| \*\*total\*\* \| (\d+) \|", open(path).read())]
+    assert totals and all(t == 2 * bench.kernels_per_step(4, True) for t in totals)
