@@ -166,10 +166,11 @@ int misat_set_instance_state(misat_ctx* ctx, const int64_t* backlog_q, const int
 /* Route one batch against the state at batch start (Sec. 3.1, Sec. 4).  Inputs and
  * outputs are device pointers; outputs are written before the call's work ends on the
  * stream.  A second route without a commit replaces the pending one.  [async]
- * When the same batch and output buffers (and sizes) come twice in a row, the route's
- * kernels are captured once into a CUDA graph (on a private stream) and replayed from then
- * on; while the caller captures the context's stream itself, or phase timing is on, they
- * are launched directly.  Errors: INVALID_ARG, BATCH_TOO_LARGE; malformed contents are
+ * The second time a set of batch and output buffers (and sizes) comes among the last four
+ * sets seen, the route's kernels are captured into a CUDA graph (on a private stream) and
+ * replayed from then on; the graphs of the four most recently used sets are kept.  While
+ * the caller captures the context's stream itself, or phase timing is on, they are launched
+ * directly.  Errors: INVALID_ARG, BATCH_TOO_LARGE; malformed contents are
  * reported by misat_sync. */
 int misat_route(misat_ctx* ctx, const misat_batch* batch, misat_decisions* out);
 

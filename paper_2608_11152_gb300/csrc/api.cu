@@ -222,8 +222,9 @@ namespace {
 
 // Launch a fixed sequence through a cached CUDA graph: `launch(stream)` enqueues the
 // sequence; it is captured once per key (the values its kernel arguments depend on) and
-// replayed with one graph launch.  When the context's stream is itself being captured by
-// the caller, or capture is unavailable, the sequence is launched directly.
+// replayed with one graph launch; the cache keeps the graphs of the four most recently used
+// keys.  When the context's stream is itself being captured by the caller, or capture is
+// unavailable, the sequence is launched directly.
 template <class F>
 int run_graph(misat_ctx* c, misat_ctx::GraphCache& gc, const std::vector<uint64_t>& key, F&& launch) {
   cudaStream_t st = c->stream;
