@@ -269,7 +269,7 @@ def setup_router(sc, torch, prefix_index):
     from paper_2608_11152_gb300 import misat
 
     r = misat.Router(sc.cap_blocks, max_batch=sc.max_batch, max_tokens=sc.max_tokens,
-                     protected_frac_q16=sc.protected_frac_q16, rounds=sc.rounds, mode=sc.mode,
+                     protected_frac_q16=sc.protected_frac_q16, mode=sc.mode,
                      hold_delay_q=sc.hold_delay_q, prior_kbar=sc.prior_kbar, prior_T_us=sc.prior_T_us,
                      prefix_index=prefix_index)
     r.set_mixture(sc.rho_ppm)
@@ -289,7 +289,7 @@ def setup_router(sc, torch, prefix_index):
 def setup_oracle(sc):
     import oracle
 
-    o = oracle.Oracle(sc.cap_blocks, protected_frac_q16=sc.protected_frac_q16, rounds=sc.rounds, mode=sc.mode,
+    o = oracle.Oracle(sc.cap_blocks, protected_frac_q16=sc.protected_frac_q16, mode=sc.mode,
                       hold_delay_q=sc.hold_delay_q, prior_kbar=sc.prior_kbar, prior_T_us=sc.prior_T_us)
     o.set_mixture(sc.rho_ppm)
     o.set_instance_state(sc.backlog_q, sc.tokcost_q, sc.contraction)

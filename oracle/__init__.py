@@ -66,7 +66,7 @@ def _load():
         "oracle_mix64": (u64, [u64]),
         "oracle_hash_prompt": (i64, [p, i64, u64, p]),
         "oracle_caps_eval": (C.c_int, [i64, p, p, p, i32, p, p, p]),
-        "oracle_create": (p, [i32, p, i32, i32, i32, i64, i32, i32, p, i64, u64]),
+        "oracle_create": (p, [i32, p, i32, i32, i64, i32, i32, p, i64, u64]),
         "oracle_destroy": (None, [p]),
         "oracle_set_mixture": (C.c_int, [p, p]),
         "oracle_set_instance_state": (C.c_int, [p, p, p, p]),
@@ -131,14 +131,14 @@ def caps_eval(Cw, N, kbar, T, mode=MODE_MISA_T, rho=(333334, 333333, 333333)):
 class Oracle:
     """Owning handle of one oracle router state (host memory)."""
 
-    def __init__(self, cap_blocks, protected_frac_q16=58982, rounds=4, mode=MODE_MISA_T,
+    def __init__(self, cap_blocks, protected_frac_q16=58982, mode=MODE_MISA_T,
                  hold_delay_q=0, hist_window=256, min_obs=8, prior_kbar=(64, 64, 64),
                  prior_T_us=30_000_000, hash_seed=0x9E3779B97F4A7C15):
         lib = _load()
         cap = _arr(cap_blocks, np.int64)
         pk = _arr(prior_kbar, np.int64)
         self.W = len(cap)
-        self._h = lib.oracle_create(self.W, _ptr(cap), protected_frac_q16, rounds, mode, hold_delay_q,
+        self._h = lib.oracle_create(self.W, _ptr(cap), protected_frac_q16, mode, hold_delay_q,
                                     hist_window, min_obs, _ptr(pk), prior_T_us, C.c_uint64(hash_seed))
         if not self._h:
             raise ValueError("invalid oracle configuration")

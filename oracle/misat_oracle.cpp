@@ -22,9 +22,10 @@
 //                      a new session needs global and class headroom
 //   Sec. 3.3           D_TV(p, q) = 1/2 |p - q|_1
 //
-// Where the paper is silent (hash function, index eviction order, batch rounds,
-// fixed-point units) the oracle follows the readings listed in the design notes
-// of this repository; each such place is marked "reading:" below.
+// Where the paper is silent (hash function, index eviction order, the order in
+// which the requests of one batch are decided, fixed-point units) the oracle
+// follows the readings listed in the design notes of this repository; each such
+// place is marked "reading:" below.
 //
 // Parity status: every function below is pinned by the -m "not gpu" tests
 // (published SplitMix64 vectors, token-by-token brute force of H, hand-worked
@@ -58,7 +59,7 @@ constexpr uint8_t ADMIT_NEW = 2;
 constexpr uint8_t ADMIT_FOLLOW = 3;
 constexpr uint8_t HOLD_GLOBAL_CAP = 16;
 constexpr uint8_t HOLD_CLASS_CAP = 17;
-constexpr uint8_t HOLD_NO_ELIGIBLE = 18;
+constexpr uint8_t HOLD_NO_ELIGIBLE = 18;  // reserved: the serial selection never produces it
 constexpr uint8_t HOLD_PREFER_CACHE = 19;
 constexpr uint8_t HOLD_LEADER_HELD = 20;
 
@@ -66,7 +67,7 @@ constexpr int SESS_PROTECTED = 1;   // s in O_w u P_w on instance `inst`
 constexpr int SESS_RELEASED = 2;    // admitted before, protected nowhere now
 
 constexpr int64_t CAP_INF = 2147483647;           // "no cap"
-constexpr int64_t BACKLOG_MAX = (int64_t)1 << 61;   // saturation of in-batch backlog
+constexpr int64_t BACKLOG_MAX = (int64_t)1 << 61;   // largest backlog d_w and hold delay
 constexpr int64_t TOKCOST_MAX = (int64_t)1 << 32;
 constexpr int64_t MAX_PROMPT_TOKENS = (int64_t)1 << 20;
 constexpr int BLOCK = 16;  // tokens per KV block
@@ -135,7 +136,6 @@ struct Oracle {
   int32_t W = 0;
   std::vector<int64_t> cap;
   int32_t pf_q16 = 0;
-  int32_t rounds = 1;
   int32_t mode = 0;
   int64_t hold_delay_q = 0;
   int32_t hist_window = 256;
@@ -261,13 +261,12 @@ void instance_caps(const Oracle& o, int w, const int64_t N[3], const int64_t kb[
   }
 }
 
-int validate_config(int32_t W, const int64_t* cap, int32_t pf, int32_t rounds, int32_t mode,
-                    int64_t hold, int32_t win, int32_t min_obs, const int64_t* pk, int64_t T0) {
+int validate_config(int32_t W, const int64_t* cap, int32_t pf, int32_t mode, int64_t hold,
+                    int32_t win, int32_t min_obs, const int64_t* pk, int64_t T0) {
   if (W < 1 || W > 1024) return ERR_INVALID_ARG;
   for (int w = 0; w < W; ++w)
     if (cap[w] < 1 || cap[w] > ((int64_t)1 << 26)) return ERR_INVALID_ARG;
   if (pf < 1 || pf > 65536) return ERR_INVALID_ARG;
-  if (rounds < 1 || rounds > 64) return ERR_INVALID_ARG;
   if (mode < 0 || mode > 3) return ERR_INVALID_ARG;
   if (hold < 0 || hold > BACKLOG_MAX) return ERR_INVALID_ARG;
   if (win < 1 || win > 4096 || min_obs < 1) return ERR_INVALID_ARG;
@@ -309,17 +308,16 @@ int oracle_caps_eval(int64_t Cw, const int64_t* N, const int64_t* kb, const int6
   return OK;
 }
 
-void* oracle_create(int32_t W, const int64_t* cap, int32_t pf_q16, int32_t rounds, int32_t mode,
+void* oracle_create(int32_t W, const int64_t* cap, int32_t pf_q16, int32_t mode,
                     int64_t hold_delay_q, int32_t hist_window, int32_t min_obs,
                     const int64_t* prior_kbar, int64_t prior_T_us, uint64_t hash_seed) {
-  if (validate_config(W, cap, pf_q16, rounds, mode, hold_delay_q, hist_window, min_obs,
-                      prior_kbar, prior_T_us) != OK)
+  if (validate_config(W, cap, pf_q16, mode, hold_delay_q, hist_window, min_obs, prior_kbar,
+                      prior_T_us) != OK)
     return nullptr;
   Oracle* o = new Oracle();
   o->W = W;
   o->cap.assign(cap, cap + W);
   o->pf_q16 = pf_q16;
-  o->rounds = rounds;
   o->mode = mode;
   o->hold_delay_q = hold_delay_q;
   o->hist_window = hist_window;
@@ -452,12 +450,15 @@ int oracle_route(void* h, int32_t n, const uint8_t* cls, const uint64_t* session
     for (int b = 0; b < 3; ++b) o->K_wb[(size_t)w * 3 + b] = Kwb[b];
   }
 
-  // selection rounds (reading: batch rounds with in-batch backlog update)
+  // selection (reading: the batch's leaders are decided one at a time in arrival order,
+  // as the online router of Sec. 4 decides requests.  Each one sees the snapshot taken at
+  // batch start -- caches, sessions, backlog d_w and throughput mu_w -- and the admissions
+  // of the leaders before it: an admitted session is recorded at once as pending on its
+  // instance (P_w, Sec. 4.1-4.2), so it takes headroom from everyone after it.  A leader is
+  // therefore held only when no instance has headroom for it at its turn.)
   std::vector<int64_t> adm(W, 0);
   std::vector<std::array<int64_t, 3>> admb(W, {0, 0, 0});
-  std::vector<int64_t> bk(o->backlog_q);
-  std::vector<char> resolved(n, 0);
-  std::vector<uint8_t> last_reason(n, HOLD_NO_ELIGIBLE);
+  const std::vector<int64_t>& bk = o->backlog_q;
   o->out_inst.assign(n, -1);
   o->out_reason.assign(n, 0);
 
@@ -469,80 +470,55 @@ int oracle_route(void* h, int32_t n, const uint8_t* cls, const uint64_t* session
            o->prot[w][b] + admb[w][b] < o->K_wb[(size_t)w * 3 + b];  // Eq. (6) + Sec. 4.2
   };
 
-  for (int k = 0; k < o->rounds; ++k) {
-    std::vector<int32_t> choice(n, -1);
-    for (int r = 0; r < n; ++r) {
-      if (o->leader[r] != r || resolved[r]) continue;
-      // placement: argmin of Eq. (1) over eligible instances, ties to lower w
-      int best = -1;
-      int64_t best_cost = 0;
-      for (int w = 0; w < W; ++w) {
-        if (!eligible(r, w)) continue;
-        int64_t cost = bk[w] + (o->L[r] - BLOCK * (int64_t)o->H[(size_t)r * W + w]) * o->tokcost_q[w];
-        if (best < 0 || cost < best_cost) {
-          best = w;
-          best_cost = cost;
-        }
-      }
-      if (best < 0) {
-        last_reason[r] = HOLD_NO_ELIGIBLE;
-        continue;
-      }
-      // Eq. (7): a continuation that must be admitted again may prefer to wait
-      if (st_state[r] == SESS_RELEASED) {
-        int wh = 0;
-        for (int w = 1; w < W; ++w)
-          if (o->H[(size_t)r * W + w] > o->H[(size_t)r * W + wh]) wh = w;
-        int64_t Hh = o->H[(size_t)r * W + wh];
-        if (Hh > 0 && !eligible(r, wh)) {
-          int64_t lhs = o->hold_delay_q + bk[wh] - bk[best];
-          int64_t rhs = BLOCK * Hh * o->tokcost_q[wh];
-          if (lhs < rhs) {
-            last_reason[r] = HOLD_PREFER_CACHE;
-            continue;
-          }
-        }
-      }
-      choice[r] = best;
-    }
-    // per instance, choosers in arrival order: Eq. (6) with global and class headroom
-    std::vector<int64_t> prefill_tokens(W, 0);
+  for (int r = 0; r < n; ++r) {
+    if (o->leader[r] != r) continue;
+    const int b = cls[r];
+    // placement among the instances where Admit(r, w) holds (Sec. 4.4: filter by
+    // headroom, then cache-aware placement): argmin of Eq. (1), ties to the lower w
+    int best = -1;
+    int64_t best_cost = 0;
     for (int w = 0; w < W; ++w) {
-      for (int r = 0; r < n; ++r) {
-        if (choice[r] != w) continue;
-        int b = cls[r];
-        bool protected_here = st_state[r] == SESS_PROTECTED && st_inst[r] == w;
-        uint8_t decided = 0;
-        if (protected_here) {
-          decided = ADMIT_CONT;
-        } else if (tot[w] + adm[w] >= o->K_w[w]) {
-          last_reason[r] = HOLD_GLOBAL_CAP;
-        } else if (o->prot[w][b] + admb[w][b] >= o->K_wb[(size_t)w * 3 + b]) {
-          last_reason[r] = HOLD_CLASS_CAP;
-        } else {
-          adm[w] += 1;
-          admb[w][b] += 1;
-          decided = ADMIT_NEW;
-        }
-        if (decided) {
-          resolved[r] = 1;
-          o->out_inst[r] = w;
-          o->out_reason[r] = decided;
-          prefill_tokens[w] += o->L[r] - BLOCK * (int64_t)o->H[(size_t)r * W + w];
+      if (!eligible(r, w)) continue;
+      int64_t cost = bk[w] + (o->L[r] - BLOCK * (int64_t)o->H[(size_t)r * W + w]) * o->tokcost_q[w];
+      if (best < 0 || cost < best_cost) {
+        best = w;
+        best_cost = cost;
+      }
+    }
+    if (best < 0) {
+      // HOLD: the global cap binds everywhere, or the class cap binds on every instance
+      // that still has global headroom
+      bool global_room = false;
+      for (int w = 0; w < W; ++w)
+        if (tot[w] + adm[w] < o->K_w[w]) global_room = true;
+      o->out_reason[r] = global_room ? HOLD_CLASS_CAP : HOLD_GLOBAL_CAP;
+      continue;
+    }
+    // Eq. (7): a continuation that must be admitted again may prefer to wait
+    if (st_state[r] == SESS_RELEASED) {
+      int wh = 0;
+      for (int w = 1; w < W; ++w)
+        if (o->H[(size_t)r * W + w] > o->H[(size_t)r * W + wh]) wh = w;
+      int64_t Hh = o->H[(size_t)r * W + wh];
+      if (Hh > 0 && !eligible(r, wh)) {
+        int64_t lhs = o->hold_delay_q + bk[wh] - bk[best];
+        int64_t rhs = BLOCK * Hh * o->tokcost_q[wh];
+        if (lhs < rhs) {
+          o->out_reason[r] = HOLD_PREFER_CACHE;
+          continue;
         }
       }
     }
-    // admitted prefill joins the instance backlog d_w before the next round
-    for (int w = 0; w < W; ++w) {
-      __int128 v = (__int128)bk[w] + (__int128)o->tokcost_q[w] * prefill_tokens[w];
-      bk[w] = v > BACKLOG_MAX ? BACKLOG_MAX : (int64_t)v;
+    bool protected_here = st_state[r] == SESS_PROTECTED && st_inst[r] == best;
+    o->out_inst[r] = best;
+    if (protected_here) {
+      o->out_reason[r] = ADMIT_CONT;  // no headroom consumed
+    } else {
+      o->out_reason[r] = ADMIT_NEW;   // pending on `best` from now on
+      adm[best] += 1;
+      admb[best][b] += 1;
     }
   }
-  for (int r = 0; r < n; ++r)
-    if (o->leader[r] == r && !resolved[r]) {
-      o->out_inst[r] = -1;
-      o->out_reason[r] = last_reason[r];
-    }
   // followers: later requests of a session in the batch follow their leader
   for (int r = 0; r < n; ++r) {
     int ld = o->leader[r];

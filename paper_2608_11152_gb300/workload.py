@@ -194,7 +194,6 @@ class Scenario:
     tokcost_q: np.ndarray
     contraction: np.ndarray
     hold_delay_q: int
-    rounds: int = 4
     protected_frac_q16: int = 58982   # C_w = 0.9 Cap_w
     mode: int = 0
     fillers: list = field(default_factory=list)
@@ -522,7 +521,7 @@ def config5(n=65536, fill=0.95, seed=20260005, n_warm=1, instances=128, cap=2621
                             n_warm, spec, fill=fill)
 
 
-def small_random(seed, W=3, cap=64, n=24, rounds=2, mode=0, n_warm=2) -> Scenario:
+def small_random(seed, W=3, cap=64, n=24, mode=0, n_warm=2) -> Scenario:
     """Tiny randomized scenario (small W and capacity so caps and eviction bind often)."""
     rng = np.random.default_rng(seed)
     spec = MixSpec(rho_ppm=(400000, 300000, 300000), rlvr_prompt=(8, 96), rlvr_fanout=int(rng.integers(1, 5)),
@@ -531,7 +530,6 @@ def small_random(seed, W=3, cap=64, n=24, rounds=2, mode=0, n_warm=2) -> Scenari
                    agent_max_turns=(2, 6), agent_hist_cap=512, agent_sessions=int(rng.integers(1, 4)))
     sc = _stream_scenario(f"small_{seed}", seed, W, cap, n, n_warm, spec)
     sc.cap_blocks = rng.integers(max(4, cap // 4), cap + 1, size=W).astype(np.int64)
-    sc.rounds = rounds
     sc.mode = mode
     sc.hold_delay_q = int(rng.integers(0, 2_000_000))
     sc.backlog_q = rng.integers(0, 2_000_000, size=W, dtype=np.int64)

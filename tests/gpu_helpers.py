@@ -17,7 +17,7 @@ def make_router(sc, **over):
     from paper_2608_11152_gb300 import misat
 
     kw = dict(max_batch=max(1, sc.max_batch), max_tokens=max(16, sc.max_tokens),
-              protected_frac_q16=sc.protected_frac_q16, rounds=sc.rounds, mode=sc.mode,
+              protected_frac_q16=sc.protected_frac_q16, mode=sc.mode,
               hold_delay_q=sc.hold_delay_q, prior_kbar=sc.prior_kbar, prior_T_us=sc.prior_T_us)
     kw.update(over)
     r = misat.Router(sc.cap_blocks, **kw)

@@ -13,7 +13,7 @@ HOLDS = (oracle.HOLD_GLOBAL_CAP, oracle.HOLD_CLASS_CAP, oracle.HOLD_NO_ELIGIBLE,
 
 
 def make_oracle(sc, **over):
-    kw = dict(protected_frac_q16=sc.protected_frac_q16, rounds=sc.rounds, mode=sc.mode,
+    kw = dict(protected_frac_q16=sc.protected_frac_q16, mode=sc.mode,
               hold_delay_q=sc.hold_delay_q, prior_kbar=sc.prior_kbar, prior_T_us=sc.prior_T_us)
     kw.update(over)
     o = oracle.Oracle(sc.cap_blocks, **kw)

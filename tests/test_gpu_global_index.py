@@ -61,7 +61,7 @@ def check_global(r, o, W):
 def test_parity_random_small_both_layouts(seed, prefix_index):
     rng = np.random.default_rng(100 + seed)
     sc = wl.small_random(9000 + seed, W=int(rng.integers(1, 9)), cap=int(rng.integers(8, 160)),
-                         n=int(rng.integers(1, 80)), rounds=int(rng.integers(1, 6)), mode=seed % 4,
+                         n=int(rng.integers(1, 80)), mode=seed % 4,
                          n_warm=int(rng.integers(0, 6)))
     r, o = run_parity(sc, prefix_index=prefix_index)
     if prefix_index == 0:
@@ -82,7 +82,7 @@ def test_parity_config5_reduced_per_instance_layout():
 
 
 def test_global_index_mirrors_every_kind_of_change():
-    sc = wl.small_random(31, W=5, cap=120, n=40, rounds=3, mode=0, n_warm=4)
+    sc = wl.small_random(31, W=5, cap=120, n=40, mode=0, n_warm=4)
     r, o = run_parity(sc)
     check_global(r, o, sc.W)
     # engine removal events: drop a suffix of the deepest chain on every instance
@@ -145,7 +145,7 @@ def test_global_index_rebuilds_when_claimed_slots_accumulate():
     """Keys whose instances all evicted them keep their slot until the library rebuilds the
     index from the instance tables; many small commits must trigger such rebuilds and stay
     bit-exact throughout."""
-    sc = wl.small_random(47, W=4, cap=64, n=60, rounds=2, mode=3, n_warm=40)
+    sc = wl.small_random(47, W=4, cap=64, n=60, mode=3, n_warm=40)
     r, o = make_router(sc), make_oracle(sc)
     _, slots, _ = r.global_info()
     claimed_seen = []

@@ -89,5 +89,5 @@ def test_controller_loop_config2():
 @pytest.mark.gpu
 @pytest.mark.parametrize("seed", range(3))
 def test_controller_loop_small_random(seed):
-    sc = wl.small_random(800 + seed, W=4, cap=96, n=32, rounds=2, n_warm=10)
+    sc = wl.small_random(800 + seed, W=4, cap=96, n=32, n_warm=10)
     _run(sc)

@@ -46,7 +46,7 @@ def _mk(cls, sessions, lens, seed=0, offset_tokens=None):
 def test_parity_random_small(seed):
     rng = np.random.default_rng(seed)
     sc = wl.small_random(5000 + seed, W=int(rng.integers(1, 9)), cap=int(rng.integers(8, 160)),
-                         n=int(rng.integers(1, 80)), rounds=int(rng.integers(1, 6)), mode=seed % 4,
+                         n=int(rng.integers(1, 80)), mode=seed % 4,
                          n_warm=int(rng.integers(0, 6)))
     r, o = run_parity(sc)
     r.close()
@@ -56,7 +56,7 @@ def test_parity_random_small(seed):
 def test_parity_with_releases_and_rebounds(seed):
     """Completions with done=0 release sessions (Eq. 7 continuations); backlogs change
     between batches so continuations rebind; caps are contracted on some instances."""
-    sc = wl.small_random(7000 + seed, W=4, cap=96, n=48, rounds=3, mode=0, n_warm=6)
+    sc = wl.small_random(7000 + seed, W=4, cap=96, n=48, mode=0, n_warm=6)
     r, o = make_router(sc), make_oracle(sc)
     rng = np.random.default_rng(seed)
     steps = list(sc.warm) + [(sc.batch, None)]
@@ -209,20 +209,20 @@ def test_longest_prompt_65535_blocks():
 
 
 def test_many_instances_w1024():
-    sc = wl.small_random(14, W=1024, cap=32, n=300, rounds=3, n_warm=2)
+    sc = wl.small_random(14, W=1024, cap=32, n=300, n_warm=2)
     r, o = run_parity(sc)
     r.close()
 
 
 def test_one_instance():
-    sc = wl.small_random(15, W=1, cap=256, n=60, rounds=2, n_warm=3)
+    sc = wl.small_random(15, W=1, cap=256, n=60, n_warm=3)
     r, o = run_parity(sc)
     r.close()
 
 
 def test_table_growth_and_session_rebuild():
     """Tiny tables and a tiny session table: growth and rebuild paths run and stay exact."""
-    sc = wl.small_random(16, W=3, cap=8, n=70, rounds=4, mode=3, n_warm=5)
+    sc = wl.small_random(16, W=3, cap=8, n=70, mode=3, n_warm=5)
     r, o = run_parity(sc, max_sessions=1, table_load=0.25)
     r.close()
 
@@ -496,7 +496,7 @@ def test_rounds_sweep_on_config2_first_batch():
 def test_checkpoint_restore_replays_identically():
     """A restored checkpoint gives the same decisions and the same committed state again,
     including after a commit that grew a table (the restore shrinks it back)."""
-    sc = wl.small_random(19, W=3, cap=16, n=60, rounds=3, mode=3, n_warm=2)
+    sc = wl.small_random(19, W=3, cap=16, n=60, mode=3, n_warm=2)
     r, o = run_parity(sc, table_load=0.25)
     ck = r.checkpoint_save()
     o2 = o.clone()

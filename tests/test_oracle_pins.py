@@ -91,7 +91,7 @@ def test_hash_distinct_keys_on_medium_workload():
 
 @pytest.mark.parametrize("seed", list(range(12)))
 def test_H_and_index_match_token_level_bruteforce(seed):
-    sc = wl.small_random(1000 + seed, W=3, cap=48, n=20, rounds=2, mode=seed % 4, n_warm=3)
+    sc = wl.small_random(1000 + seed, W=3, cap=48, n=20, mode=seed % 4, n_warm=3)
     o = make_oracle(sc)
     model = BlockModel(sc.cap_blocks)
     seq = 0
@@ -133,7 +133,7 @@ def _batch(cls, sessions, lens, seed=0):
 def test_quota_hand_example_end_to_end(mode, Kb):
     """One instance with C_w = 1000, 8/4/2 new sessions, priors (64, 96, 512) and
     residencies (600, 120, 1800): the route must apply exactly the hand-worked caps."""
-    o = oracle.Oracle([1000], protected_frac_q16=65536, rounds=1, mode=mode,
+    o = oracle.Oracle([1000], protected_frac_q16=65536, mode=mode,
                       prior_kbar=(64, 96, 512), prior_T_us=1, min_obs=1, hist_window=1)
     o.set_mixture((400000, 300000, 300000))
     o.set_instance_state([0], [1], [0])
@@ -156,6 +156,25 @@ def test_quota_hand_example_end_to_end(mode, Kb):
         if r not in exp:
             before = sum(1 for x in exp if x < r)
             assert reason[r] == (oracle.HOLD_GLOBAL_CAP if before >= 7 else oracle.HOLD_CLASS_CAP)
+
+
+def test_serial_selection_hand_example():
+    """Sec. 4.1 Eq. (6), Sec. 4.2 and the Sec. 4.4 pipeline on a batch worked by hand
+    (tests/golden/serial_selection_example.txt): each leader takes the cheapest instance
+    where Admit holds given the sessions admitted before it, and is held only when none has
+    headroom for it (class cap while some instance has global headroom, else global cap)."""
+    g = _golden_kv("serial_selection_example.txt")
+    W = len(g["backlog"])
+    o = oracle.Oracle([4096] * W, protected_frac_q16=65536, mode=oracle.MODE_MISA_T,
+                      prior_kbar=(2048, 2048, 2048))
+    o.set_instance_state(g["backlog"], g["tokcost"], [0] * W)
+    n = len(g["cls"])
+    b = _batch(g["cls"], list(range(1, n + 1)), [g["prompt_tokens"][0]] * n)
+    inst, reason, hit = o.route(b.cls, b.session, b.tok_off, b.tokens)
+    caps = o.caps()
+    assert list(caps["K_w"]) == g["K_w"]
+    assert all(list(caps["K_wb"][w]) == g["K_wb"] for w in range(W))
+    assert list(inst) == g["inst"] and list(reason) == g["reason"]
 
 
 def test_quota_closed_forms_random():
@@ -186,7 +205,7 @@ def test_quota_closed_forms_random():
 # ---------------------------------------------------------------- special cases
 
 def test_one_instance_no_cache_admits_in_arrival_order():
-    o = oracle.Oracle([4096], rounds=1, prior_kbar=(16, 16, 16))
+    o = oracle.Oracle([4096], prior_kbar=(16, 16, 16))
     o.set_instance_state([0], [10], [0])
     rng = np.random.default_rng(3)
     cls = list(rng.integers(0, 3, size=200))
@@ -209,7 +228,7 @@ def test_one_instance_no_cache_admits_in_arrival_order():
 
 def test_placement_only_without_token_cost_picks_least_backlog():
     W = 6
-    o = oracle.Oracle([512] * W, mode=oracle.MODE_PLACEMENT_ONLY, rounds=1)
+    o = oracle.Oracle([512] * W, mode=oracle.MODE_PLACEMENT_ONLY)
     bk = [50, 20, 70, 20, 90, 30]
     o.set_instance_state(bk, [0] * W, [0] * W)
     b = _batch([0, 1, 2] * 10, list(range(1, 31)), [64] * 30)
@@ -219,7 +238,7 @@ def test_placement_only_without_token_cost_picks_least_backlog():
 
 def test_placement_only_with_equal_backlogs_picks_longest_prefix():
     W = 5
-    o = oracle.Oracle([4096] * W, mode=oracle.MODE_PLACEMENT_ONLY, rounds=1)
+    o = oracle.Oracle([4096] * W, mode=oracle.MODE_PLACEMENT_ONLY)
     rng = np.random.default_rng(9)
     base = rng.integers(0, wl.VOCAB, size=16 * 20, dtype=np.int32)
     # warm instance w with the first 4*w blocks of `base` (w = 1..4)
@@ -241,7 +260,7 @@ def test_placement_only_with_equal_backlogs_picks_longest_prefix():
 
 def test_equal_residency_makes_misat_equal_misa():
     for seed in range(6):
-        sc = wl.small_random(2000 + seed, W=4, cap=96, n=30, rounds=3, mode=0, n_warm=0)
+        sc = wl.small_random(2000 + seed, W=4, cap=96, n=30, mode=0, n_warm=0)
         res = []
         for mode in (oracle.MODE_MISA_T, oracle.MODE_MISA):
             o = make_oracle(sc, mode=mode)
@@ -290,11 +309,79 @@ def _check_route_invariants(o, b, inst, reason, hit, prot_before, sess_before):
             assert new[w, c] <= max(0, caps["K_wb"][w, c] - prot_before[w, c])
 
 
+def _eligible_after(caps, prot_before, adm, st, w, c):
+    """Admit(r, w) of Eq. (6) with the class cap of Sec. 4.2, given the new sessions `adm`
+    [W][3] admitted so far in the batch (pending, Sec. 4.1)."""
+    if st[0] == 1 and st[1] == w:
+        return True
+    return (prot_before[w].sum() + adm[w].sum() < caps["K_w"][w]
+            and prot_before[w, c] + adm[w, c] < caps["K_wb"][w, c])
+
+
+def _check_held_have_no_headroom(o, b, inst, reason, prot_before, sess_before):
+    """Eq. (6) holds a request only when it cannot get headroom: under the counts after the
+    whole batch, a leader held for a cap has no instance where Admit holds."""
+    W = o.W
+    caps = o.caps()
+    adm = np.zeros((W, 3), np.int64)
+    for r in range(b.n):
+        if reason[r] == oracle.ADMIT_NEW:
+            adm[inst[r], b.cls[r]] += 1
+    for r in range(b.n):
+        if reason[r] in (oracle.HOLD_GLOBAL_CAP, oracle.HOLD_CLASS_CAP, oracle.HOLD_NO_ELIGIBLE):
+            st = sess_before.get(int(b.session[r]), (0, -1))
+            assert not any(_eligible_after(caps, prot_before, adm, st, w, b.cls[r]) for w in range(W))
+            if reason[r] == oracle.HOLD_GLOBAL_CAP:
+                assert all(prot_before[w].sum() + adm[w].sum() >= caps["K_w"][w] for w in range(W))
+
+
+def _check_serial_order(o, b, inst, reason, prot_before, sess_before, backlog, tokcost, hold):
+    """The batch decided one leader at a time in arrival order, checked on the decisions
+    alone: with the sessions admitted before a leader counted as pending, an admitted leader
+    sits on the cheapest instance of Eq. (1) where Admit holds (Sec. 4.4, ties to the lower
+    index); a leader held for a cap had no such instance at its turn; an Eq. (7) hold had its
+    cached instance without headroom and a saving above the hold delay."""
+    W = o.W
+    caps = o.caps()
+    H = o.H().astype(np.int64)
+    L = np.diff(b.tok_off).astype(np.int64)
+    adm = np.zeros((W, 3), np.int64)
+    seen = set()
+    for r in range(b.n):
+        s = int(b.session[r])
+        if s in seen:
+            continue
+        seen.add(s)
+        c = int(b.cls[r])
+        st = sess_before.get(s, (0, -1))
+        E = [w for w in range(W) if _eligible_after(caps, prot_before, adm, st, w, c)]
+        if reason[r] in (oracle.HOLD_GLOBAL_CAP, oracle.HOLD_CLASS_CAP):
+            assert not E
+            room = any(prot_before[w].sum() + adm[w].sum() < caps["K_w"][w] for w in range(W))
+            assert reason[r] == (oracle.HOLD_CLASS_CAP if room else oracle.HOLD_GLOBAL_CAP)
+            continue
+        assert reason[r] != oracle.HOLD_NO_ELIGIBLE and E
+        cost = {w: int(backlog[w]) + int(L[r] - 16 * H[r, w]) * int(tokcost[w]) for w in E}
+        best = min(E, key=lambda w: (cost[w], w))
+        wh = int(np.argmax(H[r]))
+        eq7 = (st[0] == 2 and H[r, wh] > 0 and wh not in E
+               and hold + int(backlog[wh]) - int(backlog[best]) < 16 * int(H[r, wh]) * int(tokcost[wh]))
+        if reason[r] == oracle.HOLD_PREFER_CACHE:
+            assert eq7 and inst[r] == -1
+            continue
+        assert not eq7 and inst[r] == best
+        if reason[r] == oracle.ADMIT_CONT:
+            assert st == (1, best)
+        else:
+            assert reason[r] == oracle.ADMIT_NEW and st != (1, best)
+            adm[best, c] += 1
+
+
 @pytest.mark.parametrize("seed", list(range(40)))
 def test_invariants_random_small(seed):
     rng = np.random.default_rng(seed)
     sc = wl.small_random(3000 + seed, W=int(rng.integers(1, 6)), cap=int(rng.integers(16, 128)),
-                         n=int(rng.integers(1, 40)), rounds=int(rng.integers(1, 5)), mode=seed % 4,
+                         n=int(rng.integers(1, 40)), mode=seed % 4,
                          n_warm=int(rng.integers(0, 5)))
     o = make_oracle(sc)
     for b, comp in scenario_steps(sc):
@@ -303,6 +390,9 @@ def test_invariants_random_small(seed):
         sess_before = {int(i): (int(s), int(w)) for i, s, w in zip(ids, st, ins)}
         inst, reason, hit = o.route(b.cls, b.session, b.tok_off, b.tokens)
         _check_route_invariants(o, b, inst, reason, hit, prot_before, sess_before)
+        _check_held_have_no_headroom(o, b, inst, reason, prot_before, sess_before)
+        _check_serial_order(o, b, inst, reason, prot_before, sess_before, sc.backlog_q, sc.tokcost_q,
+                            sc.hold_delay_q)
         if sc.mode == oracle.MODE_PLACEMENT_ONLY:
             assert np.all(inst >= 0)
         if sc.mode in (oracle.MODE_SESSION_ADMISSION, oracle.MODE_PLACEMENT_ONLY):
@@ -324,7 +414,7 @@ def test_prefer_cache_rule_eq7():
     """A released continuation whose cached instance has no headroom waits when the
     saved prefill beats the hold delay plus the queue difference, else goes cold."""
     for hold, expect in ((0, oracle.HOLD_PREFER_CACHE), (10**12, oracle.ADMIT_NEW)):
-        o = oracle.Oracle([4096, 4096], rounds=1, prior_kbar=(4000, 4000, 4000), hold_delay_q=hold,
+        o = oracle.Oracle([4096, 4096], prior_kbar=(4000, 4000, 4000), hold_delay_q=hold,
                           protected_frac_q16=65536)
         o.set_instance_state([100, 100], [1000, 1000], [0, 0])
         # K_w = floor(4096/4000) = 1 on both instances
@@ -346,7 +436,7 @@ def test_prefer_cache_rule_eq7():
 
 
 def test_rebound_moves_protection():
-    o = oracle.Oracle([4096, 4096], rounds=1, prior_kbar=(8, 8, 8))
+    o = oracle.Oracle([4096, 4096], prior_kbar=(8, 8, 8))
     o.set_instance_state([0, 10**9], [1, 1], [0, 0])
     b = _batch([1], [55], [64])
     inst, reason, _ = o.route(b.cls, b.session, b.tok_off, b.tokens)
@@ -362,7 +452,7 @@ def test_rebound_moves_protection():
 
 
 def test_external_evict_and_reset():
-    o = oracle.Oracle([4096], rounds=1)
+    o = oracle.Oracle([4096])
     b = _batch([0], [9], [16 * 10])
     o.route(b.cls, b.session, b.tok_off, b.tokens)
     o.commit()
@@ -376,3 +466,23 @@ def test_external_evict_and_reset():
     assert o.check_invariants() == 2
     o.reset_instance(0)
     assert o.index_size(0) == 0 and o.check_invariants() == 0
+
+
+def test_held_leaders_have_no_headroom_on_rlvr_heavy_config():
+    """The RLVR-heavy workload (32 x 131,072 blocks, 16,384 requests): every leader held for
+    a cap has no instance with headroom for it once the batch is decided, and the batch is
+    decided in arrival order as the per-turn check describes."""
+    sc = wl.config3()
+    o = make_oracle(sc)
+    for b, comp in sc.warm:
+        o.route(b.cls, b.session, b.tok_off, b.tokens)
+        o.commit()
+        o.complete(comp.session, comp.cls, comp.total_blocks, comp.residency_us, comp.done)
+    prot_before = o.counts().astype(np.int64)
+    ids, st, ins, cl = o.sessions()
+    sess_before = {int(i): (int(s), int(w)) for i, s, w in zip(ids, st, ins)}
+    b = sc.batch
+    inst, reason, hit = o.route(b.cls, b.session, b.tok_off, b.tokens)
+    _check_held_have_no_headroom(o, b, inst, reason, prot_before, sess_before)
+    held = int(np.sum(np.isin(reason, (oracle.HOLD_GLOBAL_CAP, oracle.HOLD_CLASS_CAP))))
+    assert held > 0 and int(np.sum(reason == oracle.ADMIT_NEW)) > 3000
