@@ -2,7 +2,7 @@
 """Benchmark of the MISA-T batched routing decision on GB300.
 
 One step = one pass of the whole hot path over one batch: misat_route (block hash,
-longest-prefix probe, caps, scoring, admission rounds) + misat_commit (index insert,
+longest-prefix probe, caps, serial placement and admission) + misat_commit (index insert,
 session update, eviction).  Workload: the throughput-stress configuration, 128
 instances x 262,144 KV blocks filled to 95% (33.5M resident block hashes), batches of
 65,536 mixed RLVR/RLHF/agentic requests (40/30/30), synthetic and seeded.
@@ -53,14 +53,13 @@ CLOCK_QUERY = ("timestamp,index,clocks.sm,clocks.max.sm,power.draw,clocks_event_
                "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
 
 
-def kernels_per_step(rounds, global_index):
+def kernels_per_step(global_index):
     """Kernels one route+commit launches.  Route: class parameters, prologue, leaders, hash,
-    caps, probe first, probe search, 4 per selection round (score, tile count, tile scan,
-    admit, whose last tile also ends the round; rounds after one that admitted nobody still
-    launch and exit at once), finalize.
+    caps, probe first, probe search, the three of the selection (records, initial envelopes,
+    serial selection), finalize.
     Commit: insert work list, insert, the global-index pass (global layout only), sessions,
     and the five eviction kernels (estimate, collect, select, delete, shift)."""
-    return 8 + 4 * rounds + 8 + (1 if global_index else 0)
+    return 11 + 8 + (1 if global_index else 0)
 
 
 def max_over_ranks(ms, dist, device):
@@ -80,9 +79,9 @@ def whole_job_rate(units_per_rank, world, steps, max_ms):
     return world * units_per_rank * steps / max(max_ms / 1e3, 1e-12)
 
 
-def PHASE_KERNELS(rounds, global_index):
+def PHASE_KERNELS(global_index):
     """Kernel launches per phase of one route+commit (see kernels_per_step)."""
-    return {"prologue": 2, "hash": 1, "caps": 1, "probe_first": 1, "probe_search": 1, "rounds": 4 * rounds,
+    return {"prologue": 2, "hash": 1, "caps": 1, "probe_first": 1, "probe_search": 1, "select": 3,
             "finalize": 1, "insert": 3 if global_index else 2, "sessions": 1, "evict": 5}
 
 
@@ -184,7 +183,7 @@ def workload_config(args, sc):
     return {"workload": name,
             "instances": int(sc.W), "cap_blocks": int(sc.cap_blocks[0]), "fill": args.fill if args.config == 5 else None,
             "batch_requests": int(sc.batch.n), "batch_tokens": int(sc.batch.n_tokens), "block_tokens": 16,
-            "rounds": int(sc.rounds), "mode": "MISA-T", "prefix_index": args.prefix_index,
+            "selection": "serial in arrival order", "mode": "MISA-T", "prefix_index": args.prefix_index,
             "l2": ("L2 flushed before every timed step (a %d MB write, outside the step's events) after the "
                    "state restore; tokens %.3f GB, tables %.3f GB" % (L2_FLUSH_BYTES >> 20, sc.batch.n_tokens * 4 / 1e9,
                                                                     sc.W * 2 * int(sc.cap_blocks[0]) * 16 / 1e9))}
@@ -594,7 +593,7 @@ def run_gb300(args):
     phase_ms = {p: phase_tot[p] / KP for p in phase_tot}
     # dominant kernel: the phase with the largest time per kernel launch (multi-kernel phases
     # are split evenly over their kernels); the committed ncu launch list gives the exact shares
-    per_launch = {p: phase_ms[p] / PHASE_KERNELS(sc.rounds, pidx == misat.PREFIX_GLOBAL)[p] for p in phase_ms}
+    per_launch = {p: phase_ms[p] / PHASE_KERNELS(pidx == misat.PREFIX_GLOBAL)[p] for p in phase_ms}
     dom = max(per_launch, key=lambda p: per_launch[p])
     def roof(kind):
         ms = phase_ms[kind]
@@ -629,6 +628,12 @@ def run_gb300(args):
         "scaling": "weak", "vs_baseline": None, "dtype": "u64", "data": "synthetic (seeded, shaped after the paper's workloads)",
         "config": workload_config(args, sc),
         "probes_per_s": round(world * st.probes * K / (total_ms / 1e3), 1),
+        "probes_definition": ("index lookups executed by the probe kernels per second: with the global "
+                              "prefix index one lookup of a request's block 0 answers all instances, and "
+                              "each step of a prefix search is one lookup; with per-instance tables every "
+                              "(request, instance) block-0 lookup counts"),
+        "prefix_decisions_per_s": round(world * n * sc.W * K / (total_ms / 1e3), 1),
+        "prefix_decisions_definition": "(request, instance) longest-cached-prefix values H computed per second",
         "e2e": {"value": round(e2e, 1), "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
                 "api": ("misat_stage_host_delta + misat_route_staged + misat_commit (batch in the delta layout, "
                         "rebuilt on the GPU; copy of step k+1 overlaps step k)") if e2e_delta is not None else
@@ -640,25 +645,44 @@ def run_gb300(args):
                 "full_layout_api": "misat_stage_host + misat_route_staged + misat_commit (all tokens copied)",
                 "sequential_value": round(e2e_seq, 1), "host_link_h2d_gbs": link_gbs,
                 "sequential_api": "misat_route_host + misat_commit (copy, route, read-back; CUDA events)"},
-        "gpu_launches": kernels_per_step(sc.rounds, pidx == misat.PREFIX_GLOBAL) * K,
+        "gpu_launches": kernels_per_step(pidx == misat.PREFIX_GLOBAL) * K,
         "roofline": dom_roof,
         "kernels": kernels,
         "prefix_index": args.prefix_index,
         "global_index": gidx,
+        "value_with_rebuild": (round(whole_job_rate(n, world, 1, total_ms / K + gidx["amortized_rebuild_ms_per_step"]), 1)
+                               if gidx else None),
+        "value_with_rebuild_definition": ("requests / (device time of route+commit + the global prefix index's "
+                                          "rebuild time divided by the steps one rebuild's headroom lasts at this "
+                                          "step's rate of new keys)"),
         "phase_ms": {p: round(v, 4) for p, v in phase_ms.items()},
         "clocks": clocks,
         "wall_s_timed_loop": round(wall, 3),
-        "stats": {"admitted": st.n_admitted, "held": st.n_held, "probes": st.probes, "bucket_reads": st.bucket_reads,
+        "stats": {"admitted": st.n_admitted, "held": st.n_held,
+                  "admitted_by_reason": dict(zip(("continuation", "new_session", "follower"),
+                                                 (int(x) for x in list(st.by_reason)[:3]))),
+                  "held_by_reason": dict(zip(("global_cap", "class_cap", "no_eligible", "prefer_cache",
+                                              "leader_held"), (int(x) for x in list(st.by_reason)[3:8]))),
+                  "admitted_by_class": dict(zip(("rlvr", "rlhf", "agentic"), (int(x) for x in st.admitted_by_class))),
+                  "held_by_class": dict(zip(("rlvr", "rlhf", "agentic"), (int(x) for x in st.held_by_class))),
+                  "probes": st.probes, "bucket_reads": st.bucket_reads,
                   "new_keys": st.new_keys, "evicted": st.evicted, "hit_tokens": st.hit_tokens,
                   "query_tokens": st.query_tokens, "dtv_ppm": st.dtv_ppm},
     }
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        o = setup_oracle(sc)
-        t = cpu_step(o, sc.batch)
-        log(f"oracle step: {t:.2f} s")
+        base = setup_oracle(sc)
+        times = []
+        for _ in range(3):
+            o = base.clone()
+            times.append(cpu_step(o, sc.batch))
+            o.close()
+        t = statistics.median(times)
+        log(f"oracle steps: {[round(x, 2) for x in times]} s")
         line["cpu_baseline"] = {"value": round(n / t, 1), "unit": UNIT, "cores": 1, "kind": "oracle",
-                                "sample": f"one full {n}-request batch (route+commit) from the same warmed state, "
-                                          f"single-threaded C++ oracle, {t:.2f} s; host has {os.cpu_count()} cores"}
+                                "sample": (f"median of 3 full {n}-request batches (route+commit), each from a copy "
+                                           f"of the same warmed state, single-threaded C++ oracle: "
+                                           f"{', '.join(f'{x:.2f}' for x in times)} s; host has {os.cpu_count()} cores"),
+                                "steps_s": [round(x, 3) for x in times]}
     else:
         line["cpu_baseline"] = None
     ckpt.free()

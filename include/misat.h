@@ -12,9 +12,12 @@
  *      resident-block index, held as GPU open-addressing hash tables (Sec. 4.4),
  *   3. caps K_w and K_wb (Sec. 4.1, Eqs. 9-13), eligibility (Eq. 6), prefill
  *      cost (Eq. 1) and the hold-vs-cold rule (Eq. 7), argmin placement,
- *   4. arrival-order admission under the global and class caps (Eq. 6, Sec. 4.2),
- *      then a deterministic commit: index insert, session table update and
- *      eviction down to each instance's KV block capacity.
+ *   4. admission in arrival order under the global and class caps (Eq. 6, Sec. 4.2):
+ *      the leaders of a batch (first request of each session) are decided one at a
+ *      time, each against the batch-start snapshot plus the sessions admitted before
+ *      it, which are pending on their instances; then a deterministic commit: index
+ *      insert, session table update and eviction down to each instance's KV block
+ *      capacity.
  *
  * Conventions
  *   - Return value: MISAT_OK (0) or a negative MISAT_ERR_* code.  Calls validate
@@ -67,9 +70,11 @@ extern "C" {
 #define MISAT_ADMIT_CONT 1         /* session already protected on the instance (Eq. 6, case 1) */
 #define MISAT_ADMIT_NEW 2          /* new, released or rebound session admitted with headroom */
 #define MISAT_ADMIT_FOLLOW 3       /* later request of a session whose leader was admitted */
-#define MISAT_HOLD_GLOBAL_CAP 16   /* no global headroom on the chosen instance */
-#define MISAT_HOLD_CLASS_CAP 17    /* no class headroom on the chosen instance */
-#define MISAT_HOLD_NO_ELIGIBLE 18  /* no instance has headroom for this session */
+#define MISAT_HOLD_GLOBAL_CAP 16   /* at its turn no instance had global headroom (K_w reached) */
+#define MISAT_HOLD_CLASS_CAP 17    /* at its turn every instance with global headroom had reached
+                                      the session's class cap K_wb */
+#define MISAT_HOLD_NO_ELIGIBLE 18  /* not produced (the two reasons above cover every hold for
+                                      headroom); the value stays reserved */
 #define MISAT_HOLD_PREFER_CACHE 19 /* Eq. (7): waiting for the cached instance is cheaper */
 #define MISAT_HOLD_LEADER_HELD 20  /* later request of a session whose leader was held */
 
@@ -80,7 +85,6 @@ typedef struct misat_config {
   int32_t n_instances;          /* W, 1..1024 */
   const int64_t* cap_blocks;    /* host [W]: resident-block capacity Cap_w, 1..2^26 */
   int32_t protected_frac_q16;   /* C_w = floor(Cap_w * q / 65536), 1..65536 (0.9 -> 58982) */
-  int32_t rounds;               /* selection rounds per batch, 1..64 (default 4) */
   int32_t mode;                 /* MISAT_MODE_* */
   int32_t max_batch;            /* largest n passed to misat_route, 1..2^20 */
   int64_t max_tokens;           /* largest total prompt tokens of one batch, >= 16 */
@@ -163,9 +167,15 @@ int misat_set_mixture(misat_ctx* ctx, const uint32_t rho_ppm[3]);
 int misat_set_instance_state(misat_ctx* ctx, const int64_t* backlog_q, const int64_t* tokcost_q,
                              const int32_t* cap_contraction);
 
-/* Route one batch against the state at batch start (Sec. 3.1, Sec. 4).  Inputs and
- * outputs are device pointers; outputs are written before the call's work ends on the
- * stream.  A second route without a commit replaces the pending one.  [async]
+/* Route one batch (Sec. 3.1, Sec. 4).  The leaders -- the first request of each session in
+ * the batch -- are decided in arrival order, as the router decides requests online: each
+ * sees the state at batch start (caches, sessions, d_w, mu_w) and the sessions admitted
+ * before it in the batch, pending on their instances.  A leader takes the cheapest instance
+ * of Eq. (1) where Admit (Eq. 6, with the class cap of Sec. 4.2) holds, ties to the lower
+ * index, or is held when none has headroom for it (or by Eq. 7); later requests of its
+ * session follow it.  Inputs and outputs are device pointers; outputs are written before
+ * the call's work ends on the stream.  A second route without a commit replaces the
+ * pending one.  [async]
  * The second time a set of batch and output buffers (and sizes) comes among the last four
  * sets seen, the route's kernels are captured into a CUDA graph (on a private stream) and
  * replayed from then on; the graphs of the four most recently used sets are kept.  While
@@ -340,7 +350,7 @@ int misat_checkpoint_free(misat_checkpoint* ckpt);
 #define MISAT_PHASE_CAPS 2          /* K3a caps */
 #define MISAT_PHASE_PROBE_FIRST 3   /* K2 block-0 probe of every (request, instance) pair */
 #define MISAT_PHASE_PROBE_SEARCH 4  /* K2 binary search of the hit pairs */
-#define MISAT_PHASE_ROUNDS 5        /* K3b score + K4a admission, all rounds */
+#define MISAT_PHASE_SELECT 5        /* K3b placement + K4a admission: the serial selection */
 #define MISAT_PHASE_FINALIZE 6      /* holds, followers, outputs */
 #define MISAT_PHASE_INSERT 7        /* K4b index insert */
 #define MISAT_PHASE_SESSIONS 8      /* session table update */

@@ -18,9 +18,9 @@ ROOT = os.path.dirname(HERE)
 CSRC = os.path.join(HERE, "csrc")
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "libmisat.so")
-SOURCES = ["api.cu", "hash.cu", "probe.cu", "route.cu", "commit.cu", "evict.cu", "gindex.cu", "overload.cu",
-           "stage.cu"]
-HEADERS = ["common.cuh", "gindex.cuh", "kernels.h"]
+SOURCES = ["api.cu", "hash.cu", "probe.cu", "route.cu", "select.cu", "commit.cu", "evict.cu", "gindex.cu",
+           "overload.cu", "stage.cu"]
+HEADERS = ["common.cuh", "envelope.cuh", "gindex.cuh", "kernels.h"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

@@ -17,8 +17,6 @@ using namespace misat;
 
 namespace {
 
-constexpr int kTileReq = kAdmitTile;
-constexpr int kMaxRounds = 64;
 
 // Small device block copied to the host in one transfer after each route / commit.
 // Layout (8-byte words): stats[32] | U[W] | size[W] | sess_used | err | cand[3] | work | n_hits
@@ -72,7 +70,7 @@ struct misat_ctx {
   int device = 0, num_sms = 1;
   cudaStream_t stream = nullptr;
   // configuration
-  int32_t W = 0, pf_q16 = 0, rounds = 1, mode = 0, max_batch = 0, max_sessions = 0, hist_window = 256,
+  int32_t W = 0, pf_q16 = 0, mode = 0, max_batch = 0, max_sessions = 0, hist_window = 256,
           min_obs = 8;
   int64_t max_tokens = 0, hold_delay_q = 0, prior_kbar[3] = {1, 1, 1}, prior_T = 0;
   uint64_t seed = kGold;
@@ -130,7 +128,10 @@ struct misat_ctx {
   int64_t hits_cap = 0;
   unsigned long long* d_bm_key = nullptr;
   int32_t* d_bm_val = nullptr;
-  int32_t* d_tile = nullptr;
+  int4* d_sel_rec = nullptr;     // per-request records of the selection
+  uint8_t* d_onhull = nullptr;   // initial envelopes of the selection [3W]
+  int32_t* d_rank = nullptr;     // slope order of the instances [W]
+  int32_t* d_chain_max = nullptr;  // per-chain insert limits of misat_load_chains
   // one small block of counters, mirrored to pinned host memory
   MetaLayout ml;
   unsigned long long* d_meta = nullptr;
@@ -571,14 +572,13 @@ CapsArgs caps_args(misat_ctx* c) {
   ca.pf_q16 = c->pf_q16;
   ca.mode = c->mode;
   ca.contraction = c->d_contraction;
-  ca.backlog = c->d_backlog;
   ca.ia = c->ia;
   ca.err = c->err_ptr();
   return ca;
 }
 
 // The device work of one route (n > 0), enqueued on stream st: counters reset, prologue,
-// block hash, caps, probes, selection rounds, finalize.  Captured into the route graph, or
+// block hash, caps, probes, serial selection, finalize.  Captured into the route graph, or
 // launched directly while the caller captures the context's stream.
 void enqueue_route(misat_ctx* c, const misat_batch* b, misat_decisions* out, cudaStream_t st) {
   const int32_t n = b->n;
@@ -645,18 +645,39 @@ void enqueue_route(misat_ctx* c, const misat_batch* b, misat_decisions* out, cud
   if (b->out_H)
     cudaMemcpyAsync(b->out_H, c->d_H, (size_t)n * c->W * sizeof(uint16_t), cudaMemcpyDeviceToDevice, st);
 
-  RoundArgs ra{};
-  ra.n = n;
-  ra.W = c->W;
-  ra.rq = c->rq;
-  ra.ia = c->ia;
-  ra.H = c->d_H;
-  ra.tokcost = c->d_tokcost;
-  ra.hold_delay_q = c->hold_delay_q;
-  ra.tile_counts = c->d_tile;
-  ra.n_tiles = (n + kTileReq - 1) / kTileReq;
-  ra.err = c->err_ptr();
-  for (int k = 0; k < c->rounds; ++k) launch_round(ra, c->num_sms, st);
+  SelectPrepArgs sp{};
+  sp.n = n;
+  sp.W = c->W;
+  sp.rq = c->rq;
+  sp.H = c->d_H;
+  sp.rec = c->d_sel_rec;
+  sp.err = c->err_ptr();
+  launch_select_prep(sp, st);
+  EnvInitArgs ei{};
+  ei.W = c->W;
+  ei.backlog = c->d_backlog;
+  ei.tokcost = c->d_tokcost;
+  ei.gh = c->ia.gh;
+  ei.ch = c->ia.ch;
+  ei.onhull = c->d_onhull;
+  ei.rank = c->d_rank;
+  ei.err = c->err_ptr();
+  launch_env_init(ei, st);
+  SelectArgs sa{};
+  sa.n = n;
+  sa.W = c->W;
+  sa.rec = c->d_sel_rec;
+  sa.rq = c->rq;
+  sa.gh = c->ia.gh;
+  sa.ch = c->ia.ch;
+  sa.backlog = c->d_backlog;
+  sa.tokcost = c->d_tokcost;
+  sa.onhull = c->d_onhull;
+  sa.rank = c->d_rank;
+  sa.H = c->d_H;
+  sa.hold_delay_q = c->hold_delay_q;
+  sa.err = c->err_ptr();
+  launch_select(sa, st);
   c->mark(6, st);
 
   FinalizeArgs fa{};
@@ -739,7 +760,6 @@ int misat_create(const misat_config* cfg, void* cuda_stream, misat_ctx** out) {
   for (int w = 0; w < W; ++w)
     if (cfg->cap_blocks[w] < 1 || cfg->cap_blocks[w] > ((int64_t)1 << 26)) return MISAT_ERR_INVALID_ARG;
   if (cfg->protected_frac_q16 < 1 || cfg->protected_frac_q16 > 65536) return MISAT_ERR_INVALID_ARG;
-  if (cfg->rounds < 1 || cfg->rounds > kMaxRounds) return MISAT_ERR_INVALID_ARG;
   if (cfg->mode < 0 || cfg->mode > 3) return MISAT_ERR_INVALID_ARG;
   if (cfg->max_batch < 1 || cfg->max_batch > (1 << 20)) return MISAT_ERR_INVALID_ARG;
   if (cfg->max_tokens < 16 || cfg->max_tokens > ((int64_t)1 << 36)) return MISAT_ERR_INVALID_ARG;
@@ -763,11 +783,11 @@ int misat_create(const misat_config* cfg, void* cuda_stream, misat_ctx** out) {
   if (cudaGetDevice(&c->device) != cudaSuccess) return fail(MISAT_ERR_CUDA);
   if (cudaDeviceGetAttribute(&c->num_sms, cudaDevAttrMultiProcessorCount, c->device) != cudaSuccess)
     return fail(MISAT_ERR_CUDA);
+  if (select_configure() != cudaSuccess) return fail(MISAT_ERR_CUDA);
   c->stream = (cudaStream_t)cuda_stream;
   c->W = W;
   c->cap.assign(cfg->cap_blocks, cfg->cap_blocks + W);
   c->pf_q16 = cfg->protected_frac_q16;
-  c->rounds = cfg->rounds;
   c->mode = cfg->mode;
   c->max_batch = cfg->max_batch;
   c->max_tokens = cfg->max_tokens;
@@ -800,24 +820,23 @@ int misat_create(const misat_config* cfg, void* cuda_stream, misat_ctx** out) {
   c->units_cap = (int64_t)NB + c->keys_cap / 128 + 1;  // one unit per 128 blocks of a request
   c->hits_cap = (int64_t)std::min<size_t>(NB * Ws, (size_t)1 << 27);
   const int bm_log2 = std::max(1, ceil_log2(2 * NB));
-  const size_t n_tiles = (NB + kTileReq - 1) / kTileReq;
   if ((rc = dalloc_n(c, &c->d_meta, c->ml.words)) || (rc = dalloc_n(c, &c->d_keys, (size_t)c->keys_cap)) ||
       (rc = dalloc_n(c, &c->d_units, 2 * (size_t)c->units_cap)) || (rc = dalloc_n(c, &c->d_units_n, 1)) ||
       (rc = dalloc_n(c, &c->d_H, NB * Ws)) || (rc = dalloc_n(c, &c->d_hits, (size_t)c->hits_cap)) ||
       (rc = dalloc_n(c, &c->d_bm_key, (size_t)1 << bm_log2)) ||
-      (rc = dalloc_n(c, &c->d_bm_val, (size_t)1 << bm_log2)) || (rc = dalloc_n(c, &c->d_tile, n_tiles * 3 * Ws)) ||
+      (rc = dalloc_n(c, &c->d_bm_val, (size_t)1 << bm_log2)) || (rc = dalloc_n(c, &c->d_sel_rec, 2 * NB)) ||
+      (rc = dalloc_n(c, &c->d_onhull, 3 * Ws)) || (rc = dalloc_n(c, &c->d_rank, Ws)) ||
       (rc = dalloc_n(c, &c->rq.nb, NB)) || (rc = dalloc_n(c, &c->rq.kbase, NB)) || (rc = dalloc_n(c, &c->rq.L, NB)) ||
       (rc = dalloc_n(c, &c->rq.cls, NB)) || (rc = dalloc_n(c, &c->rq.session, NB)) ||
       (rc = dalloc_n(c, &c->rq.sst, NB)) || (rc = dalloc_n(c, &c->rq.sinst, NB)) ||
       (rc = dalloc_n(c, &c->rq.leader, NB)) || (rc = dalloc_n(c, &c->rq.status, NB)) ||
-      (rc = dalloc_n(c, &c->rq.choice, NB)) || (rc = dalloc_n(c, &c->rq.last_reason, NB)) ||
+      (rc = dalloc_n(c, &c->d_chain_max, NB)) || (rc = dalloc_n(c, &c->rq.last_reason, NB)) ||
       (rc = dalloc_n(c, &c->rq.inst, NB)) || (rc = dalloc_n(c, &c->rq.reason, NB)) ||
       (rc = dalloc_n(c, &c->rq.hbest, NB)) ||
       (rc = dalloc_n(c, &c->ia.K_w, Ws)) || (rc = dalloc_n(c, &c->ia.K_wb, 3 * Ws)) ||
       (rc = dalloc_n(c, &c->ia.N_wb, 3 * Ws)) || (rc = dalloc_n(c, &c->ia.kbar_w, Ws)) ||
       (rc = dalloc_n(c, &c->ia.tot, Ws)) || (rc = dalloc_n(c, &c->ia.gh, Ws)) || (rc = dalloc_n(c, &c->ia.ch, 3 * Ws)) ||
-      (rc = dalloc_n(c, &c->ia.delta, 3 * Ws)) || (rc = dalloc_n(c, &c->ia.backlog_k, Ws)) ||
-      (rc = dalloc_n(c, &c->ia.prefill, Ws)) || (rc = dalloc_n(c, &c->ia.live, 3)) || (rc = dalloc_n(c, &c->d_params, 9)) ||
+      (rc = dalloc_n(c, &c->d_params, 9)) ||
       (rc = dalloc_n(c, &c->d_backlog, Ws)) ||
       (rc = dalloc_n(c, &c->d_tokcost, Ws)) || (rc = dalloc_n(c, &c->d_contraction, Ws)) ||
       (rc = dalloc_n(c, &c->d_prot, 3 * Ws)) || (rc = dalloc_n(c, &c->d_theta, 2 * Ws)) ||
@@ -1366,7 +1385,7 @@ int misat_load_chains(misat_ctx* c, int32_t n_chains, const int64_t* tok_off, co
   CK(cudaMemcpyAsync(c->rq.kbase, kbv.data(), (size_t)n_chains * 8, cudaMemcpyHostToDevice, st));
   CK(cudaMemcpyAsync(c->rq.inst, inst, (size_t)n_chains * 4, cudaMemcpyHostToDevice, st));
   CK(cudaMemcpyAsync(c->rq.session, seq, (size_t)n_chains * 8, cudaMemcpyHostToDevice, st));
-  CK(cudaMemcpyAsync(c->rq.choice, max_blocks, (size_t)n_chains * 4, cudaMemcpyHostToDevice, st));
+  CK(cudaMemcpyAsync(c->d_chain_max, max_blocks, (size_t)n_chains * 4, cudaMemcpyHostToDevice, st));
   CK(cudaMemcpyAsync(c->d_out_hit, arr, (size_t)n_chains * 4, cudaMemcpyHostToDevice, st));
   CK(cudaMemsetAsync(c->work_ptr(), 0, 4, st));
   HashArgs ha{};
@@ -1393,7 +1412,7 @@ int misat_load_chains(misat_ctx* c, int32_t n_chains, const int64_t* tok_off, co
   ia.keys = c->d_keys;
   ia.meta_seq = c->rq.session;
   ia.meta_arr = reinterpret_cast<const uint32_t*>(c->d_out_hit);
-  ia.max_blocks = c->rq.choice;
+  ia.max_blocks = c->d_chain_max;
   ia.size = c->size_ptr();
   ia.new_keys = c->stats_ptr() + 21;
   ia.err = c->err_ptr();

@@ -34,29 +34,23 @@ struct ReqArrays {
   int32_t* sinst;       // protected / last instance
   int32_t* leader;      // first request of the session in the batch
   uint8_t* status;      // kStUnresolved / kStResolved / kStFollower / kStHeld
-  int32_t* choice;      // this round's choice of an unresolved leader needing headroom
-  uint8_t* last_reason; // hold reason if it stays unresolved
+  uint8_t* last_reason; // hold reason of a held leader
   int32_t* inst;        // decision (internal copy)
   uint8_t* reason;      // reason (internal copy)
   uint32_t* hbest;      // max over instances of (H_rw << 16 | 65535 - w): the largest H and,
                         // among instances with it, the lowest index (set by the probe kernels)
 };
 
-// ---- per-instance round state ----
+// ---- per-instance caps of the current route ----
 struct InstArrays {
   int64_t* K_w;         // [W]
   int64_t* K_wb;        // [W*3]
   int64_t* N_wb;        // [W*3]
   int64_t* kbar_w;      // [W]
   int32_t* tot;         // [W] protected sessions at batch start
-  int32_t* gh;          // [W] global headroom at the start of the round
-  int32_t* ch;          // [W*3] class headroom at the start of the round
-  int32_t* delta;       // [W*3] admissions of the current round
-  int64_t* backlog_k;   // [W] in-batch backlog
-  unsigned long long* prefill;  // [W] admitted prefill tokens of the current round
+  int32_t* gh;          // [W] global headroom at batch start, K_w - tot (>= 0)
+  int32_t* ch;          // [W*3] class headroom at batch start, K_wb - prot_wb (>= 0)
   long long* U;         // [W] upper bound of new keys of the pending commit
-  int32_t* live;        // [3]: [0] the current round runs, [1] ADMIT_CONT of the round,
-                        //      [2] admission tiles finished in the round
 };
 
 // ---- K2 ----
@@ -112,7 +106,6 @@ struct CapsArgs {
   int32_t pf_q16;
   int32_t mode;
   const int32_t* contraction;  // [W]
-  const int64_t* backlog;      // [W]
   InstArrays ia;
   const int32_t* err;
 };
@@ -124,21 +117,49 @@ struct RouteParams {
 };
 void launch_route_params(const RouteParams& p, int64_t* dst, cudaStream_t st);
 
-constexpr int kAdmitTile = 128;  // requests per admission tile
+// ---- serial selection (select.cu) ----
+constexpr int kSelectThreads = 256;  // leaders per window of the selection CTA
 
-struct RoundArgs {
+struct SelectPrepArgs {
   int32_t n;
   int32_t W;
   ReqArrays rq;
-  InstArrays ia;
   const uint16_t* H;
-  const int64_t* tokcost;      // [W]
-  int64_t hold_delay_q;
-  int32_t* tile_counts;        // [n_tiles * 3W]
-  int32_t n_tiles;
+  int4* rec;                   // [2n] per-request records of the selection
   const int32_t* err;
 };
-void launch_round(const RoundArgs& a, int num_sms, cudaStream_t st);
+void launch_select_prep(const SelectPrepArgs& a, cudaStream_t st);
+
+struct EnvInitArgs {
+  int32_t W;
+  const int64_t* backlog;      // [W] d_w
+  const int64_t* tokcost;      // [W] 1/mu_w
+  const int32_t* gh;           // [W] global headroom at batch start
+  const int32_t* ch;           // [W*3] class headroom at batch start
+  uint8_t* onhull;             // [3*W] out: line w on the lower envelope of class b's instances
+  int32_t* rank;               // [W] out: position of line w in slope order
+  const int32_t* err;
+};
+void launch_env_init(const EnvInitArgs& a, cudaStream_t st);
+
+struct SelectArgs {
+  int32_t n;
+  int32_t W;
+  const int4* rec;             // [2n] from launch_select_prep
+  ReqArrays rq;                // out: status, inst, reason, last_reason of every leader
+  const int32_t* gh;           // [W] global headroom at batch start
+  const int32_t* ch;           // [W*3] class headroom at batch start
+  const int64_t* backlog;      // [W] d_w
+  const int64_t* tokcost;      // [W] 1/mu_w
+  const uint8_t* onhull;       // [3*W] initial envelopes (launch_env_init)
+  const int32_t* rank;         // [W] slope order (launch_env_init)
+  const uint16_t* H;           // [n*W]
+  int64_t hold_delay_q;
+  int32_t* err;
+};
+size_t select_smem_bytes(int W);
+cudaError_t select_configure();  // per device, before the first launch: shared memory of the selection CTA
+void launch_select(const SelectArgs& a, cudaStream_t st);
 
 struct FinalizeArgs {
   int32_t n;

@@ -37,7 +37,7 @@ _p = C.c_void_p
 
 class misat_config(C.Structure):
     _fields_ = [("n_instances", C.c_int32), ("cap_blocks", _p), ("protected_frac_q16", C.c_int32),
-                ("rounds", C.c_int32), ("mode", C.c_int32), ("max_batch", C.c_int32), ("max_tokens", C.c_int64),
+                ("mode", C.c_int32), ("max_batch", C.c_int32), ("max_tokens", C.c_int64),
                 ("max_sessions", C.c_int32), ("hist_window", C.c_int32), ("min_obs", C.c_int32),
                 ("hold_delay_q", C.c_int64), ("prior_kbar_blocks", C.c_int64 * 3), ("prior_T_us", C.c_int64),
                 ("hash_seed", C.c_uint64), ("table_load", C.c_double), ("prefix_index", C.c_int32)]
@@ -75,7 +75,7 @@ class misat_overload_config(C.Structure):
                 ("queue_thresh", C.c_int64), ("recover_after", C.c_int32), ("max_contraction_pct", C.c_int32)]
 
 
-PHASES = ("prologue", "hash", "caps", "probe_first", "probe_search", "rounds", "finalize", "insert",
+PHASES = ("prologue", "hash", "caps", "probe_first", "probe_search", "select", "finalize", "insert",
           "sessions", "evict")
 
 
@@ -173,7 +173,7 @@ class Router:
     """One MISA-T routing context on the current CUDA device (see include/misat.h)."""
 
     def __init__(self, cap_blocks, *, max_batch, max_tokens, max_sessions=None, protected_frac_q16=58982,
-                 rounds=4, mode=MODE_MISA_T, hold_delay_q=0, hist_window=256, min_obs=8,
+                 mode=MODE_MISA_T, hold_delay_q=0, hist_window=256, min_obs=8,
                  prior_kbar=(64, 64, 64), prior_T_us=30_000_000, hash_seed=0x9E3779B97F4A7C15,
                  table_load=0.75, prefix_index=None, stream=None):
         import torch
@@ -186,7 +186,6 @@ class Router:
         cfg.n_instances = self.W
         cfg.cap_blocks = _nptr(cap)
         cfg.protected_frac_q16 = protected_frac_q16
-        cfg.rounds = rounds
         cfg.mode = mode
         cfg.max_batch = int(max_batch)
         cfg.max_tokens = int(max(16, max_tokens))
