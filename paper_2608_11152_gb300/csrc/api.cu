@@ -11,6 +11,7 @@
 #include <vector>
 
 #include "common.cuh"
+#include "envelope.cuh"
 #include "kernels.h"
 
 using namespace misat;
@@ -131,6 +132,9 @@ struct misat_ctx {
   int4* d_sel_rec = nullptr;     // per-request records of the selection
   uint8_t* d_onhull = nullptr;   // initial envelopes of the selection [3W]
   int32_t* d_rank = nullptr;     // slope order of the instances [W]
+  int32_t* d_rank_a = nullptr;   // (d_w, w) order of the instances [W]
+  // every d_w and every 1/mu_w below 2^25: the selection's envelope arithmetic fits in 64 bits
+  bool bk_small = true, tc_small = true;
   int32_t* d_chain_max = nullptr;  // per-chain insert limits of misat_load_chains
   // one small block of counters, mirrored to pinned host memory
   MetaLayout ml;
@@ -661,6 +665,8 @@ void enqueue_route(misat_ctx* c, const misat_batch* b, misat_decisions* out, cud
   ei.ch = c->ia.ch;
   ei.onhull = c->d_onhull;
   ei.rank = c->d_rank;
+  ei.rank_a = c->d_rank_a;
+  ei.small = c->bk_small && c->tc_small;
   ei.err = c->err_ptr();
   launch_env_init(ei, st);
   SelectArgs sa{};
@@ -674,6 +680,8 @@ void enqueue_route(misat_ctx* c, const misat_batch* b, misat_decisions* out, cud
   sa.tokcost = c->d_tokcost;
   sa.onhull = c->d_onhull;
   sa.rank = c->d_rank;
+  sa.rank_a = c->d_rank_a;
+  sa.small = c->bk_small && c->tc_small;
   sa.H = c->d_H;
   sa.hold_delay_q = c->hold_delay_q;
   sa.err = c->err_ptr();
@@ -826,6 +834,7 @@ int misat_create(const misat_config* cfg, void* cuda_stream, misat_ctx** out) {
       (rc = dalloc_n(c, &c->d_bm_key, (size_t)1 << bm_log2)) ||
       (rc = dalloc_n(c, &c->d_bm_val, (size_t)1 << bm_log2)) || (rc = dalloc_n(c, &c->d_sel_rec, 2 * NB)) ||
       (rc = dalloc_n(c, &c->d_onhull, 3 * Ws)) || (rc = dalloc_n(c, &c->d_rank, Ws)) ||
+      (rc = dalloc_n(c, &c->d_rank_a, Ws)) ||
       (rc = dalloc_n(c, &c->rq.nb, NB)) || (rc = dalloc_n(c, &c->rq.kbase, NB)) || (rc = dalloc_n(c, &c->rq.L, NB)) ||
       (rc = dalloc_n(c, &c->rq.cls, NB)) || (rc = dalloc_n(c, &c->rq.session, NB)) ||
       (rc = dalloc_n(c, &c->rq.sst, NB)) || (rc = dalloc_n(c, &c->rq.sinst, NB)) ||
@@ -904,6 +913,13 @@ int misat_set_instance_state(misat_ctx* c, const int64_t* backlog_q, const int64
     if (tokcost_q && (tokcost_q[w] < 0 || tokcost_q[w] > ((int64_t)1 << 32))) return MISAT_ERR_INVALID_ARG;
     if (cap_contraction && cap_contraction[w] < 0) return MISAT_ERR_INVALID_ARG;
   }
+  auto below = [&](const int64_t* v) {
+    for (int w = 0; w < c->W; ++w)
+      if (v[w] >= kEnvSmall) return false;
+    return true;
+  };
+  if (backlog_q) c->bk_small = below(backlog_q);
+  if (tokcost_q) c->tc_small = below(tokcost_q);
   if (backlog_q) CK(cudaMemcpyAsync(c->d_backlog, backlog_q, c->W * 8, cudaMemcpyHostToDevice, c->stream));
   if (tokcost_q) CK(cudaMemcpyAsync(c->d_tokcost, tokcost_q, c->W * 8, cudaMemcpyHostToDevice, c->stream));
   if (cap_contraction)
@@ -959,7 +975,8 @@ int misat_route(misat_ctx* c, const misat_batch* b, misat_decisions* out) {
                                   (uint64_t)c->sess.log2n,
                                   reinterpret_cast<uint64_t>(c->gix.keys),
                                   reinterpret_cast<uint64_t>(c->gix.masks),
-                                  (uint64_t)c->gix.log2nb};
+                                  (uint64_t)c->gix.log2nb,
+                                  (uint64_t)(c->bk_small && c->tc_small)};
   if (c->timing) {
     // phase events bracket the kernels directly (events recorded inside a graph do not time)
     enqueue_route(c, b, out, st);

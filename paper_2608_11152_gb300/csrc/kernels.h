@@ -118,7 +118,7 @@ struct RouteParams {
 void launch_route_params(const RouteParams& p, int64_t* dst, cudaStream_t st);
 
 // ---- serial selection (select.cu) ----
-constexpr int kSelectThreads = 256;  // leaders per window of the selection CTA
+constexpr int kSelectThreads = 512;  // leaders per window of the selection CTA
 
 struct SelectPrepArgs {
   int32_t n;
@@ -138,6 +138,8 @@ struct EnvInitArgs {
   const int32_t* ch;           // [W*3] class headroom at batch start
   uint8_t* onhull;             // [3*W] out: line w on the lower envelope of class b's instances
   int32_t* rank;               // [W] out: position of line w in slope order
+  int32_t* rank_a;             // [W] out: position of line w in (d_w, w) order
+  bool small;                  // every d_w and 1/mu_w below 2^25: 64-bit envelope arithmetic
   const int32_t* err;
 };
 void launch_env_init(const EnvInitArgs& a, cudaStream_t st);
@@ -153,8 +155,10 @@ struct SelectArgs {
   const int64_t* tokcost;      // [W] 1/mu_w
   const uint8_t* onhull;       // [3*W] initial envelopes (launch_env_init)
   const int32_t* rank;         // [W] slope order (launch_env_init)
+  const int32_t* rank_a;       // [W] (d_w, w) order (launch_env_init)
   const uint16_t* H;           // [n*W]
   int64_t hold_delay_q;
+  bool small;                  // as EnvInitArgs::small
   int32_t* err;
 };
 size_t select_smem_bytes(int W);

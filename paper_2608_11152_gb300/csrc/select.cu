@@ -15,10 +15,9 @@
 //      current start: for a cold prompt (nothing cached) the cheapest instance with
 //      headroom for its class is a query of the lower envelope of the lines
 //      d_w + L / mu_w (envelope.cuh), plus its few cached or protected instances;
-//   2. the warps then take turns in arrival order (a chain of named barriers): each checks
-//      its 32 leaders against the headroom left by the leaders before them and takes their
-//      admissions out of it, up to the first leader whose instance has no headroom left at
-//      its turn;
+//   2. the admissions are counted per (instance, class); where an instance would be
+//      over-subscribed, arrival-order ranks (warp counts, one scan over the warps) find the
+//      first leader whose instance has no headroom left at its turn;
 //   3. the leaders before that one are final (their instance still had headroom, and every
 //      other instance only lost headroom, so the argmin stands); instances that ran out leave
 //      the envelopes of the classes they no longer admit, and the window continues from
@@ -36,7 +35,8 @@ constexpr unsigned kFull = 0xffffffffu;
 constexpr int kNT = kSelectThreads;
 constexpr int kNW = kNT / 32;
 constexpr int kMaxGaps = 32;   // envelope gaps handled incrementally per update
-static_assert(kNW >= 2 && kNW <= 16, "the admission chain uses named barriers 1 .. kNW - 1");
+constexpr int kSlotInst = kNT / (4 * kNW);  // over-subscribed instances given exact ranks per pass
+static_assert(kNW == 16 && kSlotInst == 8, "one thread per (counter, warp) in the rank scan");
 }  // namespace
 
 // ---------------------------------------------------------------------------
@@ -67,16 +67,10 @@ __global__ void __launch_bounds__(256) k3_select_prep(SelectPrepArgs a) {
 }
 
 // ---------------------------------------------------------------------------
-// Initial envelopes and slope order.  blockIdx.y = class b (0..2): is line i on the lower
-// envelope of the instances with headroom for class b?  blockIdx.y = 3: position of line i
-// in slope order.  Eight lanes share line i, each taking every eighth other line.
-__device__ __forceinline__ __int128 shfl_xor_i128(__int128 v, int o) {
-  uint64_t lo = (uint64_t)v, hi = (uint64_t)((unsigned __int128)v >> 64);
-  lo = __shfl_xor_sync(kFull, lo, o);
-  hi = __shfl_xor_sync(kFull, hi, o);
-  return (__int128)(((unsigned __int128)hi << 64) | lo);
-}
-
+// Initial envelopes and orders.  blockIdx.y = class b (0..2): is line i on the lower envelope
+// of the instances with headroom for class b?  blockIdx.y = 3: position of line i in slope
+// order; 4: its position in (d_w, w) order.  Eight lanes share line i, each taking every
+// eighth other line.
 __global__ void __launch_bounds__(1024) k3_env_init(EnvInitArgs a) {
   if (block_error(a.err)) return;
   const int i = blockIdx.x * 128 + (threadIdx.x >> 3);
@@ -84,14 +78,17 @@ __global__ void __launch_bounds__(1024) k3_env_init(EnvInitArgs a) {
   const int b = blockIdx.y;
   const bool line = i < a.W;
   const int64_t bki = line ? a.backlog[i] : 0, tci = line ? a.tokcost[i] : 0;
-  if (b == 3) {
+  if (b >= 3) {  // 3: position in slope order; 4: position in (d_w, w) order
     int cnt = 0;
     if (line)
-      for (int j = sub; j < a.W; j += 8)
-        if (j != i && env_slope_before(a.backlog[j], a.tokcost[j], j, bki, tci, i)) ++cnt;
+      for (int j = sub; j < a.W; j += 8) {
+        const int64_t bkj = a.backlog[j];
+        if (j != i && (b == 3 ? env_slope_before(bkj, a.tokcost[j], j, bki, tci, i) : (bkj < bki || (bkj == bki && j < i))))
+          ++cnt;
+      }
 #pragma unroll
     for (int o = 4; o > 0; o >>= 1) cnt += __shfl_xor_sync(kFull, cnt, o);
-    if (line && sub == 0) a.rank[i] = cnt;
+    if (line && sub == 0) (b == 3 ? a.rank : a.rank_a)[i] = cnt;
     return;
   }
   auto avail = [&](int w) { return a.gh[w] > 0 && a.ch[w * 3 + b] > 0; };
@@ -100,19 +97,19 @@ __global__ void __launch_bounds__(1024) k3_env_init(EnvInitArgs a) {
   env_test_init(t);
   if (ai)
     for (int j = sub; j < a.W; j += 8)
-      if (j != i && avail(j)) env_test_add(t, bki, tci, i, a.backlog[j], a.tokcost[j], j);
+      if (j != i && avail(j)) env_test_add(t, bki, tci, i, a.backlog[j], a.tokcost[j], j, a.small);
 #pragma unroll
   for (int o = 4; o > 0; o >>= 1) {
     EnvTest u;
-    u.lo_num = shfl_xor_i128(t.lo_num, o);
-    u.lo_den = __shfl_xor_sync(kFull, t.lo_den, o);
-    u.hi_num = shfl_xor_i128(t.hi_num, o);
-    u.hi_den = __shfl_xor_sync(kFull, t.hi_den, o);
+    u.lo = EnvFrac{__shfl_xor_sync(kFull, t.lo.dbk, o), __shfl_xor_sync(kFull, t.lo.dw, o),
+                   __shfl_xor_sync(kFull, t.lo.dtc, o)};
+    u.hi = EnvFrac{__shfl_xor_sync(kFull, t.hi.dbk, o), __shfl_xor_sync(kFull, t.hi.dw, o),
+                   __shfl_xor_sync(kFull, t.hi.dtc, o)};
     u.has_hi = __shfl_xor_sync(kFull, t.has_hi, o);
     u.dominated = __shfl_xor_sync(kFull, t.dominated, o);
-    env_test_merge(t, u);
+    env_test_merge(t, u, a.small);
   }
-  if (line && sub == 0) a.onhull[b * a.W + i] = ai && env_test_on(t) ? 1 : 0;
+  if (line && sub == 0) a.onhull[b * a.W + i] = ai && env_test_on(t, a.small) ? 1 : 0;
 }
 
 void launch_select_prep(const SelectPrepArgs& a, cudaStream_t st) {
@@ -121,89 +118,99 @@ void launch_select_prep(const SelectPrepArgs& a, cudaStream_t st) {
 }
 
 void launch_env_init(const EnvInitArgs& a, cudaStream_t st) {
-  dim3 grid((a.W + 127) / 128, 4);
+  dim3 grid((a.W + 127) / 128, 5);
   k3_env_init<<<grid, 1024, 0, st>>>(a);
 }
 
 // ---------------------------------------------------------------------------
 // Shared state of the selection CTA.  Per class, the headroom flags are kept both by instance
-// (queries) and in slope order (envelope updates read them as contiguous bytes).
+// (queries) and in slope order (envelope updates read them as contiguous bytes); the envelope
+// keeps its lines' d_w and 1/mu_w beside their indices, so a query step is one load level.
 struct SelSmem {
   int64_t* bk;     // [W] d_w
   int64_t* tc;     // [W] 1/mu_w
+  int64_t* hbk;    // [3][W] d_w of the envelope lines
+  int64_t* htc;    // [3][W] 1/mu_w of the envelope lines
   int32_t* gh;     // [W] global headroom
   int32_t* ch;     // [3][W] class headroom
+  int32_t* T;      // [W] admissions of the window's current choices
+  int32_t* Tb;     // [3][W]
+  int32_t* slot;   // [W] exact-rank slot of an over-subscribed instance, -1
+  int32_t* wc;     // [4 * kSlotInst counters][kNW warps]
   int32_t* surv;   // [3][W] envelope candidates of each class's update
   int16_t* ord;    // [W] instances in slope order
   int16_t* pos;    // [W] position in slope order
+  int16_t* aord;   // [W] instances in (d_w, w) order
   int16_t* hull;   // [3][W] envelope lines per class, slope order
   uint8_t* av;     // [3][W] headroom for the class (gh > 0 and ch > 0), by instance
   uint8_t* avp;    // [3][W] the same by slope position
   uint8_t* onp;    // [3][W] on the envelope of the class, by slope position
 };
 
-// Per-class scratch of an envelope update (one warp per class).
+// Per-class scratch of an envelope update (one warp per class).  headroom only shrinks, so
+// the first line with headroom in (d_w, w) order (the one that wins at x = 0) and the last in
+// slope order (the least 1/mu_w) are found by pointers that only move forward.
 struct EnvScratch {
   int gp[kMaxGaps];
   int gq[kMaxGaps];
+  int first_a;     // position in (d_w, w) order of the first line that may have headroom
+  int last_s;      // position in slope order of the last line that may have headroom
 };
 
 // Rebuild hull[b] from the on-envelope flags (compaction in slope order).  One warp.
 __device__ void env_compact_warp(const SelSmem& s, int W, int b, int* hm) {
   const int lane = threadIdx.x & 31;
   int base = 0;
-#pragma unroll 4
-  for (int x0 = 0; x0 < W; x0 += 32) {
-    const int x = x0 + lane;
-    const bool f = x < W && s.onp[b * W + x];
-    const unsigned m = __ballot_sync(kFull, f);
-    if (f) s.hull[b * W + base + __popc(m & lanemask_lt())] = s.ord[x];
-    base += __popc(m);
+  for (int x0 = 0; x0 < W; x0 += 128) {
+    bool f[4];
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const int x = x0 + 32 * u + lane;
+      f[u] = x < W && s.onp[b * W + x];
+    }
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const int x = x0 + 32 * u + lane;
+      const unsigned m = __ballot_sync(kFull, f[u]);
+      if (f[u]) {
+        const int k = base + __popc(m & lanemask_lt());
+        const int w = s.ord[x];
+        s.hull[b * W + k] = (int16_t)w;
+        s.hbk[b * W + k] = s.bk[w];
+        s.htc[b * W + k] = s.tc[w];
+      }
+      base += __popc(m);
+    }
   }
   if (lane == 0) *hm = base;
   __syncwarp();
 }
 
-// Dual point i strictly below the segment p-q (slopes p > i > q): below every chord, a line
-// may join the envelope between p and q; above it, it cannot.
-__device__ __forceinline__ bool env_below_chord(const SelSmem& s, int i, int p, int q) {
-  const __int128 lhs = env_adiff(s.bk[i], i, s.bk[p], p) * (__int128)((s.tc[p] - s.tc[q]) * 1024);
-  const __int128 rhs = env_adiff(s.bk[q], q, s.bk[p], p) * (__int128)((s.tc[p] - s.tc[i]) * 1024);
-  return lhs < rhs;
+// The line of class b with headroom that wins at x = 0 (least (d_w, w)), -1 if none.  One warp
+// (warp-uniform result).
+__device__ __forceinline__ int env_first_line(const SelSmem& s, int W, int b, EnvScratch& sc) {
+  int k = sc.first_a;
+  while (k < W && !s.av[b * W + s.aord[k]]) ++k;
+  __syncwarp();
+  if ((threadIdx.x & 31) == 0) sc.first_a = k;
+  __syncwarp();
+  return k < W ? s.aord[k] : -1;
 }
 
-// The line of class b's available ones at slope positions [x0, x1] with the least key:
-// by_slope = 0: (d_w, w) -- the line that wins at x = 0; by_slope = 1: (1/mu_w, d_w, w) -- the
-// line that wins as x grows.  -1 if none.  One warp.
-__device__ int env_end_line_warp(const SelSmem& s, int W, int b, int x0, int x1, int by_slope) {
-  const int lane = threadIdx.x & 31;
-  int64_t k1 = INT64_MAX, k2 = INT64_MAX;
-  int bw = INT32_MAX;
-  auto better = [](int64_t a1, int64_t a2, int aw, int64_t c1, int64_t c2, int cw) {
-    return a1 < c1 || (a1 == c1 && (a2 < c2 || (a2 == c2 && aw < cw)));
-  };
-  for (int x = x0 + lane; x <= x1; x += 32) {
-    if (!s.avp[b * W + x]) continue;
-    const int i = s.ord[x];
-    const int64_t c1 = by_slope ? s.tc[i] : s.bk[i];
-    const int64_t c2 = by_slope ? s.bk[i] : 0;
-    if (better(c1, c2, i, k1, k2, bw)) {
-      k1 = c1;
-      k2 = c2;
-      bw = i;
-    }
-  }
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) {
-    const int64_t o1 = __shfl_xor_sync(kFull, k1, o), o2 = __shfl_xor_sync(kFull, k2, o);
-    const int ow = __shfl_xor_sync(kFull, bw, o);
-    if (better(o1, o2, ow, k1, k2, bw)) {
-      k1 = o1;
-      k2 = o2;
-      bw = ow;
-    }
-  }
-  return bw == INT32_MAX ? -1 : bw;
+// The line of class b with headroom that wins for large x: least 1/mu_w, then least d_w (the
+// first of the last run of equal slopes in slope order), -1 if none.  One warp.
+__device__ __forceinline__ int env_last_line(const SelSmem& s, int W, int b, EnvScratch& sc) {
+  int x = sc.last_s;
+  while (x >= 0 && !s.avp[b * W + x]) --x;
+  __syncwarp();
+  if ((threadIdx.x & 31) == 0) sc.last_s = x;
+  __syncwarp();
+  if (x < 0) return -1;
+  const int64_t t = s.tc[s.ord[x]];
+  int y = x;
+  for (int z = x - 1; z >= 0 && s.tc[s.ord[z]] == t; --z)
+    if (s.avp[b * W + z]) y = z;
+  return s.ord[y];
 }
 
 // Remove the lines of class b that lost their headroom from its envelope.  One warp.
@@ -213,7 +220,7 @@ __device__ int env_end_line_warp(const SelSmem& s, int W, int b, int x0, int x1,
 // for large x (least 1/mu_w).  Between p and q the envelope is that of p, q and the lines of
 // slope strictly between them that lie below the chord p-q: a line above it cannot be on the
 // envelope there, and does not change the envelope of the ones below it.
-__device__ void env_update_warp(const SelSmem& s, int W, int b, int* hm, EnvScratch& sc) {
+__device__ void env_update_warp(const SelSmem& s, int W, int b, int* hm, EnvScratch& sc, bool small) {
   const int lane = threadIdx.x & 31;
   const int m = *hm;
   const int16_t* hull = s.hull + b * W;
@@ -249,8 +256,8 @@ __device__ void env_update_warp(const SelSmem& s, int W, int b, int* hm, EnvScra
         EnvTest t;
         env_test_init(t);
         for (int j = 0; j < W; ++j)
-          if (j != i && s.av[b * W + j]) env_test_add(t, s.bk[i], s.tc[i], i, s.bk[j], s.tc[j], j);
-        on = env_test_on(t);
+          if (j != i && s.av[b * W + j]) env_test_add(t, s.bk[i], s.tc[i], i, s.bk[j], s.tc[j], j, small);
+        on = env_test_on(t, small);
       }
       s.onp[b * W + x] = on;
     }
@@ -261,42 +268,53 @@ __device__ void env_update_warp(const SelSmem& s, int W, int b, int* hm, EnvScra
     for (int g = 0; g < ng; ++g) {
       int p = sc.gp[g], q = sc.gq[g];
       if (p < 0) {  // the envelope's start was removed: the line that now wins at x = 0
-        p = env_end_line_warp(s, W, b, 0, q >= 0 ? s.pos[q] : W - 1, 0);
+        p = env_first_line(s, W, b, sc);
         if (p >= 0 && lane == 0) s.onp[b * W + s.pos[p]] = 1;
       }
       if (p >= 0 && q < 0) {  // the end was removed: the line that now wins for large x
-        q = env_end_line_warp(s, W, b, s.pos[p], W - 1, 1);
+        q = env_last_line(s, W, b, sc);
         if (lane == 0) s.onp[b * W + s.pos[q]] = 1;
       }
       if (p < 0 || q < 0 || p == q) continue;
       const int g0 = ns;
       const int xp = s.pos[p], xq = s.pos[q];
-      const int64_t tcp = s.tc[p];
-      for (int x0 = xp + 1; x0 < xq; x0 += 32) {
-        const int x = x0 + lane;
-        bool c = false;
-        int i = 0;
-        if (x < xq && s.avp[b * W + x]) {
-          i = s.ord[x];
-          c = s.tc[i] != tcp && env_below_chord(s, i, p, q);
+      const int64_t bkp = s.bk[p], tcp = s.tc[p], bkq = s.bk[q], tcq = s.tc[q];
+      for (int x0 = xp + 1; x0 < xq; x0 += 128) {
+        bool c[4];
+        int iv[4];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+          const int x = x0 + 32 * u + lane;
+          c[u] = false;
+          iv[u] = 0;
+          if (x < xq && s.avp[b * W + x]) {
+            const int i = s.ord[x];
+            const int64_t tci = s.tc[i];
+            iv[u] = i;
+            c[u] = tci != tcp && env_below_chord(s.bk[i], tci, i, bkp, tcp, p, bkq, tcq, q, small);
+          }
         }
-        const unsigned mc = __ballot_sync(kFull, c);
-        if (c) surv[ns + __popc(mc & lanemask_lt())] = i;
-        ns += __popc(mc);
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+          const unsigned mc = __ballot_sync(kFull, c[u]);
+          if (c[u]) surv[ns + __popc(mc & lanemask_lt())] = iv[u];
+          ns += __popc(mc);
+        }
       }
       __syncwarp();
       // each candidate against p, q and the other candidates of this gap
       for (int e = g0 + lane; e < ns; e += 32) {
         const int i = surv[e];
+        const int64_t bki = s.bk[i], tci = s.tc[i];
         EnvTest t;
         env_test_init(t);
-        env_test_add(t, s.bk[i], s.tc[i], i, s.bk[p], s.tc[p], p);
-        env_test_add(t, s.bk[i], s.tc[i], i, s.bk[q], s.tc[q], q);
+        env_test_add(t, bki, tci, i, bkp, tcp, p, small);
+        env_test_add(t, bki, tci, i, bkq, tcq, q, small);
         for (int f = g0; f < ns; ++f) {
           const int j = surv[f];
-          if (j != i) env_test_add(t, s.bk[i], s.tc[i], i, s.bk[j], s.tc[j], j);
+          if (j != i) env_test_add(t, bki, tci, i, s.bk[j], s.tc[j], j, small);
         }
-        if (env_test_on(t)) s.onp[b * W + s.pos[i]] = 1;
+        if (env_test_on(t, small)) s.onp[b * W + s.pos[i]] = 1;
       }
       __syncwarp();
     }
@@ -314,17 +332,20 @@ __device__ __forceinline__ int sel_choose(const SelSmem& s, const int* s_hm, int
   int best_w = INT32_MAX;
   const int m = s_hm[b];
   const int16_t* hull = s.hull + b * W;
+  const int64_t* hbk = s.hbk + b * W;
+  const int64_t* htc = s.htc + b * W;
   const int64_t x = L;
   if (m > 0) {
     int lo = 0, hi = m - 1;
     while (lo < hi) {
       const int mid = (lo + hi) >> 1;
-      const int u = hull[mid], v = hull[mid + 1];
-      if (env_beats(s.bk[v], s.tc[v], v, s.bk[u], s.tc[u], u, x)) lo = mid + 1;
+      const int64_t cu = hbk[mid] + x * htc[mid], cv = hbk[mid + 1] + x * htc[mid + 1];
+      // line mid + 1 beats line mid at x (ties to the lower index)
+      if (cv < cu || (cv == cu && hull[mid + 1] < hull[mid])) lo = mid + 1;
       else hi = mid;
     }
     best_w = hull[lo];
-    best_c = s.bk[best_w] + x * s.tc[best_w];
+    best_c = hbk[lo] + x * htc[lo];
   }
   auto consider = [&](int w, int64_t h) {
     const int64_t c = s.bk[w] + (x - 16 * h) * s.tc[w];
@@ -378,43 +399,23 @@ __device__ __forceinline__ int first_set_from(unsigned word, int lane, int from)
   return w * 32 + __ffs(__shfl_sync(kFull, m, w)) - 1;
 }
 
-// Named barrier k of the admission chain: warp k - 1 arrives, warp k waits (64 threads).
-__device__ __forceinline__ void chain_wait(int k) { asm volatile("bar.sync %0, 64;" ::"r"(k) : "memory"); }
-__device__ __forceinline__ void chain_pass(int k) { asm volatile("bar.arrive %0, 64;" ::"r"(k) : "memory"); }
-
-// An instance's headroom drops: clear its flags for the classes it no longer admits.
-__device__ __forceinline__ void sel_take(const SelSmem& s, int W, int w, int b, int kg, int kc, int* s_nglobal,
-                                         int* s_dirty) {
-  if (kg) {
-    const int g = s.gh[w] - kg;
-    s.gh[w] = g;
-    if (g <= 0) {
-      atomicSub(s_nglobal, 1);
+// An instance's headroom dropped to `g` (global) or its class b headroom to `c`: clear its
+// flags for the classes it no longer admits.
+__device__ __forceinline__ void sel_flags(const SelSmem& s, int W, int w, int b, bool gone_g, bool gone_c,
+                                          int* s_dirty) {
+  const int x = s.pos[w];
 #pragma unroll
-      for (int c = 0; c < 3; ++c)
-        if (s.av[c * W + w]) {
-          s.av[c * W + w] = 0;
-          const int x = s.pos[w];
-          s.avp[c * W + x] = 0;
-          if (s.onp[c * W + x]) s_dirty[c] = 1;
-        }
+  for (int c = 0; c < 3; ++c)
+    if ((gone_g || (gone_c && c == b)) && s.av[c * W + w]) {
+      s.av[c * W + w] = 0;
+      s.avp[c * W + x] = 0;
+      if (s.onp[c * W + x]) s_dirty[c] = 1;
     }
-  }
-  if (kc) {
-    const int c = s.ch[b * W + w] - kc;
-    s.ch[b * W + w] = c;
-    if (c <= 0 && s.av[b * W + w]) {
-      s.av[b * W + w] = 0;
-      const int x = s.pos[w];
-      s.avp[b * W + x] = 0;
-      if (s.onp[b * W + x]) s_dirty[b] = 1;
-    }
-  }
 }
 
 __global__ void __launch_bounds__(kNT, 1) k4_select(SelectArgs a) {
   extern __shared__ __align__(16) unsigned char smem[];
-  __shared__ int s_hm[3], s_q, s_nglobal, s_dirty[3];
+  __shared__ int s_hm[3], s_q, s_nslot, s_nglobal, s_f, s_dirty[3];
   __shared__ unsigned s_lead[kNW], s_sens[kNW];
   __shared__ EnvScratch s_env[3];
   if (block_error(a.err)) return;
@@ -427,15 +428,29 @@ __global__ void __launch_bounds__(kNT, 1) k4_select(SelectArgs a) {
     p += (size_t)W * 8;
     s.tc = reinterpret_cast<int64_t*>(p);
     p += (size_t)W * 8;
+    s.hbk = reinterpret_cast<int64_t*>(p);
+    p += (size_t)W * 24;
+    s.htc = reinterpret_cast<int64_t*>(p);
+    p += (size_t)W * 24;
     s.gh = reinterpret_cast<int32_t*>(p);
     p += (size_t)W * 4;
     s.ch = reinterpret_cast<int32_t*>(p);
     p += (size_t)W * 12;
+    s.T = reinterpret_cast<int32_t*>(p);
+    p += (size_t)W * 4;
+    s.Tb = reinterpret_cast<int32_t*>(p);
+    p += (size_t)W * 12;
+    s.slot = reinterpret_cast<int32_t*>(p);
+    p += (size_t)W * 4;
+    s.wc = reinterpret_cast<int32_t*>(p);
+    p += (size_t)kNT * 4;
     s.surv = reinterpret_cast<int32_t*>(p);
     p += (size_t)W * 12;
     s.ord = reinterpret_cast<int16_t*>(p);
     p += (size_t)W * 2;
     s.pos = reinterpret_cast<int16_t*>(p);
+    p += (size_t)W * 2;
+    s.aord = reinterpret_cast<int16_t*>(p);
     p += (size_t)W * 2;
     s.hull = reinterpret_cast<int16_t*>(p);
     p += (size_t)W * 6;
@@ -448,6 +463,8 @@ __global__ void __launch_bounds__(kNT, 1) k4_select(SelectArgs a) {
   if (tid == 0) {
     s_nglobal = 0;
     s_q = kNT;
+    s_nslot = 0;
+    s_f = -1;
     s_dirty[0] = s_dirty[1] = s_dirty[2] = 0;
   }
   __syncthreads();
@@ -455,20 +472,29 @@ __global__ void __launch_bounds__(kNT, 1) k4_select(SelectArgs a) {
     const int r = a.rank[w];
     s.ord[r] = (int16_t)w;
     s.pos[w] = (int16_t)r;
+    s.aord[a.rank_a[w]] = (int16_t)w;
     s.bk[w] = a.backlog[w];
     s.tc[w] = a.tokcost[w];
     const int32_t g = a.gh[w];
     s.gh[w] = g;
     if (g > 0) atomicAdd(&s_nglobal, 1);
+    s.T[w] = 0;
+    s.slot[w] = -1;
 #pragma unroll
     for (int b = 0; b < 3; ++b) {
       const int32_t c = a.ch[w * 3 + b];
       const uint8_t v = g > 0 && c > 0;
       s.ch[b * W + w] = c;
+      s.Tb[b * W + w] = 0;
       s.av[b * W + w] = v;
       s.avp[b * W + r] = v;
       s.onp[b * W + r] = a.onhull[b * W + w];
     }
+  }
+  s.wc[tid] = 0;
+  if (tid < 3) {
+    s_env[tid].first_a = 0;
+    s_env[tid].last_s = W - 1;
   }
   __syncthreads();
   if (wid < 3) env_compact_warp(s, W, wid, &s_hm[wid]);
@@ -529,46 +555,104 @@ __global__ void __launch_bounds__(kNT, 1) k4_select(SelectArgs a) {
       // the first undecided Eq. (7) leader: the leaders before it are decided now, and an
       // Eq. (7) leader at the head is decided alone
       const int qcut = max(first_set_from(sens_word, lane, head), head + 1);
+      const int ng0 = s_nglobal;
       const bool act = lead && tid >= head && tid < qcut;
+      // 1. choices against the state at the window's current start
       if (act && !have) {
-        dw = sel_choose(s, s_hm, W, s_nglobal, L, b, sst, pw, hb, nh, h0, h1, a.H + (int64_t)i * W, a.hold_delay_q,
-                        &dec);
+        dw = sel_choose(s, s_hm, W, ng0, L, b, sst, pw, hb, nh, h0, h1, a.H + (int64_t)i * W, a.hold_delay_q, &dec);
         have = true;
       }
       const bool cons = act && dec == MISAT_ADMIT_NEW;
+      // 2. admissions per (instance, class)
       const unsigned pm = __match_any_sync(kFull, cons ? dw : -1 - lane);
       const unsigned pc = __match_any_sync(kFull, cons ? dw * 3 + b : -1 - lane);
-      // 2. the admission chain: warps in arrival order
-      bool fin = false;  // this lane's decision is final in this iteration
-      if (wid > 0) chain_wait(wid);
-      if (s_q == kNT) {
-        const int ng_before = s_nglobal;
-        const unsigned lt = lanemask_lt();
-        const bool ok = !cons || ((int)__popc(pm & lt) < s.gh[dw] && (int)__popc(pc & lt) < s.ch[b * W + dw]);
-        const unsigned bad = __ballot_sync(kFull, !ok);
-        const int f = bad ? __ffs(bad) - 1 : 32;  // first lane without headroom at its turn
-        const unsigned below = f == 32 ? kFull : ((1u << f) - 1);
-        const bool cc = cons && lane < f;
-        const unsigned pmc = pm & below, pcc = pc & below;
-        const bool gl = cc && lane == __ffs(pmc) - 1, cl = cc && lane == __ffs(pcc) - 1;
-        if (gl || cl) sel_take(s, W, dw, b, gl ? __popc(pmc) : 0, cl ? __popc(pcc) : 0, &s_nglobal, s_dirty);
-        __syncwarp();
-        fin = act && lane < f;
-        const unsigned adm = __ballot_sync(kFull, cc);
-        if (fin && (dec == MISAT_HOLD_CLASS_CAP || dec == MISAT_HOLD_GLOBAL_CAP)) {
-          // at its turn, is there global headroom left?  None before this warp, or the last
-          // one filled by an earlier admission of this warp
-          const bool gone = ng_before == 0 ||
-                            (s_nglobal == 0 && adm != 0 && lane > 31 - (int)__clz(adm));
-          dec = gone ? MISAT_HOLD_GLOBAL_CAP : MISAT_HOLD_CLASS_CAP;
-        }
-        if (f < 32 && lane == 0) s_q = wid * 32 + f;
-      }
-      if (wid < kNW - 1) chain_pass(wid + 1);
+      const bool gl = cons && lane == __ffs(pm) - 1;  // first lane of its instance in the warp
+      const bool cl = cons && lane == __ffs(pc) - 1;
+      if (gl) atomicAdd(&s.T[dw], __popc(pm));
+      if (cl) atomicAdd(&s.Tb[b * W + dw], __popc(pc));
       __syncthreads();
-      const int q = min(s_q, qcut);
-      // 3. final decisions; a tentative admission whose instance lost headroom chooses again
-      if (fin && tid < q) {
+      bool any;
+      {
+        const bool over = gl && s.T[dw] > s.gh[dw];
+        const bool overc = cl && s.Tb[b * W + dw] > s.ch[b * W + dw];
+        if ((over || overc) && atomicCAS(&s.slot[dw], -1, -2) == -1) s.slot[dw] = atomicAdd(&s_nslot, 1);
+        any = __syncthreads_or(over || overc);
+      }
+      int qv = kNT;
+      if (any) {
+        // exact arrival-order ranks at the over-subscribed instances, kSlotInst at a time: a
+        // consumer is invalid when the consumers before it fill its instance or its class
+        const int nslot = s_nslot;
+        for (int p0 = 0; p0 < nslot; p0 += kSlotInst) {
+          const int sl = cons ? s.slot[dw] - p0 : -1;
+          const bool mine = sl >= 0 && sl < kSlotInst;
+          if (mine && gl) s.wc[(sl * 4) * kNW + wid] = __popc(pm);
+          if (mine && cl) s.wc[(sl * 4 + 1 + b) * kNW + wid] = __popc(pc);
+          __syncthreads();
+          {  // exclusive scan over the warps of each counter: thread = (counter, warp)
+            const int v = s.wc[tid];
+            int incl = v;
+#pragma unroll
+            for (int o = 1; o < kNW; o <<= 1) {
+              const int t = __shfl_up_sync(kFull, incl, o, kNW);
+              if ((lane & (kNW - 1)) >= o) incl += t;
+            }
+            s.wc[tid] = incl - v;
+          }
+          __syncthreads();
+          bool bad = false;
+          if (mine) {
+            const unsigned lt = lanemask_lt();
+            const int ag = __popc(pm & lt) + s.wc[(sl * 4) * kNW + wid];
+            const int ac = __popc(pc & lt) + s.wc[(sl * 4 + 1 + b) * kNW + wid];
+            bad = ag >= s.gh[dw] || ac >= s.ch[b * W + dw];
+          }
+          const unsigned mb = __ballot_sync(kFull, bad);
+          if (lane == 0 && mb) atomicMin(&s_q, wid * 32 + __ffs(mb) - 1);
+          __syncthreads();
+          s.wc[tid] = 0;
+          __syncthreads();
+        }
+        qv = s_q;
+      }
+      const int q = min(qv, qcut);
+      // 3. the leaders before q are final: take their admissions out of the headroom (per
+      //    warp, atomically; the one that empties an instance or class clears its flags)
+      {
+        const bool cc = cons && tid < q;
+        const int qw = q - wid * 32;  // lanes of this warp before q
+        const unsigned below = qw >= 32 ? kFull : (qw <= 0 ? 0u : ((1u << qw) - 1));
+        const unsigned qm = pm & below, qc = pc & below;
+        if (cc && lane == __ffs(qm) - 1) {
+          const int k = __popc(qm);
+          const int g = atomicSub(&s.gh[dw], k);
+          if (g > 0 && g - k <= 0) {
+            atomicSub(&s_nglobal, 1);
+            sel_flags(s, W, dw, b, true, false, s_dirty);
+          }
+        }
+        if (cc && lane == __ffs(qc) - 1) {
+          const int k = __popc(qc);
+          const int c = atomicSub(&s.ch[b * W + dw], k);
+          if (c > 0 && c - k <= 0) sel_flags(s, W, dw, b, false, true, s_dirty);
+        }
+      }
+      __syncthreads();
+      if (gl) {
+        s.T[dw] = 0;
+        s.slot[dw] = -1;
+      }
+      if (cl) s.Tb[b * W + dw] = 0;
+      // the last instance with global headroom filled in this prefix: the holds after the
+      // admission that filled it found no global headroom at their turn
+      const bool exhausted = ng0 > 0 && s_nglobal == 0;
+      if (exhausted) {  // uniform
+        const unsigned mf = __ballot_sync(kFull, cons && tid < q);
+        if (lane == 0 && mf) atomicMax(&s_f, wid * 32 + 31 - __clz(mf));
+        __syncthreads();
+      }
+      if (act && tid < q) {
+        if (dec == MISAT_HOLD_CLASS_CAP && (ng0 == 0 || (exhausted && tid > s_f))) dec = MISAT_HOLD_GLOBAL_CAP;
         if (dec == MISAT_ADMIT_NEW || dec == MISAT_ADMIT_CONT) {
           a.rq.status[i] = kStResolved;
           a.rq.inst[i] = dw;
@@ -578,24 +662,27 @@ __global__ void __launch_bounds__(kNT, 1) k4_select(SelectArgs a) {
           a.rq.last_reason[i] = dec;
         }
       } else if (have && dec == MISAT_ADMIT_NEW && !s.av[b * W + dw]) {
-        have = false;
+        have = false;  // its instance has no headroom for the class any more: choose again
       }
       done = q;
       // envelopes of the classes that lost an envelope line: one warp per class
-      if (wid < 3 && s_dirty[wid]) env_update_warp(s, W, wid, &s_hm[wid], s_env[wid]);
+      if (wid < 3 && s_dirty[wid]) env_update_warp(s, W, wid, &s_hm[wid], s_env[wid], a.small);
       __syncthreads();
+      // nobody reads these again before the next iteration's first barrier
       if (tid == 0) {
         s_q = kNT;
+        s_nslot = 0;
+        s_f = -1;
         s_dirty[0] = s_dirty[1] = s_dirty[2] = 0;
       }
-      __syncwarp();  // warp 0 reads them next; the other warps after warp 0 passes the chain
     }
     __syncthreads();  // the window's bitmasks are read until here
   }
 }
 
 size_t select_smem_bytes(int W) {
-  return (size_t)W * 8 * 2 + (size_t)W * 4 * 4 + (size_t)W * 12 + (size_t)W * 2 * 5 + (size_t)W * 9 + 16;
+  return (size_t)W * 8 * 2 + (size_t)W * 48 + (size_t)W * 4 * 4 + (size_t)W * 4 * 4 + (size_t)W * 4 +
+         (size_t)kNT * 4 + (size_t)W * 12 + (size_t)W * 2 * 6 + (size_t)W * 9 + 16;
 }
 
 cudaError_t select_configure() {
