@@ -79,12 +79,6 @@ def whole_job_rate(units_per_rank, world, steps, max_ms):
     return world * units_per_rank * steps / max(max_ms / 1e3, 1e-12)
 
 
-def PHASE_KERNELS(global_index):
-    """Kernel launches per phase of one route+commit (see kernels_per_step)."""
-    return {"prologue": 2, "hash": 1, "caps": 1, "probe_first": 1, "probe_search": 1, "select": 3,
-            "finalize": 1, "insert": 3 if global_index else 2, "sessions": 1, "evict": 5}
-
-
 def parse_args():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -93,7 +87,7 @@ def parse_args():
     ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
     ap.add_argument("--n", type=int, default=65536, help="requests per batch")
     ap.add_argument("--fill", type=float, default=0.95, help="resident fraction of the KV block capacity")
-    ap.add_argument("--e2e-steps", type=int, default=10)
+    ap.add_argument("--e2e-steps", type=int, default=6, help="distinct batches in the end-to-end stream")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--instances", type=int, default=128, help="fewer only for small profiling captures")
     ap.add_argument("--cap", type=int, default=262144, help="blocks per instance; smaller only for profiling captures")
@@ -105,6 +99,8 @@ def parse_args():
 
 
 L2_FLUSH_BYTES = 256 << 20  # twice the 129 MB L2
+ROUTE_PHASES = ("prologue", "hash", "caps", "probe_first", "probe_search", "select", "finalize")
+COMMIT_PHASES = ("insert", "gix_insert", "sessions", "evict")
 
 HASH_SOURCES = ("paper_2608_11152_gb300/csrc/hash.cu", "paper_2608_11152_gb300/csrc/common.cuh")
 HASH_PROFILE = os.path.join(ROOT, "profiles", "k1_block_hash_stress_n65536.md")
@@ -275,7 +271,9 @@ def setup_router(sc, torch, prefix_index):
     r.set_instance_state(sc.backlog_q, sc.tokcost_q, sc.contraction)
     for f in sc.fillers:
         r.load_entries(f.w, f.keys, f.metas)
-    log("gpu: filler entries loaded")
+    for c in sc.chains:
+        r.load_chains(c.tok_off, c.tokens, c.inst, c.seq, c.arr, c.max_blocks)
+    log("gpu: resident fill loaded")
     for b, c in sc.warm:
         r.route(r.device_batch(b))
         r.commit()
@@ -294,7 +292,9 @@ def setup_oracle(sc):
     o.set_instance_state(sc.backlog_q, sc.tokcost_q, sc.contraction)
     for f in sc.fillers:
         o.load_entries(f.w, f.keys, f.metas)
-    log("oracle: filler entries loaded")
+    for c in sc.chains:
+        o.load_chains(c.tok_off, c.tokens, c.inst, c.seq, c.arr, c.max_blocks)
+    log("oracle: resident fill loaded")
     for b, c in sc.warm:
         o.route(b.cls, b.session, b.tok_off, b.tokens)
         o.commit()
@@ -310,9 +310,11 @@ def cpu_step(o, b):
     return time.perf_counter() - t
 
 
-def algorithmic_bytes(sc, st, mask_words=None):
-    """Algorithmic HBM bytes per launch of the hash and probe kernels (see the design notes).
-    mask_words: words per key of the global prefix index, None for the per-instance probe."""
+def algorithmic_bytes(sc, st, mask_words=None, admitted_blocks=0, evict_buckets=0):
+    """Algorithmic HBM bytes per launch of the hash, probe and commit kernels (see the design
+    notes).  mask_words: words per key of the global prefix index, None for the per-instance
+    probe; admitted_blocks: full blocks of the admitted requests (the insert's key operations);
+    evict_buckets: buckets of the tables above capacity after the inserts (the collect scan)."""
     b = sc.batch
     L = np.diff(b.tok_off)
     nb = L // 16
@@ -330,7 +332,24 @@ def algorithmic_bytes(sc, st, mask_words=None):
         first_b = 32 * st.bucket_reads_first + 8 * mask_words * st.probes_first + 2 * b.n * sc.W + 20 * b.n
     # K2 phase 2: one 32-byte key group per probe of the binary searches
     search_b = 32 * (st.probes - st.probes_first)
-    return {"hash": hash_b, "probe_first": first_b, "probe_search": search_b, "n_blocks": n_blocks}
+    mw = mask_words or 0
+    return {
+        "hash": hash_b, "probe_first": first_b, "probe_search": search_b, "n_blocks": n_blocks,
+        # K3b/K4a selection: one 32-byte record per request read, the decision fields written
+        "select": 32 * b.n + 10 * b.n,
+        # K4b insert: per admitted block, its key read (8 B), its home key group (32 B) and the
+        # read-modify-write of its meta (16 B); per new key its (key, instance) entry (16 B)
+        "insert": 56 * admitted_blocks + 16 * st.new_keys,
+        # global index: per new key, its entry read (16 B), a key group (32 B), its mask word RMW (16 B)
+        "gix_insert": (64 * st.new_keys) if mask_words else 0,
+        # K4c collect: the meta group of every bucket of a table above capacity (32 B)
+        "evict_collect": 32 * evict_buckets,
+        # delete: per evicted entry its key group (32 B) and slot cleared (16 B), its global-index
+        # key group and mask word (32 + 8 mw B), its deleted-slot bit (8 B)
+        "evict_delete": (88 + 8 * mw) * st.evicted,
+        # shift: per evicted entry one bucket of its run read and written (64 + 64 B)
+        "evict_shift": 128 * st.evicted,
+    }
 
 
 def run_gb300(args):
@@ -355,6 +374,14 @@ def run_gb300(args):
 
     sc = workload(args)
     log(f"workload generated: {sc.name}, {sc.batch.n_tokens} tokens in the measured batch")
+    # the stream of the end-to-end measurement: the measured batch, then the generator's next ones
+    stream_batches = []
+    if args.e2e_steps > 0 and sc.stream is not None:
+        stream_batches = [(sc.batch, sc.batch_completion, sc.batch_delta)]
+        while len(stream_batches) < args.e2e_steps:
+            stream_batches.append(sc.stream.next_batch(sc.batch.n, delta=True))
+        sc.max_tokens = max(sc.max_tokens, max(x.n_tokens for x, _, _ in stream_batches))
+        log(f"stream of {len(stream_batches)} batches generated for the end-to-end measurement")
     pidx = misat.PREFIX_GLOBAL if args.prefix_index == "global" else misat.PREFIX_PER_INSTANCE
     r = setup_router(sc, torch, pidx)
     ckpt = r.checkpoint_save()
@@ -485,88 +512,94 @@ def run_gb300(args):
     e2e_seq = whole_job_rate(n, world, args.e2e_steps, e2e_ms)
     log(f"e2e (one call per step, copy then route) done: {e2e_ms / max(1, args.e2e_steps):.3f} ms/step {e2e_each}")
 
-    # end to end, pipelined: the batch of step k+1 is copied (library copy stream) while step k
-    # is routed and committed; every step's copy and its decisions' read-back are inside the
-    # timed region, and so is the state restore that lets each step repeat the same batch
-    # (host wall clock, the device idle at both ends)
-    KE = args.e2e_steps
-    e2e_pipe = None
-    pipe_runs = []
-
-    def pipelined(steps):
-        r.checkpoint_restore(ckpt)
-        torch.cuda.synchronize()
-        t0 = time.perf_counter()
-        r.stage_host(hb, 0)
-        for k in range(steps):
-            if k > 0:
-                r.checkpoint_restore(ckpt)
-            if k + 1 < steps:
-                r.stage_host(hb, (k + 1) % 2)
-            r.route_staged(k % 2, hout)
-            r.commit()
-        torch.cuda.synchronize()
-        return (time.perf_counter() - t0) * 1e3
-
-    if KE > 0:
-        pipelined(4)  # untimed: each slot's route graph is captured on its second use
-        # three runs of KE steps; the median is reported (the host link is shared with the
-        # machine's other tenants, and one stall inside a run moves its mean)
-        pipe_runs = [pipelined(KE) for _ in range(3)]
-        pipe_ms = sorted(pipe_runs)[1]
-        log(f"e2e pipelined runs: {[round(x / KE, 3) for x in pipe_runs]} ms/step")
-        pipe_ms = max_over_ranks(pipe_ms, dist, "cuda")
-        e2e_pipe = whole_job_rate(n, world, KE, pipe_ms)
-        log(f"e2e pipelined done: {pipe_ms / KE:.3f} ms/step")
     h2d_full = int(b.cls.nbytes + b.session.nbytes + b.tok_off.nbytes + b.tokens.nbytes)
     d2h = int(n * (4 + 1 + 4))
 
-    # end to end, pipelined, with the batch in the delta layout: each prompt is sent as the
-    # tokens that follow an earlier prompt of the batch it extends (an agentic turn after the
-    # session's previous turn, a fan-out sample after its group's first sample); the library
-    # rebuilds the full batch on the GPU before the same route.  The layout is the caller's
-    # input format, built once outside the timed region.
-    e2e_delta, delta_runs, h2d_delta = None, [], None
+    # end to end over a stream of distinct batches: the measured batch and the batches the
+    # workload's generator produces after it, each staged from pinned host memory (the copy of
+    # batch k+1 overlaps the route and commit of batch k), routed, its decisions read back to
+    # host memory, committed, and followed by the completion events of its sessions; no state
+    # restore anywhere, host wall clock with the device idle at both ends.  Held requests are
+    # not resubmitted (the generator does not model retries).
+    def pinned(a):
+        return torch.from_numpy(np.ascontiguousarray(a)).pin_memory().numpy()
+
+    def pin_batch(bb):
+        return Batch(cls=pinned(bb.cls), session=pinned(bb.session.view(np.int64)).view(np.uint64), group=bb.group,
+                     tok_off=pinned(bb.tok_off), tokens=pinned(bb.tokens))
+
+    def pin_delta(dd):
+        return DeltaBatch(cls=pinned(dd.cls), session=pinned(dd.session.view(np.int64)).view(np.uint64),
+                          base=pinned(dd.base), delta_off=pinned(dd.delta_off), delta_tokens=pinned(dd.delta_tokens))
+
+    def pin_comp(c):
+        return Completion(session=pinned(c.session.view(np.int64)).view(np.uint64), cls=pinned(c.cls),
+                          total_blocks=pinned(c.total_blocks), residency_us=pinned(c.residency_us), done=pinned(c.done))
+
+    from paper_2608_11152_gb300.workload import Completion, DeltaBatch
+
+    KE = len(stream_batches)
+    e2e_stream = e2e_delta = stream_device = None
+    stream_runs, delta_runs = [], []
+    h2d_stream = h2d_delta = comp_bytes = None
     if KE > 0:
-        from paper_2608_11152_gb300.workload import DeltaBatch, encode_delta
+        sb = [(pin_batch(x), pin_delta(dl), pin_comp(c)) for x, c, dl in stream_batches]
+        houts = [{k: torch.empty(max(1, x.n), dtype=d).pin_memory().numpy() for k, d in
+                  (("inst", torch.int32), ("reason", torch.uint8), ("hit_blocks", torch.int32))} for x, _, _ in sb]
+        n_stream = sum(x.n for x, _, _ in sb)
+        comp_bytes = sum(int(c.session.nbytes + c.cls.nbytes + c.total_blocks.nbytes + c.residency_us.nbytes + c.done.nbytes)
+                         for _, _, c in sb)
+        h2d_stream = (sum(int(x.cls.nbytes + x.session.nbytes + x.tok_off.nbytes + x.tokens.nbytes) for x, _, _ in sb)
+                      + comp_bytes) // KE
+        h2d_delta = (sum(int(dl.cls.nbytes + dl.session.nbytes + dl.base.nbytes + dl.delta_off.nbytes +
+                             dl.delta_tokens.nbytes + 8 * (dl.n + 1)) for _, dl, _ in sb) + comp_bytes) // KE
 
-        enc = encode_delta(b)
-
-        def pinned(a):
-            return torch.from_numpy(np.ascontiguousarray(a)).pin_memory().numpy()
-
-        henc = DeltaBatch(cls=pinned(enc.cls), session=pinned(enc.session.view(np.int64)).view(np.uint64),
-                          base=pinned(enc.base), delta_off=pinned(enc.delta_off),
-                          delta_tokens=pinned(enc.delta_tokens))
-        # bytes copied per step: the layout, plus the full offsets the library computes
-        h2d_delta = int(enc.cls.nbytes + enc.session.nbytes + enc.base.nbytes + enc.delta_off.nbytes
-                        + enc.delta_tokens.nbytes + 8 * (n + 1))
-
-        def pipelined_delta(steps):
+        def run_stream(delta):
             r.checkpoint_restore(ckpt)
             torch.cuda.synchronize()
             t0 = time.perf_counter()
-            r.stage_host_delta(henc, 0)
-            for k in range(steps):
-                if k > 0:
-                    r.checkpoint_restore(ckpt)
-                if k + 1 < steps:
-                    r.stage_host_delta(henc, (k + 1) % 2)
-                r.route_staged(k % 2, hout)
+            stage = (lambda k, slot: r.stage_host_delta(sb[k][1], slot)) if delta else \
+                    (lambda k, slot: r.stage_host(sb[k][0], slot))
+            stage(0, 0)
+            for k in range(KE):
+                if k + 1 < KE:
+                    stage(k + 1, (k + 1) % 2)
+                r.route_staged(k % 2, houts[k])
                 r.commit()
+                c = sb[k][2]
+                r.complete(c.session, c.cls, c.total_blocks, c.residency_us, c.done)
             torch.cuda.synchronize()
             return (time.perf_counter() - t0) * 1e3
 
-        pipelined_delta(4)
-        delta_runs = [pipelined_delta(KE) for _ in range(3)]
+        run_stream(False)  # untimed: route graphs of both slots captured
+        run_stream(True)
+        stream_runs = [run_stream(False) for _ in range(3)]
+        delta_runs = [run_stream(True) for _ in range(3)]
+        # device time of the stream's route and commit (a separate pass with phase events)
+        r.set_timing(True)
+        r.checkpoint_restore(ckpt)
+        dev = []
+        for k in range(KE):
+            r.stage_host(sb[k][0], 0)
+            r.route_staged(0, houts[k])
+            ph = r.phase_times()
+            r.commit()
+            pc = r.phase_times()
+            c = sb[k][2]
+            r.complete(c.session, c.cls, c.total_blocks, c.residency_us, c.done)
+            dev.append((sum(ph[x] for x in ROUTE_PHASES), sum(pc[x] for x in COMMIT_PHASES), ph["select"]))
+        r.set_timing(False)
+        stream_device = [round(sum(x[i] for x in dev) / KE, 3) for i in range(3)]
+        log(f"stream device time per batch: route {stream_device[0]} ms (selection {stream_device[2]}), "
+            f"commit {stream_device[1]} ms")
+        sms = max_over_ranks(sorted(stream_runs)[1], dist, "cuda")
         dms = max_over_ranks(sorted(delta_runs)[1], dist, "cuda")
-        e2e_delta = whole_job_rate(n, world, KE, dms)
-        log(f"e2e pipelined, delta layout ({h2d_delta / 1e6:.0f} MB per step): "
-            f"{[round(x / KE, 3) for x in delta_runs]} ms/step")
-    if e2e_delta is not None:
-        e2e, h2d = e2e_delta, h2d_delta
-    else:
-        e2e, h2d = (e2e_pipe if e2e_pipe is not None else e2e_seq), h2d_full
+        e2e_stream = whole_job_rate(n_stream / KE, world, KE, sms)
+        e2e_delta = whole_job_rate(n_stream / KE, world, KE, dms)
+        log(f"e2e stream of {KE} batches, full layout: {[round(x / KE, 3) for x in stream_runs]} ms/batch; "
+            f"delta layout: {[round(x / KE, 3) for x in delta_runs]} ms/batch")
+    e2e = e2e_stream if e2e_stream is not None else e2e_seq
+    h2d = h2d_stream if h2d_stream is not None else h2d_full
 
     # roofline: dominant kernel of the step, plus the hash and probe kernels
     peak, peak_kind = peaks()
@@ -589,35 +622,48 @@ def run_gb300(args):
                 "rebuild_ms": round(rb_ms, 3), "steps_between_rebuilds": round(steps_between, 1),
                 "amortized_rebuild_ms_per_step": round(rb_ms / steps_between, 4)}
         log(f"global index: {gidx}")
-    ab = algorithmic_bytes(sc, st, mask_words=gidx["mask_words"] if gidx else None)
+    # the insert's key operations: full blocks of the admitted requests; the collect's scan:
+    # buckets of the tables above capacity after the inserts (the committed sizes plus the
+    # evictions of the step)
+    inst_h = out["inst"][: n].cpu().numpy()
+    nb_all = np.diff(sc.batch.tok_off) // 16
+    admitted_blocks = int(nb_all[inst_h >= 0].sum())
+    evict_buckets = 0
+    for w in range(sc.W):
+        if r.index_size(w) >= int(sc.cap_blocks[w]):
+            evict_buckets += r.table_buckets(w)
+    ab = algorithmic_bytes(sc, st, mask_words=gidx["mask_words"] if gidx else None,
+                           admitted_blocks=admitted_blocks, evict_buckets=evict_buckets)
     phase_ms = {p: phase_tot[p] / KP for p in phase_tot}
-    # dominant kernel: the phase with the largest time per kernel launch (multi-kernel phases
-    # are split evenly over their kernels); the committed ncu launch list gives the exact shares
-    per_launch = {p: phase_ms[p] / PHASE_KERNELS(pidx == misat.PREFIX_GLOBAL)[p] for p in phase_ms}
-    dom = max(per_launch, key=lambda p: per_launch[p])
+    # one kernel per phase below (the insert phase adds the small work-list kernel)
+    KERNEL_NAMES = {"hash": "k1_block_hash", "probe_first": "k2_probe_first_gix" if gidx else "k2_probe_first_group",
+                    "probe_search": "k2_probe_search", "select": "k4_select", "insert": "k4_insert",
+                    "gix_insert": "k4_gix_insert", "evict_collect": "k4_evict_collect",
+                    "evict_delete": "k4_evict_delete", "evict_shift": "k4_evict_shift"}
+
     def roof(kind):
-        ms = phase_ms[kind]
+        ms = phase_ms.get(kind, 0.0)
         byts = ab.get(kind)
         if byts is None or ms <= 0:
             return None
         ach = byts / (ms / 1e3) / 1e9
         return {"bound": "hbm", "achieved": round(ach, 1), "peak": peak, "unit": "GB/s",
                 "frac": round(ach / peak, 4), "traffic": None, "bytes_per_launch": int(byts),
-                "ms_per_launch": round(ms, 4), "peak_kind": peak_kind}
+                "ms_per_launch": round(ms, 4), "peak_kind": peak_kind, "kernel": KERNEL_NAMES[kind]}
 
-    kernels = {k: roof(k) for k in ("hash", "probe_first", "probe_search")}
+    kernels = {k: roof(k) for k in KERNEL_NAMES}
     if kernels["hash"] is not None:
         kernels["hash"]["traffic"] = profiled_traffic(sc.batch.n_tokens)
         hf = profiled_hash_fields(sc.batch.n_tokens)
         if "alu_pipe_active_frac" in hf:
             # the kernel's actual limiter: integer ALU issue (ncu sm__pipe_alu_cycles_active)
             kernels["hash"]["alu_pipe_active_frac_ncu"] = float(hf["alu_pipe_active_frac"])
-    dom_roof = dict(kernels[dom]) if kernels.get(dom) else roof(dom)
-    if dom_roof is None:
-        dom_roof = {"bound": "hbm", "achieved": None, "peak": peak, "unit": "GB/s", "frac": None, "traffic": None,
-                    "kernel": dom, "ms_per_launch": round(phase_ms[dom], 4),
-                    "note": "no algorithmic byte model for this phase yet"}
-    dom_roof["kernel"] = {"hash": "k1_block_hash", "probe_first": "k2_probe_first", "probe_search": "k2_probe_search"}.get(dom, dom)
+    if kernels["select"] is not None:
+        kernels["select"]["limiter"] = ("one CTA walks the batch in arrival order; bound by the chain of "
+                                        "headroom-exhaustion events, not by memory")
+    # dominant kernel: the largest time per launch
+    dom = max((k for k in kernels if kernels[k]), key=lambda k: kernels[k]["ms_per_launch"])
+    dom_roof = dict(kernels[dom])
     if dom == "hash":
         dom_roof["traffic_source"] = "profiles/k1_block_hash_stress_n65536.md (ncu dram__bytes_read.sum + dram__bytes_write.sum)"
 
@@ -635,16 +681,24 @@ def run_gb300(args):
         "prefix_decisions_per_s": round(world * n * sc.W * K / (total_ms / 1e3), 1),
         "prefix_decisions_definition": "(request, instance) longest-cached-prefix values H computed per second",
         "e2e": {"value": round(e2e, 1), "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
-                "api": ("misat_stage_host_delta + misat_route_staged + misat_commit (batch in the delta layout, "
-                        "rebuilt on the GPU; copy of step k+1 overlaps step k)") if e2e_delta is not None else
-                       "misat_stage_host + misat_route_staged + misat_commit (copy of step k+1 overlaps step k)",
-                "timer": "host wall clock over all steps, device idle at both ends; state restore inside; median of 3 runs",
-                "runs_ms_per_step": [round(x / KE, 3) for x in (delta_runs or pipe_runs)] if KE > 0 else None,
-                "full_layout_value": round(e2e_pipe, 1) if e2e_pipe is not None else None,
-                "full_layout_h2d_bytes_per_step": h2d_full,
-                "full_layout_api": "misat_stage_host + misat_route_staged + misat_commit (all tokens copied)",
+                "api": ("misat_stage_host + misat_route_staged + misat_commit + misat_complete over a stream of "
+                        f"{KE} distinct batches (the measured one and the generator's next ones), every token "
+                        "copied; the copy of batch k+1 overlaps batch k; no state restore"),
+                "timer": "host wall clock over the stream, device idle at both ends; median of 3 runs",
+                "runs_ms_per_step": [round(x / KE, 3) for x in stream_runs] if KE > 0 else None,
+                "h2d_includes": "cls, session, tok_off, tokens of each batch and the completion events that follow it",
+                "delta_layout_value": round(e2e_delta, 1) if e2e_delta is not None else None,
+                "delta_layout_h2d_bytes_per_step": h2d_delta,
+                "delta_layout_runs_ms_per_step": [round(x / KE, 3) for x in delta_runs] if KE > 0 else None,
+                "delta_layout_api": ("misat_stage_host_delta (each prompt sent as the tokens after the earlier "
+                                     "prompt of the batch it extends, as the generator emits it; rebuilt on the "
+                                     "GPU) + misat_route_staged + misat_commit + misat_complete, same stream"),
+                "stream_device_ms_per_batch": ({"route": stream_device[0], "selection": stream_device[2],
+                                                "commit": stream_device[1]} if stream_device else None),
                 "sequential_value": round(e2e_seq, 1), "host_link_h2d_gbs": link_gbs,
-                "sequential_api": "misat_route_host + misat_commit (copy, route, read-back; CUDA events)"},
+                "sequential_h2d_bytes_per_step": h2d_full,
+                "sequential_api": ("misat_route_host + misat_commit on the measured batch from the same state "
+                                   "(copy, route, read-back; CUDA events)")},
         "gpu_launches": kernels_per_step(pidx == misat.PREFIX_GLOBAL) * K,
         "roofline": dom_roof,
         "kernels": kernels,

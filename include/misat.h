@@ -288,6 +288,10 @@ int misat_load_entries(misat_ctx* ctx, int32_t w, const misat_entry* entries, in
 /* Number of resident blocks of instance w.  [sync] */
 int misat_index_size(misat_ctx* ctx, int32_t w, int64_t* out);
 
+/* Buckets (4 slots each) of instance w's table: 2^k, at least 2 Cap_w slots at creation,
+ * doubled when a commit would fill it past table_load.  [host] */
+int misat_index_buckets(misat_ctx* ctx, int32_t w, int64_t* out);
+
 /* Copy instance w's index to host_out sorted by key (cap entries available; *n_out =
  * count).  [sync] */
 int misat_dump_index(misat_ctx* ctx, int32_t w, misat_entry* host_out, int64_t cap,
@@ -342,9 +346,11 @@ int misat_checkpoint_restore(misat_ctx* ctx, const misat_checkpoint* ckpt);
 int misat_checkpoint_free(misat_checkpoint* ckpt);
 
 /* ---- per-phase device time (measurement; the paper has no counterpart) ----
- * With timing enabled, CUDA events on the context's stream bracket each phase of
- * misat_route and misat_commit.  misat_phase_times waits and writes the durations (ms)
- * of the last route / commit, indexed by MISAT_PHASE_*. */
+ * With timing enabled, the route and commit kernels are launched directly (no graph
+ * replay, the global-index pass on the context's stream instead of beside the session
+ * update) with CUDA events on the context's stream between them.  misat_phase_times waits
+ * and writes the durations (ms) of the last route / commit, indexed by MISAT_PHASE_*
+ * (MISAT_N_PHASES values). */
 #define MISAT_PHASE_PROLOGUE 0      /* validation, session snapshot, leaders */
 #define MISAT_PHASE_HASH 1          /* K1 chained block hash */
 #define MISAT_PHASE_CAPS 2          /* K3a caps */
@@ -352,10 +358,16 @@ int misat_checkpoint_free(misat_checkpoint* ckpt);
 #define MISAT_PHASE_PROBE_SEARCH 4  /* K2 binary search of the hit pairs */
 #define MISAT_PHASE_SELECT 5        /* K3b placement + K4a admission: the serial selection */
 #define MISAT_PHASE_FINALIZE 6      /* holds, followers, outputs */
-#define MISAT_PHASE_INSERT 7        /* K4b index insert */
+#define MISAT_PHASE_INSERT 7        /* K4b index insert (work list + table inserts) */
 #define MISAT_PHASE_SESSIONS 8      /* session table update */
-#define MISAT_PHASE_EVICT 9         /* K4c eviction select + compaction */
-#define MISAT_N_PHASES 10
+#define MISAT_PHASE_EVICT 9         /* K4c eviction, all five kernels */
+#define MISAT_PHASE_GIX_INSERT 10   /* global prefix index bits of the new keys (inline while timing) */
+#define MISAT_PHASE_EVICT_ESTIMATE 11
+#define MISAT_PHASE_EVICT_COLLECT 12
+#define MISAT_PHASE_EVICT_SELECT 13
+#define MISAT_PHASE_EVICT_DELETE 14
+#define MISAT_PHASE_EVICT_SHIFT 15
+#define MISAT_N_PHASES 16
 int misat_set_timing(misat_ctx* ctx, int enable);
 int misat_phase_times(misat_ctx* ctx, float* ms_out);
 

@@ -197,7 +197,7 @@ struct misat_ctx {
   cudaEvent_t ev_fork = nullptr, ev_join = nullptr;
   // phase timing: events 0..7 bracket the route phases, 8..11 the commit phases
   bool timing = false;
-  cudaEvent_t ev[12] = {};
+  cudaEvent_t ev[17] = {};
 
   void mark(int i) {
     if (timing) cudaEventRecord(ev[i], stream);
@@ -234,7 +234,9 @@ template <class F>
 int run_graph(misat_ctx* c, misat_ctx::GraphCache& gc, const std::vector<uint64_t>& key, F&& launch) {
   cudaStream_t st = c->stream;
   cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
-  if (gc.failed || !c->cap_stream || cudaStreamIsCapturing(st, &cs) != cudaSuccess ||
+  // direct launches while phase timing is on (events inside a graph do not time), after a
+  // failed capture, and while the caller captures the stream itself
+  if (c->timing || gc.failed || !c->cap_stream || cudaStreamIsCapturing(st, &cs) != cudaSuccess ||
       cs != cudaStreamCaptureStatusNone) {
     cudaGetLastError();
     launch(st);
@@ -560,10 +562,14 @@ int evict_all(misat_ctx* c, unsigned long long* evicted_counter, cudaEvent_t joi
   const int chunks = (int)std::min<uint64_t>(256, std::max<uint64_t>(1, ((uint64_t)1 << maxlg) / (4 * 256)));
   const std::vector<uint64_t> key{(uint64_t)chunks, reinterpret_cast<uint64_t>(ev.gix.keys),
                                   (uint64_t)ev.gix.log2nb, reinterpret_cast<uint64_t>(evicted_counter)};
-  int rc = run_graph(c, c->g_evict, key, [&](cudaStream_t s) { launch_evict_select(ev, chunks, c->num_sms, s); });
+  // with phase timing the kernels are launched directly with an event after each
+  const cudaEvent_t* marks = c->timing ? c->ev + 12 : nullptr;
+  int rc = run_graph(c, c->g_evict, key,
+                     [&](cudaStream_t s) { launch_evict_select(ev, chunks, c->num_sms, s, marks); });
   if (rc) return rc;
   if (join) CK(cudaStreamWaitEvent(c->stream, join, 0));
-  return run_graph(c, c->g_evict_apply, key, [&](cudaStream_t s) { launch_evict_apply(ev, chunks, c->num_sms, s); });
+  return run_graph(c, c->g_evict_apply, key,
+                   [&](cudaStream_t s) { launch_evict_apply(ev, chunks, c->num_sms, s, marks ? marks + 3 : nullptr); });
 }
 
 CapsArgs caps_args(misat_ctx* c) {
@@ -1231,7 +1237,7 @@ int misat_commit(misat_ctx* c) {
     c->mark(9);
     cudaEvent_t join = nullptr;
     if (ia.gix.keys) {
-      if (c->side_stream) {
+      if (c->side_stream && !c->timing) {
         CK(cudaEventRecord(c->ev_fork, st));
         CK(cudaStreamWaitEvent(c->side_stream, c->ev_fork, 0));
         launch_insert_gix(ia, c->num_sms * 4, c->side_stream);
@@ -1241,16 +1247,15 @@ int misat_commit(misat_ctx* c) {
         launch_insert_gix(ia, c->num_sms * 8, st);
       }
     }
+    c->mark(10);
     SessUpdateArgs sa{n, c->rq, c->sess, c->d_prot, c->err_ptr()};
     launch_session_update(sa, st);
-    c->mark(10);
+    c->mark(11);
     int rc = evict_all(c, c->stats_ptr() + 19, join);
     if (rc) return rc;
   } else {
-    c->mark(9);
-    c->mark(10);
+    for (int i = 9; i <= 16; ++i) c->mark(i);
   }
-  c->mark(11);
   CK(cudaGetLastError());
   CK(enqueue_meta(c));
   c->seq += 1;
@@ -1262,11 +1267,21 @@ int misat_complete(misat_ctx* c, int32_t n, const uint64_t* session, const uint8
   if (!c || n < 0) return MISAT_ERR_INVALID_ARG;
   if (n == 0) return MISAT_OK;
   if (!session || !cls || !total_blocks || !residency_us || !done) return MISAT_ERR_INVALID_ARG;
-  std::unordered_set<uint64_t> seen;
-  seen.reserve((size_t)n * 2);
-  for (int i = 0; i < n; ++i) {
-    if (cls[i] > 2 || total_blocks[i] < 0 || residency_us[i] < 0 || session[i] == 0) return MISAT_ERR_INVALID_ARG;
-    if (!seen.insert(session[i]).second) return MISAT_ERR_INVALID_ARG;
+  {
+    // distinct sessions: open addressing in one flat table (session ids are nonzero)
+    const int lg = ceil_log2(2 * (uint64_t)n);
+    const uint64_t mask = ((uint64_t)1 << lg) - 1;
+    std::vector<uint64_t> seen(mask + 1, 0);
+    for (int i = 0; i < n; ++i) {
+      if (cls[i] > 2 || total_blocks[i] < 0 || residency_us[i] < 0 || session[i] == 0) return MISAT_ERR_INVALID_ARG;
+      uint64_t h = session[i] * kGold;
+      h = (h ^ (h >> 29)) & mask;
+      while (seen[h] != 0) {
+        if (seen[h] == session[i]) return MISAT_ERR_INVALID_ARG;
+        h = (h + 1) & mask;
+      }
+      seen[h] = session[i];
+    }
   }
   for (int i = 0; i < n; ++i) {
     if (!done[i]) continue;
@@ -1450,6 +1465,12 @@ int misat_index_size(misat_ctx* c, int32_t w, int64_t* out) {
   if (rc) return rc;
   *out = c->h_size(w);
   return c->h_err();
+}
+
+int misat_index_buckets(misat_ctx* c, int32_t w, int64_t* out) {
+  if (!c || !out || w < 0 || w >= c->W) return MISAT_ERR_INVALID_ARG;
+  *out = (int64_t)1 << c->h_desc[w].log2nb;
+  return MISAT_OK;
 }
 
 int misat_dump_index(misat_ctx* c, int32_t w, misat_entry* host_out, int64_t cap, int64_t* n_out) {
@@ -1636,11 +1657,13 @@ int misat_phase_times(misat_ctx* c, float* ms) {
   if (!c || !ms) return MISAT_ERR_INVALID_ARG;
   if (!c->timing) return MISAT_ERR_STATE;
   CK(cudaStreamSynchronize(c->stream));
-  // route phases: consecutive events 0..7; commit phases: 8..11
-  const int from[MISAT_N_PHASES] = {0, 1, 2, 3, 4, 5, 6, 8, 9, 10};
+  // route phases: consecutive events 0..7; commit: 8 start, 9 tables inserted, 10 global index,
+  // 11 sessions, 12..16 after each eviction kernel
+  const int from[MISAT_N_PHASES] = {0, 1, 2, 3, 4, 5, 6, 8, 10, 11, 9, 11, 12, 13, 14, 15};
+  const int to[MISAT_N_PHASES] = {1, 2, 3, 4, 5, 6, 7, 9, 11, 16, 10, 12, 13, 14, 15, 16};
   for (int i = 0; i < MISAT_N_PHASES; ++i) {
     float t = 0.f;
-    if (cudaEventElapsedTime(&t, c->ev[from[i]], c->ev[from[i] + 1]) != cudaSuccess) {
+    if (cudaEventElapsedTime(&t, c->ev[from[i]], c->ev[to[i]]) != cudaSuccess) {
       cudaGetLastError();
       t = 0.f;  // phase not recorded (e.g. empty batch)
     }

@@ -578,27 +578,34 @@ int stream_grid(const EvictArgs& a, int chunks_per_inst, int num_sms) {
 }
 }  // namespace
 
-void launch_evict_select(const EvictArgs& a, int chunks_per_inst, int num_sms, cudaStream_t st) {
+void launch_evict_select(const EvictArgs& a, int chunks_per_inst, int num_sms, cudaStream_t st,
+                         const cudaEvent_t* marks) {
   const int W = a.only_w ? 1 : a.W;
   cudaMemsetAsync(a.n_act, 0, sizeof(unsigned), st);
   k4_evict_estimate<<<W, kSelThreads, 0, st>>>(a);
+  if (marks) cudaEventRecord(marks[0], st);
   k4_evict_collect<<<stream_grid(a, chunks_per_inst, num_sms), 256, 0, st>>>(a, (uint32_t)chunks_per_inst);
+  if (marks) cudaEventRecord(marks[1], st);
   k4_evict_select<<<W, kSelThreads, 0, st>>>(a);
+  if (marks) cudaEventRecord(marks[2], st);
 }
 
-void launch_evict_apply(const EvictArgs& a, int chunks_per_inst, int num_sms, cudaStream_t st) {
+void launch_evict_apply(const EvictArgs& a, int chunks_per_inst, int num_sms, cudaStream_t st,
+                        const cudaEvent_t* marks) {
   // the eviction lists (about E entries per instance) are split into fewer, larger pieces
   // than the tables: each piece then holds several entries per thread
   (void)chunks_per_inst;
   constexpr int kListChunks = 32;
   const int grid = stream_grid(a, kListChunks, num_sms);
   k4_evict_delete<<<grid, 256, 0, st>>>(a, (uint32_t)kListChunks);
+  if (marks) cudaEventRecord(marks[0], st);
   k4_evict_shift<<<grid, 256, 0, st>>>(a, (uint32_t)kListChunks);
+  if (marks) cudaEventRecord(marks[1], st);
 }
 
 void launch_evict(const EvictArgs& a, int chunks_per_inst, int num_sms, cudaStream_t st) {
-  launch_evict_select(a, chunks_per_inst, num_sms, st);
-  launch_evict_apply(a, chunks_per_inst, num_sms, st);
+  launch_evict_select(a, chunks_per_inst, num_sms, st, nullptr);
+  launch_evict_apply(a, chunks_per_inst, num_sms, st, nullptr);
 }
 
 // Compaction of one instance table: delete entries with meta == 0 (marked) or

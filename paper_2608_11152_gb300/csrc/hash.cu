@@ -218,62 +218,59 @@ static __device__ __align__(256) unsigned long long g_noalloc_scratch[kNoAllocWo
 namespace {
 
 // One CTA: clear the counters, validate the offsets and write the exclusive prefix of
-// floor(L_r / 16) (compact key positions) into the scratch array.
+// floor(L_r / 16) (compact key positions) into the scratch array.  The offsets are read in
+// coalesced tiles of blockDim.x requests (thread t takes request tile + t); each tile is
+// scanned across the block and carried into the next.
 __global__ void __launch_bounds__(1024) k1na_offsets(const int64_t* tok_off, int32_t n, int64_t n_tokens,
                                                      int64_t keys_cap, unsigned long long* scratch) {
-  __shared__ long long s_warp[32];
+  __shared__ long long s_wsum[32], s_wex[32], s_tot;
   __shared__ int s_bad;
   const int t = threadIdx.x, lane = t & 31, wid = t >> 5;
+  const int nw = (blockDim.x + 31) >> 5;
   if (t == 0) {
     scratch[0] = 0;
     scratch[1] = 0;
     s_bad = 0;
   }
-  __syncthreads();
-  const int per = (n + blockDim.x - 1) / blockDim.x;
-  const int lo = t * per, hi = min(n, lo + per);
-  long long local = 0;
-  bool bad = false;
-  for (int r = lo; r < hi; ++r) {
-    const int64_t t0 = tok_off[r], t1 = tok_off[r + 1];
-    if (t0 < 0 || t1 < t0 || t1 > n_tokens || (t1 - t0) >= (1 << 20)) bad = true;
-    local += (t1 - t0) >> 4;
-  }
-  if (t == 0 && tok_off[0] != 0) bad = true;
-  if (t == 0 && tok_off[n] != n_tokens) bad = true;
-  if (bad) atomicOr(&s_bad, 1);
-  long long incl = local;
-#pragma unroll
-  for (int o = 1; o < 32; o <<= 1) {
-    const long long v = __shfl_up_sync(kFull, incl, o);
-    if (lane >= o) incl += v;
-  }
-  if (lane == 31) s_warp[wid] = incl;
-  __syncthreads();
-  if (wid == 0) {
-    const long long v = s_warp[lane];
-    long long sc = v;
+  bool bad = t == 0 && (tok_off[0] != 0 || tok_off[n] != n_tokens);
+  long long carry = 0;  // key positions of the tiles before this one (block-uniform)
+  for (int base = 0; base < n; base += blockDim.x) {
+    const int r = base + t;
+    long long v = 0;
+    if (r < n) {
+      const int64_t t0 = tok_off[r], t1 = tok_off[r + 1];
+      if (t0 < 0 || t1 < t0 || t1 > n_tokens || (t1 - t0) >= (1 << 20)) bad = true;
+      v = (t1 - t0) >> 4;
+    }
+    long long incl = v;
 #pragma unroll
     for (int o = 1; o < 32; o <<= 1) {
-      const long long u = __shfl_up_sync(kFull, sc, o);
-      if (lane >= o) sc += u;
+      const long long u = __shfl_up_sync(kFull, incl, o);
+      if (lane >= o) incl += u;
     }
-    s_warp[lane] = sc - v;
+    if (lane == 31) s_wsum[wid] = incl;
+    __syncthreads();
+    if (wid == 0) {
+      const long long w = lane < nw ? s_wsum[lane] : 0;
+      long long sc = w;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const long long u = __shfl_up_sync(kFull, sc, o);
+        if (lane >= o) sc += u;
+      }
+      s_wex[lane] = sc - w;
+      if (lane == 31) s_tot = sc;
+    }
+    __syncthreads();
+    if (r < n) scratch[8 + r] = (unsigned long long)(carry + s_wex[wid] + incl - v);
+    carry += s_tot;
   }
-  __syncthreads();
-  long long run = s_warp[wid] + incl - local;
-  for (int r = lo; r < hi; ++r) {
-    scratch[8 + r] = (unsigned long long)run;
-    run += (tok_off[r + 1] - tok_off[r]) >> 4;
-  }
-  if (t == blockDim.x - 1) {
-    scratch[8 + n] = (unsigned long long)run;
-    scratch[2] = (unsigned long long)run;
-  }
+  if (bad) atomicOr(&s_bad, 1);
   __syncthreads();
   if (t == 0) {
-    const long long total = (long long)scratch[2];
-    if (s_bad || total > keys_cap) scratch[1] = (unsigned long long)(long long)MISAT_ERR_INVALID_ARG;
+    scratch[8 + n] = (unsigned long long)carry;
+    scratch[2] = (unsigned long long)carry;
+    if (s_bad || carry > keys_cap) scratch[1] = (unsigned long long)(long long)MISAT_ERR_INVALID_ARG;
   }
 }
 

@@ -76,7 +76,8 @@ class misat_overload_config(C.Structure):
 
 
 PHASES = ("prologue", "hash", "caps", "probe_first", "probe_search", "select", "finalize", "insert",
-          "sessions", "evict")
+          "sessions", "evict", "gix_insert", "evict_estimate", "evict_collect", "evict_select", "evict_delete",
+          "evict_shift")
 
 
 _SIG = {
@@ -96,6 +97,7 @@ _SIG = {
     "misat_load_chains": [_p, C.c_int32, _p, _p, _p, _p, _p, _p],
     "misat_load_entries": [_p, C.c_int32, _p, C.c_int64],
     "misat_index_size": [_p, C.c_int32, C.POINTER(C.c_int64)],
+    "misat_index_buckets": [_p, C.c_int32, C.POINTER(C.c_int64)],
     "misat_dump_index": [_p, C.c_int32, _p, C.c_int64, C.POINTER(C.c_int64)],
     "misat_dump_keys": [_p, _p, C.c_int64, C.POINTER(C.c_int64)],
     "misat_dump_caps": [_p, _p, _p, _p, _p, _p, _p],
@@ -336,6 +338,11 @@ class Router:
         v = C.c_int64(0)
         _ck(_lib.misat_index_size(self._h, w, C.byref(v)), "misat_index_size")
         return v.value
+
+    def table_buckets(self, w):
+        v = C.c_int64(0)
+        _ck(_lib.misat_index_buckets(self._h, w, C.byref(v)), "misat_index_buckets")
+        return int(v.value)
 
     def dump_index(self, w):
         cap = self.index_size(w) + 16

@@ -165,6 +165,20 @@ class Filler:
 
 
 @dataclass
+class ChainBatch:
+    """Prompt chains resident before the first batch, in the layout of the load_chains call:
+    chain c is tokens[tok_off[c]:tok_off[c+1]]; its first max_blocks[c] full blocks are
+    resident on instance inst[c] with the tick (seq[c], arr[c]) -- whole prefixes with one
+    tick, so depth orders their eviction."""
+    tok_off: np.ndarray     # int64 [m+1]
+    tokens: np.ndarray      # int32
+    inst: np.ndarray        # int32 [m]
+    seq: np.ndarray         # uint64 [m]
+    arr: np.ndarray         # uint32 [m]
+    max_blocks: np.ndarray  # int32 [m]
+
+
+@dataclass
 class MixSpec:
     rho_ppm: tuple
     rlvr_prompt: tuple
@@ -196,9 +210,13 @@ class Scenario:
     hold_delay_q: int
     protected_frac_q16: int = 58982   # C_w = 0.9 Cap_w
     mode: int = 0
-    fillers: list = field(default_factory=list)
+    fillers: list = field(default_factory=list)  # list of Filler (loaded entries)
+    chains: list = field(default_factory=list)   # list of ChainBatch (loaded prompt chains)
     warm: list = field(default_factory=list)   # list of (Batch, Completion)
     batch: Batch | None = None
+    batch_completion: Completion | None = None  # completion events of the measured batch's sessions
+    batch_delta: DeltaBatch | None = None       # the measured batch in the delta layout
+    stream: object = None                       # generator of the batches after the measured one
     max_tokens: int = 0
     max_batch: int = 0
 
@@ -247,13 +265,29 @@ class MixedStream:
         v = int(round(median * math.exp(sigma * self.rng.standard_normal())))
         return max(1, min(cap, v))
 
+    def seed_sessions(self, histories):
+        """Put agentic sessions with the given histories (token arrays) at the front of the pool:
+        they continue with their next turn, which appends to the history."""
+        s = self.spec
+        seeded = []
+        for h in histories:
+            mt = int(self.rng.integers(max(2, s.agent_max_turns[0]), s.agent_max_turns[1] + 1))
+            a = _AgentSession(self._sid(), h, mt, max(len(h), s.agent_hist_cap) + s.agent_append[1])
+            a.turn = 1
+            seeded.append(a)
+        self.pool = seeded + self.pool
+
     def _new_agent(self):
         s = self.spec
         L0 = int(self.rng.integers(s.agent_initial[0], s.agent_initial[1] + 1))
         mt = int(self.rng.integers(s.agent_max_turns[0], s.agent_max_turns[1] + 1))
         return _AgentSession(self._sid(), self._tokens(L0), mt, s.agent_hist_cap + s.agent_append[1])
 
-    def next_batch(self, n: int) -> tuple[Batch, Completion]:
+    def next_batch(self, n: int, delta: bool = False):
+        """The next batch of n requests and the completion events of its sessions; with
+        delta=True also the batch in the delta layout, built from what the generator knows
+        (an agentic turn extends its session's previous turn in the batch, a fan-out sample
+        its group's first sample) without comparing tokens."""
         s = self.spec
         rng = self.rng
         n_rlvr, n_rlhf, n_agent = split_classes(n, s.rho_ppm)
@@ -347,7 +381,43 @@ class MixedStream:
             residency_us=np.array([c[3] for c in comp], dtype=np.int64),
             done=np.ones(len(comp), dtype=np.uint8),
         )
-        return batch, completion
+        if not delta:
+            return batch, completion
+        return batch, completion, _structural_delta(reqs, batch)
+
+
+def _structural_delta(reqs, batch: Batch) -> DeltaBatch:
+    """Delta layout of a generated batch from its structure: the base of a request is the
+    latest earlier request of its session (agentic turns), else the first earlier request of
+    its prompt group (fan-out samples), chains at most DELTA_MAX_DEPTH long."""
+    n = len(reqs)
+    base = np.full(n, -1, np.int32)
+    depth = np.zeros(n, np.int32)
+    last_of_session, first_of_group = {}, {}
+    lens = np.diff(batch.tok_off)
+    parts, off = [], np.zeros(n + 1, np.int64)
+    for r, (c, sid, g, prompt, akey) in enumerate(reqs):
+        b = -1
+        if akey is not None and sid in last_of_session:
+            b = last_of_session[sid]
+        elif g and g in first_of_group:
+            b = first_of_group[g]
+        if b >= 0 and depth[b] < DELTA_MAX_DEPTH:
+            base[r] = b
+            depth[r] = depth[b] + 1
+            own = prompt[int(lens[b]):]
+        else:
+            depth[r] = 1
+            own = prompt
+        parts.append(own)
+        off[r + 1] = off[r] + len(own)
+        if akey is not None:
+            last_of_session[sid] = r
+        if g and g not in first_of_group:
+            first_of_group[g] = r
+    tok = np.concatenate(parts).astype(np.int32) if parts else np.zeros(0, np.int32)
+    return DeltaBatch(cls=batch.cls.copy(), session=batch.session.copy(), base=base, delta_off=off,
+                      delta_tokens=tok)
 
 
 def _prior_kbar(spec: MixSpec) -> tuple:
@@ -374,13 +444,65 @@ MIX2 = dict(rlvr_prompt=(64, 1024), rlvr_fanout=8, rlvr_decode_median=4096, rlvr
             agent_hist_cap=32768)
 
 
-def _stream_scenario(name, seed, W, cap, n, n_warm, spec: MixSpec, fill=0.0):
+CHAIN_BLOCKS = (32, 1024)   # blocks per fill chain, uniform (512 to 16,384 tokens)
+CHAIN_TOKENS_PER_LOAD = 1 << 25   # tokens per ChainBatch (the load call's staging limit)
+CHAIN_PER_LOAD = 16384            # chains per ChainBatch
+
+
+def _chain_fill(rng, W, cap, fill, n_sessions):
+    """Resident prompt chains filling every instance to `fill` of its capacity: chains of
+    CHAIN_BLOCKS random-token blocks, each older than any commit (seq 0, its own arrival
+    tick).  The first n_sessions chains are also returned as the histories of agentic sessions
+    that continue later; those are resident only 60-90% deep (uniform per chain)."""
+    target = int(fill * cap)
+    lens, insts = [], []
+    for w in range(W):
+        left = target
+        while left > 0:
+            k = min(left, int(rng.integers(CHAIN_BLOCKS[0], CHAIN_BLOCKS[1] + 1)))
+            lens.append(k)
+            insts.append(w)
+            left -= k
+    m = len(lens)
+    perm = rng.permutation(m)  # the session histories come from every instance
+    lens = np.array(lens, np.int64)[perm]
+    insts = np.array(insts, np.int32)[perm]
+    maxb = lens.astype(np.int32).copy()
+    ns = min(n_sessions, m)
+    maxb[:ns] = np.maximum(1, (lens[:ns] * rng.uniform(0.6, 0.9, size=ns)).astype(np.int32))
+    arr = rng.integers(0, 1 << 20, size=m, dtype=np.int64).astype(np.uint32)
+    tok_len = 16 * lens
+    batches, histories = [], []
+    c0 = 0
+    while c0 < m:
+        c1 = c0
+        t = 0
+        while c1 < m and c1 - c0 < CHAIN_PER_LOAD and (t + tok_len[c1] <= CHAIN_TOKENS_PER_LOAD or c1 == c0):
+            t += tok_len[c1]
+            c1 += 1
+        off = np.zeros(c1 - c0 + 1, np.int64)
+        np.cumsum(tok_len[c0:c1], out=off[1:])
+        toks = rng.integers(0, VOCAB, size=int(off[-1]), dtype=np.int32)
+        batches.append(ChainBatch(tok_off=off, tokens=toks, inst=insts[c0:c1].copy(),
+                                  seq=np.zeros(c1 - c0, np.uint64), arr=arr[c0:c1].copy(),
+                                  max_blocks=maxb[c0:c1].copy()))
+        for c in range(c0, min(c1, ns)):
+            histories.append(toks[off[c - c0]:off[c - c0 + 1]].copy())
+        c0 = c1
+    return batches, histories
+
+
+def _stream_scenario(name, seed, W, cap, n, n_warm, spec: MixSpec, fill=0.0, chain_fill=False):
     rng = np.random.default_rng(seed + 7)
     backlog, tokcost, contraction = _instance_state(rng, W)
     sc = Scenario(name=name, W=W, cap_blocks=np.full(W, cap, dtype=np.int64), rho_ppm=spec.rho_ppm,
                   prior_kbar=_prior_kbar(spec), prior_T_us=30_000_000, backlog_q=backlog,
                   tokcost_q=tokcost, contraction=contraction, hold_delay_q=50_000_000)
-    if fill > 0:
+    histories = []
+    if fill > 0 and chain_fill:
+        n_hist = max(1, spec.agent_sessions // 4)
+        sc.chains, histories = _chain_fill(rng, W, cap, fill, n_hist)
+    elif fill > 0:
         nf = int(fill * cap)
         for w in range(W):
             # full 64-bit keys (like block hashes), 0 and 1 excluded
@@ -397,9 +519,14 @@ def _stream_scenario(name, seed, W, cap, n, n_warm, spec: MixSpec, fill=0.0):
     stream = MixedStream(spec, seed, sid_base=(seed % 4096) << 40)
     for _ in range(n_warm):
         sc.warm.append(stream.next_batch(n))
-    sc.batch, _ = stream.next_batch(n)
-    sc.max_batch = max([b.n for b, _ in sc.warm] + [sc.batch.n])
-    sc.max_tokens = max([b.n_tokens for b, _ in sc.warm] + [sc.batch.n_tokens])
+    if histories:
+        # agentic sessions whose history is (60-90% deep) resident on some instance continue in
+        # the measured batch; the router has not seen them (they are new sessions to it)
+        stream.seed_sessions(histories)
+    sc.batch, sc.batch_completion, sc.batch_delta = stream.next_batch(n, delta=True)
+    sc.stream = stream   # continues with the batches after the measured one
+    sc.max_batch = max([b.n for b, _ in sc.warm] + [sc.batch.n] + [len(c.inst) for c in sc.chains])
+    sc.max_tokens = max([b.n_tokens for b, _ in sc.warm] + [sc.batch.n_tokens] + [int(c.tok_off[-1]) for c in sc.chains])
     return sc
 
 
@@ -514,11 +641,12 @@ def _concat_batches(batches, rng):
 
 
 def config5(n=65536, fill=0.95, seed=20260005, n_warm=1, instances=128, cap=262144) -> Scenario:
-    """Throughput stress: 128 x 262,144 blocks filled to `fill`, batches of n requests 40/30/30
-    (fewer instances only for small profiling captures)."""
+    """Throughput stress: 128 x 262,144 blocks filled to `fill` with resident prompt chains (a
+    quarter of the batch's agentic sessions continue histories that are 60-90% resident),
+    batches of n requests 40/30/30 (fewer instances only for small profiling captures)."""
     spec = MixSpec(rho_ppm=(400000, 300000, 300000), agent_sessions=max(1, round(0.3 * n / 4.8)), **MIX2)
     return _stream_scenario(f"cfg5_stress_{instances}x{cap}_n{n}_fill{int(fill * 100)}", seed, instances, cap, n,
-                            n_warm, spec, fill=fill)
+                            n_warm, spec, fill=fill, chain_fill=True)
 
 
 def small_random(seed, W=3, cap=64, n=24, mode=0, n_warm=2) -> Scenario:

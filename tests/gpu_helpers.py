@@ -10,7 +10,7 @@ import time
 import numpy as np
 
 import oracle
-from tests.helpers import make_oracle
+from tests.helpers import load_fill, make_oracle
 
 
 def make_router(sc, **over):
@@ -93,12 +93,10 @@ def run_parity(sc, index_every_step=True, check_H=True, check_keys=True, final_i
     r = make_router(sc, **router_over)
     o = make_oracle(sc)
     try:
-        for f in sc.fillers:
-            r.load_entries(f.w, f.keys, f.metas)
-        progress("gpu fillers loaded")
-        for f in sc.fillers:
-            o.load_entries(f.w, f.keys, f.metas)
-        progress("oracle fillers loaded")
+        load_fill(r, sc)
+        progress("gpu fill loaded")
+        load_fill(o, sc)
+        progress("oracle fill loaded")
         steps = list(sc.warm) + [(sc.batch, None)]
         for i, (b, comp) in enumerate(steps):
             route_both(r, o, b, sc.W, check_H=check_H, check_keys=check_keys)

@@ -22,6 +22,14 @@ def make_oracle(sc, **over):
     return o
 
 
+def load_fill(x, sc):
+    """Load a scenario's resident fill (entries and prompt chains) into a router or an oracle."""
+    for f in sc.fillers:
+        x.load_entries(f.w, f.keys, f.metas)
+    for c in sc.chains:
+        x.load_chains(c.tok_off, c.tokens, c.inst, c.seq, c.arr, c.max_blocks)
+
+
 def scenario_steps(sc):
     """Yield ("route", batch, completion_after) for the warm-up batches and the measured batch."""
     for b, c in sc.warm:

@@ -44,3 +44,20 @@ def test_decode_follows_chains():
     off, tok = wl.decode_delta(d)
     assert off.tolist() == [0, 3, 8, 14, 17]
     assert tok.tolist() == [1, 2, 3, 1, 2, 3, 4, 5, 1, 2, 3, 4, 5, 6, 1, 2, 3]
+
+
+def test_generator_layout_equals_token_comparison():
+    """The layout the generator emits from its structure (turns extend their session's
+    previous turn, fan-out samples their group's first sample) is the one found by comparing
+    tokens, and rebuilds the batch exactly."""
+    for sc in (wl.config1(), wl.config2(), wl.small_random(5, n=60, n_warm=2)):
+        for _ in range(2):
+            b, _, d = sc.stream.next_batch(sc.batch.n, delta=True)
+            e = wl.encode_delta(b)
+            assert np.array_equal(d.base, e.base)
+            assert np.array_equal(d.delta_off, e.delta_off) and np.array_equal(d.delta_tokens, e.delta_tokens)
+            off, tok = wl.decode_delta(d)
+            assert np.array_equal(off, b.tok_off) and np.array_equal(tok, b.tokens)
+        e = wl.encode_delta(sc.batch)
+        assert np.array_equal(sc.batch_delta.base, e.base)
+        assert np.array_equal(sc.batch_delta.delta_tokens, e.delta_tokens)

@@ -12,7 +12,7 @@ from oracle import overload as ovo
 from paper_2608_11152_gb300 import misat
 from paper_2608_11152_gb300 import workload as wl
 from tests.gpu_helpers import assert_equal, compare_state, make_router
-from tests.helpers import make_oracle
+from tests.helpers import load_fill, make_oracle
 
 # reactive thresholds so that contractions happen within a few batches
 CFG = dict(ref_windows=4, min_ref=1, gap_ppm=0, confirm=1, queue_thresh=2, recover_after=1, max_contraction_pct=60)
@@ -41,9 +41,8 @@ def _run(sc):
     ctl_o = ovo.OverloadOracle(W, **CFG)
     contracted = 0
     try:
-        for f in sc.fillers:
-            r.load_entries(f.w, f.keys, f.metas)
-            o.load_entries(f.w, f.keys, f.metas)
+        for x in (r, o):
+            load_fill(x, sc)
         for b, comp in list(sc.warm) + [(sc.batch, None)]:
             out = r.route(r.device_batch(b))
             torch.cuda.synchronize()

@@ -18,7 +18,7 @@ else:
 import oracle  # noqa: E402
 from paper_2608_11152_gb300 import workload as wl  # noqa: E402
 from tests.gpu_helpers import assert_equal, compare_state, make_router, route_both, run_parity  # noqa: E402
-from tests.helpers import make_oracle  # noqa: E402
+from tests.helpers import load_fill, make_oracle  # noqa: E402
 
 pytestmark = [pytest.mark.gpu]
 
@@ -104,8 +104,9 @@ def test_parity_config5_reduced():
 
 
 def test_parity_config5_full_size():
-    """The benchmark workload itself: 128 x 262,144 blocks at 95% fill, 65,536 requests,
-    in the launch configuration the benchmark times: the measured batch is routed as the
+    """The benchmark workload itself: 128 x 262,144 blocks at 95% fill (resident prompt chains,
+    some of them histories that agentic sessions of the batch continue), 65,536 requests, in
+    the launch configuration the benchmark times: the measured batch is routed as the
     benchmark routes it (same buffers every call, so the route is launched directly, then
     captured, then replayed from its CUDA graph) and every one of those routes must give the
     oracle's decisions; then the commit and every instance's index are compared."""
@@ -115,9 +116,8 @@ def test_parity_config5_full_size():
     r = make_router(sc)
     o = make_oracle(sc)
     try:
-        for f in sc.fillers:
-            r.load_entries(f.w, f.keys, f.metas)
-            o.load_entries(f.w, f.keys, f.metas)
+        load_fill(r, sc)
+        load_fill(o, sc)
         for b, comp in sc.warm:
             route_both(r, o, b, sc.W, check_H=False, check_keys=False)
             r.commit()
