@@ -133,6 +133,8 @@ struct misat_ctx {
   uint8_t* d_onhull = nullptr;   // initial envelopes of the selection [3W]
   int32_t* d_rank = nullptr;     // slope order of the instances [W]
   int32_t* d_rank_a = nullptr;   // (d_w, w) order of the instances [W]
+  int32_t* d_sel_list = nullptr; // [3 max_batch] each class's leaders (per-class selection)
+  int32_t* d_sel_x = nullptr;    // [W + 2] admissions per instance, ticket, coupled flag
   // every d_w and every 1/mu_w below 2^25: the selection's envelope arithmetic fits in 64 bits
   bool bk_small = true, tc_small = true;
   int32_t* d_chain_max = nullptr;  // per-chain insert limits of misat_load_chains
@@ -661,6 +663,9 @@ void enqueue_route(misat_ctx* c, const misat_batch* b, misat_decisions* out, cud
   sp.rq = c->rq;
   sp.H = c->d_H;
   sp.rec = c->d_sel_rec;
+  sp.adm = c->d_sel_x;
+  sp.ticket = reinterpret_cast<unsigned*>(c->d_sel_x + c->W);
+  sp.coupled = c->d_sel_x + c->W + 1;
   sp.err = c->err_ptr();
   launch_select_prep(sp, st);
   EnvInitArgs ei{};
@@ -675,6 +680,27 @@ void enqueue_route(misat_ctx* c, const misat_batch* b, misat_decisions* out, cud
   ei.small = c->bk_small && c->tc_small;
   ei.err = c->err_ptr();
   launch_env_init(ei, st);
+  SelectClassArgs sc{};
+  sc.n = n;
+  sc.W = c->W;
+  sc.rec = c->d_sel_rec;
+  sc.rq = c->rq;
+  sc.gh = c->ia.gh;
+  sc.ch = c->ia.ch;
+  sc.backlog = c->d_backlog;
+  sc.tokcost = c->d_tokcost;
+  sc.onhull = c->d_onhull;
+  sc.rank = c->d_rank;
+  sc.rank_a = c->d_rank_a;
+  sc.H = c->d_H;
+  sc.hold_delay_q = c->hold_delay_q;
+  sc.small = c->bk_small && c->tc_small;
+  sc.list = c->d_sel_list;
+  sc.adm = c->d_sel_x;
+  sc.ticket = reinterpret_cast<unsigned*>(c->d_sel_x + c->W);
+  sc.coupled = c->d_sel_x + c->W + 1;
+  sc.err = c->err_ptr();
+  launch_select_class(sc, st);
   SelectArgs sa{};
   sa.n = n;
   sa.W = c->W;
@@ -690,6 +716,7 @@ void enqueue_route(misat_ctx* c, const misat_batch* b, misat_decisions* out, cud
   sa.small = c->bk_small && c->tc_small;
   sa.H = c->d_H;
   sa.hold_delay_q = c->hold_delay_q;
+  sa.coupled = c->d_sel_x + c->W + 1;
   sa.err = c->err_ptr();
   launch_select(sa, st);
   c->mark(6, st);
@@ -797,7 +824,7 @@ int misat_create(const misat_config* cfg, void* cuda_stream, misat_ctx** out) {
   if (cudaGetDevice(&c->device) != cudaSuccess) return fail(MISAT_ERR_CUDA);
   if (cudaDeviceGetAttribute(&c->num_sms, cudaDevAttrMultiProcessorCount, c->device) != cudaSuccess)
     return fail(MISAT_ERR_CUDA);
-  if (select_configure() != cudaSuccess) return fail(MISAT_ERR_CUDA);
+  if (select_configure() != cudaSuccess || select_class_configure() != cudaSuccess) return fail(MISAT_ERR_CUDA);
   c->stream = (cudaStream_t)cuda_stream;
   c->W = W;
   c->cap.assign(cfg->cap_blocks, cfg->cap_blocks + W);
@@ -840,7 +867,8 @@ int misat_create(const misat_config* cfg, void* cuda_stream, misat_ctx** out) {
       (rc = dalloc_n(c, &c->d_bm_key, (size_t)1 << bm_log2)) ||
       (rc = dalloc_n(c, &c->d_bm_val, (size_t)1 << bm_log2)) || (rc = dalloc_n(c, &c->d_sel_rec, 2 * NB)) ||
       (rc = dalloc_n(c, &c->d_onhull, 3 * Ws)) || (rc = dalloc_n(c, &c->d_rank, Ws)) ||
-      (rc = dalloc_n(c, &c->d_rank_a, Ws)) ||
+      (rc = dalloc_n(c, &c->d_rank_a, Ws)) || (rc = dalloc_n(c, &c->d_sel_list, 3 * NB)) ||
+      (rc = dalloc_n(c, &c->d_sel_x, Ws + 2)) ||
       (rc = dalloc_n(c, &c->rq.nb, NB)) || (rc = dalloc_n(c, &c->rq.kbase, NB)) || (rc = dalloc_n(c, &c->rq.L, NB)) ||
       (rc = dalloc_n(c, &c->rq.cls, NB)) || (rc = dalloc_n(c, &c->rq.session, NB)) ||
       (rc = dalloc_n(c, &c->rq.sst, NB)) || (rc = dalloc_n(c, &c->rq.sinst, NB)) ||

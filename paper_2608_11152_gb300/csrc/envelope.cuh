@@ -51,9 +51,9 @@ constexpr int64_t kEnvSmall = (int64_t)1 << 25;
 
 // a < b as fractions; small: every |dbk| and |dtc| of the instance set is below 2^25
 MISAT_HD bool env_frac_lt(const EnvFrac& a, const EnvFrac& b, bool small) {
-  if (small) {
-    const int64_t d1 = a.dbk * b.dtc - b.dbk * a.dtc;
-    const int64_t d2 = a.dw * b.dtc - b.dw * a.dtc;
+  if (small) {  // every factor fits in 32 bits: one widening multiply per product
+    const int64_t d1 = (int64_t)(int32_t)a.dbk * (int32_t)b.dtc - (int64_t)(int32_t)b.dbk * (int32_t)a.dtc;
+    const int64_t d2 = (int64_t)(int32_t)a.dw * (int32_t)b.dtc - (int64_t)(int32_t)b.dw * (int32_t)a.dtc;
     return 1024 * d1 + d2 < 0;
   }
   const __int128 na = (__int128)a.dbk * 1024 + a.dw, nb = (__int128)b.dbk * 1024 + b.dw;

@@ -118,7 +118,8 @@ struct RouteParams {
 void launch_route_params(const RouteParams& p, int64_t* dst, cudaStream_t st);
 
 // ---- serial selection (select.cu) ----
-constexpr int kSelectThreads = 512;  // leaders per window of the selection CTA
+constexpr int kSelectThreads = 512;        // leaders per window of the joint selection CTA
+constexpr int kSelectClassThreads = 512;   // leaders per window of a per-class selection CTA
 
 struct SelectPrepArgs {
   int32_t n;
@@ -126,6 +127,9 @@ struct SelectPrepArgs {
   ReqArrays rq;
   const uint16_t* H;
   int4* rec;                   // [2n] per-request records of the selection
+  int32_t* adm;                // [W] zeroed here: admissions per instance of the per-class path
+  unsigned* ticket;            // zeroed here
+  int32_t* coupled;            // zeroed here
   const int32_t* err;
 };
 void launch_select_prep(const SelectPrepArgs& a, cudaStream_t st);
@@ -159,11 +163,39 @@ struct SelectArgs {
   const uint16_t* H;           // [n*W]
   int64_t hold_delay_q;
   bool small;                  // as EnvInitArgs::small
+  const int32_t* coupled;      // the joint selection runs only when the per-class path set this
   int32_t* err;
 };
 size_t select_smem_bytes(int W);
 cudaError_t select_configure();  // per device, before the first launch: shared memory of the selection CTA
 void launch_select(const SelectArgs& a, cudaStream_t st);
+
+// Per-class selection (one CTA per class), valid while no instance runs out of global
+// headroom; otherwise it sets *coupled and launch_select decides the batch.
+struct SelectClassArgs {
+  int32_t n;
+  int32_t W;
+  const int4* rec;             // [2n] from launch_select_prep
+  ReqArrays rq;                // out: status, inst, reason, last_reason of every leader
+  const int32_t* gh;           // [W] global headroom at batch start
+  const int32_t* ch;           // [W*3] class headroom at batch start
+  const int64_t* backlog;      // [W] d_w
+  const int64_t* tokcost;      // [W] 1/mu_w
+  const uint8_t* onhull;       // [3*W] initial envelopes (launch_env_init)
+  const int32_t* rank;         // [W] slope order (launch_env_init)
+  const int32_t* rank_a;       // [W] (d_w, w) order (launch_env_init)
+  const uint16_t* H;           // [n*W]
+  int64_t hold_delay_q;
+  bool small;                  // as EnvInitArgs::small
+  int32_t* list;               // [3n] scratch: each class's leaders in arrival order
+  int32_t* adm;                // [W] zeroed by launch_select_prep
+  unsigned* ticket;            // zeroed by launch_select_prep
+  int32_t* coupled;            // zeroed by launch_select_prep; set when the joint kernel must run
+  int32_t* err;
+};
+size_t select_class_smem_bytes(int W);
+cudaError_t select_class_configure();
+void launch_select_class(const SelectClassArgs& a, cudaStream_t st);
 
 struct FinalizeArgs {
   int32_t n;

@@ -44,6 +44,13 @@ static_assert(kNW == 16 && kSlotInst == 8, "one thread per (counter, warp) in th
 //   rec[2r]   = {L, cls | sst << 8 | leader << 16, protected / last instance, hbest}
 //   rec[2r+1] = {instances with H > 0, first two of them as (w << 16 | H), 0}
 __global__ void __launch_bounds__(256) k3_select_prep(SelectPrepArgs a) {
+  if (blockIdx.x == 0) {
+    for (int w = threadIdx.x; w < a.W; w += blockDim.x) a.adm[w] = 0;
+    if (threadIdx.x == 0) {
+      *a.ticket = 0;
+      *a.coupled = 0;
+    }
+  }
   if (block_error(a.err)) return;
   const int r = blockIdx.x * blockDim.x + threadIdx.x;
   if (r >= a.n) return;
@@ -419,6 +426,8 @@ __global__ void __launch_bounds__(kNT, 1) k4_select(SelectArgs a) {
   __shared__ unsigned s_lead[kNW], s_sens[kNW];
   __shared__ EnvScratch s_env[3];
   if (block_error(a.err)) return;
+  // the per-class path decided the batch unless it raised the flag (no flag: always run)
+  if (a.coupled != nullptr && *(volatile const int32_t*)a.coupled == 0) return;
   const int W = a.W;
   const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
   SelSmem s;
@@ -657,8 +666,9 @@ __global__ void __launch_bounds__(kNT, 1) k4_select(SelectArgs a) {
           a.rq.status[i] = kStResolved;
           a.rq.inst[i] = dw;
           a.rq.reason[i] = dec;
-        } else {
+        } else {  // (inst may hold an admission of the per-class path, which this replaces)
           a.rq.status[i] = kStHeld;
+          a.rq.inst[i] = -1;
           a.rq.last_reason[i] = dec;
         }
       } else if (have && dec == MISAT_ADMIT_NEW && !s.av[b * W + dw]) {
@@ -693,6 +703,597 @@ cudaError_t select_configure() {
 void launch_select(const SelectArgs& a, cudaStream_t st) {
   if (a.n <= 0) return;
   k4_select<<<1, kNT, select_smem_bytes(a.W), st>>>(a);
+}
+
+// ---------------------------------------------------------------------------
+// Per-class selection: the path taken when no instance runs out of global headroom.
+//
+// A leader of class b is eligible on w when w has global headroom and class-b headroom
+// (Eq. 6 with the class cap of Sec. 4.2).  As long as every instance keeps global headroom,
+// eligibility depends only on the admissions of the leader's own class, so the leaders of the
+// three classes form three independent chains.  One CTA per class decides its class's leaders
+// in arrival order with the window scheme of k4_select, on one envelope and per-instance
+// counters.  At the end the CTAs add up their admissions per instance: if every instance that
+// had global headroom at batch start keeps some, no decision could have depended on the global
+// cap, and the result is exactly that of the joint arrival order (by induction over the arrival
+// order: each instance's global headroom stays positive at every leader's turn, so the joint
+// eligibility equals the per-class one, and a hold's reason -- class cap while some instance
+// has global headroom -- is the class cap exactly when some instance had it at batch start).
+// Otherwise the last CTA sets `coupled` and k4_select decides the whole batch again.
+//
+// Within a window a tentative admission is final once the registered choosers of its
+// instance before it leave it headroom; the first leader that finds none cuts the window.
+// Exact cut positions come from per-instance ballots over the window's choices (one warp per
+// over-subscribed instance).  An instance that runs out leaves the envelope by a local repair
+// (the lines between its neighbours that lie below their chord, envelope.cuh), and only the
+// leaders that had chosen it choose again.
+namespace {
+constexpr int kCT = kSelectClassThreads;
+constexpr int kCW = kCT / 32;
+static_assert(kCW <= 32 && (kCW & (kCW - 1)) == 0, "the window bitmask is at most one word per lane of a warp");
+}  // namespace
+
+struct ClsSmem {
+  int16_t* chs;    // [kCT] registered choice of each window slot, -1 (16-byte aligned)
+  longlong2* ln;   // [W] {d_w, 1/mu_w}
+  longlong2* hl;   // [W] {d_w, 1/mu_w} of the envelope lines, slope order
+  longlong2* tl;   // [W] scratch of the envelope repair
+  int32_t* ch;     // [W] class headroom (0 for an instance without global headroom)
+  int32_t* T;      // [W] registered choosers in the window
+  int32_t* fpos;   // [W] window slot of the chooser that takes an instance's last headroom, kCT
+  int32_t* cand;   // [W] envelope repair candidates
+  int32_t* rem;    // [W] instances that ran out in this iteration
+  int16_t* hull;   // [W] envelope lines, slope order
+  int16_t* th;     // [W] scratch of the envelope repair
+  int16_t* hp;     // [W] position of an instance on the envelope, -1 if it is not on it
+  int16_t* ord;    // [W] instances in slope order
+  int16_t* pos;    // [W] position in slope order
+  int16_t* aord;   // [W] instances in (d_w, w) order
+  uint8_t* av;     // [W] class headroom left
+  unsigned* tm;    // [32] "tight" instances: registered choosers >= class headroom > 0
+};
+
+size_t select_class_smem_bytes(int W) {
+  return (size_t)kCT * 2 + 128 + (size_t)W * (16 * 3 + 4 * 5 + 2 * 6 + 1) + 64;
+}
+
+// First set position >= from in a kCT-bit mask held one word per lane (kCT if none).  Warp-uniform.
+__device__ __forceinline__ int cls_first_set(unsigned word, int lane, int from) {
+  if (from >= kCT) return kCT;
+  const int fw = from >> 5;
+  unsigned m = lane < fw ? 0u : word;
+  if (lane == fw) m &= ~0u << (from & 31);
+  const unsigned nz = __ballot_sync(kFull, m != 0);
+  if (!nz) return kCT;
+  const int w = __ffs(nz) - 1;
+  return w * 32 + __ffs(__shfl_sync(kFull, m, w)) - 1;
+}
+
+// Position of the (k+1)-th set bit of m (k < popc(m)).
+__device__ __forceinline__ int nth_set(unsigned m, int k) {
+  for (int i = 0; i < k; ++i) m &= m - 1;
+  return __ffs(m) - 1;
+}
+
+// Decision of one leader of the CTA's class against the current state; see sel_choose.
+__device__ __forceinline__ int cls_choose(const ClsSmem& s, int m, int nglobal, int64_t x, int sst, int pw,
+                                          uint32_t hb, int nh, uint32_t h0, uint32_t h1, const uint16_t* Hrow,
+                                          int W, int64_t hold, uint8_t* dec) {
+  int64_t best_c = INT64_MAX;
+  int best_w = INT32_MAX;
+  if (m > 0) {
+    int lo = 0, hi = m - 1;
+    while (lo < hi) {
+      const int mid = (lo + hi) >> 1;
+      const longlong2 u = s.hl[mid], v = s.hl[mid + 1];
+      const int64_t cu = u.x + x * u.y, cv = v.x + x * v.y;
+      // line mid + 1 beats line mid at x (ties to the lower index)
+      if (cv < cu || (cv == cu && s.hull[mid + 1] < s.hull[mid])) lo = mid + 1;
+      else hi = mid;
+    }
+    const longlong2 t = s.hl[lo];
+    best_w = s.hull[lo];
+    best_c = t.x + x * t.y;
+  }
+  auto consider = [&](int w, int64_t h) {
+    const longlong2 t = s.ln[w];
+    const int64_t c = t.x + (x - 16 * h) * t.y;
+    if (c < best_c || (c == best_c && w < best_w)) {
+      best_c = c;
+      best_w = w;
+    }
+  };
+  if (nh > 0 && nh <= 2) {
+    const int w0 = (int)(h0 >> 16);
+    if (s.av[w0] || w0 == pw) consider(w0, h0 & 0xffff);
+    if (nh == 2) {
+      const int w1 = (int)(h1 >> 16);
+      if (s.av[w1] || w1 == pw) consider(w1, h1 & 0xffff);
+    }
+  } else if (nh > 2) {
+    for (int w = 0; w < W; ++w) {
+      const int h = Hrow[w];
+      if (h && (s.av[w] || w == pw)) consider(w, h);
+    }
+  }
+  if (pw >= 0) consider(pw, 0);
+  if (best_w == INT32_MAX) {
+    *dec = nglobal > 0 ? MISAT_HOLD_CLASS_CAP : MISAT_HOLD_GLOBAL_CAP;
+    return -1;
+  }
+  const int hmax = (int)(hb >> 16), whit = 65535 - (int)(hb & 0xffffu);
+  if (sst == kSessReleased && hmax > 0 && !s.av[whit]) {
+    const int64_t lhs = hold + s.ln[whit].x - s.ln[best_w].x;
+    const int64_t rhs = 16 * (int64_t)hmax * s.ln[whit].y;
+    if (lhs < rhs) {
+      *dec = MISAT_HOLD_PREFER_CACHE;
+      return -1;
+    }
+  }
+  *dec = best_w == pw ? MISAT_ADMIT_CONT : MISAT_ADMIT_NEW;
+  return best_w;
+}
+
+__device__ __forceinline__ bool cls_present(const ClsSmem& s, int i) { return s.av[i] || s.hp[i] >= 0; }
+
+// Envelope repair after instance w ran out of headroom (one warp).  The lines p and q that bound
+// the repaired stretch are w's neighbours on the envelope, or, where w was the first (last)
+// line, the line that now wins at x = 0 (for large x).  The lines strictly between p and q in
+// slope order that lie below the chord p-q are the candidates; each is tested against p, q and
+// the other candidates (EnvTest over the domain x >= 0), and the ones on the envelope replace
+// w.  A line that ran out in the same iteration but is still on the envelope counts as present
+// until its own repair, so that every repair computes the envelope of a well-defined set; the
+// order of the repairs does not change the final envelope.  first_a / last_s: forward-only
+// pointers to the lines that may win at x = 0 ((d_w, w) order) and for large x (slope order).
+__device__ __forceinline__ void cls_repair(const ClsSmem& s, int W, int w, int* hm, int* first_a, int* last_s,
+                                           bool small) {
+  const int lane = threadIdx.x & 31;
+  const int k = s.hp[w];
+  __syncwarp();
+  if (k < 0) return;
+  if (lane == 0) s.hp[w] = -1;
+  __syncwarp();
+  const int m = *hm;
+  const int P = k > 0 ? s.hull[k - 1] : -1, Q = k + 1 < m ? s.hull[k + 1] : -1;
+  int p = P, q = Q;
+  if (p < 0) {  // the line that now wins at x = 0
+    int a = *first_a;
+    while (a < W && !cls_present(s, s.aord[a])) ++a;
+    p = a < W ? s.aord[a] : -1;
+    __syncwarp();
+    if (lane == 0) *first_a = a;
+  }
+  if (q < 0 && p >= 0) {  // the line that now wins for large x: least 1/mu_w, then least d_w
+    int x = *last_s;
+    while (x >= 0 && !cls_present(s, s.ord[x])) --x;
+    __syncwarp();
+    if (lane == 0) *last_s = x;
+    const int64_t t = s.ln[s.ord[x]].y;
+    int y = x;
+    for (int z = x - 1; z >= 0 && s.ln[s.ord[z]].y == t; --z)
+      if (cls_present(s, s.ord[z])) y = z;
+    q = s.ord[y];
+  }
+  int nnew = 0;
+  if (P < 0 && p >= 0 && p != Q) {
+    if (lane == 0) s.th[0] = (int16_t)p;
+    nnew = 1;
+  }
+  if (p >= 0 && q != p) {
+    const int xp = s.pos[p], xq = s.pos[q];
+    const longlong2 lp = s.ln[p], lq = s.ln[q];
+    int nc = 0;
+    for (int x0 = xp + 1; x0 < xq; x0 += 32) {
+      const int x = x0 + lane;
+      bool c = false;
+      int i = 0;
+      if (x < xq) {
+        i = s.ord[x];
+        if (s.av[i]) {
+          const longlong2 li = s.ln[i];
+          c = li.y != lp.y && env_below_chord(li.x, li.y, i, lp.x, lp.y, p, lq.x, lq.y, q, small);
+        }
+      }
+      const unsigned mc = __ballot_sync(kFull, c);
+      if (c) s.cand[nc + __popc(mc & lanemask_lt())] = i;
+      nc += __popc(mc);
+    }
+    __syncwarp();
+    for (int e0 = 0; e0 < nc; e0 += 32) {
+      const int e = e0 + lane;
+      bool on = false;
+      int i = 0;
+      if (e < nc) {
+        i = s.cand[e];
+        const longlong2 li = s.ln[i];
+        EnvTest t;
+        env_test_init(t);
+        env_test_add(t, li.x, li.y, i, lp.x, lp.y, p, small);
+        env_test_add(t, li.x, li.y, i, lq.x, lq.y, q, small);
+        for (int f = 0; f < nc; ++f) {
+          const int j = s.cand[f];
+          if (j != i) {
+            const longlong2 lj = s.ln[j];
+            env_test_add(t, li.x, li.y, i, lj.x, lj.y, j, small);
+          }
+        }
+        on = env_test_on(t, small);
+      }
+      const unsigned mo = __ballot_sync(kFull, on);
+      if (on) s.th[nnew + __popc(mo & lanemask_lt())] = (int16_t)i;
+      nnew += __popc(mo);
+    }
+    if (Q < 0 && q != P) {
+      if (lane == 0) s.th[nnew] = (int16_t)q;
+      nnew += 1;
+    }
+  }
+  __syncwarp();
+  // splice: hull[0..k-1] ++ th[0..nnew-1] ++ hull[k+1..m-1]
+  const int tail = m - k - 1;
+  for (int t = lane; t < tail; t += 32) {
+    s.th[nnew + t] = s.hull[k + 1 + t];
+    s.tl[nnew + t] = s.hl[k + 1 + t];
+  }
+  for (int t = lane; t < nnew; t += 32) s.tl[t] = s.ln[s.th[t]];
+  __syncwarp();
+  const int total = nnew + tail;
+  for (int t = lane; t < total; t += 32) {
+    const int v = s.th[t];
+    s.hull[k + t] = (int16_t)v;
+    s.hl[k + t] = s.tl[t];
+    s.hp[v] = (int16_t)(k + t);
+  }
+  if (lane == 0) *hm = k + total;
+  __syncwarp();
+}
+
+__global__ void __launch_bounds__(kCT, 1) k4_select_class(SelectClassArgs a) {
+  extern __shared__ __align__(16) unsigned char smem[];
+  __shared__ int s_nc, s_q, s_hm, s_first_a, s_last_s, s_nglobal, s_last;
+  __shared__ int s_ws[kCW];
+  __shared__ unsigned s_lead[kCW], s_sens[kCW];
+  if (block_error(a.err)) return;
+  const int W = a.W, b = blockIdx.x;
+  const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
+  ClsSmem s;
+  {
+    unsigned char* p = smem;
+    s.chs = reinterpret_cast<int16_t*>(p);
+    p += (size_t)kCT * 2;
+    s.tm = reinterpret_cast<unsigned*>(p);
+    p += 128;
+    s.ln = reinterpret_cast<longlong2*>(p);
+    p += (size_t)W * 16;
+    s.hl = reinterpret_cast<longlong2*>(p);
+    p += (size_t)W * 16;
+    s.tl = reinterpret_cast<longlong2*>(p);
+    p += (size_t)W * 16;
+    s.ch = reinterpret_cast<int32_t*>(p);
+    p += (size_t)W * 4;
+    s.T = reinterpret_cast<int32_t*>(p);
+    p += (size_t)W * 4;
+    s.fpos = reinterpret_cast<int32_t*>(p);
+    p += (size_t)W * 4;
+    s.cand = reinterpret_cast<int32_t*>(p);
+    p += (size_t)W * 4;
+    s.rem = reinterpret_cast<int32_t*>(p);
+    p += (size_t)W * 4;
+    s.hull = reinterpret_cast<int16_t*>(p);
+    p += (size_t)W * 2;
+    s.th = reinterpret_cast<int16_t*>(p);
+    p += (size_t)W * 2;
+    s.hp = reinterpret_cast<int16_t*>(p);
+    p += (size_t)W * 2;
+    s.ord = reinterpret_cast<int16_t*>(p);
+    p += (size_t)W * 2;
+    s.pos = reinterpret_cast<int16_t*>(p);
+    p += (size_t)W * 2;
+    s.aord = reinterpret_cast<int16_t*>(p);
+    p += (size_t)W * 2;
+    s.av = p;
+  }
+  if (tid == 0) {
+    s_nglobal = 0;
+    s_q = kCT;
+    s_first_a = 0;
+    s_last_s = W - 1;
+  }
+  __syncthreads();
+  for (int w = tid; w < W; w += kCT) {
+    const int r = a.rank[w];
+    s.ord[r] = (int16_t)w;
+    s.pos[w] = (int16_t)r;
+    s.aord[a.rank_a[w]] = (int16_t)w;
+    s.ln[w] = make_longlong2(a.backlog[w], a.tokcost[w]);
+    const int g = a.gh[w];
+    if (g > 0) atomicAdd(&s_nglobal, 1);
+    const int c = g > 0 ? a.ch[w * 3 + b] : 0;
+    s.ch[w] = c;
+    s.av[w] = c > 0;
+    s.T[w] = 0;
+    s.fpos[w] = kCT;
+    s.hp[w] = -1;
+  }
+  s.chs[tid] = -1;
+  if (tid < 32) s.tm[tid] = 0;
+  __syncthreads();
+  // initial envelope of the class (launch_env_init), compacted in slope order
+  if (wid == 0) {
+    int base = 0;
+    for (int x0 = 0; x0 < W; x0 += 32) {
+      const int x = x0 + lane;
+      const int w = x < W ? s.ord[x] : 0;
+      const bool f = x < W && a.onhull[b * W + w];
+      const unsigned mf = __ballot_sync(kFull, f);
+      if (f) {
+        const int k = base + __popc(mf & lanemask_lt());
+        s.hull[k] = (int16_t)w;
+        s.hl[k] = s.ln[w];
+        s.hp[w] = (int16_t)k;
+      }
+      base += __popc(mf);
+    }
+    if (lane == 0) s_hm = base;
+  }
+  // The class's leaders in arrival order.  A request is a leader iff its status is not
+  // kStFollower; the other CTAs only turn leaders' statuses into decisions, so the test is
+  // stable while they run.  Each thread takes 8 consecutive requests per pass.
+  int32_t* lst = a.list + (int64_t)b * a.n;
+  int nc = 0;
+  for (int c0 = 0; c0 < a.n; c0 += 8 * kCT) {
+    const int r0 = c0 + 8 * tid;
+    uint32_t fm = 0;
+    if (r0 + 8 <= a.n) {
+      const uint2 cl = *reinterpret_cast<const uint2*>(a.rq.cls + r0);
+      const uint2 st = *reinterpret_cast<const uint2*>(a.rq.status + r0);
+#pragma unroll
+      for (int u = 0; u < 8; ++u) {
+        const uint32_t cu = ((u < 4 ? cl.x : cl.y) >> (8 * (u & 3))) & 0xff;
+        const uint32_t su = ((u < 4 ? st.x : st.y) >> (8 * (u & 3))) & 0xff;
+        if (cu == (uint32_t)b && su != kStFollower) fm |= 1u << u;
+      }
+    } else {
+      for (int u = 0; u < 8 && r0 + u < a.n; ++u)
+        if (a.rq.cls[r0 + u] == b && a.rq.status[r0 + u] != kStFollower) fm |= 1u << u;
+    }
+    const int cnt = __popc(fm);
+    int incl = cnt;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int t = __shfl_up_sync(kFull, incl, o);
+      if (lane >= o) incl += t;
+    }
+    if (lane == 31) s_ws[wid] = incl;
+    __syncthreads();
+    if (wid == 0) {
+      const int v = lane < kCW ? s_ws[lane] : 0;
+      int wi = v;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const int t = __shfl_up_sync(kFull, wi, o);
+        if (lane >= o) wi += t;
+      }
+      if (lane < kCW) s_ws[lane] = wi - v;
+      if (lane == 31) s_nc = wi;
+    }
+    __syncthreads();
+    int off = nc + s_ws[wid] + incl - cnt;
+    for (uint32_t t = fm; t; t &= t - 1) lst[off++] = r0 + __ffs(t) - 1;
+    nc += s_nc;
+    __syncthreads();
+  }
+  const int nglobal = s_nglobal;
+
+  // records of the first window
+  int rn = tid < nc ? lst[tid] : 0;
+  int4 n0 = make_int4(0, 0, 0, 0), n1 = make_int4(0, 0, 0, 0);
+  if (tid < nc) {
+    n0 = a.rec[2 * rn];
+    n1 = a.rec[2 * rn + 1];
+  }
+#pragma unroll 1
+  for (int base = 0; base < nc; base += kCT) {
+    const int i = base + tid;
+    const bool valid = i < nc;
+    const int r = rn;
+    const int4 r0 = n0, r1 = n1;
+    if (i + kCT < nc) {  // the next window's records, in flight during this one
+      rn = lst[i + kCT];
+      n0 = a.rec[2 * rn];
+      n1 = a.rec[2 * rn + 1];
+    }
+    const int64_t L = r0.x;
+    const int sst = (r0.y >> 8) & 0xff;
+    const int pw = sst == (int)kSessProtected ? r0.z : -1;
+    const uint32_t hb = (uint32_t)r0.w;
+    const int nh = r1.x;
+    const uint32_t h0 = (uint32_t)r1.y, h1 = (uint32_t)r1.z;
+    const bool sens = valid && sst == (int)kSessReleased && (hb >> 16) > 0;
+    {
+      const unsigned ml = __ballot_sync(kFull, valid), ms = __ballot_sync(kFull, sens);
+      if (lane == 0) {
+        s_lead[wid] = ml;
+        s_sens[wid] = ms;
+      }
+    }
+    __syncthreads();
+    const unsigned lead_word = lane < kCW ? s_lead[lane] : 0u;
+    const unsigned sens_word = lane < kCW ? s_sens[lane] : 0u;
+    int done = 0;
+    bool have = false, reg = false;
+    uint8_t dec = 0;
+    int dw = -1;
+    int guard = 0;
+#pragma unroll 1
+    while (true) {
+      const int head = cls_first_set(lead_word, lane, done);
+      if (head == kCT) break;
+      if (++guard > 2 * kCT) {  // every iteration decides at least the leader at `head`
+        if (tid == 0) set_error(a.err, MISAT_ERR_INTERNAL);
+        return;
+      }
+      // an Eq. (7) leader is decided alone, at the head, against the exact state of its turn
+      const int qcut = max(cls_first_set(sens_word, lane, head), head + 1);
+      const bool act = valid && tid >= head && tid < qcut;
+      // 1. a registered choice whose instance ran out is taken again; choices and registration
+      if (reg && !s.av[dw]) {
+        atomicSub(&s.T[dw], 1);
+        s.chs[tid] = -1;
+        reg = false;
+        have = false;
+      }
+      if (act && !have) {
+        dw = cls_choose(s, s_hm, nglobal, L, sst, pw, hb, nh, h0, h1, a.H + (int64_t)r * W, W, a.hold_delay_q, &dec);
+        have = true;
+        if (dec == MISAT_ADMIT_NEW) {
+          reg = true;
+          if (atomicAdd(&s.T[dw], 1) + 1 >= s.ch[dw]) atomicOr(&s.tm[dw >> 5], 1u << (dw & 31));
+          s.chs[tid] = (int16_t)dw;
+        }
+      }
+      __syncthreads();
+      // 2. instances with as many registered choosers as headroom (or more): the slot of the
+      //    chooser that takes the last headroom (fpos) and of the first one that finds none
+      //    (the cut); the k-th such instance goes to warp k mod kCW.  The tight set is kept
+      //    exactly: a registration that reaches the headroom adds its instance, and an instance
+      //    leaves it only when it runs out (a decided prefix lowers both counts alike).
+      {
+        const unsigned word = s.tm[lane];
+        const unsigned nzw = __ballot_sync(kFull, word != 0);
+        int seen = 0;
+        for (unsigned zz = nzw; zz; zz &= zz - 1) {
+          const int wi = __ffs(zz) - 1;
+          const unsigned bits = __shfl_sync(kFull, word, wi);
+          unsigned mine = 0;
+          for (unsigned t = bits; t; t &= t - 1) {
+            if ((seen & (kCW - 1)) == wid) mine |= t & (0u - t);
+            ++seen;
+          }
+          while (mine) {
+            const int w = 32 * wi + __ffs(mine) - 1;
+            mine &= mine - 1;
+            const int need = s.ch[w];
+            // lane j counts the registered choosers of w among slots [kSL j, kSL (j + 1))
+            constexpr int kSL = kCT / 32;
+            int c = 0;
+            const int4* v = reinterpret_cast<const int4*>(s.chs + kSL * lane);
+#pragma unroll
+            for (int u = 0; u < kSL / 8; ++u) {
+              const int4 z = v[u];
+              const int zv[4] = {z.x, z.y, z.z, z.w};
+#pragma unroll
+              for (int h = 0; h < 4; ++h) c += ((int16_t)(zv[h] & 0xffff) == w) + ((zv[h] >> 16) == w);
+            }
+            int incl = c;
+#pragma unroll
+            for (int o = 1; o < 32; o <<= 1) {
+              const int t = __shfl_up_sync(kFull, incl, o);
+              if (lane >= o) incl += t;
+            }
+            // slot of the k-th (1-based) registered chooser of w, kCT if there are fewer
+            auto kth_slot = [&](int k) -> int {
+              const unsigned mx = __ballot_sync(kFull, incl >= k);
+              if (!mx) return kCT;
+              const int l = __ffs(mx) - 1;
+              const int before = __shfl_sync(kFull, incl - c, l);
+              const unsigned mb = __ballot_sync(kFull, lane < kSL && s.chs[kSL * l + lane] == w);
+              return kSL * l + (int)__fns(mb, 0, k - before);
+            };
+            const int f = kth_slot(need);
+            const int p = kth_slot(need + 1);
+            if (lane == 0) {
+              s.fpos[w] = f;
+              if (p < kCT) atomicMin(&s_q, p);
+            }
+          }
+        }
+      }
+      __syncthreads();
+      const int q = min(s_q, qcut);
+      // 3. the leaders before q are decided; warp 0 then takes the instances whose last
+      //    headroom went to one of them out of the envelope
+      if (act && tid < q) {
+        if (dec == MISAT_ADMIT_NEW || dec == MISAT_ADMIT_CONT) {
+          a.rq.status[r] = kStResolved;
+          a.rq.inst[r] = dw;
+          a.rq.reason[r] = dec;
+        } else {
+          a.rq.status[r] = kStHeld;
+          a.rq.inst[r] = -1;
+          a.rq.last_reason[r] = dec;
+        }
+        if (reg) {
+          atomicSub(&s.T[dw], 1);
+          atomicSub(&s.ch[dw], 1);
+          s.chs[tid] = -1;
+          reg = false;
+        }
+      }
+      if (wid == 0) {
+        int nrem = 0;
+        const unsigned word = s.tm[lane];
+        unsigned keep = word;
+        for (unsigned t = word; t; t &= t - 1) {  // lane-local: the tight instances of word `lane`
+          const int w = 32 * lane + __ffs(t) - 1;
+          const int f = s.fpos[w];
+          s.fpos[w] = kCT;
+          if (f < q) keep &= ~(t & (0u - t));
+        }
+        const unsigned out = word & ~keep;
+        s.tm[lane] = keep;
+        // instances that ran out, in index order
+        int cnt = __popc(out), excl = cnt;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+          const int v = __shfl_up_sync(kFull, excl, o);
+          if (lane >= o) excl += v;
+        }
+        nrem = __shfl_sync(kFull, excl, 31);
+        excl -= cnt;
+        for (unsigned t = out; t; t &= t - 1) {
+          const int w = 32 * lane + __ffs(t) - 1;
+          s.av[w] = 0;
+          s.rem[excl++] = w;
+        }
+        __syncwarp();
+        for (int e = 0; e < nrem; ++e) cls_repair(s, W, s.rem[e], &s_hm, &s_first_a, &s_last_s, a.small);
+      }
+      __syncthreads();
+      if (tid == 0) s_q = kCT;  // read by every thread before the barrier above
+      done = q;
+    }
+    __syncthreads();  // s_lead / s_sens are rewritten by the next window
+  }
+  // admissions per instance, and the check that no instance ran out of global headroom
+  for (int w = tid; w < W; w += kCT) {
+    const int c0 = a.gh[w] > 0 ? a.ch[w * 3 + b] : 0;
+    const int used = c0 - s.ch[w];
+    if (used) atomicAdd(&a.adm[w], used);
+  }
+  __threadfence();
+  __syncthreads();
+  if (tid == 0) s_last = atomicAdd(a.ticket, 1u) == gridDim.x - 1;
+  __syncthreads();
+  if (s_last) {
+    __threadfence();
+    bool bad = false;
+    for (int w = tid; w < W; w += kCT) {
+      const int g = a.gh[w];
+      if (g > 0 && __ldcg(&a.adm[w]) >= g) bad = true;
+    }
+    if (__syncthreads_or(bad) && tid == 0) *a.coupled = 1;
+  }
+}
+
+cudaError_t select_class_configure() {
+  return cudaFuncSetAttribute(k4_select_class, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                              (int)select_class_smem_bytes(kMaxW));
+}
+
+void launch_select_class(const SelectClassArgs& a, cudaStream_t st) {
+  if (a.n <= 0) return;
+  k4_select_class<<<3, kCT, select_class_smem_bytes(a.W), st>>>(a);
 }
 
 }  // namespace misat
