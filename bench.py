@@ -637,7 +637,7 @@ def run_gb300(args):
     phase_ms = {p: phase_tot[p] / KP for p in phase_tot}
     # one kernel per phase below (the insert phase adds the small work-list kernel)
     KERNEL_NAMES = {"hash": "k1_block_hash", "probe_first": "k2_probe_first_gix" if gidx else "k2_probe_first_group",
-                    "probe_search": "k2_probe_search", "select": "k4_select", "insert": "k4_insert",
+                    "probe_search": "k2_probe_search", "select": "k4_select_class", "insert": "k4_insert",
                     "gix_insert": "k4_gix_insert", "evict_collect": "k4_evict_collect",
                     "evict_delete": "k4_evict_delete", "evict_shift": "k4_evict_shift"}
 
@@ -659,8 +659,8 @@ def run_gb300(args):
             # the kernel's actual limiter: integer ALU issue (ncu sm__pipe_alu_cycles_active)
             kernels["hash"]["alu_pipe_active_frac_ncu"] = float(hf["alu_pipe_active_frac"])
     if kernels["select"] is not None:
-        kernels["select"]["limiter"] = ("one CTA walks the batch in arrival order; bound by the chain of "
-                                        "headroom-exhaustion events, not by memory")
+        kernels["select"]["limiter"] = ("one CTA per class walks its leaders in arrival order; bound by the "
+                                        "chain of headroom-exhaustion events (barrier-separated steps), not by memory")
     # dominant kernel: the largest time per launch
     dom = max((k for k in kernels if kernels[k]), key=lambda k: kernels[k]["ms_per_launch"])
     dom_roof = dict(kernels[dom])
