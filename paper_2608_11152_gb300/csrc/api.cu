@@ -135,6 +135,9 @@ struct misat_ctx {
   int32_t* d_rank_a = nullptr;   // (d_w, w) order of the instances [W]
   int32_t* d_sel_list = nullptr; // [3 max_batch] each class's leaders (per-class selection)
   int32_t* d_sel_x = nullptr;    // [W + 2] admissions per instance, ticket, coupled flag
+  ulonglong2* d_grp = nullptr;   // (first key, instance) groups of a route's admitted requests
+  uint32_t grp_log2 = 1;
+  int32_t* d_skip = nullptr;     // [max_batch] leading blocks a later request of the group inserts
   // every d_w and every 1/mu_w below 2^25: the selection's envelope arithmetic fits in 64 bits
   bool bk_small = true, tc_small = true;
   int32_t* d_chain_max = nullptr;  // per-chain insert limits of misat_load_chains
@@ -601,6 +604,7 @@ void enqueue_route(misat_ctx* c, const misat_batch* b, misat_decisions* out, cud
   const int bm_log2 = std::max(1, ceil_log2(2 * (uint64_t)n));
   cudaMemsetAsync(c->d_bm_key, 0, ((size_t)1 << bm_log2) * 8, st);
   cudaMemsetAsync(c->d_bm_val, 0x7f, ((size_t)1 << bm_log2) * 4, st);
+  cudaMemsetAsync(c->d_grp, 0, ((size_t)1 << bm_log2) * sizeof(ulonglong2), st);
 
   c->mark(0, st);
   PrologueArgs pa{};
@@ -731,6 +735,9 @@ void enqueue_route(misat_ctx* c, const misat_batch* b, misat_decisions* out, cud
   fa.out_hit = out->hit_blocks;
   fa.U = c->U_ptr();
   fa.stats = c->stats_ptr();
+  fa.grp = c->d_grp;
+  fa.grp_log2 = (uint32_t)bm_log2;
+  fa.keys = c->d_keys;
   fa.err = c->err_ptr();
   launch_finalize(fa, st);
   c->mark(7, st);
@@ -868,7 +875,8 @@ int misat_create(const misat_config* cfg, void* cuda_stream, misat_ctx** out) {
       (rc = dalloc_n(c, &c->d_bm_val, (size_t)1 << bm_log2)) || (rc = dalloc_n(c, &c->d_sel_rec, 2 * NB)) ||
       (rc = dalloc_n(c, &c->d_onhull, 3 * Ws)) || (rc = dalloc_n(c, &c->d_rank, Ws)) ||
       (rc = dalloc_n(c, &c->d_rank_a, Ws)) || (rc = dalloc_n(c, &c->d_sel_list, 3 * NB)) ||
-      (rc = dalloc_n(c, &c->d_sel_x, Ws + 2)) ||
+      (rc = dalloc_n(c, &c->d_sel_x, Ws + 2)) || (rc = dalloc_n(c, &c->d_skip, NB)) ||
+      (rc = dalloc_n(c, &c->d_grp, (size_t)1 << bm_log2)) ||
       (rc = dalloc_n(c, &c->rq.nb, NB)) || (rc = dalloc_n(c, &c->rq.kbase, NB)) || (rc = dalloc_n(c, &c->rq.L, NB)) ||
       (rc = dalloc_n(c, &c->rq.cls, NB)) || (rc = dalloc_n(c, &c->rq.session, NB)) ||
       (rc = dalloc_n(c, &c->rq.sst, NB)) || (rc = dalloc_n(c, &c->rq.sinst, NB)) ||
@@ -974,6 +982,7 @@ int misat_route(misat_ctx* c, const misat_batch* b, misat_decisions* out) {
   estimate_classes(c);
   c->last_n = n;
   c->last_ntok = b->n_tokens;
+  c->grp_log2 = (uint32_t)std::max(1, ceil_log2(2 * (uint64_t)std::max(n, 1)));  // as enqueue_route
   RouteParams prm{};
   for (int i = 0; i < 3; ++i) {
     prm.v[i] = c->kbar_b[i];
@@ -1261,6 +1270,9 @@ int misat_commit(misat_ctx* c) {
     ia.gnew = c->d_gnew;
     ia.n_gnew = c->d_gnew_n;
     ia.gnew_cap = c->keys_cap;
+    ia.grp = c->d_grp;
+    ia.grp_log2 = c->grp_log2;
+    ia.skip = c->d_skip;
     launch_insert_tables(ia, c->num_sms, st);
     c->mark(9);
     cudaEvent_t join = nullptr;

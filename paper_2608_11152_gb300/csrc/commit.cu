@@ -109,12 +109,13 @@ __device__ __forceinline__ void load_unit_keys(const UnitRec& u, int lane, uint6
 __global__ void __launch_bounds__(256) k4_units(InsertArgs a) {
   const int r = blockIdx.x * blockDim.x + threadIdx.x;
   const int lane = threadIdx.x & 31;
-  int u = 0, c = 0, w = 0;
+  int u = 0, c = 0, w = 0, s0 = 0;
   if (r < a.n && *a.err == 0 && a.inst[r] >= 0) {
     w = a.inst[r];
     c = a.nb[r];
     if (a.max_blocks && a.max_blocks[r] < c) c = a.max_blocks[r];
-    u = (c + kUnitBlocks - 1) / kUnitBlocks;
+    if (a.skip) s0 = min(a.skip[r], c);
+    u = (c - s0 + kUnitBlocks - 1) / kUnitBlocks;
   }
   int incl = u;
 #pragma unroll
@@ -140,7 +141,7 @@ __global__ void __launch_bounds__(256) k4_units(InsertArgs a) {
       set_error(a.err, MISAT_ERR_TABLE_FULL);
       break;
     }
-    const int j0 = i * kUnitBlocks;
+    const int j0 = s0 + i * kUnitBlocks;
     const int cnt = min(kUnitBlocks, c - j0);
     const uint64_t k0 = kp + 8ull * (uint64_t)j0;
     units[2 * ((int64_t)base + i)] = make_int4((int)(uint32_t)k0, (int)(uint32_t)(k0 >> 32), (int)(uint32_t)tp,
@@ -149,6 +150,56 @@ __global__ void __launch_bounds__(256) k4_units(InsertArgs a) {
         make_int4((int)(uint32_t)mhi, (int)(uint32_t)(mhi >> 32), j0,
                   (int)((uint32_t)w | (d.log2nb << 16) | ((uint32_t)(cnt - 1) << 24)));
   }
+}
+
+// Insert work that a later request does anyway.  Keys chain the whole prefix, so request r
+// and a later request r' of the same instance whose keys agree on blocks 0 .. p-1 insert the
+// same p keys at the same depths, and r' with the larger tick (same commit, later arrival):
+// after r' the index holds exactly what it holds after both, for every order of the atomics
+// (max-merged ticks, a key claimed once).  Per request, r' is the latest admitted request of
+// its (first key, instance) group (grp_note at route time), and skip[r] = p is the length of
+// the common prefix, compared key by key (one warp per request, 32 keys per step).  An agentic
+// turn and the next turn of its session, or two samples of one prompt, share their prefix.
+__global__ void __launch_bounds__(256) k4_dedup(InsertArgs a) {
+  const int r = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+  const int lane = threadIdx.x & 31;
+  if (r >= a.n) return;
+  int p = 0;
+  const int w = a.inst[r];
+  const int c = a.nb[r];
+  if (w >= 0 && c > 0 && *a.err == 0) {
+    const uint64_t* kr = a.keys + a.kbase[r];
+    const int last = grp_last(a.grp, a.grp_log2, __ldg(kr), w);
+    if (last > r) {
+      const uint64_t* kl = a.keys + a.kbase[last];
+      const int m = min(c, a.nb[last]);
+      p = m;
+      // 128 keys per step: four loads per lane in flight
+      for (int j0 = 0; j0 < m; j0 += 128) {
+        bool ne[4];
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+          const int j = j0 + 32 * k + lane;
+          ne[k] = j < m && __ldg(kr + j) != __ldg(kl + j);
+        }
+        unsigned first = 0;
+        int at = -1;
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+          const unsigned b = __ballot_sync(kFull, ne[k]);
+          if (at < 0 && b) {
+            first = b;
+            at = k;
+          }
+        }
+        if (at >= 0) {
+          p = j0 + 32 * at + __ffs(first) - 1;
+          break;
+        }
+      }
+    }
+  }
+  if (lane == 0) a.skip[r] = p;
 }
 
 __global__ void __launch_bounds__(kInsThreads, 3) k4_insert(InsertArgs a) {
@@ -254,6 +305,7 @@ void launch_insert_tables(const InsertArgs& a, int num_sms, cudaStream_t st) {
   if (a.n <= 0) return;
   cudaMemsetAsync(a.n_units, 0, sizeof(unsigned), st);
   if (a.gix.keys) cudaMemsetAsync(a.n_gnew, 0, sizeof(unsigned), st);
+  if (a.grp && a.skip) k4_dedup<<<(a.n + 7) / 8, 256, 0, st>>>(a);
   k4_units<<<(a.n + 255) / 256, 256, 0, st>>>(a);
   k4_insert<<<num_sms * 3, kInsThreads, 0, st>>>(a);  // resident CTAs: 3 per SM
 }

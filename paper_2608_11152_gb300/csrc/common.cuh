@@ -167,4 +167,48 @@ __device__ __forceinline__ int table_contains(const InstDesc& d, uint64_t key, u
   return 0;
 }
 
+// ---- groups of the admitted requests of a batch (commit work dedup) ----
+// Open-addressing table over (first block key, instance): per group the latest admitted
+// request.  Slot {key0, tag}: tag = (instance + 1) << 32 | (arrival + 1), 0 = empty.  A slot's
+// key is claimed first, then its instance; a slot whose instance differs is passed over, so
+// every (key0, instance) pair owns exactly one slot of its probe sequence.
+__device__ __forceinline__ uint32_t grp_home(uint64_t key0, int w, uint32_t log2n) {
+  return (uint32_t)(mix64(key0 ^ ((uint64_t)(w + 1) * kGold)) >> (64 - log2n));
+}
+
+__device__ __forceinline__ void grp_note(ulonglong2* tab, uint32_t log2n, uint64_t key0, int w, int r) {
+  const uint32_t mask = (1u << log2n) - 1;
+  uint32_t h = grp_home(key0, w, log2n);
+  for (uint32_t it = 0; it <= mask; ++it) {
+    unsigned long long* kp = &tab[h].x;
+    unsigned long long k = __ldcg(kp);
+    if (k == 0) {
+      k = atomicCAS(kp, 0ull, (unsigned long long)key0);
+      if (k == 0) k = key0;
+    }
+    if (k == key0) {
+      unsigned* tag = reinterpret_cast<unsigned*>(&tab[h].y);  // [0] arrival + 1, [1] instance + 1
+      const unsigned wv = atomicCAS(tag + 1, 0u, (unsigned)(w + 1));
+      if (wv == 0 || wv == (unsigned)(w + 1)) {
+        atomicMax(tag, (unsigned)(r + 1));
+        return;
+      }
+    }
+    h = (h + 1) & mask;
+  }
+}
+
+// The latest admitted request of group (key0, w), -1 if the group is not in the table.
+__device__ __forceinline__ int grp_last(const ulonglong2* tab, uint32_t log2n, uint64_t key0, int w) {
+  const uint32_t mask = (1u << log2n) - 1;
+  uint32_t h = grp_home(key0, w, log2n);
+  for (uint32_t it = 0; it <= mask; ++it) {
+    const ulonglong2 e = __ldcg(&tab[h]);
+    if (e.x == 0) return -1;
+    if (e.x == key0 && (uint32_t)(e.y >> 32) == (uint32_t)(w + 1)) return (int)(uint32_t)e.y - 1;
+    h = (h + 1) & mask;
+  }
+  return -1;
+}
+
 }  // namespace misat

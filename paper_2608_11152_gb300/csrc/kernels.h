@@ -207,6 +207,9 @@ struct FinalizeArgs {
   int32_t* out_hit;
   long long* U;
   unsigned long long* stats;   // route stats block (see api)
+  ulonglong2* grp;             // zeroed before the launch: (first key, instance) groups of the
+  uint32_t grp_log2;           //   admitted requests (grp_note), read back at commit
+  const uint64_t* keys;
   const int32_t* err;
 };
 void launch_finalize(const FinalizeArgs& a, cudaStream_t st);
@@ -234,6 +237,9 @@ struct InsertArgs {
   ulonglong2* gnew;            // keys new to an instance table, (key, instance), for the
   unsigned* n_gnew;            //   global index pass (zeroed by the launcher)
   int64_t gnew_cap;
+  const ulonglong2* grp;       // groups of the admitted requests (NULL: insert every block)
+  uint32_t grp_log2;
+  int32_t* skip;               // [n] leading blocks a later request of the group inserts
 };
 void launch_insert(const InsertArgs& a, int num_sms, cudaStream_t st);  // tables, then global index
 void launch_insert_tables(const InsertArgs& a, int num_sms, cudaStream_t st);

@@ -234,7 +234,9 @@ __global__ void __launch_bounds__(256) k4_finalize(FinalizeArgs a) {
     b = a.rq.cls[r];
     if (w >= 0) {
       L = a.rq.L[r];
-      atomic_add_i64(&a.U[w], (long long)(a.rq.nb[r] - hb));
+      const int nbr = a.rq.nb[r];
+      atomic_add_i64(&a.U[w], (long long)(nbr - hb));
+      if (a.grp && nbr > 0) grp_note(a.grp, a.grp_log2, a.keys[a.rq.kbase[r]], w, r);
     }
   }
   // statistics: warp ballots and sums, one shared-memory add per warp and counter

@@ -1191,17 +1191,14 @@ __global__ void __launch_bounds__(kCT, 1) k4_select_class(SelectClassArgs a) {
               const int t = __shfl_up_sync(kFull, incl, o);
               if (lane >= o) incl += t;
             }
-            // slot of the k-th (1-based) registered chooser of w, kCT if there are fewer
-            auto kth_slot = [&](int k) -> int {
-              const unsigned mx = __ballot_sync(kFull, incl >= k);
-              if (!mx) return kCT;
-              const int l = __ffs(mx) - 1;
-              const int before = __shfl_sync(kFull, incl - c, l);
-              const unsigned mb = __ballot_sync(kFull, lane < kSL && s.chs[kSL * l + lane] == w);
-              return kSL * l + (int)__fns(mb, 0, k - before);
-            };
-            const int f = kth_slot(need);
-            const int p = kth_slot(need + 1);
+            // slots of the need-th and (need + 1)-th registered choosers of w (kCT if fewer)
+            const unsigned mx1 = __ballot_sync(kFull, incl >= need), mx2 = __ballot_sync(kFull, incl > need);
+            const int l1 = mx1 ? __ffs(mx1) - 1 : 31, l2 = mx2 ? __ffs(mx2) - 1 : 31;
+            const int before1 = __shfl_sync(kFull, incl - c, l1), before2 = __shfl_sync(kFull, incl - c, l2);
+            const unsigned mb1 = __ballot_sync(kFull, lane < kSL && s.chs[kSL * l1 + lane] == w);
+            const unsigned mb2 = l2 == l1 ? mb1 : __ballot_sync(kFull, lane < kSL && s.chs[kSL * l2 + lane] == w);
+            const int f = mx1 ? kSL * l1 + (int)__fns(mb1, 0, need - before1) : kCT;
+            const int p = mx2 ? kSL * l2 + (int)__fns(mb2, 0, need + 1 - before2) : kCT;
             if (lane == 0) {
               s.fpos[w] = f;
               if (p < kCT) atomicMin(&s_q, p);
