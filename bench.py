@@ -55,11 +55,12 @@ CLOCK_QUERY = ("timestamp,index,clocks.sm,clocks.max.sm,power.draw,clocks_event_
 
 def kernels_per_step(global_index):
     """Kernels one route+commit launches.  Route: class parameters, prologue, leaders, hash,
-    caps, probe first, probe search, the three of the selection (records, initial envelopes,
-    serial selection), finalize.
-    Commit: insert work list, insert, the global-index pass (global layout only), sessions,
-    and the five eviction kernels (estimate, collect, select, delete, shift)."""
-    return 11 + 8 + (1 if global_index else 0)
+    caps, probe first, probe search, the four of the selection (records, initial envelopes,
+    per-class selection, joint selection: it returns at once unless the per-class path hands
+    it the batch), finalize.
+    Commit: insert dedup, insert work list, insert, the global-index pass (global layout only),
+    sessions, and the five eviction kernels (estimate, collect, select, delete, shift)."""
+    return 12 + 9 + (1 if global_index else 0)
 
 
 def max_over_ranks(ms, dist, device):
