@@ -311,11 +311,13 @@ def cpu_step(o, b):
     return time.perf_counter() - t
 
 
-def algorithmic_bytes(sc, st, mask_words=None, admitted_blocks=0, evict_buckets=0):
+def algorithmic_bytes(sc, st, mask_words=None, admitted_blocks=0, evict_buckets=0, insert_ops=None):
     """Algorithmic HBM bytes per launch of the hash, probe and commit kernels (see the design
     notes).  mask_words: words per key of the global prefix index, None for the per-instance
-    probe; admitted_blocks: full blocks of the admitted requests (the insert's key operations);
-    evict_buckets: buckets of the tables above capacity after the inserts (the collect scan)."""
+    probe; admitted_blocks: full blocks of the admitted requests; insert_ops: the insert's key
+    operations (admitted blocks less those a later request of the same instance inserts; None:
+    all of them); evict_buckets: buckets of the tables above capacity after the inserts (the
+    collect scan)."""
     b = sc.batch
     L = np.diff(b.tok_off)
     nb = L // 16
@@ -334,13 +336,15 @@ def algorithmic_bytes(sc, st, mask_words=None, admitted_blocks=0, evict_buckets=
     # K2 phase 2: one 32-byte key group per probe of the binary searches
     search_b = 32 * (st.probes - st.probes_first)
     mw = mask_words or 0
+    ops = admitted_blocks if insert_ops is None else insert_ops
     return {
         "hash": hash_b, "probe_first": first_b, "probe_search": search_b, "n_blocks": n_blocks,
         # K3b/K4a selection: one 32-byte record per request read, the decision fields written
         "select": 32 * b.n + 10 * b.n,
-        # K4b insert: per admitted block, its key read (8 B), its home key group (32 B) and the
-        # read-modify-write of its meta (16 B); per new key its (key, instance) entry (16 B)
-        "insert": 56 * admitted_blocks + 16 * st.new_keys,
+        # K4b insert: per key operation, its key read (8 B), its home key group (32 B) and the
+        # read-modify-write of its meta (16 B); per new key its (key, instance) entry (16 B);
+        # per block left to a later request, its key and the later request's key compared (16 B)
+        "insert": 56 * ops + 16 * st.new_keys + 16 * (admitted_blocks - ops),
         # global index: per new key, its entry read (16 B), a key group (32 B), its mask word RMW (16 B)
         "gix_insert": (64 * st.new_keys) if mask_words else 0,
         # K4c collect: the meta group of every bucket of a table above capacity (32 B)
@@ -634,7 +638,8 @@ def run_gb300(args):
         if r.index_size(w) >= int(sc.cap_blocks[w]):
             evict_buckets += r.table_buckets(w)
     ab = algorithmic_bytes(sc, st, mask_words=gidx["mask_words"] if gidx else None,
-                           admitted_blocks=admitted_blocks, evict_buckets=evict_buckets)
+                           admitted_blocks=admitted_blocks, evict_buckets=evict_buckets,
+                           insert_ops=int(st.insert_ops))
     phase_ms = {p: phase_tot[p] / KP for p in phase_tot}
     # one kernel per phase below (the insert phase adds the small work-list kernel)
     KERNEL_NAMES = {"hash": "k1_block_hash", "probe_first": "k2_probe_first_gix" if gidx else "k2_probe_first_group",
@@ -722,7 +727,8 @@ def run_gb300(args):
                   "held_by_class": dict(zip(("rlvr", "rlhf", "agentic"), (int(x) for x in st.held_by_class))),
                   "probes": st.probes, "bucket_reads": st.bucket_reads,
                   "new_keys": st.new_keys, "evicted": st.evicted, "hit_tokens": st.hit_tokens,
-                  "query_tokens": st.query_tokens, "dtv_ppm": st.dtv_ppm},
+                  "query_tokens": st.query_tokens, "dtv_ppm": st.dtv_ppm,
+                  "admitted_blocks": admitted_blocks, "insert_key_ops": int(st.insert_ops)},
     }
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         base = setup_oracle(sc)

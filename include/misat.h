@@ -145,6 +145,9 @@ typedef struct misat_batch_stats {
   int64_t new_keys;              /* keys inserted by the last commit */
   int64_t evicted;               /* keys evicted by the last commit */
   int64_t seq;                   /* commits applied so far */
+  int64_t insert_ops;            /* key operations of the last commit's insert: full blocks of the
+                                    admitted requests, less the leading blocks that a later request
+                                    of the same instance inserts with the same keys */
 } misat_batch_stats;
 
 /* Create a router on the current CUDA device.  cuda_stream: a cudaStream_t (NULL =

@@ -1249,6 +1249,7 @@ int misat_commit(misat_ctx* c) {
     if (rc) return rc;
   }
   CK(cudaMemsetAsync(c->stats_ptr() + 18, 0, 2 * 8, st));
+  CK(cudaMemsetAsync(c->stats_ptr() + 24, 0, 8, st));
   c->mark(8);
   if (n > 0) {
     InsertArgs ia{};
@@ -1273,6 +1274,7 @@ int misat_commit(misat_ctx* c) {
     ia.grp = c->d_grp;
     ia.grp_log2 = c->grp_log2;
     ia.skip = c->d_skip;
+    ia.ops = c->stats_ptr() + 24;
     launch_insert_tables(ia, c->num_sms, st);
     c->mark(9);
     cudaEvent_t join = nullptr;
@@ -1623,6 +1625,7 @@ int misat_stats(misat_ctx* c, misat_batch_stats* o) {
   o->new_keys = (int64_t)s[18];
   o->evicted = (int64_t)s[19];
   o->seq = (int64_t)c->seq;
+  o->insert_ops = (int64_t)s[24];
   // D_TV (Sec. 3.3) of the admitted class mix against rho, in ppm
   const int64_t A = o->n_admitted;
   if (A > 0) {

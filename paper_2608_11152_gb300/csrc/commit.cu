@@ -124,6 +124,10 @@ __global__ void __launch_bounds__(256) k4_units(InsertArgs a) {
     if (lane >= o) incl += t;
   }
   const int tot = __shfl_sync(kFull, incl, 31);
+  if (a.ops) {
+    const int blocks = __reduce_add_sync(kFull, (unsigned)(c - s0));
+    if (lane == 0 && blocks) atomicAdd(a.ops, (unsigned long long)blocks);
+  }
   if (tot == 0) return;
   unsigned base = 0;
   if (lane == 31) base = atomicAdd(a.n_units, (unsigned)tot);

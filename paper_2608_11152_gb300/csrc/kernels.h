@@ -240,6 +240,7 @@ struct InsertArgs {
   const ulonglong2* grp;       // groups of the admitted requests (NULL: insert every block)
   uint32_t grp_log2;
   int32_t* skip;               // [n] leading blocks a later request of the group inserts
+  unsigned long long* ops;     // blocks in the work list (NULL: not counted)
 };
 void launch_insert(const InsertArgs& a, int num_sms, cudaStream_t st);  // tables, then global index
 void launch_insert_tables(const InsertArgs& a, int num_sms, cudaStream_t st);

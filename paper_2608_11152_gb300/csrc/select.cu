@@ -734,7 +734,7 @@ static_assert(kCW <= 32 && (kCW & (kCW - 1)) == 0, "the window bitmask is at mos
 }  // namespace
 
 struct ClsSmem {
-  int16_t* chs;    // [kCT] registered choice of each window slot, -1 (16-byte aligned)
+  unsigned* regm;  // [W][kCW] registered choosers of each instance: one bit per window slot
   longlong2* ln;   // [W] {d_w, 1/mu_w}
   longlong2* hl;   // [W] {d_w, 1/mu_w} of the envelope lines, slope order
   longlong2* tl;   // [W] scratch of the envelope repair
@@ -754,7 +754,7 @@ struct ClsSmem {
 };
 
 size_t select_class_smem_bytes(int W) {
-  return (size_t)kCT * 2 + 128 + (size_t)W * (16 * 3 + 4 * 5 + 2 * 6 + 1) + 64;
+  return (size_t)128 + (size_t)W * (4 * kCW + 16 * 3 + 4 * 5 + 2 * 6 + 1) + 64;
 }
 
 // First set position >= from in a kCT-bit mask held one word per lane (kCT if none).  Warp-uniform.
@@ -899,7 +899,13 @@ __device__ __forceinline__ void cls_repair(const ClsSmem& s, int W, int w, int* 
       nc += __popc(mc);
     }
     __syncwarp();
-    for (int e0 = 0; e0 < nc; e0 += 32) {
+    if (nc == 1) {
+      // a single line below the chord beats p and q around their crossing (x >= 0): it is on
+      // the envelope, and nothing else enters between p and q
+      if (lane == 0) s.th[nnew] = (int16_t)s.cand[0];
+      nnew += 1;
+    }
+    for (int e0 = 0; nc > 1 && e0 < nc; e0 += 32) {
       const int e = e0 + lane;
       bool on = false;
       int i = 0;
@@ -959,10 +965,10 @@ __global__ void __launch_bounds__(kCT, 1) k4_select_class(SelectClassArgs a) {
   ClsSmem s;
   {
     unsigned char* p = smem;
-    s.chs = reinterpret_cast<int16_t*>(p);
-    p += (size_t)kCT * 2;
     s.tm = reinterpret_cast<unsigned*>(p);
     p += 128;
+    s.regm = reinterpret_cast<unsigned*>(p);
+    p += (size_t)W * kCW * 4;
     s.ln = reinterpret_cast<longlong2*>(p);
     p += (size_t)W * 16;
     s.hl = reinterpret_cast<longlong2*>(p);
@@ -1015,7 +1021,7 @@ __global__ void __launch_bounds__(kCT, 1) k4_select_class(SelectClassArgs a) {
     s.fpos[w] = kCT;
     s.hp[w] = -1;
   }
-  s.chs[tid] = -1;
+  for (int i = tid; i < W * kCW; i += kCT) s.regm[i] = 0;
   if (tid < 32) s.tm[tid] = 0;
   __syncthreads();
   // initial envelope of the class (launch_env_init), compacted in slope order
@@ -1139,7 +1145,7 @@ __global__ void __launch_bounds__(kCT, 1) k4_select_class(SelectClassArgs a) {
       // 1. a registered choice whose instance ran out is taken again; choices and registration
       if (reg && !s.av[dw]) {
         atomicSub(&s.T[dw], 1);
-        s.chs[tid] = -1;
+        atomicAnd(&s.regm[dw * kCW + wid], ~(1u << lane));
         reg = false;
         have = false;
       }
@@ -1149,7 +1155,7 @@ __global__ void __launch_bounds__(kCT, 1) k4_select_class(SelectClassArgs a) {
         if (dec == MISAT_ADMIT_NEW) {
           reg = true;
           if (atomicAdd(&s.T[dw], 1) + 1 >= s.ch[dw]) atomicOr(&s.tm[dw >> 5], 1u << (dw & 31));
-          s.chs[tid] = (int16_t)dw;
+          atomicOr(&s.regm[dw * kCW + wid], 1u << lane);
         }
       }
       __syncthreads();
@@ -1174,31 +1180,23 @@ __global__ void __launch_bounds__(kCT, 1) k4_select_class(SelectClassArgs a) {
             const int w = 32 * wi + __ffs(mine) - 1;
             mine &= mine - 1;
             const int need = s.ch[w];
-            // lane j counts the registered choosers of w among slots [kSL j, kSL (j + 1))
-            constexpr int kSL = kCT / 32;
-            int c = 0;
-            const int4* v = reinterpret_cast<const int4*>(s.chs + kSL * lane);
-#pragma unroll
-            for (int u = 0; u < kSL / 8; ++u) {
-              const int4 z = v[u];
-              const int zv[4] = {z.x, z.y, z.z, z.w};
-#pragma unroll
-              for (int h = 0; h < 4; ++h) c += ((int16_t)(zv[h] & 0xffff) == w) + ((zv[h] >> 16) == w);
-            }
+            // lane j holds the registered choosers of w among slots [32 j, 32 j + 32)
+            const unsigned word = lane < kCW ? s.regm[w * kCW + lane] : 0u;
+            const int c = __popc(word);
             int incl = c;
 #pragma unroll
-            for (int o = 1; o < 32; o <<= 1) {
+            for (int o = 1; o < kCW; o <<= 1) {
               const int t = __shfl_up_sync(kFull, incl, o);
               if (lane >= o) incl += t;
             }
             // slots of the need-th and (need + 1)-th registered choosers of w (kCT if fewer)
-            const unsigned mx1 = __ballot_sync(kFull, incl >= need), mx2 = __ballot_sync(kFull, incl > need);
-            const int l1 = mx1 ? __ffs(mx1) - 1 : 31, l2 = mx2 ? __ffs(mx2) - 1 : 31;
+            const unsigned mx1 = __ballot_sync(kFull, lane < kCW && incl >= need);
+            const unsigned mx2 = __ballot_sync(kFull, lane < kCW && incl > need);
+            const int l1 = mx1 ? __ffs(mx1) - 1 : 0, l2 = mx2 ? __ffs(mx2) - 1 : 0;
+            const unsigned w1 = __shfl_sync(kFull, word, l1), w2 = __shfl_sync(kFull, word, l2);
             const int before1 = __shfl_sync(kFull, incl - c, l1), before2 = __shfl_sync(kFull, incl - c, l2);
-            const unsigned mb1 = __ballot_sync(kFull, lane < kSL && s.chs[kSL * l1 + lane] == w);
-            const unsigned mb2 = l2 == l1 ? mb1 : __ballot_sync(kFull, lane < kSL && s.chs[kSL * l2 + lane] == w);
-            const int f = mx1 ? kSL * l1 + (int)__fns(mb1, 0, need - before1) : kCT;
-            const int p = mx2 ? kSL * l2 + (int)__fns(mb2, 0, need + 1 - before2) : kCT;
+            const int f = mx1 ? 32 * l1 + (int)__fns(w1, 0, need - before1) : kCT;
+            const int p = mx2 ? 32 * l2 + (int)__fns(w2, 0, need + 1 - before2) : kCT;
             if (lane == 0) {
               s.fpos[w] = f;
               if (p < kCT) atomicMin(&s_q, p);
@@ -1223,7 +1221,7 @@ __global__ void __launch_bounds__(kCT, 1) k4_select_class(SelectClassArgs a) {
         if (reg) {
           atomicSub(&s.T[dw], 1);
           atomicSub(&s.ch[dw], 1);
-          s.chs[tid] = -1;
+          atomicAnd(&s.regm[dw * kCW + wid], ~(1u << lane));
           reg = false;
         }
       }
