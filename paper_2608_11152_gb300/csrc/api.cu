@@ -133,7 +133,8 @@ struct misat_ctx {
   uint8_t* d_onhull = nullptr;   // initial envelopes of the selection [3W]
   int32_t* d_rank = nullptr;     // slope order of the instances [W]
   int32_t* d_rank_a = nullptr;   // (d_w, w) order of the instances [W]
-  int32_t* d_sel_list = nullptr; // [3 max_batch] each class's leaders (per-class selection)
+  int32_t* d_sel_list = nullptr; // [3 max_batch] each class's leaders per block of 256 requests
+  int32_t* d_sel_cnt = nullptr;  // [3 * blocks] leaders per class and block
   int32_t* d_sel_x = nullptr;    // [W + 2] admissions per instance, ticket, coupled flag
   ulonglong2* d_grp = nullptr;   // (first key, instance) groups of a route's admitted requests
   uint32_t grp_log2 = 1;
@@ -670,6 +671,8 @@ void enqueue_route(misat_ctx* c, const misat_batch* b, misat_decisions* out, cud
   sp.adm = c->d_sel_x;
   sp.ticket = reinterpret_cast<unsigned*>(c->d_sel_x + c->W);
   sp.coupled = c->d_sel_x + c->W + 1;
+  sp.seg = c->d_sel_list;
+  sp.segcnt = c->d_sel_cnt;
   sp.err = c->err_ptr();
   launch_select_prep(sp, st);
   EnvInitArgs ei{};
@@ -699,7 +702,8 @@ void enqueue_route(misat_ctx* c, const misat_batch* b, misat_decisions* out, cud
   sc.H = c->d_H;
   sc.hold_delay_q = c->hold_delay_q;
   sc.small = c->bk_small && c->tc_small;
-  sc.list = c->d_sel_list;
+  sc.seg = c->d_sel_list;
+  sc.segcnt = c->d_sel_cnt;
   sc.adm = c->d_sel_x;
   sc.ticket = reinterpret_cast<unsigned*>(c->d_sel_x + c->W);
   sc.coupled = c->d_sel_x + c->W + 1;
@@ -875,6 +879,7 @@ int misat_create(const misat_config* cfg, void* cuda_stream, misat_ctx** out) {
       (rc = dalloc_n(c, &c->d_bm_val, (size_t)1 << bm_log2)) || (rc = dalloc_n(c, &c->d_sel_rec, 2 * NB)) ||
       (rc = dalloc_n(c, &c->d_onhull, 3 * Ws)) || (rc = dalloc_n(c, &c->d_rank, Ws)) ||
       (rc = dalloc_n(c, &c->d_rank_a, Ws)) || (rc = dalloc_n(c, &c->d_sel_list, 3 * NB)) ||
+      (rc = dalloc_n(c, &c->d_sel_cnt, 3 * ((NB + 255) / 256))) ||
       (rc = dalloc_n(c, &c->d_sel_x, Ws + 2)) || (rc = dalloc_n(c, &c->d_skip, NB)) ||
       (rc = dalloc_n(c, &c->d_grp, (size_t)1 << bm_log2)) ||
       (rc = dalloc_n(c, &c->rq.nb, NB)) || (rc = dalloc_n(c, &c->rq.kbase, NB)) || (rc = dalloc_n(c, &c->rq.L, NB)) ||

@@ -130,6 +130,8 @@ struct SelectPrepArgs {
   int32_t* adm;                // [W] zeroed here: admissions per instance of the per-class path
   unsigned* ticket;            // zeroed here
   int32_t* coupled;            // zeroed here
+  int32_t* seg;                // [3n] out: per class and block of 256 requests, its leaders in order
+  int32_t* segcnt;             // [3 * blocks] out: leaders per class and block
   const int32_t* err;
 };
 void launch_select_prep(const SelectPrepArgs& a, cudaStream_t st);
@@ -187,13 +189,14 @@ struct SelectClassArgs {
   const uint16_t* H;           // [n*W]
   int64_t hold_delay_q;
   bool small;                  // as EnvInitArgs::small
-  int32_t* list;               // [3n] scratch: each class's leaders in arrival order
+  const int32_t* seg;          // [3n] per class and block of 256 requests, its leaders (prep)
+  const int32_t* segcnt;       // [3 * blocks] leaders per class and block (prep)
   int32_t* adm;                // [W] zeroed by launch_select_prep
   unsigned* ticket;            // zeroed by launch_select_prep
   int32_t* coupled;            // zeroed by launch_select_prep; set when the joint kernel must run
   int32_t* err;
 };
-size_t select_class_smem_bytes(int W);
+size_t select_class_smem_bytes(int W, int n);
 cudaError_t select_class_configure();
 void launch_select_class(const SelectClassArgs& a, cudaStream_t st);
 

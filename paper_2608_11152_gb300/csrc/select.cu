@@ -44,6 +44,7 @@ static_assert(kNW == 16 && kSlotInst == 8, "one thread per (counter, warp) in th
 //   rec[2r]   = {L, cls | sst << 8 | leader << 16, protected / last instance, hbest}
 //   rec[2r+1] = {instances with H > 0, first two of them as (w << 16 | H), 0}
 __global__ void __launch_bounds__(256) k3_select_prep(SelectPrepArgs a) {
+  __shared__ int s_wc[3][8];
   if (blockIdx.x == 0) {
     for (int w = threadIdx.x; w < a.W; w += blockDim.x) a.adm[w] = 0;
     if (threadIdx.x == 0) {
@@ -53,6 +54,29 @@ __global__ void __launch_bounds__(256) k3_select_prep(SelectPrepArgs a) {
   }
   if (block_error(a.err)) return;
   const int r = blockIdx.x * blockDim.x + threadIdx.x;
+  const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+  // this block's leaders of each class, in arrival order, for the per-class selection
+  {
+    const int c = r < a.n && a.rq.status[r] == kStUnresolved ? a.rq.cls[r] : 3;
+    unsigned mine = 0;
+#pragma unroll
+    for (int b = 0; b < 3; ++b) {
+      const unsigned m = __ballot_sync(kFull, c == b);
+      if (lane == 0) s_wc[b][wid] = __popc(m);
+      if (c == b) mine = m;
+    }
+    __syncthreads();
+    if (c < 3) {
+      int off = __popc(mine & lanemask_lt());
+      for (int k = 0; k < wid; ++k) off += s_wc[c][k];
+      a.seg[(int64_t)c * a.n + blockIdx.x * 256 + off] = r;
+    }
+    if (threadIdx.x < 3) {
+      int t = 0;
+      for (int k = 0; k < 8; ++k) t += s_wc[threadIdx.x][k];
+      a.segcnt[threadIdx.x * gridDim.x + blockIdx.x] = t;
+    }
+  }
   if (r >= a.n) return;
   const int lead = a.rq.status[r] == kStUnresolved;
   const uint32_t hb = a.rq.hbest[r];
@@ -729,6 +753,7 @@ void launch_select(const SelectArgs& a, cudaStream_t st) {
 // leaders that had chosen it choose again.
 namespace {
 constexpr int kCT = kSelectClassThreads;
+constexpr int kMaxBatchBlocks = 4096;  // blocks of 256 requests: batches of up to 2^20 requests
 constexpr int kCW = kCT / 32;
 static_assert(kCW <= 32 && (kCW & (kCW - 1)) == 0, "the window bitmask is at most one word per lane of a warp");
 }  // namespace
@@ -753,8 +778,10 @@ struct ClsSmem {
   unsigned* tm;    // [32] "tight" instances: registered choosers >= class headroom > 0
 };
 
-size_t select_class_smem_bytes(int W) {
-  return (size_t)128 + (size_t)W * (4 * kCW + 16 * 3 + 4 * 5 + 2 * 6 + 1) + 64;
+size_t select_class_smem_bytes(int W, int n) {
+  const size_t nblk = ((size_t)n + 255) >> 8;
+  return (size_t)128 + (size_t)W * (4 * kCW + 16 * 3 + 4 * 5 + 2 * 6) + (((size_t)W + 15) & ~(size_t)15) +
+         nblk * 4 + 64;
 }
 
 // First set position >= from in a kCT-bit mask held one word per lane (kCT if none).  Warp-uniform.
@@ -956,7 +983,7 @@ __device__ __forceinline__ void cls_repair(const ClsSmem& s, int W, int w, int* 
 
 __global__ void __launch_bounds__(kCT, 1) k4_select_class(SelectClassArgs a) {
   extern __shared__ __align__(16) unsigned char smem[];
-  __shared__ int s_nc, s_q, s_hm, s_first_a, s_last_s, s_nglobal, s_last;
+  __shared__ int s_nc, s_q, s_hm, s_first_a, s_last_s, s_nglobal, s_last, s_navail;
   __shared__ int s_ws[kCW];
   __shared__ unsigned s_lead[kCW], s_sens[kCW];
   if (block_error(a.err)) return;
@@ -1004,6 +1031,7 @@ __global__ void __launch_bounds__(kCT, 1) k4_select_class(SelectClassArgs a) {
     s_q = kCT;
     s_first_a = 0;
     s_last_s = W - 1;
+    s_navail = 0;
   }
   __syncthreads();
   for (int w = tid; w < W; w += kCT) {
@@ -1017,6 +1045,7 @@ __global__ void __launch_bounds__(kCT, 1) k4_select_class(SelectClassArgs a) {
     const int c = g > 0 ? a.ch[w * 3 + b] : 0;
     s.ch[w] = c;
     s.av[w] = c > 0;
+    if (c > 0) atomicAdd(&s_navail, 1);
     s.T[w] = 0;
     s.fpos[w] = kCT;
     s.hp[w] = -1;
@@ -1042,57 +1071,65 @@ __global__ void __launch_bounds__(kCT, 1) k4_select_class(SelectClassArgs a) {
     }
     if (lane == 0) s_hm = base;
   }
-  // The class's leaders in arrival order.  A request is a leader iff its status is not
-  // kStFollower; the other CTAs only turn leaders' statuses into decisions, so the test is
-  // stable while they run.  Each thread takes 8 consecutive requests per pass.
-  int32_t* lst = a.list + (int64_t)b * a.n;
-  int nc = 0;
-  for (int c0 = 0; c0 < a.n; c0 += 8 * kCT) {
-    const int r0 = c0 + 8 * tid;
-    uint32_t fm = 0;
-    if (r0 + 8 <= a.n) {
-      const uint2 cl = *reinterpret_cast<const uint2*>(a.rq.cls + r0);
-      const uint2 st = *reinterpret_cast<const uint2*>(a.rq.status + r0);
+  // The class's leaders in arrival order: the prep kernel listed them per block of 256
+  // requests; the block offsets are an exclusive scan of its counts (s_pre), and the class
+  // index g of a leader maps to its block by binary search.
+  const int nblk = (a.n + 255) >> 8;
+  const int32_t* seg = a.seg + (int64_t)b * a.n;
+  int* s_pre = reinterpret_cast<int*>(s.av + ((W + 15) & ~15));
+  {
+    constexpr int kPer = (kMaxBatchBlocks + kCT - 1) / kCT;
+    int v[kPer], t = 0;
 #pragma unroll
-      for (int u = 0; u < 8; ++u) {
-        const uint32_t cu = ((u < 4 ? cl.x : cl.y) >> (8 * (u & 3))) & 0xff;
-        const uint32_t su = ((u < 4 ? st.x : st.y) >> (8 * (u & 3))) & 0xff;
-        if (cu == (uint32_t)b && su != kStFollower) fm |= 1u << u;
-      }
-    } else {
-      for (int u = 0; u < 8 && r0 + u < a.n; ++u)
-        if (a.rq.cls[r0 + u] == b && a.rq.status[r0 + u] != kStFollower) fm |= 1u << u;
+    for (int u = 0; u < kPer; ++u) {
+      const int j = tid * kPer + u;
+      v[u] = j < nblk ? a.segcnt[b * nblk + j] : 0;
+      t += v[u];
     }
-    const int cnt = __popc(fm);
-    int incl = cnt;
+    int incl = t;
 #pragma unroll
     for (int o = 1; o < 32; o <<= 1) {
-      const int t = __shfl_up_sync(kFull, incl, o);
-      if (lane >= o) incl += t;
+      const int x = __shfl_up_sync(kFull, incl, o);
+      if (lane >= o) incl += x;
     }
     if (lane == 31) s_ws[wid] = incl;
     __syncthreads();
     if (wid == 0) {
-      const int v = lane < kCW ? s_ws[lane] : 0;
-      int wi = v;
+      const int x = lane < kCW ? s_ws[lane] : 0;
+      int wi = x;
 #pragma unroll
       for (int o = 1; o < 32; o <<= 1) {
-        const int t = __shfl_up_sync(kFull, wi, o);
-        if (lane >= o) wi += t;
+        const int y = __shfl_up_sync(kFull, wi, o);
+        if (lane >= o) wi += y;
       }
-      if (lane < kCW) s_ws[lane] = wi - v;
+      if (lane < kCW) s_ws[lane] = wi - x;
       if (lane == 31) s_nc = wi;
     }
     __syncthreads();
-    int off = nc + s_ws[wid] + incl - cnt;
-    for (uint32_t t = fm; t; t &= t - 1) lst[off++] = r0 + __ffs(t) - 1;
-    nc += s_nc;
+    int off = s_ws[wid] + incl - t;
+#pragma unroll
+    for (int u = 0; u < kPer; ++u) {
+      const int j = tid * kPer + u;
+      if (j < nblk) s_pre[j] = off;
+      off += v[u];
+    }
     __syncthreads();
   }
+  const int nc = s_nc;
+  // request of class index g (< nc): the last block whose offset is <= g
+  auto leader_at = [&](int g) -> int {
+    int lo = 0, hi = nblk - 1;
+    while (lo < hi) {
+      const int mid = (lo + hi + 1) >> 1;
+      if (s_pre[mid] <= g) lo = mid;
+      else hi = mid - 1;
+    }
+    return seg[(int64_t)lo * 256 + (g - s_pre[lo])];
+  };
   const int nglobal = s_nglobal;
 
   // records of the first window
-  int rn = tid < nc ? lst[tid] : 0;
+  int rn = tid < nc ? leader_at(tid) : 0;
   int4 n0 = make_int4(0, 0, 0, 0), n1 = make_int4(0, 0, 0, 0);
   if (tid < nc) {
     n0 = a.rec[2 * rn];
@@ -1100,12 +1137,30 @@ __global__ void __launch_bounds__(kCT, 1) k4_select_class(SelectClassArgs a) {
   }
 #pragma unroll 1
   for (int base = 0; base < nc; base += kCT) {
+    if (s_navail == 0) {
+      // no instance has headroom for the class any more: every remaining leader is decided
+      // on its own (a protected session continues on its instance, anyone else is held)
+      for (int i = base + tid; i < nc; i += kCT) {
+        const int r = leader_at(i);
+        const int4 r0 = a.rec[2 * r];
+        if (((r0.y >> 8) & 0xff) == (int)kSessProtected) {
+          a.rq.status[r] = kStResolved;
+          a.rq.inst[r] = r0.z;
+          a.rq.reason[r] = MISAT_ADMIT_CONT;
+        } else {
+          a.rq.status[r] = kStHeld;
+          a.rq.inst[r] = -1;
+          a.rq.last_reason[r] = nglobal > 0 ? MISAT_HOLD_CLASS_CAP : MISAT_HOLD_GLOBAL_CAP;
+        }
+      }
+      break;
+    }
     const int i = base + tid;
     const bool valid = i < nc;
     const int r = rn;
     const int4 r0 = n0, r1 = n1;
     if (i + kCT < nc) {  // the next window's records, in flight during this one
-      rn = lst[i + kCT];
+      rn = leader_at(i + kCT);
       n0 = a.rec[2 * rn];
       n1 = a.rec[2 * rn + 1];
     }
@@ -1246,6 +1301,7 @@ __global__ void __launch_bounds__(kCT, 1) k4_select_class(SelectClassArgs a) {
         }
         nrem = __shfl_sync(kFull, excl, 31);
         excl -= cnt;
+        if (lane == 0) s_navail -= nrem;
         for (unsigned t = out; t; t &= t - 1) {
           const int w = 32 * lane + __ffs(t) - 1;
           s.av[w] = 0;
@@ -1283,12 +1339,12 @@ __global__ void __launch_bounds__(kCT, 1) k4_select_class(SelectClassArgs a) {
 
 cudaError_t select_class_configure() {
   return cudaFuncSetAttribute(k4_select_class, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                              (int)select_class_smem_bytes(kMaxW));
+                              (int)select_class_smem_bytes(kMaxW, 256 * kMaxBatchBlocks));
 }
 
 void launch_select_class(const SelectClassArgs& a, cudaStream_t st) {
   if (a.n <= 0) return;
-  k4_select_class<<<3, kCT, select_class_smem_bytes(a.W), st>>>(a);
+  k4_select_class<<<3, kCT, select_class_smem_bytes(a.W, a.n), st>>>(a);
 }
 
 }  // namespace misat
