@@ -728,7 +728,8 @@ def run_gb300(args):
                   "probes": st.probes, "bucket_reads": st.bucket_reads,
                   "new_keys": st.new_keys, "evicted": st.evicted, "hit_tokens": st.hit_tokens,
                   "query_tokens": st.query_tokens, "dtv_ppm": st.dtv_ppm,
-                  "admitted_blocks": admitted_blocks, "insert_key_ops": int(st.insert_ops)},
+                  "admitted_blocks": admitted_blocks, "insert_key_ops": int(st.insert_ops),
+                  "selection_path": "joint" if int(st.joint_selection) else "per-class"},
     }
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         base = setup_oracle(sc)

@@ -148,6 +148,9 @@ typedef struct misat_batch_stats {
   int64_t insert_ops;            /* key operations of the last commit's insert: full blocks of the
                                     admitted requests, less the leading blocks that a later request
                                     of the same instance inserts with the same keys */
+  int64_t joint_selection;       /* 1 if some instance ran out of global headroom during the last
+                                    route, so its leaders were decided by the joint chain over all
+                                    classes; 0 if the per-class chains decided them */
 } misat_batch_stats;
 
 /* Create a router on the current CUDA device.  cuda_stream: a cudaStream_t (NULL =

@@ -707,6 +707,7 @@ void enqueue_route(misat_ctx* c, const misat_batch* b, misat_decisions* out, cud
   sc.adm = c->d_sel_x;
   sc.ticket = reinterpret_cast<unsigned*>(c->d_sel_x + c->W);
   sc.coupled = c->d_sel_x + c->W + 1;
+  sc.stats = c->stats_ptr();
   sc.err = c->err_ptr();
   launch_select_class(sc, st);
   SelectArgs sa{};
@@ -1631,6 +1632,7 @@ int misat_stats(misat_ctx* c, misat_batch_stats* o) {
   o->evicted = (int64_t)s[19];
   o->seq = (int64_t)c->seq;
   o->insert_ops = (int64_t)s[24];
+  o->joint_selection = (int64_t)s[25];
   // D_TV (Sec. 3.3) of the admitted class mix against rho, in ppm
   const int64_t A = o->n_admitted;
   if (A > 0) {

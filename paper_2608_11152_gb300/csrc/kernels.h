@@ -194,6 +194,7 @@ struct SelectClassArgs {
   int32_t* adm;                // [W] zeroed by launch_select_prep
   unsigned* ticket;            // zeroed by launch_select_prep
   int32_t* coupled;            // zeroed by launch_select_prep; set when the joint kernel must run
+  unsigned long long* stats;   // route stats block: [25] = 1 when the joint kernel runs
   int32_t* err;
 };
 size_t select_class_smem_bytes(int W, int n);

@@ -1333,7 +1333,10 @@ __global__ void __launch_bounds__(kCT, 1) k4_select_class(SelectClassArgs a) {
       const int g = a.gh[w];
       if (g > 0 && __ldcg(&a.adm[w]) >= g) bad = true;
     }
-    if (__syncthreads_or(bad) && tid == 0) *a.coupled = 1;
+    if (__syncthreads_or(bad) && tid == 0) {
+      *a.coupled = 1;
+      a.stats[25] = 1;
+    }
   }
 }
 

@@ -512,6 +512,32 @@ def test_serial_selection_many_windows_and_fills(seed, W):
     r.close()
 
 
+def test_per_class_and_joint_selection_paths_match_the_oracle():
+    """While no instance runs out of global headroom, the per-class chains decide a batch;
+    otherwise the joint chain over all classes decides it again.  Across these scenarios both
+    paths decide some batches (session admission, which has no class caps, makes the global cap
+    bind), and every batch equals the oracle's decisions and committed state."""
+    seen = {0: 0, 1: 0}
+    for seed in range(12):
+        rng = np.random.default_rng(300 + seed)
+        W = int(rng.integers(2, 9))
+        sc = wl.small_random(9300 + seed, W=W, cap=int(rng.integers(40, 200)), n=int(rng.integers(100, 600)),
+                             mode=seed % 4, n_warm=3)
+        r, o = make_router(sc), make_oracle(sc)
+        for b, comp in list(sc.warm) + [(sc.batch, None)]:
+            route_both(r, o, b, W)
+            seen[int(r.stats().joint_selection)] += 1
+            r.commit()
+            o.commit()
+            compare_state(r, o, W, index=False)
+            if comp is not None:
+                for x in (r, o):
+                    x.complete(comp.session, comp.cls, comp.total_blocks, comp.residency_us, comp.done)
+        compare_state(r, o, W)
+        r.close()
+    assert seen[0] > 0 and seen[1] > 0, seen
+
+
 def test_checkpoint_restore_replays_identically():
     """A restored checkpoint gives the same decisions and the same committed state again,
     including after a commit that grew a table (the restore shrinks it back)."""
