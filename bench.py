@@ -122,10 +122,10 @@ def hash_sources_sha256():
     return h.hexdigest()
 
 
-def profiled_hash_fields(batch_tokens):
-    """Figures of the block-hash kernel from the committed ncu summary (DRAM bytes per launch,
-    ALU pipe occupancy), if that capture was taken on the same batch with the kernel's current
-    sources; else {}."""
+def profiled_hash_fields():
+    """Figures of the block-hash kernel from the committed ncu summary (DRAM bytes per launch
+    and the batch's token count, ALU pipe occupancy), if that capture was taken with the
+    kernel's current sources; else {}."""
     try:
         fields = {}
         for line in open(HASH_PROFILE):
@@ -134,17 +134,19 @@ def profiled_hash_fields(batch_tokens):
                 fields[k.strip()] = v.strip().strip("`")
         if fields.get("sources_sha256") != hash_sources_sha256():
             return {}
-        if int(fields["batch_tokens"]) != int(batch_tokens):
-            return {}
         return fields
     except Exception:
         return {}
 
 
 def profiled_traffic(batch_tokens):
-    """DRAM bytes per launch of the block-hash kernel (see profiled_hash_fields), or None."""
-    f = profiled_hash_fields(batch_tokens)
-    return int(f["traffic_bytes_per_launch"]) if "traffic_bytes_per_launch" in f else None
+    """DRAM bytes per launch of the block-hash kernel, scaled from the captured batch to this
+    one by the token count (every token is read once, so the traffic grows with the tokens),
+    or None without a current capture."""
+    f = profiled_hash_fields()
+    if "traffic_bytes_per_launch" not in f:
+        return None
+    return int(round(int(f["traffic_bytes_per_launch"]) * int(batch_tokens) / int(f["batch_tokens"])))
 
 
 def peaks():
@@ -660,7 +662,7 @@ def run_gb300(args):
     kernels = {k: roof(k) for k in KERNEL_NAMES}
     if kernels["hash"] is not None:
         kernels["hash"]["traffic"] = profiled_traffic(sc.batch.n_tokens)
-        hf = profiled_hash_fields(sc.batch.n_tokens)
+        hf = profiled_hash_fields()
         if "alu_pipe_active_frac" in hf:
             # the kernel's actual limiter: integer ALU issue (ncu sm__pipe_alu_cycles_active)
             kernels["hash"]["alu_pipe_active_frac_ncu"] = float(hf["alu_pipe_active_frac"])

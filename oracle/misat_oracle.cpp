@@ -82,16 +82,20 @@ uint64_t mix64(uint64_t z) {
   return z ^ (z >> 31);
 }
 
+// Odd word multiplier of the content hash: the second SplitMix64 multiplier.
+constexpr uint64_t WORD_MUL = 0x94d049bb133111ebULL;
+
 // Content hash of one full block of 16 token ids: the 16 ids are read as eight
 // 64-bit words (even id in the low half), each word is offset by its position
-// times G and mixed, the eight results are XOR-ed and mixed once more.
+// times G and multiplied by the odd constant WORD_MUL (a bijection of the word), the
+// eight products are XOR-ed and mixed once.
 uint64_t block_content_hash(const int32_t* t) {
   uint64_t acc = 0;
   for (int i = 0; i < 8; ++i) {
     uint64_t lo = (uint32_t)t[2 * i];
     uint64_t hi = (uint32_t)t[2 * i + 1];
     uint64_t x = lo | (hi << 32);
-    acc ^= mix64(x + (uint64_t)(i + 1) * G);
+    acc ^= (x + (uint64_t)(i + 1) * G) * WORD_MUL;
   }
   return mix64(acc);
 }

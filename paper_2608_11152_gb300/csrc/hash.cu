@@ -1,8 +1,9 @@
 // K1: chained 16-token block hash (Sec. 4.4: the router's prefix index is keyed by
 // block hashes of the engine's prefix cache).
 //
-// Key of block j of a prompt:  c_j = mix64(XOR_i mix64(x_i + (i+1)G)) over the
-// block's eight 64-bit token pairs, a_j = a_{j-1} G + c_j (a_{-1} = seed),
+// Key of block j of a prompt:  c_j = mix64(XOR_i (x_i + (i+1)G) M) over the block's
+// eight 64-bit token pairs x_i (M odd: a bijection of each word), a_j = a_{j-1} G + c_j
+// (a_{-1} = seed),
 // k_j = mix64(a_j ^ (j+1)) (+2 if < 2).  The chain step is affine mod 2^64, so a
 // warp evaluates 32 consecutive blocks as an inclusive scan of affine maps:
 // in-chunk sums s_j = sum_{i<=j} c_i G^{j-i} (Hillis-Steele, multiplier G^d at
@@ -19,8 +20,9 @@
 // chunk with a two-step reduce-scatter (lane 4m+q ends with block 8q+m), then one
 // shuffle moves block j to lane j for the scan.  Keys are written coalesced.
 //
-// The kernel is bound by integer issue (ten 64-bit mixes per block), so the
-// structure above is chosen to spend as few instructions as possible around them.
+// Per block: eight 64-bit multiplies and two 64-bit mixes (the content hash's and the
+// key's), so the kernel streams tokens near the memory roof; the structure above keeps
+// the instructions around them few.
 #include <mutex>
 
 #include "common.cuh"
@@ -37,6 +39,7 @@ __host__ __device__ constexpr uint64_t gold_pow(int k) {
 }
 
 constexpr unsigned kFull = 0xffffffffu;
+constexpr uint64_t kWordMul = 0x94d049bb133111ebull;  // the content hash's odd word multiplier
 
 __device__ __forceinline__ int4 load_tok4(const int4* base, int64_t idx, int64_t n_int4) {
   if (idx < n_int4) return ld_stream_v4(base + idx);
@@ -112,7 +115,7 @@ __device__ __forceinline__ void hash_chain(const int4* tok4, int64_t n_int4, int
     for (int i = 0; i < 4; ++i) vn[i] = more ? load_tok4(tok4, nbase + 32 * i + lane, n_int4) : make_int4(0, 0, 0, 0);
     if (OFF != 0 && more && lane == 0) exn = load_tok4(tok4, nbase + 128, n_int4);
 
-    // partial XOR of the lane's two pre-mixed token pairs, per sub-row
+    // partial XOR of the lane's two multiplied token pairs, per sub-row
     uint64_t p[4];
 #pragma unroll
     for (int i = 0; i < 4; ++i) {
@@ -120,7 +123,7 @@ __device__ __forceinline__ void hash_chain(const int4* tok4, int64_t n_int4, int
       if (OFF != 0) t = align_words<OFF>(v[i], next_words<OFF>(v[i], i < 3 ? v[i + 1] : ex, lane));
       const uint64_t xa = (uint64_t)(uint32_t)t.x | ((uint64_t)(uint32_t)t.y << 32);
       const uint64_t xb = (uint64_t)(uint32_t)t.z | ((uint64_t)(uint32_t)t.w << 32);
-      p[i] = mix64(xa + lc.addA) ^ mix64(xb + lc.addB);
+      p[i] = ((xa + lc.addA) * kWordMul) ^ ((xb + lc.addB) * kWordMul);
     }
     // reduce-scatter over the quad: after the exchange with lane^1 a lane keeps the
     // sub-rows with bit 0 = its q's bit 0, after lane^2 the sub-row i = q: block 8q + m
