@@ -92,8 +92,9 @@ def parse_args():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--instances", type=int, default=128, help="fewer only for small profiling captures")
     ap.add_argument("--cap", type=int, default=262144, help="blocks per instance; smaller only for profiling captures")
-    ap.add_argument("--prefix-index", default="global", choices=["global", "per-instance"],
-                    help="block-0 probe through the global key->instance-mask index or per instance table")
+    ap.add_argument("--prefix-index", default="per-instance", choices=["global", "per-instance"],
+                    help="block-0 probe per instance table (default: the faster step at this admission "
+                         "volume) or through the global key->instance-mask index")
     ap.add_argument("--config", type=int, default=5, choices=[1, 2, 3, 4, 5],
                     help="workload: 1-4 the smaller mixed configurations, 5 the throughput stress sweep")
     return ap.parse_args()

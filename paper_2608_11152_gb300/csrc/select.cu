@@ -747,10 +747,13 @@ void launch_select(const SelectArgs& a, cudaStream_t st) {
 //
 // Within a window a tentative admission is final once the registered choosers of its
 // instance before it leave it headroom; the first leader that finds none cuts the window.
-// Exact cut positions come from per-instance ballots over the window's choices (one warp per
-// over-subscribed instance).  An instance that runs out leaves the envelope by a local repair
-// (the lines between its neighbours that lie below their chord, envelope.cuh), and only the
-// leaders that had chosen it choose again.
+// Registrations stay in place for the whole window (decided ones included), so the slot where
+// an instance runs out (the ch-th registered chooser, ch its headroom at the window's start)
+// and the slot of its first chooser that finds none only move earlier as leaders register,
+// and are recomputed (one warp per instance) only for the instances that received
+// registrations since their last scan.  An instance that runs out leaves the envelope by a
+// local repair (the lines between its neighbours that lie below their chord, envelope.cuh),
+// and only the undecided leaders that had chosen it choose again.
 namespace {
 constexpr int kCT = kSelectClassThreads;
 constexpr int kMaxBatchBlocks = 4096;  // blocks of 256 requests: batches of up to 2^20 requests
@@ -759,13 +762,14 @@ static_assert(kCW <= 32 && (kCW & (kCW - 1)) == 0, "the window bitmask is at mos
 }  // namespace
 
 struct ClsSmem {
-  unsigned* regm;  // [W][kCW] registered choosers of each instance: one bit per window slot
+  unsigned* regm;  // [W][kCW] registered choosers of each instance in the window: one bit per slot
   longlong2* ln;   // [W] {d_w, 1/mu_w}
   longlong2* hl;   // [W] {d_w, 1/mu_w} of the envelope lines, slope order
   longlong2* tl;   // [W] scratch of the envelope repair
-  int32_t* ch;     // [W] class headroom (0 for an instance without global headroom)
+  int32_t* ch;     // [W] class headroom at the window's start (0 without global headroom)
   int32_t* T;      // [W] registered choosers in the window
   int32_t* fpos;   // [W] window slot of the chooser that takes an instance's last headroom, kCT
+  int32_t* pp;     // [W] window slot of its first chooser that finds no headroom, kCT
   int32_t* cand;   // [W] envelope repair candidates
   int32_t* rem;    // [W] instances that ran out in this iteration
   int16_t* hull;   // [W] envelope lines, slope order
@@ -776,11 +780,12 @@ struct ClsSmem {
   int16_t* aord;   // [W] instances in (d_w, w) order
   uint8_t* av;     // [W] class headroom left
   unsigned* tm;    // [32] "tight" instances: registered choosers >= class headroom > 0
+  unsigned* dm;    // [32] tight instances with registrations since their last scan
 };
 
 size_t select_class_smem_bytes(int W, int n) {
   const size_t nblk = ((size_t)n + 255) >> 8;
-  return (size_t)128 + (size_t)W * (4 * kCW + 16 * 3 + 4 * 5 + 2 * 6) + (((size_t)W + 15) & ~(size_t)15) +
+  return (size_t)256 + (size_t)W * (4 * kCW + 16 * 3 + 4 * 6 + 2 * 6) + (((size_t)W + 15) & ~(size_t)15) +
          nblk * 4 + 64;
 }
 
@@ -796,10 +801,19 @@ __device__ __forceinline__ int cls_first_set(unsigned word, int lane, int from) 
   return w * 32 + __ffs(__shfl_sync(kFull, m, w)) - 1;
 }
 
-// Position of the (k+1)-th set bit of m (k < popc(m)).
-__device__ __forceinline__ int nth_set(unsigned m, int k) {
-  for (int i = 0; i < k; ++i) m &= m - 1;
-  return __ffs(m) - 1;
+// Position of the (k+1)-th set bit of x (0 <= k < popc(x)): a binary search on bit counts.
+__device__ __forceinline__ int nth_set(unsigned x, int k) {
+  int pos = 0;
+  int c = __popc(x & 0xffffu);
+  if (k >= c) { k -= c; x >>= 16; pos += 16; }
+  c = __popc(x & 0xffu);
+  if (k >= c) { k -= c; x >>= 8; pos += 8; }
+  c = __popc(x & 0xfu);
+  if (k >= c) { k -= c; x >>= 4; pos += 4; }
+  c = __popc(x & 0x3u);
+  if (k >= c) { k -= c; x >>= 2; pos += 2; }
+  if (k >= (int)(x & 1u)) pos += 1;
+  return pos;
 }
 
 // Decision of one leader of the CTA's class against the current state; see sel_choose.
@@ -983,7 +997,8 @@ __device__ __forceinline__ void cls_repair(const ClsSmem& s, int W, int w, int* 
 
 __global__ void __launch_bounds__(kCT, 1) k4_select_class(SelectClassArgs a) {
   extern __shared__ __align__(16) unsigned char smem[];
-  __shared__ int s_nc, s_q, s_hm, s_first_a, s_last_s, s_nglobal, s_last, s_navail;
+  __shared__ int s_nc, s_hm, s_first_a, s_last_s, s_nglobal, s_last, s_navail;
+  __shared__ int s_qb[2];  // cut bound of the current and the next iteration
   __shared__ int s_ws[kCW];
   __shared__ unsigned s_lead[kCW], s_sens[kCW];
   if (block_error(a.err)) return;
@@ -993,7 +1008,8 @@ __global__ void __launch_bounds__(kCT, 1) k4_select_class(SelectClassArgs a) {
   {
     unsigned char* p = smem;
     s.tm = reinterpret_cast<unsigned*>(p);
-    p += 128;
+    s.dm = s.tm + 32;
+    p += 256;
     s.regm = reinterpret_cast<unsigned*>(p);
     p += (size_t)W * kCW * 4;
     s.ln = reinterpret_cast<longlong2*>(p);
@@ -1007,6 +1023,8 @@ __global__ void __launch_bounds__(kCT, 1) k4_select_class(SelectClassArgs a) {
     s.T = reinterpret_cast<int32_t*>(p);
     p += (size_t)W * 4;
     s.fpos = reinterpret_cast<int32_t*>(p);
+    p += (size_t)W * 4;
+    s.pp = reinterpret_cast<int32_t*>(p);
     p += (size_t)W * 4;
     s.cand = reinterpret_cast<int32_t*>(p);
     p += (size_t)W * 4;
@@ -1028,7 +1046,7 @@ __global__ void __launch_bounds__(kCT, 1) k4_select_class(SelectClassArgs a) {
   }
   if (tid == 0) {
     s_nglobal = 0;
-    s_q = kCT;
+    s_qb[0] = kCT;
     s_first_a = 0;
     s_last_s = W - 1;
     s_navail = 0;
@@ -1048,10 +1066,11 @@ __global__ void __launch_bounds__(kCT, 1) k4_select_class(SelectClassArgs a) {
     if (c > 0) atomicAdd(&s_navail, 1);
     s.T[w] = 0;
     s.fpos[w] = kCT;
+    s.pp[w] = kCT;
     s.hp[w] = -1;
   }
   for (int i = tid; i < W * kCW; i += kCT) s.regm[i] = 0;
-  if (tid < 32) s.tm[tid] = 0;
+  if (tid < 64) s.tm[tid] = 0;  // tm and dm
   __syncthreads();
   // initial envelope of the class (launch_env_init), compacted in slope order
   if (wid == 0) {
@@ -1181,7 +1200,7 @@ __global__ void __launch_bounds__(kCT, 1) k4_select_class(SelectClassArgs a) {
     __syncthreads();
     const unsigned lead_word = lane < kCW ? s_lead[lane] : 0u;
     const unsigned sens_word = lane < kCW ? s_sens[lane] : 0u;
-    int done = 0;
+    int done = 0, par = 0;
     bool have = false, reg = false;
     uint8_t dec = 0;
     int dw = -1;
@@ -1197,30 +1216,39 @@ __global__ void __launch_bounds__(kCT, 1) k4_select_class(SelectClassArgs a) {
       // an Eq. (7) leader is decided alone, at the head, against the exact state of its turn
       const int qcut = max(cls_first_set(sens_word, lane, head), head + 1);
       const bool act = valid && tid >= head && tid < qcut;
-      // 1. a registered choice whose instance ran out is taken again; choices and registration
-      if (reg && !s.av[dw]) {
-        atomicSub(&s.T[dw], 1);
-        atomicAnd(&s.regm[dw * kCW + wid], ~(1u << lane));
+      // 1. an undecided leader whose instance ran out chooses again (its stale registration
+      //    stays with that instance, which is never scanned again); choices and registration,
+      //    one shared-memory update per (warp, instance)
+      if (tid >= done && reg && !s.av[dw]) {
         reg = false;
         have = false;
       }
+      bool nreg = false;
       if (act && !have) {
         dw = cls_choose(s, s_hm, nglobal, L, sst, pw, hb, nh, h0, h1, a.H + (int64_t)r * W, W, a.hold_delay_q, &dec);
         have = true;
-        if (dec == MISAT_ADMIT_NEW) {
-          reg = true;
-          if (atomicAdd(&s.T[dw], 1) + 1 >= s.ch[dw]) atomicOr(&s.tm[dw >> 5], 1u << (dw & 31));
-          atomicOr(&s.regm[dw * kCW + wid], 1u << lane);
+        nreg = dec == MISAT_ADMIT_NEW;
+        reg = nreg;
+      }
+      if (__any_sync(kFull, nreg)) {
+        const unsigned grp = __match_any_sync(kFull, nreg ? dw : -1 - lane);
+        if (nreg && lane == __ffs(grp) - 1) {
+          s.regm[dw * kCW + wid] |= grp;  // word (dw, wid) is written by this warp only
+          const int t1 = atomicAdd(&s.T[dw], __popc(grp)) + __popc(grp);
+          if (t1 >= s.ch[dw]) {
+            const unsigned bit = 1u << (dw & 31);
+            if (!(s.tm[dw >> 5] & bit)) atomicOr(&s.tm[dw >> 5], bit);
+            if (!(s.dm[dw >> 5] & bit)) atomicOr(&s.dm[dw >> 5], bit);
+          }
         }
       }
       __syncthreads();
-      // 2. instances with as many registered choosers as headroom (or more): the slot of the
-      //    chooser that takes the last headroom (fpos) and of the first one that finds none
-      //    (the cut); the k-th such instance goes to warp k mod kCW.  The tight set is kept
-      //    exactly: a registration that reaches the headroom adds its instance, and an instance
-      //    leaves it only when it runs out (a decided prefix lowers both counts alike).
+      // 2. tight instances with new registrations: the slot of the chooser that takes the last
+      //    headroom (fpos) and of the first one that finds none (pp); the k-th such instance
+      //    goes to warp k mod kCW.  Both slots only move earlier while the instance is tight,
+      //    so the cut bound starts from the others' pp (set by step 3 of the last iteration).
       {
-        const unsigned word = s.tm[lane];
+        const unsigned word = s.tm[lane] & s.dm[lane];
         const unsigned nzw = __ballot_sync(kFull, word != 0);
         int seen = 0;
         for (unsigned zz = nzw; zz; zz &= zz - 1) {
@@ -1250,19 +1278,20 @@ __global__ void __launch_bounds__(kCT, 1) k4_select_class(SelectClassArgs a) {
             const int l1 = mx1 ? __ffs(mx1) - 1 : 0, l2 = mx2 ? __ffs(mx2) - 1 : 0;
             const unsigned w1 = __shfl_sync(kFull, word, l1), w2 = __shfl_sync(kFull, word, l2);
             const int before1 = __shfl_sync(kFull, incl - c, l1), before2 = __shfl_sync(kFull, incl - c, l2);
-            const int f = mx1 ? 32 * l1 + (int)__fns(w1, 0, need - before1) : kCT;
-            const int p = mx2 ? 32 * l2 + (int)__fns(w2, 0, need + 1 - before2) : kCT;
+            const int f = mx1 ? 32 * l1 + nth_set(w1, need - 1 - before1) : kCT;
+            const int p = mx2 ? 32 * l2 + nth_set(w2, need - before2) : kCT;
             if (lane == 0) {
               s.fpos[w] = f;
-              if (p < kCT) atomicMin(&s_q, p);
+              s.pp[w] = p;
+              if (p < kCT) atomicMin(&s_qb[par], p);
             }
           }
         }
       }
       __syncthreads();
-      const int q = min(s_q, qcut);
-      // 3. the leaders before q are decided; warp 0 then takes the instances whose last
-      //    headroom went to one of them out of the envelope
+      const int q = min(s_qb[par], qcut);
+      // 3. the leaders before q are decided; warp 0 takes the instances whose last headroom
+      //    went to one of them out of the envelope, and sets the next iteration's cut bound
       if (act && tid < q) {
         if (dec == MISAT_ADMIT_NEW || dec == MISAT_ADMIT_CONT) {
           a.rq.status[r] = kStResolved;
@@ -1273,25 +1302,26 @@ __global__ void __launch_bounds__(kCT, 1) k4_select_class(SelectClassArgs a) {
           a.rq.inst[r] = -1;
           a.rq.last_reason[r] = dec;
         }
-        if (reg) {
-          atomicSub(&s.T[dw], 1);
-          atomicSub(&s.ch[dw], 1);
-          atomicAnd(&s.regm[dw * kCW + wid], ~(1u << lane));
-          reg = false;
-        }
       }
       if (wid == 0) {
-        int nrem = 0;
         const unsigned word = s.tm[lane];
-        unsigned keep = word;
+        unsigned out = 0;
+        int mn = kCT;
         for (unsigned t = word; t; t &= t - 1) {  // lane-local: the tight instances of word `lane`
           const int w = 32 * lane + __ffs(t) - 1;
-          const int f = s.fpos[w];
-          s.fpos[w] = kCT;
-          if (f < q) keep &= ~(t & (0u - t));
+          if (s.fpos[w] < q) {
+            out |= t & (0u - t);
+            s.fpos[w] = kCT;
+            s.pp[w] = kCT;
+          } else {
+            mn = min(mn, s.pp[w]);
+          }
         }
-        const unsigned out = word & ~keep;
-        s.tm[lane] = keep;
+        s.tm[lane] = word & ~out;
+        s.dm[lane] = 0;
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) mn = min(mn, __shfl_xor_sync(kFull, mn, o));
+        if (lane == 0) s_qb[par ^ 1] = mn;  // last read before the barrier above
         // instances that ran out, in index order
         int cnt = __popc(out), excl = cnt;
 #pragma unroll
@@ -1299,7 +1329,7 @@ __global__ void __launch_bounds__(kCT, 1) k4_select_class(SelectClassArgs a) {
           const int v = __shfl_up_sync(kFull, excl, o);
           if (lane >= o) excl += v;
         }
-        nrem = __shfl_sync(kFull, excl, 31);
+        const int nrem = __shfl_sync(kFull, excl, 31);
         excl -= cnt;
         if (lane == 0) s_navail -= nrem;
         for (unsigned t = out; t; t &= t - 1) {
@@ -1311,9 +1341,17 @@ __global__ void __launch_bounds__(kCT, 1) k4_select_class(SelectClassArgs a) {
         for (int e = 0; e < nrem; ++e) cls_repair(s, W, s.rem[e], &s_hm, &s_first_a, &s_last_s, a.small);
       }
       __syncthreads();
-      if (tid == 0) s_q = kCT;  // read by every thread before the barrier above
       done = q;
+      par ^= 1;
     }
+    // end of the window: every tight instance ran out (its last headroom went to a decided
+    // leader); the others lose the window's admissions
+    for (int w = tid; w < W; w += kCT) {
+      s.ch[w] = s.av[w] ? s.ch[w] - s.T[w] : 0;
+      s.T[w] = 0;
+    }
+    for (int i = tid; i < W * kCW; i += kCT) s.regm[i] = 0;
+    if (tid == 0) s_qb[0] = kCT;
     __syncthreads();  // s_lead / s_sens are rewritten by the next window
   }
   // admissions per instance, and the check that no instance ran out of global headroom

@@ -37,5 +37,7 @@ def test_launch_count_claim_matches_the_committed_launch_list():
     import re
 
     path = os.path.join(os.path.dirname(bench.__file__), "profiles", "launches_route_commit_cfg5_n65536_fill95.md")
-    totals = [int(m.group(1)) for m in re.finditer(r"\| \*\*total\*\* \| (\d+) \|", open(path).read())]
-    assert totals and all(t == 2 * bench.kernels_per_step(True) for t in totals)
+    text = open(path).read()
+    global_index = "prefix index: global" in text
+    totals = [int(m.group(1)) for m in re.finditer(r"\| \*\*total\*\* \| (\d+) \|", text)]
+    assert totals and all(t == 2 * bench.kernels_per_step(global_index) for t in totals)
