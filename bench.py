@@ -55,12 +55,13 @@ CLOCK_QUERY = ("timestamp,index,clocks.sm,clocks.max.sm,power.draw,clocks_event_
 
 def kernels_per_step(global_index):
     """Kernels one route+commit launches.  Route: class parameters, prologue, leaders, hash,
-    caps, probe first, probe search, the four of the selection (records, initial envelopes,
-    per-class selection, joint selection: it returns at once unless the per-class path hands
-    it the batch), finalize.
+    caps, the block-0 probe (one kernel with the global index; with per-instance tables three:
+    claim of the distinct block-0 keys, their probes, the per-request expansion), probe search,
+    the four of the selection (records, initial envelopes, per-class selection, joint
+    selection: it returns at once unless the per-class path hands it the batch), finalize.
     Commit: insert dedup, insert work list, insert, the global-index pass (global layout only),
     sessions, and the five eviction kernels (estimate, collect, select, delete, shift)."""
-    return 12 + 9 + (1 if global_index else 0)
+    return (12 + 9 + 1) if global_index else (14 + 9)
 
 
 def max_over_ranks(ms, dist, device):
@@ -329,9 +330,13 @@ def algorithmic_bytes(sc, st, mask_words=None, admitted_blocks=0, evict_buckets=
     # plus two 8-byte offsets per request
     hash_b = 72 * n_blocks + 16 * b.n
     if mask_words is None:
-        # K2 phase 1 per instance: one 32-byte key group per block-0 probe, the H row written
-        # (2 B per pair), block-0 key, block count and key base read per request
-        first_b = 32 * st.probes_first + 2 * b.n * sc.W + 20 * b.n
+        # K2 phase 1 per instance: one 32-byte key group per block-0 probe of a distinct key
+        # (each distinct block-0 key is probed once per instance), that key's instance mask
+        # written and its slot listed; per request its H row written (2 B per pair), its
+        # block-0 key, block count and key base read (the batch-local index of distinct keys
+        # stays in L2 and is not counted)
+        mw = (sc.W + 63) // 64
+        first_b = 32 * st.probes_first + (8 * mw + 12) * st.first_block_keys + 2 * b.n * sc.W + 20 * b.n
     else:
         # K2 phase 1 through the global index: one 32-byte key group per bucket read, the mask
         # of each looked-up key, the H row, request fields (the hit list is not counted)
@@ -645,7 +650,8 @@ def run_gb300(args):
                            insert_ops=int(st.insert_ops))
     phase_ms = {p: phase_tot[p] / KP for p in phase_tot}
     # one kernel per phase below (the insert phase adds the small work-list kernel)
-    KERNEL_NAMES = {"hash": "k1_block_hash", "probe_first": "k2_probe_first_gix" if gidx else "k2_probe_first_group",
+    KERNEL_NAMES = {"hash": "k1_block_hash",
+                    "probe_first": "k2_probe_first_gix" if gidx else "k2_first_claim + k2_probe_distinct + k2_probe_first_gix",
                     "probe_search": "k2_probe_search", "select": "k4_select_class", "insert": "k4_insert",
                     "gix_insert": "k4_gix_insert", "evict_collect": "k4_evict_collect",
                     "evict_delete": "k4_evict_delete", "evict_shift": "k4_evict_shift"}
@@ -686,7 +692,8 @@ def run_gb300(args):
         "probes_definition": ("index lookups executed by the probe kernels per second: with the global "
                               "prefix index one lookup of a request's block 0 answers all instances, and "
                               "each step of a prefix search is one lookup; with per-instance tables every "
-                              "(request, instance) block-0 lookup counts"),
+                              "(distinct block-0 key, instance) lookup counts (requests that share their "
+                              "block-0 key share its lookups)"),
         "prefix_decisions_per_s": round(world * n * sc.W * K / (total_ms / 1e3), 1),
         "prefix_decisions_definition": "(request, instance) longest-cached-prefix values H computed per second",
         "e2e": {"value": round(e2e, 1), "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
@@ -732,6 +739,7 @@ def run_gb300(args):
                   "new_keys": st.new_keys, "evicted": st.evicted, "hit_tokens": st.hit_tokens,
                   "query_tokens": st.query_tokens, "dtv_ppm": st.dtv_ppm,
                   "admitted_blocks": admitted_blocks, "insert_key_ops": int(st.insert_ops),
+                  "first_block_keys": int(st.first_block_keys),
                   "selection_path": "joint" if int(st.joint_selection) else "per-class"},
     }
     if rank == 0 and world == 1 and not args.no_cpu_baseline:

@@ -151,6 +151,10 @@ typedef struct misat_batch_stats {
   int64_t joint_selection;       /* 1 if some instance ran out of global headroom during the last
                                     route, so its leaders were decided by the joint chain over all
                                     classes; 0 if the per-class chains decided them */
+  int64_t first_block_keys;      /* per-instance layout: distinct block-0 keys of the last route
+                                    (each probed once per instance); 0 with the global index */
+  int64_t first_block_lookups;   /* per-instance layout: lookups of the requests' block-0 keys in
+                                    the route's index of distinct keys; 0 with the global index */
 } misat_batch_stats;
 
 /* Create a router on the current CUDA device.  cuda_stream: a cudaStream_t (NULL =

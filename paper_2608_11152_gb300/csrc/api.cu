@@ -137,6 +137,8 @@ struct misat_ctx {
   int32_t* d_sel_cnt = nullptr;  // [3 * blocks] leaders per class and block
   int32_t* d_sel_x = nullptr;    // [W + 2] admissions per instance, ticket, coupled flag
   ulonglong2* d_grp = nullptr;   // (first key, instance) groups of a route's admitted requests
+  GIndex fb{};                   // per-instance layout: batch-local index of the distinct block-0 keys
+  int32_t* d_fb_list = nullptr;  // [max_batch] its claimed slots
   uint32_t grp_log2 = 1;
   int32_t* d_skip = nullptr;     // [max_batch] leading blocks a later request of the group inserts
   // every d_w and every 1/mu_w below 2^25: the selection's envelope arithmetic fits in 64 bits
@@ -606,6 +608,12 @@ void enqueue_route(misat_ctx* c, const misat_batch* b, misat_decisions* out, cud
   cudaMemsetAsync(c->d_bm_key, 0, ((size_t)1 << bm_log2) * 8, st);
   cudaMemsetAsync(c->d_bm_val, 0x7f, ((size_t)1 << bm_log2) * 4, st);
   cudaMemsetAsync(c->d_grp, 0, ((size_t)1 << bm_log2) * sizeof(ulonglong2), st);
+  GIndex fb{};
+  if (c->fb.keys) {
+    fb = c->fb;
+    fb.log2nb = (uint32_t)std::max(0, bm_log2 - 2);
+    cudaMemsetAsync(fb.keys, 0, ((size_t)4 << fb.log2nb) * 8, st);
+  }
 
   c->mark(0, st);
   PrologueArgs pa{};
@@ -655,6 +663,10 @@ void enqueue_route(misat_ctx* c, const misat_batch* b, misat_decisions* out, cud
   pr.stats_search = c->stats_ptr() + 22;
   pr.err = c->err_ptr();
   pr.gix = gix_or_null(c);
+  pr.fb = fb;
+  pr.fb_list = c->d_fb_list;
+  pr.fb_count = c->stats_ptr() + 26;
+  pr.stats_fb = c->stats_ptr() + 27;
   launch_probe_first(pr, c->num_sms, st);
   c->mark(4, st);
   launch_probe_search(pr, c->num_sms, st);
@@ -929,6 +941,14 @@ int misat_create(const misat_config* cfg, void* cuda_stream, misat_ctx** out) {
       return fail(MISAT_ERR_CUDA);
     c->sess.log2n = lg;
     c->sess.used = c->d_meta + c->ml.sess_used;
+  }
+  // per-instance layout: the batch-local index of distinct block-0 keys (2 max_batch slots)
+  if (cfg->prefix_index == MISAT_PREFIX_PER_INSTANCE) {
+    c->fb.mw = (uint32_t)((W + 63) / 64);
+    const size_t fslots = (size_t)4 << std::max(0, bm_log2 - 2);
+    if ((rc = dalloc_n(c, &c->fb.keys, fslots)) || (rc = dalloc_n(c, &c->fb.masks, fslots * c->fb.mw)) ||
+        (rc = dalloc_n(c, &c->d_fb_list, NB)))
+      return fail(rc);
   }
   // global prefix index, sized for full tables (up to 2^26 keys; rebuilds grow it)
   if (cfg->prefix_index == MISAT_PREFIX_GLOBAL) {
@@ -1633,6 +1653,8 @@ int misat_stats(misat_ctx* c, misat_batch_stats* o) {
   o->seq = (int64_t)c->seq;
   o->insert_ops = (int64_t)s[24];
   o->joint_selection = (int64_t)s[25];
+  o->first_block_keys = (int64_t)s[26];
+  o->first_block_lookups = (int64_t)s[27];
   // D_TV (Sec. 3.3) of the admitted class mix against rho, in ppm
   const int64_t A = o->n_admitted;
   if (A > 0) {

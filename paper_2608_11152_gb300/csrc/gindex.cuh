@@ -94,6 +94,37 @@ __device__ __forceinline__ int gix_set(const GIndex& g, uint64_t key, int w) {
   return -1;
 }
 
+// Find-or-claim `key` without touching its mask.  Returns its slot (and sets *claimed when
+// this call took it), or -1 if the index has no free slot.
+__device__ __forceinline__ int64_t gix_claim(const GIndex& g, uint64_t key, bool* claimed) {
+  const uint32_t mask = (1u << g.log2nb) - 1;
+  uint32_t b = home_bucket(key, g.log2nb);
+  *claimed = false;
+  for (uint32_t it = 0; it <= mask; ++it) {
+    unsigned long long* kb = g.keys + 4 * (size_t)b;
+    for (int tries = 0; tries < 2 * kSlots; ++tries) {
+      const ulonglong2* p = reinterpret_cast<const ulonglong2*>(kb);
+      const ulonglong2 x = __ldcg(p), y = __ldcg(p + 1);
+      const unsigned long long k[4] = {x.x, x.y, y.x, y.y};
+      int s = -1, e = -1;
+#pragma unroll
+      for (int i = 3; i >= 0; --i) {
+        if (k[i] == key) s = i;
+        if (k[i] == kEmpty) e = i;
+      }
+      if (s >= 0) return 4 * (int64_t)b + s;
+      if (e < 0) break;  // full without the key: next bucket
+      const unsigned long long old = atomicCAS(kb + e, kEmpty, (unsigned long long)key);
+      if (old == kEmpty || old == key) {
+        *claimed = old == kEmpty;
+        return 4 * (int64_t)b + e;
+      }
+    }
+    b = (b + 1) & mask;
+  }
+  return -1;
+}
+
 // Clear bit w of `key`.  Returns 0, or -1 if the key is not in the index (an index that
 // no longer mirrors the tables).
 __device__ __forceinline__ int gix_clear(const GIndex& g, uint64_t key, int w) {

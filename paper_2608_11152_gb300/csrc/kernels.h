@@ -70,6 +70,13 @@ struct ProbeArgs {
   unsigned long long* stats_search;  // phase 2: [0] probes, [1] bucket reads
   int32_t* err;
   GIndex gix;                        // phase 1 reads the global index when gix.keys != NULL
+  // per-instance layout: a batch-local index of the distinct block-0 keys (GIndex layout,
+  // keys cleared per batch), the list of its claimed slots, the list's length (also the
+  // distinct-key count reported by the statistics) and the counters of its lookups
+  GIndex fb;
+  int32_t* fb_list;
+  unsigned long long* fb_count;
+  unsigned long long* stats_fb;      // [0] batch-index lookups, [1] their bucket reads
 };
 void launch_probe_first(const ProbeArgs& a, int num_sms, cudaStream_t st);
 void launch_probe_search(const ProbeArgs& a, int num_sms, cudaStream_t st);

@@ -6,11 +6,13 @@
 // tick and eviction takes the deepest block of a tick first), so "block h-1 is
 // resident" is monotone in h and H is found by binary search.
 //
-// Phase 1 (k2_probe_first_group): every (r, w) pair probes block 0.  A probe reads
-// one 32-byte sector (the four keys of the home bucket) and continues to the next
-// bucket only when the bucket is full without a match.  Most pairs miss and finish
-// after one sector.  Pairs with block 0 resident and at least two blocks are
-// appended to a compact hit list (warp-aggregated).
+// Phase 1: block 0 of every request on every instance.  With the global index one lookup
+// per request answers all instances (k2_probe_first_gix).  With per-instance tables every
+// distinct block-0 key of the batch is probed once per instance (k2_first_claim,
+// k2_probe_distinct) and the requests' rows are expanded from the keys' instance masks by
+// the same kernel.  A table probe reads one 32-byte sector (the four keys of the home
+// bucket) and continues to the next bucket only when the bucket is full without a match.
+// Pairs with block 0 resident and at least two blocks are appended to a compact hit list.
 // Phase 2 (k2_probe_search): a group of 16 lanes per hit pair searches [1, nb] with 16
 // parallel lookups per step (monotone predicate under prefix closure).
 #include "common.cuh"
@@ -46,12 +48,43 @@ __device__ __forceinline__ void block_add_stats(unsigned long long* stats, unsig
 
 }  // namespace
 
-// Phase 1, sub-warp layout: a group of S lanes (S = min(32, pow2 >= W)) owns one request;
-// its block-0 key is read once and broadcast, each lane probes instances w = lane, lane+S,
-// ... with up to kIlp independent sector loads in flight before any of them is consumed.
-template <int S>
-__global__ void __launch_bounds__(256) k2_probe_first_group(ProbeArgs a) {
-  constexpr int kIlp = 4;
+// Phase 1, per-instance layout with the block-0 lookups of a batch shared by key: requests
+// that start with the same block (the members of a rollout group, the turns of a session)
+// have the same block-0 residency on every instance, so each distinct key is probed once.
+// (a) k2_first_claim: every request finds or claims its block-0 key in the batch-local index;
+//     a claimer zeroes the key's instance mask and lists its slot (one atomic per warp).
+// (b) k2_probe_distinct: a warp per listed key looks it up in the W instance tables (lane j
+//     takes the instances congruent to j mod 32) and writes the key's instance mask, one
+//     64-bit word per two ballots.
+// (c) k2_probe_first_gix on the batch-local index writes every request's H row, hbest and
+//     hit-list entries from its key's mask, as with the global index.
+__global__ void __launch_bounds__(256) k2_first_claim(ProbeArgs a) {
+  if (block_error(a.err)) return;
+  const int lane = threadIdx.x & 31;
+  const int stride = gridDim.x * blockDim.x;
+  const uint32_t mw = a.fb.mw;
+  for (int r0 = blockIdx.x * blockDim.x + (threadIdx.x & ~31); r0 < a.n; r0 += stride) {
+    const int r = r0 + lane;
+    bool claimed = false;
+    int64_t slot = -1;
+    if (r < a.n && a.nb[r] > 0) {
+      slot = gix_claim(a.fb, a.keys[a.kbase[r]], &claimed);
+      if (slot < 0) set_error(a.err, MISAT_ERR_TABLE_FULL);
+    }
+    if (claimed)
+      for (uint32_t i = 0; i < mw; ++i) a.fb.masks[(size_t)slot * mw + i] = 0ull;
+    const unsigned m = __ballot_sync(0xffffffffu, claimed);
+    if (m) {
+      const int leader = __ffs(m) - 1;
+      unsigned long long base = 0;
+      if (lane == leader) base = atomicAdd(a.fb_count, (unsigned long long)__popc(m));
+      base = __shfl_sync(0xffffffffu, base, leader);
+      if (claimed) a.fb_list[base + __popc(m & lanemask_lt())] = (int32_t)slot;
+    }
+  }
+}
+
+__global__ void __launch_bounds__(256) k2_probe_distinct(ProbeArgs a) {
   __shared__ Bucket* s_tab[kMaxW];
   __shared__ uint32_t s_lg[kMaxW];
   if (block_error(a.err)) return;
@@ -61,68 +94,36 @@ __global__ void __launch_bounds__(256) k2_probe_first_group(ProbeArgs a) {
   }
   __syncthreads();
   const int lane = threadIdx.x & 31;
-  const int sub = lane & (S - 1);
-  const int gid = (blockIdx.x * blockDim.x + threadIdx.x) / S;  // group index
-  const int ngroups = (gridDim.x * blockDim.x) / S;
+  const int nd = (int)*a.fb_count;
+  const uint32_t mw = a.fb.mw;
   unsigned long long probes = 0, reads = 0;
-  // groups per warp iterate in lockstep so that the warp-wide ballots see every lane
-  const int warp_first_group = ((blockIdx.x * blockDim.x + (threadIdx.x & ~31)) / S);
-  for (int rb = warp_first_group; rb < a.n; rb += ngroups) {
-    const int r = rb + (gid - warp_first_group);
-    const bool live = r < a.n;
-    int32_t nb = 0;
-    uint64_t key = 0;
-    if (live) {
-      nb = a.nb[r];
-      if (nb > 0) key = a.keys[a.kbase[r]];
-    }
-    int wmin = INT32_MAX;  // lowest instance holding block 0
-    for (int w0 = 0; w0 < a.W; w0 += S * kIlp) {
-      int res[kIlp];
-      uint32_t rd[kIlp];
-#pragma unroll
-      for (int i = 0; i < kIlp; ++i) {
-        const int w = w0 + i * S + sub;
-        res[i] = 0;
-        rd[i] = 0;
-        if (live && nb > 0 && w < a.W) {
-          InstDesc d;
-          d.tab = s_tab[w];
-          d.log2nb = s_lg[w];
-          res[i] = table_contains(d, key, &rd[i]);
-        }
+  for (int d = (blockIdx.x * blockDim.x + threadIdx.x) >> 5; d < nd; d += (gridDim.x * blockDim.x) >> 5) {
+    const int64_t slot = a.fb_list[d];
+    const uint64_t key = a.fb.keys[slot];
+    for (int w0 = 0; w0 < a.W; w0 += 64) {
+      int h0 = 0, h1 = 0;
+      const int wa = w0 + lane, wb = w0 + 32 + lane;
+      if (wa < a.W) {
+        InstDesc dd;
+        dd.tab = s_tab[wa];
+        dd.log2nb = s_lg[wa];
+        uint32_t rd = 0;
+        h0 = table_contains(dd, key, &rd);
+        probes += 1;
+        reads += rd;
       }
-#pragma unroll
-      for (int i = 0; i < kIlp; ++i) {
-        const int w = w0 + i * S + sub;
-        const bool valid = live && w < a.W;
-        if (valid && res[i]) wmin = min(wmin, w);
-        if (valid) {
-          a.H[(int64_t)r * a.W + w] = (uint16_t)res[i];
-          if (nb > 0) {
-            probes += 1;
-            reads += rd[i];
-          }
-        }
-        const bool hl = valid && res[i] && nb > 1;
-        const unsigned m = __ballot_sync(0xffffffffu, hl);
-        if (m) {
-          unsigned pos = 0;
-          const int leader = __ffs(m) - 1;
-          if (lane == leader) pos = atomicAdd(a.n_hits, (unsigned)__popc(m));
-          pos = __shfl_sync(0xffffffffu, pos, leader) + __popc(m & lanemask_lt());
-          if (hl) {
-            if ((int64_t)pos < a.hits_cap)
-              a.hits[pos] = make_int2(r, w);
-            else
-              set_error(a.err, MISAT_ERR_TABLE_FULL);
-          }
-        }
+      if (wb < a.W) {
+        InstDesc dd;
+        dd.tab = s_tab[wb];
+        dd.log2nb = s_lg[wb];
+        uint32_t rd = 0;
+        h1 = table_contains(dd, key, &rd);
+        probes += 1;
+        reads += rd;
       }
+      const unsigned m0 = __ballot_sync(0xffffffffu, h0), m1 = __ballot_sync(0xffffffffu, h1);
+      if (lane == 0) a.fb.masks[(size_t)slot * mw + (w0 >> 6)] = (unsigned long long)m0 | ((unsigned long long)m1 << 32);
     }
-#pragma unroll
-    for (int o = S / 2; o > 0; o >>= 1) wmin = min(wmin, __shfl_xor_sync(0xffffffffu, wmin, o, S));
-    if (live && sub == 0) a.hbest[r] = wmin < a.W ? (1u << 16) | (65535u - (uint32_t)wmin) : 65535u;
   }
   block_add_stats(a.stats, probes, reads);
 }
@@ -325,26 +326,20 @@ __global__ void __launch_bounds__(256) k2_probe_first_gix(ProbeArgs a) {
 void launch_probe_first(const ProbeArgs& a, int num_sms, cudaStream_t st) {
   const int64_t total = (int64_t)a.n * a.W;
   if (total <= 0) return;
+  const int groups = (a.n + 31) / 32;
+  const int gblocks = (groups + 7) / 8;
+  const int ggrid = gblocks < num_sms * 8 ? gblocks : num_sms * 8;
   if (a.gix.keys) {
-    const int groups = (a.n + 31) / 32;
-    const int blocks = (groups + 7) / 8;
-    const int grid = blocks < num_sms * 8 ? blocks : num_sms * 8;
-    k2_probe_first_gix<<<grid, 256, 8 * 32 * (a.gix.mw * sizeof(unsigned long long) + sizeof(int2)), st>>>(a);
+    k2_probe_first_gix<<<ggrid, 256, 8 * 32 * (a.gix.mw * sizeof(unsigned long long) + sizeof(int2)), st>>>(a);
     return;
   }
-  int S = 1;
-  while (S < a.W && S < 32) S <<= 1;
-  const int64_t threads = (int64_t)a.n * S;
-  int64_t blocks = (threads + 255) / 256;
-  const int grid = (int)(blocks < (int64_t)num_sms * 8 ? blocks : (int64_t)num_sms * 8);
-  switch (S) {
-    case 1: k2_probe_first_group<1><<<grid, 256, 0, st>>>(a); break;
-    case 2: k2_probe_first_group<2><<<grid, 256, 0, st>>>(a); break;
-    case 4: k2_probe_first_group<4><<<grid, 256, 0, st>>>(a); break;
-    case 8: k2_probe_first_group<8><<<grid, 256, 0, st>>>(a); break;
-    case 16: k2_probe_first_group<16><<<grid, 256, 0, st>>>(a); break;
-    default: k2_probe_first_group<32><<<grid, 256, 0, st>>>(a); break;
-  }
+  // per-instance tables: the context allocates the batch-local index with the tables
+  k2_first_claim<<<ggrid, 256, 0, st>>>(a);
+  k2_probe_distinct<<<num_sms * 8, 256, 0, st>>>(a);
+  ProbeArgs e = a;
+  e.gix = a.fb;
+  e.stats = a.stats_fb;
+  k2_probe_first_gix<<<ggrid, 256, 8 * 32 * (a.fb.mw * sizeof(unsigned long long) + sizeof(int2)), st>>>(e);
 }
 
 void launch_probe_search(const ProbeArgs& a, int num_sms, cudaStream_t st) {

@@ -68,7 +68,8 @@ class misat_batch_stats(C.Structure):
                 ("dtv_ppm", C.c_int64), ("probes", C.c_int64), ("bucket_reads", C.c_int64),
                 ("probes_first", C.c_int64), ("bucket_reads_first", C.c_int64),
                 ("new_keys", C.c_int64), ("evicted", C.c_int64), ("seq", C.c_int64),
-                ("insert_ops", C.c_int64), ("joint_selection", C.c_int64)]
+                ("insert_ops", C.c_int64), ("joint_selection", C.c_int64),
+                ("first_block_keys", C.c_int64), ("first_block_lookups", C.c_int64)]
 
 
 class misat_overload_config(C.Structure):
