@@ -84,36 +84,46 @@ def test_parity_with_releases_and_rebounds(seed):
 
 # ------------------------------------------------------------------ workload configurations
 
+# both block-0 probe layouts: 0 = through the global index, 1 = per-instance tables with the
+# lookups shared by the requests that start with the same block (the benchmark's layout)
+LAYOUTS = [0, 1]
+
+
+@pytest.mark.parametrize("prefix_index", LAYOUTS)
 @pytest.mark.parametrize("cfg", [1, 2, 3])
-def test_parity_config(cfg):
+def test_parity_config(cfg, prefix_index):
     sc = wl.CONFIGS[cfg]()
-    r, o = run_parity(sc, index_every_step=cfg == 1)
+    r, o = run_parity(sc, index_every_step=cfg == 1, prefix_index=prefix_index)
     r.close()
 
 
-def test_parity_config4_agentic_long_sessions():
+@pytest.mark.parametrize("prefix_index", LAYOUTS)
+def test_parity_config4_agentic_long_sessions(prefix_index):
     sc = wl.config4()
-    r, o = run_parity(sc, index_every_step=False)
+    r, o = run_parity(sc, index_every_step=False, prefix_index=prefix_index)
     r.close()
 
 
-def test_parity_config5_reduced():
+@pytest.mark.parametrize("prefix_index", LAYOUTS)
+def test_parity_config5_reduced(prefix_index):
     sc = wl.config5(n=4096, fill=0.5)
-    r, o = run_parity(sc, index_every_step=False)
+    r, o = run_parity(sc, index_every_step=False, prefix_index=prefix_index)
     r.close()
 
 
-def test_parity_config5_full_size():
+@pytest.mark.parametrize("prefix_index", LAYOUTS)
+def test_parity_config5_full_size(prefix_index):
     """The benchmark workload itself: 128 x 262,144 blocks at 95% fill (resident prompt chains,
     some of them histories that agentic sessions of the batch continue), 65,536 requests, in
-    the launch configuration the benchmark times: the measured batch is routed as the
-    benchmark routes it (same buffers every call, so the route is launched directly, then
-    captured, then replayed from its CUDA graph) and every one of those routes must give the
-    oracle's decisions; then the commit and every instance's index are compared."""
+    the launch configuration the benchmark times (per-instance tables; the global index as
+    well): the measured batch is routed as the benchmark routes it (same buffers every call,
+    so the route is launched directly, then captured, then replayed from its CUDA graph) and
+    every one of those routes must give the oracle's decisions; then the commit and every
+    instance's index are compared."""
     import torch
 
     sc = wl.config5(n=65536, fill=0.95)
-    r = make_router(sc)
+    r = make_router(sc, prefix_index=prefix_index)
     o = make_oracle(sc)
     try:
         load_fill(r, sc)
@@ -208,16 +218,48 @@ def test_longest_prompt_65535_blocks():
     r.close()
 
 
-def test_many_instances_w1024():
+@pytest.mark.parametrize("prefix_index", LAYOUTS)
+def test_many_instances_w1024(prefix_index):
     sc = wl.small_random(14, W=1024, cap=32, n=300, n_warm=2)
-    r, o = run_parity(sc)
+    r, o = run_parity(sc, prefix_index=prefix_index)
     r.close()
 
 
-def test_one_instance():
+@pytest.mark.parametrize("prefix_index", LAYOUTS)
+def test_one_instance(prefix_index):
     sc = wl.small_random(15, W=1, cap=256, n=60, n_warm=3)
-    r, o = run_parity(sc)
+    r, o = run_parity(sc, prefix_index=prefix_index)
     r.close()
+
+
+def test_shared_block0_lookups_count_the_distinct_first_blocks():
+    """Per-instance tables: every distinct block-0 key of a batch is probed once per instance.
+    The statistics must report the number of distinct first blocks (16-token prefixes,
+    counted on the host from the tokens) and exactly that many probes per instance, and
+    the decisions and H rows must still equal the oracle's (route_both)."""
+    sc = wl.config3()
+    r = make_router(sc, prefix_index=1)
+    o = make_oracle(sc)
+    try:
+        load_fill(r, sc)
+        load_fill(o, sc)
+        for b, comp in list(sc.warm) + [(sc.batch, None)]:
+            route_both(r, o, b, sc.W)
+            s = r.stats()
+            L = np.diff(b.tok_off)
+            firsts = {b.tokens[b.tok_off[i]:b.tok_off[i] + 16].tobytes() for i in range(b.n) if L[i] >= 16}
+            assert s.first_block_keys == len(firsts), (s.first_block_keys, len(firsts))
+            assert s.probes_first == len(firsts) * sc.W
+            assert s.first_block_lookups == int((L >= 16).sum())
+            assert len(firsts) < int((L >= 16).sum())  # the workload does share first blocks
+            r.commit()
+            o.commit()
+            if comp is not None:
+                for x in (r, o):
+                    x.complete(comp.session, comp.cls, comp.total_blocks, comp.residency_us, comp.done)
+        compare_state(r, o, sc.W, index=True)
+    finally:
+        r.close()
 
 
 def test_table_growth_and_session_rebuild():
