@@ -220,9 +220,9 @@ int misat_route_host(misat_ctx* ctx, const misat_batch* host_batch, misat_decisi
  *
  * Typical loop: stage(0, batch 0); for k: stage((k+1)%2, batch k+1); route_staged(k%2);
  * commit.  The GPU's copy engine takes host-to-device copies in order, so a host copy that
- * another call enqueues on the context's stream (misat_set_instance_state, misat_complete,
- * misat_load_*) while a staged batch is being copied starts after that batch's copy;
- * misat_route_staged and misat_commit make no host-to-device copy. */
+ * another call enqueues on the context's stream (misat_set_instance_state, misat_load_*)
+ * while a staged batch is being copied starts after that batch's copy; misat_route_staged,
+ * misat_commit and misat_complete make no host-to-device copy. */
 int misat_stage_host(misat_ctx* ctx, const misat_batch* host_batch, int32_t slot);
 int misat_route_staged(misat_ctx* ctx, int32_t slot, misat_decisions* host_out);
 
@@ -271,7 +271,14 @@ int misat_commit(misat_ctx* ctx);
  *              protected set and is forgotten;
  *   done == 0: protection is released but the session is remembered; its next
  *              request is a continuation that must be admitted again (Eq. 7).
- * Unknown sessions only update the histories.  [async] */
+ * Unknown sessions only update the histories.  The arrays are copied into one of two
+ * library buffers of mapped pinned host memory before the call returns, so the caller may
+ * reuse them at once; the first call allocates them (2 x 9 max_batch bytes).  The device
+ * update is a kernel on the context's stream that reads that buffer over the host link (no
+ * copy-engine transfer, so it does not queue behind a staged batch's copy), and the call
+ * does not wait for it.
+ * [async]  Errors: INVALID_ARG (a class above 2, a negative count, session 0 or a session
+ * listed twice), OOM, CUDA. */
 int misat_complete(misat_ctx* ctx, int32_t n, const uint64_t* session, const uint8_t* cls,
                    const int32_t* total_blocks, const int64_t* residency_us, const uint8_t* done);
 

@@ -154,6 +154,17 @@ struct misat_ctx {
   int64_t* d_stage_off = nullptr;
   uint8_t* d_stage_cls = nullptr;
   uint64_t* d_stage_ses = nullptr;
+  // completion events: two pinned host copies (so that the caller's arrays are free when
+  // misat_complete returns), read by the completion kernel in place, and the event after the
+  // kernel that last read each
+  struct CompBuf {
+    uint64_t* h_ses = nullptr;   // mapped pinned host memory
+    uint8_t* h_done = nullptr;
+    uint64_t* d_ses = nullptr;   // the same memory as the device addresses it
+    uint8_t* d_done = nullptr;
+    cudaEvent_t ev = nullptr;
+  } comp[2];
+  int comp_turn = 0;
   int32_t* d_out_inst = nullptr;
   uint8_t* d_out_reason = nullptr;
   int32_t* d_out_hit = nullptr;
@@ -794,6 +805,11 @@ int misat_destroy(misat_ctx* c) {
     cudaStreamSynchronize(c->copy_stream);
     cudaStreamDestroy(c->copy_stream);
   }
+  for (auto& cb : c->comp) {
+    if (cb.ev) cudaEventDestroy(cb.ev);
+    if (cb.h_ses) cudaFreeHost(cb.h_ses);
+    if (cb.h_done) cudaFreeHost(cb.h_done);
+  }
   for (auto& sl : c->slot) {
     if (sl.ev_copied) cudaEventDestroy(sl.ev_copied);
     if (sl.ev_free) cudaEventDestroy(sl.ev_free);
@@ -1359,16 +1375,32 @@ int misat_complete(misat_ctx* c, int32_t n, const uint64_t* session, const uint8
     while ((int32_t)c->hist_blocks[b].size() > c->hist_window) c->hist_blocks[b].pop_front();
     while ((int32_t)c->hist_res[b].size() > c->hist_window) c->hist_res[b].pop_front();
   }
-  // device part: sessions and done flags through the route staging buffers (in chunks)
+  // device part: sessions and done flags, in chunks of max_batch, through one of two pinned
+  // host copies (reused once the kernel that last read it has run); nothing here waits for
+  // the stream
   cudaStream_t st = c->stream;
   for (int off = 0; off < n; off += c->max_batch) {
     const int m = std::min(c->max_batch, n - off);
-    CK(cudaMemcpyAsync(c->d_stage_ses, session + off, (size_t)m * 8, cudaMemcpyHostToDevice, st));
-    CK(cudaMemcpyAsync(c->d_stage_cls, done + off, (size_t)m, cudaMemcpyHostToDevice, st));
-    CompleteArgs a{m, c->d_stage_ses, c->d_stage_cls, c->sess, c->d_prot};
+    misat_ctx::CompBuf& cb = c->comp[c->comp_turn];
+    c->comp_turn ^= 1;
+    if (!cb.h_ses) {
+      if (cudaHostAlloc(&cb.h_ses, (size_t)c->max_batch * 8, cudaHostAllocMapped) != cudaSuccess ||
+          cudaHostAlloc(&cb.h_done, (size_t)c->max_batch, cudaHostAllocMapped) != cudaSuccess)
+        return MISAT_ERR_OOM;
+      CK(cudaHostGetDevicePointer(reinterpret_cast<void**>(&cb.d_ses), cb.h_ses, 0));
+      CK(cudaHostGetDevicePointer(reinterpret_cast<void**>(&cb.d_done), cb.h_done, 0));
+      CK(cudaEventCreateWithFlags(&cb.ev, cudaEventDisableTiming));
+    } else {
+      CK(cudaEventSynchronize(cb.ev));
+    }
+    std::memcpy(cb.h_ses, session + off, (size_t)m * 8);
+    std::memcpy(cb.h_done, done + off, (size_t)m);
+    // the kernel reads the pinned copy over the host link: no copy-engine transfer, so the
+    // update does not queue behind a staged batch's copy
+    CompleteArgs a{m, cb.d_ses, cb.d_done, c->sess, c->d_prot};
     launch_complete(a, st);
     CK(cudaGetLastError());
-    CK(cudaStreamSynchronize(st));  // staging is reused
+    CK(cudaEventRecord(cb.ev, st));
   }
   return MISAT_OK;
 }
