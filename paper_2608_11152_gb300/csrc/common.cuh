@@ -151,6 +151,22 @@ __device__ __forceinline__ void ld_bucket_keys_cg(const Bucket* b, unsigned long
 
 // Look a key up in one instance table (no concurrent writers).  Returns 1 if
 // resident.  Adds the number of buckets read to *reads.  Bounded by the table size.
+// Look a key up from bucket b0 on (the later buckets of its probe sequence, after a full
+// home bucket without it).  Adds the buckets read to *reads.
+__device__ __forceinline__ int table_contains_from(const InstDesc& d, uint64_t key, uint32_t b0, uint32_t* reads) {
+  const uint32_t mask = (1u << d.log2nb) - 1;
+  uint32_t b = b0;
+  for (uint32_t it = 0; it < mask; ++it) {
+    unsigned long long k[4];
+    ld_bucket_keys(d.tab + b, k);
+    *reads += 1;
+    if ((k[0] == key) | (k[1] == key) | (k[2] == key) | (k[3] == key)) return 1;
+    if ((k[0] == kEmpty) | (k[1] == kEmpty) | (k[2] == kEmpty) | (k[3] == kEmpty)) return 0;
+    b = (b + 1) & mask;
+  }
+  return 0;
+}
+
 __device__ __forceinline__ int table_contains(const InstDesc& d, uint64_t key, uint32_t* reads) {
   const uint32_t mask = (1u << d.log2nb) - 1;
   uint32_t b = home_bucket(key, d.log2nb);

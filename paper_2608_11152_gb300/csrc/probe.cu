@@ -84,6 +84,8 @@ __global__ void __launch_bounds__(256) k2_first_claim(ProbeArgs a) {
   }
 }
 
+constexpr int kDistIlp = 4;  // tables per lane with their home sectors in flight together
+
 __global__ void __launch_bounds__(256) k2_probe_distinct(ProbeArgs a) {
   __shared__ Bucket* s_tab[kMaxW];
   __shared__ uint32_t s_lg[kMaxW];
@@ -100,29 +102,48 @@ __global__ void __launch_bounds__(256) k2_probe_distinct(ProbeArgs a) {
   for (int d = (blockIdx.x * blockDim.x + threadIdx.x) >> 5; d < nd; d += (gridDim.x * blockDim.x) >> 5) {
     const int64_t slot = a.fb_list[d];
     const uint64_t key = a.fb.keys[slot];
-    for (int w0 = 0; w0 < a.W; w0 += 64) {
-      int h0 = 0, h1 = 0;
-      const int wa = w0 + lane, wb = w0 + 32 + lane;
-      if (wa < a.W) {
-        InstDesc dd;
-        dd.tab = s_tab[wa];
-        dd.log2nb = s_lg[wa];
-        uint32_t rd = 0;
-        h0 = table_contains(dd, key, &rd);
-        probes += 1;
-        reads += rd;
+    for (int w0 = 0; w0 < a.W; w0 += 32 * kDistIlp) {
+      // the home-bucket sectors of the lane's kDistIlp tables are requested before any is
+      // examined; a full home bucket without the key continues its probe sequence after
+      ulonglong2 k01[kDistIlp], k23[kDistIlp];
+#pragma unroll
+      for (int i = 0; i < kDistIlp; ++i) {
+        const int w = w0 + 32 * i + lane;
+        k01[i] = make_ulonglong2(kEmpty, kEmpty);
+        k23[i] = k01[i];
+        if (w < a.W) {
+          const ulonglong2* p = reinterpret_cast<const ulonglong2*>(s_tab[w][home_bucket(key, s_lg[w])].key);
+          k01[i] = __ldg(p);
+          k23[i] = __ldg(p + 1);
+        }
       }
-      if (wb < a.W) {
-        InstDesc dd;
-        dd.tab = s_tab[wb];
-        dd.log2nb = s_lg[wb];
-        uint32_t rd = 0;
-        h1 = table_contains(dd, key, &rd);
-        probes += 1;
-        reads += rd;
+#pragma unroll
+      for (int i = 0; i < kDistIlp; ++i) {
+        const int w = w0 + 32 * i + lane;
+        int h = 0;
+        if (w < a.W) {
+          h = (k01[i].x == key) | (k01[i].y == key) | (k23[i].x == key) | (k23[i].y == key);
+          const bool open =
+              (k01[i].x == kEmpty) | (k01[i].y == kEmpty) | (k23[i].x == kEmpty) | (k23[i].y == kEmpty);
+          uint32_t rd = 1;
+          if (!h && !open) {
+            InstDesc dd;
+            dd.tab = s_tab[w];
+            dd.log2nb = s_lg[w];
+            h = table_contains_from(dd, key, (home_bucket(key, dd.log2nb) + 1) & ((1u << dd.log2nb) - 1), &rd);
+          }
+          probes += 1;
+          reads += rd;
+        }
+        const unsigned m = __ballot_sync(0xffffffffu, h);
+        if (lane == 0) {
+          const int wb = w0 + 32 * i;
+          if (wb < a.W) {
+            unsigned* mw32 = reinterpret_cast<unsigned*>(a.fb.masks + (size_t)slot * mw);
+            mw32[wb >> 5] = m;  // 32-bit halves of the little-endian 64-bit mask words
+          }
+        }
       }
-      const unsigned m0 = __ballot_sync(0xffffffffu, h0), m1 = __ballot_sync(0xffffffffu, h1);
-      if (lane == 0) a.fb.masks[(size_t)slot * mw + (w0 >> 6)] = (unsigned long long)m0 | ((unsigned long long)m1 << 32);
     }
   }
   block_add_stats(a.stats, probes, reads);
