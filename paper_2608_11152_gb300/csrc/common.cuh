@@ -8,6 +8,28 @@
 
 namespace misat {
 
+// Blocks of `kernel` that fit on the GPU at once at this block size and dynamic shared memory
+// (resident blocks per SM x SMs; queried once per kernel).  A grid-stride loop with a static
+// split over this many blocks runs in one wave: with more blocks than fit, the blocks of the
+// second wave start only as the first finish, and a latency-bound pass takes about twice its
+// one-wave time.
+template <auto Kernel>
+inline int resident_grid(int block, size_t smem, int num_sms) {
+  static int per_sm = 0, last_block = -1;
+  static size_t last_smem = 0;
+  if (per_sm == 0 || block != last_block || smem != last_smem) {
+    int v = 0;
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&v, Kernel, block, smem) != cudaSuccess || v < 1) {
+      cudaGetLastError();
+      v = 1;
+    }
+    per_sm = v;
+    last_block = block;
+    last_smem = smem;
+  }
+  return per_sm * num_sms;
+}
+
 constexpr int kBlockTokens = 16;
 constexpr uint64_t kGold = 0x9e3779b97f4a7c15ull;  // SplitMix64 increment, chain multiplier
 constexpr uint64_t kEmpty = 0;                     // empty slot key (block keys are >= 2)

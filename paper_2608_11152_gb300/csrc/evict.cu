@@ -413,6 +413,49 @@ __global__ void __launch_bounds__(kSelThreads) k4_evict_select(EvictArgs a) {
 }
 
 namespace {
+// The apply passes take the entries of all instances over capacity as one index space, so
+// that every thread gets about the same number whatever the instances' shares: entry g
+// belongs to the k-th active instance with s_pre[k] <= g < s_pre[k + 1] (its D list first,
+// then its candidates).  Built by each CTA in shared memory; returns the total.
+__device__ unsigned long long list_prefix(const EvictArgs& a, unsigned long long* s_pre, int nact) {
+  // the lengths are loaded in parallel, then warp 0 scans them 32 at a time
+  for (int k = threadIdx.x; k < nact; k += blockDim.x) {
+    const int w = a.act[k];
+    s_pre[k + 1] = (unsigned long long)a.n_d[w] + a.n_cand[w];
+  }
+  __syncthreads();
+  if (threadIdx.x < 32) {
+    const int lane = threadIdx.x;
+    unsigned long long carry = 0;
+    for (int k0 = 0; k0 < nact; k0 += 32) {
+      const int k = k0 + lane;
+      const unsigned long long v = k < nact ? s_pre[k + 1] : 0;
+      unsigned long long incl = v;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const unsigned long long t = __shfl_up_sync(kFull, incl, o);
+        if (lane >= o) incl += t;
+      }
+      if (k < nact) s_pre[k + 1] = carry + incl;
+      carry += __shfl_sync(kFull, incl, 31);
+    }
+    if (lane == 0) s_pre[0] = 0;
+  }
+  __syncthreads();
+  return s_pre[nact];
+}
+
+// The k with s_pre[k] <= g < s_pre[k + 1] (binary search over nact entries).
+__device__ __forceinline__ int list_owner(const unsigned long long* s_pre, int nact, unsigned long long g) {
+  int lo = 0, hi = nact - 1;
+  while (lo < hi) {
+    const int mid = (lo + hi + 1) >> 1;
+    if (s_pre[mid] <= g) lo = mid;
+    else hi = mid - 1;
+  }
+  return lo;
+}
+
 // Delete slot sl of instance w's table; the global index (if any) loses bit w of its key.
 __device__ __forceinline__ void delete_slot(const GIndex& g, int w, Bucket* tab, uint32_t* dmask, uint32_t sl,
                                             int32_t* err) {
@@ -425,61 +468,66 @@ __device__ __forceinline__ void delete_slot(const GIndex& g, int w, Bucket* tab,
 }  // namespace
 
 // Delete D and the candidates at or below theta; record them in the deleted-slot masks.
-__device__ __forceinline__ void delete_chunk(const EvictArgs& a, int w, uint32_t cidx, uint32_t chunks) {
-  const unsigned nd = a.n_d[w], n = a.n_cand[w];
-  const uint32_t* dsl = a.dslots[w];
-  const uint4* c0 = a.cand_a[w];
-  const uint32_t* slots = a.slots[w];
-  uint32_t* dmask = a.dmask[w];
-  Bucket* tab = a.desc[w].tab;
-  const unsigned long long tm = a.theta[2 * w], tk = a.theta[2 * w + 1];
-  long long deleted = 0;
-  const unsigned stride = chunks * blockDim.x;
-  for (unsigned i = cidx * blockDim.x + threadIdx.x; i < nd + n; i += stride) {
+// Deletions are counted per instance in shared memory and added to the sizes once per CTA.
+__global__ void __launch_bounds__(256) k4_evict_delete(EvictArgs a) {
+  __shared__ unsigned long long s_pre[kMaxW + 1];
+  __shared__ unsigned s_del[kMaxW];
+  if (block_error(a.err)) return;
+  const int nact = (int)*(volatile const unsigned*)a.n_act;
+  for (int k = threadIdx.x; k < nact; k += blockDim.x) s_del[k] = 0;
+  const unsigned long long total = list_prefix(a, s_pre, nact);
+  const unsigned long long stride = (unsigned long long)gridDim.x * blockDim.x;
+  for (unsigned long long g = (unsigned long long)blockIdx.x * blockDim.x + threadIdx.x; g < total; g += stride) {
+    const int k = list_owner(s_pre, nact, g);
+    const int w = a.act[k];
+    const unsigned i = (unsigned)(g - s_pre[k]), nd = a.n_d[w];
+    uint32_t sl;
     if (i < nd) {
-      delete_slot(a.gix, w, tab, dmask, dsl[i], a.err);
-      ++deleted;
+      sl = a.dslots[w][i];
     } else {
-      const uint4 v = c0[i - nd];
-      if (!le128(v_hi(v), v_lo(v), tm, tk)) continue;
-      delete_slot(a.gix, w, tab, dmask, slots[i - nd], a.err);
-      ++deleted;
+      const uint4 v = a.cand_a[w][i - nd];
+      if (!le128(v_hi(v), v_lo(v), a.theta[2 * w], a.theta[2 * w + 1])) continue;
+      sl = a.slots[w][i - nd];
+    }
+    delete_slot(a.gix, w, a.desc[w].tab, a.dmask[w], sl, a.err);
+    atomicAdd(&s_del[k], 1u);
+  }
+  __syncthreads();
+  unsigned long long mine = 0;
+  for (int k = threadIdx.x; k < nact; k += blockDim.x) {
+    const unsigned d = s_del[k];
+    if (d) {
+      atomic_add_i64(&a.size[a.act[k]], -(long long)d);
+      mine += d;
     }
   }
-  const long long tot = block_sum(deleted);
-  if (threadIdx.x == 0 && tot) {
-    atomic_add_i64(&a.size[w], -tot);
-    atomicAdd(a.evicted, (unsigned long long)tot);
-  }
-}
-
-__global__ void __launch_bounds__(256) k4_evict_delete(EvictArgs a, uint32_t chunks) {
-  if (block_error(a.err)) return;
-  const uint32_t items = *(volatile const unsigned*)a.n_act * chunks;
-  for (uint32_t it = blockIdx.x; it < items; it += gridDim.x) delete_chunk(a, a.act[it / chunks], it % chunks, chunks);
+  const long long tot = block_sum((long long)mine);
+  if (threadIdx.x == 0 && tot) atomicAdd(a.evicted, (unsigned long long)tot);
 }
 
 // Refill the holes of every run of full buckets that lost an entry.  The thread of the
 // run's first deleted slot (lowest bucket, then lowest slot) owns the run.
-__device__ __forceinline__ void shift_chunk(const EvictArgs& a, int w, uint32_t cidx, uint32_t chunks) {
-  const unsigned nd = a.n_d[w], n = a.n_cand[w];
-  const uint32_t* dsl = a.dslots[w];
-  const uint4* c0 = a.cand_a[w];
-  const uint32_t* slots = a.slots[w];
-  const uint32_t* full = a.bitmaps[w];
-  const uint32_t* dmask = a.dmask[w];
-  const InstDesc d = a.desc[w];
-  const uint32_t NB = 1u << d.log2nb, mask = NB - 1;
-  const unsigned long long tm = a.theta[2 * w], tk = a.theta[2 * w + 1];
-  const unsigned stride = chunks * blockDim.x;
-  for (unsigned i = cidx * blockDim.x + threadIdx.x; i < nd + n; i += stride) {
+__global__ void __launch_bounds__(256) k4_evict_shift(EvictArgs a) {
+  __shared__ unsigned long long s_pre[kMaxW + 1];
+  if (block_error(a.err)) return;
+  const int nact = (int)*(volatile const unsigned*)a.n_act;
+  const unsigned long long total = list_prefix(a, s_pre, nact);
+  const unsigned long long stride = (unsigned long long)gridDim.x * blockDim.x;
+  for (unsigned long long g = (unsigned long long)blockIdx.x * blockDim.x + threadIdx.x; g < total; g += stride) {
+    const int k = list_owner(s_pre, nact, g);
+    const int w = a.act[k];
+    const unsigned i = (unsigned)(g - s_pre[k]), nd = a.n_d[w];
+    const uint32_t* full = a.bitmaps[w];
+    const uint32_t* dmask = a.dmask[w];
+    const InstDesc d = a.desc[w];
+    const uint32_t NB = 1u << d.log2nb, mask = NB - 1;
     uint32_t sl;
     if (i < nd) {
-      sl = dsl[i];
+      sl = a.dslots[w][i];
     } else {
-      const uint4 v = c0[i - nd];
-      if (!le128(v_hi(v), v_lo(v), tm, tk)) continue;
-      sl = slots[i - nd];
+      const uint4 v = a.cand_a[w][i - nd];
+      if (!le128(v_hi(v), v_lo(v), a.theta[2 * w], a.theta[2 * w + 1])) continue;
+      sl = a.slots[w][i - nd];
     }
     // the bitmap and deleted-mask words last read (runs are short: mostly one word each)
     uint32_t fw_i = 0xffffffffu, fw = 0, dw_i = 0xffffffffu, dw = 0;
@@ -564,17 +612,12 @@ __device__ __forceinline__ void shift_chunk(const EvictArgs& a, int w, uint32_t 
   }
 }
 
-__global__ void __launch_bounds__(256) k4_evict_shift(EvictArgs a, uint32_t chunks) {
-  if (block_error(a.err)) return;
-  const uint32_t items = *(volatile const unsigned*)a.n_act * chunks;
-  for (uint32_t it = blockIdx.x; it < items; it += gridDim.x) shift_chunk(a, a.act[it / chunks], it % chunks, chunks);
-}
 
 namespace {
-int stream_grid(const EvictArgs& a, int chunks_per_inst, int num_sms) {
+int stream_grid(const EvictArgs& a, int chunks_per_inst, int resident) {
   // streaming passes: resident CTAs over (active instance, chunk) items
   const int64_t items = (int64_t)(a.only_w ? 1 : a.W) * chunks_per_inst;
-  return (int)(items < (int64_t)num_sms * 8 ? items : (int64_t)num_sms * 8);
+  return (int)(items < (int64_t)resident ? items : (int64_t)resident);
 }
 }  // namespace
 
@@ -584,7 +627,8 @@ void launch_evict_select(const EvictArgs& a, int chunks_per_inst, int num_sms, c
   cudaMemsetAsync(a.n_act, 0, sizeof(unsigned), st);
   k4_evict_estimate<<<W, kSelThreads, 0, st>>>(a);
   if (marks) cudaEventRecord(marks[0], st);
-  k4_evict_collect<<<stream_grid(a, chunks_per_inst, num_sms), 256, 0, st>>>(a, (uint32_t)chunks_per_inst);
+  k4_evict_collect<<<stream_grid(a, chunks_per_inst, resident_grid<k4_evict_collect>(256, 0, num_sms)), 256, 0, st>>>(
+      a, (uint32_t)chunks_per_inst);
   if (marks) cudaEventRecord(marks[1], st);
   k4_evict_select<<<W, kSelThreads, 0, st>>>(a);
   if (marks) cudaEventRecord(marks[2], st);
@@ -592,14 +636,11 @@ void launch_evict_select(const EvictArgs& a, int chunks_per_inst, int num_sms, c
 
 void launch_evict_apply(const EvictArgs& a, int chunks_per_inst, int num_sms, cudaStream_t st,
                         const cudaEvent_t* marks) {
-  // the eviction lists (about E entries per instance) are split into fewer, larger pieces
-  // than the tables: each piece then holds several entries per thread
+  // one grid-stride pass over the list entries of every instance over capacity, one wave each
   (void)chunks_per_inst;
-  constexpr int kListChunks = 32;
-  const int grid = stream_grid(a, kListChunks, num_sms);
-  k4_evict_delete<<<grid, 256, 0, st>>>(a, (uint32_t)kListChunks);
+  k4_evict_delete<<<resident_grid<k4_evict_delete>(256, 0, num_sms), 256, 0, st>>>(a);
   if (marks) cudaEventRecord(marks[0], st);
-  k4_evict_shift<<<grid, 256, 0, st>>>(a, (uint32_t)kListChunks);
+  k4_evict_shift<<<resident_grid<k4_evict_shift>(256, 0, num_sms), 256, 0, st>>>(a);
   if (marks) cudaEventRecord(marks[1], st);
 }
 

@@ -349,14 +349,16 @@ void launch_probe_first(const ProbeArgs& a, int num_sms, cudaStream_t st) {
   if (total <= 0) return;
   const int groups = (a.n + 31) / 32;
   const int gblocks = (groups + 7) / 8;
-  const int ggrid = gblocks < num_sms * 8 ? gblocks : num_sms * 8;
+  const size_t gsmem = 8 * 32 * ((a.gix.keys ? a.gix.mw : a.fb.mw) * sizeof(unsigned long long) + sizeof(int2));
+  const int gres = resident_grid<k2_probe_first_gix>(256, gsmem, num_sms);
+  const int ggrid = gblocks < gres ? gblocks : gres;
   if (a.gix.keys) {
     k2_probe_first_gix<<<ggrid, 256, 8 * 32 * (a.gix.mw * sizeof(unsigned long long) + sizeof(int2)), st>>>(a);
     return;
   }
   // per-instance tables: the context allocates the batch-local index with the tables
   k2_first_claim<<<ggrid, 256, 0, st>>>(a);
-  k2_probe_distinct<<<num_sms * 8, 256, 0, st>>>(a);
+  k2_probe_distinct<<<num_sms * 8, 256, 0, st>>>(a);  // two waves: measured faster than one for this pass
   ProbeArgs e = a;
   e.gix = a.fb;
   e.stats = a.stats_fb;
@@ -365,7 +367,7 @@ void launch_probe_first(const ProbeArgs& a, int num_sms, cudaStream_t st) {
 
 void launch_probe_search(const ProbeArgs& a, int num_sms, cudaStream_t st) {
   if ((int64_t)a.n * a.W <= 0) return;
-  k2_probe_search<<<num_sms * 8, 256, 0, st>>>(a);
+  k2_probe_search<<<resident_grid<k2_probe_search>(256, 0, num_sms), 256, 0, st>>>(a);
 }
 
 }  // namespace misat
