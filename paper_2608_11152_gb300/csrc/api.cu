@@ -588,7 +588,7 @@ int evict_all(misat_ctx* c, unsigned long long* evicted_counter, cudaEvent_t joi
   if (rc) return rc;
   if (join) CK(cudaStreamWaitEvent(c->stream, join, 0));
   return run_graph(c, c->g_evict_apply, key,
-                   [&](cudaStream_t s) { launch_evict_apply(ev, chunks, c->num_sms, s, marks ? marks + 3 : nullptr); });
+                   [&](cudaStream_t s) { launch_evict_apply(ev, c->num_sms, s, marks ? marks + 3 : nullptr); });
 }
 
 CapsArgs caps_args(misat_ctx* c) {

@@ -634,10 +634,8 @@ void launch_evict_select(const EvictArgs& a, int chunks_per_inst, int num_sms, c
   if (marks) cudaEventRecord(marks[2], st);
 }
 
-void launch_evict_apply(const EvictArgs& a, int chunks_per_inst, int num_sms, cudaStream_t st,
-                        const cudaEvent_t* marks) {
+void launch_evict_apply(const EvictArgs& a, int num_sms, cudaStream_t st, const cudaEvent_t* marks) {
   // one grid-stride pass over the list entries of every instance over capacity, one wave each
-  (void)chunks_per_inst;
   k4_evict_delete<<<resident_grid<k4_evict_delete>(256, 0, num_sms), 256, 0, st>>>(a);
   if (marks) cudaEventRecord(marks[0], st);
   k4_evict_shift<<<resident_grid<k4_evict_shift>(256, 0, num_sms), 256, 0, st>>>(a);
@@ -646,7 +644,7 @@ void launch_evict_apply(const EvictArgs& a, int chunks_per_inst, int num_sms, cu
 
 void launch_evict(const EvictArgs& a, int chunks_per_inst, int num_sms, cudaStream_t st) {
   launch_evict_select(a, chunks_per_inst, num_sms, st, nullptr);
-  launch_evict_apply(a, chunks_per_inst, num_sms, st, nullptr);
+  launch_evict_apply(a, num_sms, st, nullptr);
 }
 
 // Compaction of one instance table: delete entries with meta == 0 (marked) or

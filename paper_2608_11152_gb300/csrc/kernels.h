@@ -316,7 +316,7 @@ void launch_evict(const EvictArgs& a, int chunks_per_inst, int num_sms, cudaStre
 // marks (may be NULL): events recorded after each kernel (select: 3, apply: 2), for phase timing
 void launch_evict_select(const EvictArgs& a, int chunks_per_inst, int num_sms, cudaStream_t st,
                          const cudaEvent_t* marks);
-void launch_evict_apply(const EvictArgs& a, int chunks_per_inst, int num_sms, cudaStream_t st,
+void launch_evict_apply(const EvictArgs& a, int num_sms, cudaStream_t st,
                         const cudaEvent_t* marks);
 void launch_compact_marked(const EvictArgs& a, cudaStream_t st);
 
