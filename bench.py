@@ -107,15 +107,18 @@ COMMIT_PHASES = ("insert", "gix_insert", "sessions", "evict")
 
 HASH_SOURCES = ("paper_2608_11152_gb300/csrc/hash.cu", "paper_2608_11152_gb300/csrc/common.cuh")
 HASH_PROFILE = os.path.join(ROOT, "profiles", "k1_block_hash_stress_n65536.md")
+SELECT_SOURCES = ("paper_2608_11152_gb300/csrc/select.cu", "paper_2608_11152_gb300/csrc/envelope.cuh",
+                  "paper_2608_11152_gb300/csrc/common.cuh")
+SELECT_PROFILE = os.path.join(ROOT, "profiles", "k4_select_class_stress_n65536.md")
 
 
-def hash_sources_sha256():
-    """sha256 of the block-hash kernel's sources with comments and blank space removed (a
-    comment edit does not make the committed ncu figures stale; a code edit does)."""
+def hash_sources_sha256(files=HASH_SOURCES):
+    """sha256 of a kernel's sources with comments and blank space removed (a comment edit
+    does not make the committed ncu figures stale; a code edit does)."""
     import re
 
     h = hashlib.sha256()
-    for f in HASH_SOURCES:
+    for f in files:
         with open(os.path.join(ROOT, f)) as fh:
             text = fh.read()
         text = re.sub(r"/\*.*?\*/", " ", text, flags=re.S)
@@ -124,21 +127,35 @@ def hash_sources_sha256():
     return h.hexdigest()
 
 
-def profiled_hash_fields():
-    """Figures of the block-hash kernel from the committed ncu summary (DRAM bytes per launch
-    and the batch's token count, ALU pipe occupancy), if that capture was taken with the
-    kernel's current sources; else {}."""
+def profiled_fields(path, sources):
+    """The machine-readable figures of a committed ncu summary, if that capture was taken with
+    the kernel's current sources; else {}."""
     try:
         fields = {}
-        for line in open(HASH_PROFILE):
+        for line in open(path):
             if ":" in line and line.startswith("- `"):
                 k, v = line[3:].split("`:", 1)
                 fields[k.strip()] = v.strip().strip("`")
-        if fields.get("sources_sha256") != hash_sources_sha256():
+        if fields.get("sources_sha256") != hash_sources_sha256(sources):
             return {}
         return fields
     except Exception:
         return {}
+
+
+def profiled_hash_fields():
+    """Figures of the block-hash kernel from its committed ncu summary (DRAM bytes per launch
+    and the batch's token count, ALU pipe occupancy), or {}."""
+    return profiled_fields(HASH_PROFILE, HASH_SOURCES)
+
+
+def profiled_select_traffic(n, instances):
+    """DRAM bytes per launch of the per-class selection from its committed ncu summary, when
+    that capture's workload is this one (the stress batch at 128 instances), else None."""
+    f = profiled_fields(SELECT_PROFILE, SELECT_SOURCES)
+    if not f or int(f["batch_requests"]) != int(n) or int(f["instances"]) != int(instances):
+        return None
+    return int(f["traffic_bytes_per_launch"])
 
 
 def profiled_traffic(batch_tokens):
@@ -674,13 +691,17 @@ def run_gb300(args):
             # the kernel's actual limiter: integer ALU issue (ncu sm__pipe_alu_cycles_active)
             kernels["hash"]["alu_pipe_active_frac_ncu"] = float(hf["alu_pipe_active_frac"])
     if kernels["select"] is not None:
+        if args.config == 5:
+            kernels["select"]["traffic"] = profiled_select_traffic(sc.batch.n, sc.W)
         kernels["select"]["limiter"] = ("one CTA per class walks its leaders in arrival order; bound by the "
                                         "chain of headroom-exhaustion events (barrier-separated steps), not by memory")
     # dominant kernel: the largest time per launch
     dom = max((k for k in kernels if kernels[k]), key=lambda k: kernels[k]["ms_per_launch"])
     dom_roof = dict(kernels[dom])
-    if dom == "hash":
+    if dom == "hash" and dom_roof.get("traffic") is not None:
         dom_roof["traffic_source"] = "profiles/k1_block_hash_stress_n65536.md (ncu dram__bytes_read.sum + dram__bytes_write.sum)"
+    if dom == "select" and dom_roof.get("traffic") is not None:
+        dom_roof["traffic_source"] = "profiles/k4_select_class_stress_n65536.md (ncu dram__bytes_read.sum + dram__bytes_write.sum)"
 
     clocks = sampler.summary()
     line = {
