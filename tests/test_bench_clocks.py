@@ -41,3 +41,35 @@ def test_launch_count_claim_matches_the_committed_launch_list():
     global_index = "prefix index: global" in text
     totals = [int(m.group(1)) for m in re.finditer(r"\| \*\*total\*\* \| (\d+) \|", text)]
     assert totals and all(t == 2 * bench.kernels_per_step(global_index) for t in totals)
+
+
+def test_profiled_figures_are_read_only_while_the_sources_match(tmp_path):
+    """A committed ncu summary's machine-readable figures count only while the kernel's
+    sources (comments and blank space aside) hash to the recorded value."""
+    src = tmp_path / "k.cu"
+    src.write_text("__global__ void k() { int x = 1; }  // first version\n")
+    sha = bench.hash_sources_sha256((str(src),))
+    summ = tmp_path / "k.md"
+    summ.write_text("# ncu\n\n- `traffic_bytes_per_launch`: `123`\n- `batch_requests`: `65536`\n"
+                    f"- `instances`: `128`\n- `sources_sha256`: `{sha}`\n")
+    f = bench.profiled_fields(str(summ), (str(src),))
+    assert f["traffic_bytes_per_launch"] == "123" and f["instances"] == "128"
+    src.write_text("__global__ void k() { int x = 1; }  /* a comment edit */\n")
+    assert bench.profiled_fields(str(summ), (str(src),))["traffic_bytes_per_launch"] == "123"
+    src.write_text("__global__ void k() { int x = 2; }\n")
+    assert bench.profiled_fields(str(summ), (str(src),)) == {}
+
+
+def test_selection_traffic_is_reported_for_the_captured_workload_only():
+    """The per-class selection's DRAM bytes were captured on the stress batch (65,536 requests,
+    128 instances): another workload gets no figure."""
+    import os
+
+    f = bench.profiled_fields(bench.SELECT_PROFILE, bench.SELECT_SOURCES)
+    if not f:  # the kernel changed since the capture: nothing is reported at all
+        assert bench.profiled_select_traffic(65536, 128) is None
+        return
+    assert bench.profiled_select_traffic(65536, 128) == int(f["traffic_bytes_per_launch"])
+    assert bench.profiled_select_traffic(4096, 128) is None
+    assert bench.profiled_select_traffic(65536, 64) is None
+    assert os.path.exists(bench.SELECT_PROFILE)
