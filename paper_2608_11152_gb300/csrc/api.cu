@@ -1383,13 +1383,22 @@ int misat_complete(misat_ctx* c, int32_t n, const uint64_t* session, const uint8
     const int m = std::min(c->max_batch, n - off);
     misat_ctx::CompBuf& cb = c->comp[c->comp_turn];
     c->comp_turn ^= 1;
-    if (!cb.h_ses) {
-      if (cudaHostAlloc(&cb.h_ses, (size_t)c->max_batch * 8, cudaHostAllocMapped) != cudaSuccess ||
-          cudaHostAlloc(&cb.h_done, (size_t)c->max_batch, cudaHostAllocMapped) != cudaSuccess)
+    if (!cb.ev) {
+      // first use: mapped pinned buffers and their event; on any failure nothing is kept
+      const bool ok =
+          cudaHostAlloc(&cb.h_ses, (size_t)c->max_batch * 8, cudaHostAllocMapped) == cudaSuccess &&
+          cudaHostAlloc(&cb.h_done, (size_t)c->max_batch, cudaHostAllocMapped) == cudaSuccess &&
+          cudaHostGetDevicePointer(reinterpret_cast<void**>(&cb.d_ses), cb.h_ses, 0) == cudaSuccess &&
+          cudaHostGetDevicePointer(reinterpret_cast<void**>(&cb.d_done), cb.h_done, 0) == cudaSuccess &&
+          cudaEventCreateWithFlags(&cb.ev, cudaEventDisableTiming) == cudaSuccess;
+      if (!ok) {
+        cudaGetLastError();
+        if (cb.h_ses) cudaFreeHost(cb.h_ses);
+        if (cb.h_done) cudaFreeHost(cb.h_done);
+        if (cb.ev) cudaEventDestroy(cb.ev);
+        cb = misat_ctx::CompBuf{};
         return MISAT_ERR_OOM;
-      CK(cudaHostGetDevicePointer(reinterpret_cast<void**>(&cb.d_ses), cb.h_ses, 0));
-      CK(cudaHostGetDevicePointer(reinterpret_cast<void**>(&cb.d_done), cb.h_done, 0));
-      CK(cudaEventCreateWithFlags(&cb.ev, cudaEventDisableTiming));
+      }
     } else {
       CK(cudaEventSynchronize(cb.ev));
     }
